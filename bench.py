@@ -1,0 +1,322 @@
+"""Benchmark: budgeted KV-cache repair on the Llama-3-8B-shaped workload.
+
+Workload: random-init bf16 Llama-3-8B-shaped model (32 layers, d 4096,
+32/8 heads, FFN 14336, vocab 128256), a cached document of 5000 uniform
+random tokens, an 8-token same-length edit at position 2500, EditLocal
+K = 32, so P = 40 rows recomputed through all 32 layers.
+
+One step = the hot path once: kvr_select (EditLocal) + kvr_repair (edit
+apply, then the 40 rows through every layer, K/V written back in place).
+The full re-prefill of the edited 5000-token document is timed separately
+as the baseline the speedup is quoted against.
+
+Prints one JSON line (rank 0).  --impl reference times the CPU oracle on a
+bounded sample of the same workload instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+WORKLOAD = "llama8b"
+N_CTX, EDIT_START, EDIT_LEN, K_BUDGET = 5000, 2500, 8, 32
+METRIC = "repair latency ms & positions/s at K=32, 5k ctx; speedup vs full re-prefill"
+
+
+def load_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+class Clocks:
+    """Samples nvidia-smi clocks and throttle reasons while running."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.rows = []
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except Exception:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.rows.append([x.strip() for x in line.split(",")])
+
+    def __exit__(self, *a):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in self.rows:
+            try:
+                sm.append(float(r[1]))
+                mx = float(r[2])
+                for i, nm in enumerate(names):
+                    if r[5 + i].lower() == "active":
+                        reasons.add(nm)
+            except (ValueError, IndexError):
+                continue
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def edit_inputs(cfg):
+    from paper_2609_17983_gb300 import synth
+    doc = synth.document(1, N_CTX, cfg["vocab"], cfg["delim_id"])
+    new = synth.edit_tokens(2, doc[EDIT_START:EDIT_START + EDIT_LEN], cfg["vocab"],
+                            cfg["delim_id"])
+    return doc, new
+
+
+# ------------------------------------------------------------- CPU oracle
+
+def oracle_sample(cfg, layers: int):
+    """Time the oracle's operator R for the 40 rows of the workload through
+    `layers` layers of the 8B shape (one layer's seeded weights reused for
+    every sampled layer; a seeded synthetic stale cache of the document's
+    length).  Returns (seconds per layer, threads)."""
+    import oracle
+    from paper_2609_17983_gb300 import synth
+    threads = oracle.set_threads(os.cpu_count() or 1)
+    doc, new = edit_inputs(cfg)
+    edited = doc.copy()
+    edited[EDIT_START:EDIT_START + EDIT_LEN] = new
+    P = np.arange(EDIT_START, EDIT_START + EDIT_LEN + K_BUDGET)
+    used = np.unique(edited[P])
+    remap = {int(t): i for i, t in enumerate(used)}
+    ly = synth.layer_weights(cfg, 0, 0)
+    W = dict(embed=synth.rows(0, synth.TID_EMBED, used, cfg["d_model"], cfg["dtype"]),
+             final_norm=synth.ones(cfg["d_model"], cfg["dtype"]), lm_head=None,
+             layers=[ly] * layers)
+    ocfg = dict(cfg, n_layers=layers, vocab=len(used))
+    toks = np.zeros(N_CTX, np.int32)
+    toks[P] = [remap[int(t)] for t in edited[P]]
+    cache = oracle.empty_cache(ocfg, N_CTX)
+    g = synth.tensor(3, 999, cache.k.shape, "fp32")
+    cache.k[:] = g
+    cache.v[:] = g[::-1]
+    t0 = time.perf_counter()
+    oracle.recompute(ocfg, W, cache, toks, P)
+    dt = time.perf_counter() - t0
+    return dt / layers, threads
+
+
+def run_reference(args, cfg, rank):
+    if rank != 0:
+        return None
+    M = EDIT_LEN + K_BUDGET
+    times = []
+    threads = 1
+    for i in range(args.warmup + args.steps):
+        per_layer, threads = oracle_sample(cfg, args.oracle_layers)
+        if i >= args.warmup:
+            times.append(per_layer * cfg["n_layers"])
+    t = statistics.median(times)
+    val = M / t
+    sample = (f"oracle operator R on the {M} rows through {args.oracle_layers} of "
+              f"{cfg['n_layers']} layers per step, scaled to all layers")
+    return {"metric": METRIC, "value": val, "unit": "positions/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": t * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "impl": "reference",
+            "config": {"workload": f"{WORKLOAD}: n={N_CTX}, edit {EDIT_LEN}@{EDIT_START}, "
+                                   f"editlocal K={K_BUDGET}"},
+            "cpu_baseline": {"value": val, "unit": "positions/s", "cores": threads,
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": val, "unit": "positions/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+
+
+# ------------------------------------------------------------- GPU arm
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="kvrepair", choices=["kvrepair", "reference"])
+    ap.add_argument("--prefill-steps", type=int, default=3)
+    ap.add_argument("--oracle-layers", type=int, default=4)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+
+    from paper_2609_17983_gb300 import synth
+    cfg = synth.preset(WORKLOAD)
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+
+    if args.impl == "reference":
+        out = run_reference(args, cfg, rank)
+        if out is not None:
+            print(json.dumps(out), flush=True)
+        return
+
+    # the CPU baseline runs before any GPU work (no forked workers after CUDA init)
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        per_layer, threads = oracle_sample(cfg, args.oracle_layers)
+        M = EDIT_LEN + K_BUDGET
+        cpu = {"value": M / (per_layer * cfg["n_layers"]), "unit": "positions/s",
+               "cores": threads, "kind": "oracle",
+               "sample": f"oracle operator R on the {M} rows through {args.oracle_layers} of "
+                         f"{cfg['n_layers']} layers (one step), scaled to all layers"}
+
+    import torch
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    from paper_2609_17983_gb300 import kvrepair as kv
+
+    stream = torch.cuda.current_stream()
+    model = kv.Model(cfg, None, seed=0, max_context=8192, max_rows=4096)
+    model.set_stream(stream.cuda_stream)
+    doc, new = edit_inputs(cfg)
+    cache = model.prefill(doc)
+    model.synchronize()
+    M = EDIT_LEN + K_BUDGET
+
+    def step():
+        A = model.select(cache, "editlocal", K_BUDGET, EDIT_START, new)
+        cache.repair(new, EDIT_START, A)
+
+    def barrier():
+        torch.cuda.synchronize()
+        if world > 1:
+            torch.distributed.barrier()
+        torch.cuda.synchronize()
+
+    for _ in range(args.warmup):
+        step()
+    barrier()
+    l0 = model.launches()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with Clocks(local) as clk:
+        ev0.record(stream)
+        for _ in range(args.steps):
+            step()
+        ev1.record(stream)
+        barrier()
+    ms = ev0.elapsed_time(ev1) / args.steps
+    launches = model.launches() - l0
+    if world > 1:
+        t = torch.tensor([ms], device="cuda")
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms = float(t.item())
+    value = world * M / (ms / 1e3)
+
+    # per-kernel-class device time over the same steps (CUDA events on the stream)
+    kv.kvr_profile_reset(model.h)
+    kv.kvr_profile_enable(model.h, True)
+    for _ in range(args.steps):
+        step()
+    model.synchronize()
+    prof = kv.kvr_profile_read(model.h)
+    kv.kvr_profile_enable(model.h, False)
+    gemms = {k: v for k, v in prof.items() if k.startswith("gemm") and v["launches"]}
+    dom = max(gemms, key=lambda k: gemms[k]["ms"])
+    d = gemms[dom]
+    peak, peak_kind = load_peaks()
+    achieved = d["bytes"] / d["launches"] / (d["ms"] / d["launches"] / 1e3) / 1e9
+    all_w = sum(v["bytes"] for v in gemms.values())
+    all_ms = sum(v["ms"] for v in gemms.values())
+
+    # e2e through the public API: host inputs in, repaired rows out
+    P = np.concatenate([np.arange(EDIT_START, EDIT_START + EDIT_LEN),
+                        np.arange(EDIT_START + EDIT_LEN, EDIT_START + EDIT_LEN + K_BUDGET)])
+    barrier()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        A = model.select(cache, "editlocal", K_BUDGET, EDIT_START, new)
+        cache.repair(new, EDIT_START, A)
+        k_rows, v_rows = cache.read(P)
+    barrier()
+    e2e_s = (time.perf_counter() - t0) / args.steps
+    h2d = int(new.nbytes + 4 * K_BUDGET + 4 * M)
+    d2h = int(k_rows.nbytes + v_rows.nbytes + 4 * K_BUDGET)
+
+    # the baseline: full re-prefill of the edited document
+    edited = doc.copy()
+    edited[EDIT_START:EDIT_START + EDIT_LEN] = new
+    pre = []
+    for i in range(1 + args.prefill_steps):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        c2 = model.prefill(edited)
+        b.record(stream)
+        torch.cuda.synchronize()
+        c2.close()
+        if i:
+            pre.append(a.elapsed_time(b))
+    prefill_ms = statistics.median(pre)
+
+    if rank == 0:
+        out = {"metric": METRIC, "value": value, "unit": "positions/s", "n_gpus": world,
+               "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+               "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+               "dtype": "bf16", "data": "synthetic (seeded random-init weights and tokens)",
+               "config": {"workload": f"{WORKLOAD}: Llama-3-8B shape, n={N_CTX}, "
+                                      f"edit {EDIT_LEN}@{EDIT_START}, editlocal K={K_BUDGET}",
+                          "rows": M, "layers": cfg["n_layers"],
+                          "parallelism": "replicas" if world > 1 else "single",
+                          "l2": "inputs larger than L2 (14 GB of weights streamed per step)"},
+               "repair_ms": ms, "prefill_ms": prefill_ms, "speedup_vs_prefill": prefill_ms / ms,
+               "token_layers_per_s": value * cfg["n_layers"],
+               "gpu_launches": launches,
+               "e2e": {"value": world * M / e2e_s, "unit": "positions/s",
+                       "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+               "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peak,
+                            "unit": "GB/s", "frac": achieved / peak, "traffic": None,
+                            "peak_kind": peak_kind,
+                            "all_gemms_gbs": all_w / (all_ms / 1e3) / 1e9},
+               "kernel_ms_per_step": {k: v["ms"] / args.steps for k, v in prof.items()
+                                      if v["launches"]},
+               "clocks": clk.summary(),
+               "cpu_baseline": cpu}
+        print(json.dumps(out), flush=True)
+    cache.close()
+    model.close()
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,214 @@
+/*
+ * kvrepair.h -- C ABI of libkvrepair: budgeted in-place repair of a stale KV
+ * cache after a same-length document edit, on one GB300 GPU (sm_103a).
+ *
+ * Method: "Contiguity, Not Importance: Budgeted Repair of Stale KV Caches
+ * After Document Edits", Sec. 3.  A context C of n tokens is prefilled and
+ * its key/value states K(C) are cached.  An edit replaces the half-open span
+ * S = [s_start, s_end) with the same number of new tokens, giving C'.  Repair
+ * recomputes the positions P = S u A, A a subset of the pool D = [s_end, n),
+ * from C' layer by layer against the otherwise-stale cache and writes the
+ * refreshed K/V back in place (operator R, Eq. 1).  A is chosen by one of the
+ * five selection policies of Table 1.
+ *
+ * Conventions for every entry point:
+ *   - Return value: KVR_OK (0) or an error code below; kvr_last_error()
+ *     returns a message for the calling thread's last failure.
+ *   - Token, position and output arrays are HOST pointers (int32 / float),
+ *     owned by the caller and only read/written during the call.
+ *   - Model and cache handles are owned by the library and freed with
+ *     kvr_model_free / kvr_cache_free.  A cache must be freed before its model.
+ *   - Device work is enqueued on the model's stream (kvr_model_set_stream;
+ *     default: the legacy default stream).  Calls that return data to the host
+ *     (kvr_select, kvr_logits, kvr_cache_read*) synchronise that stream;
+ *     kvr_prefill and kvr_repair return once the work is enqueued.
+ *   - Argument errors are detected on the host before any device work and
+ *     leave the cache unchanged.  A CUDA error during device work marks the
+ *     cache poisoned; every later call on it returns KVR_E_POISONED.
+ *   - Device waits (mbarrier spins in the tensor-core kernels) are bounded;
+ *     a wait that runs out sets a device flag that kvr_synchronize (and the
+ *     synchronising calls) report as KVR_E_DEVICE_TIMEOUT.
+ *   - Not thread-safe per model: calls on one model (and its caches) must not
+ *     overlap.
+ */
+#ifndef KVREPAIR_H
+#define KVREPAIR_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int32_t kvr_status;
+#define KVR_OK 0
+#define KVR_E_INVAL 1          /* malformed argument (NULL handle, bad config) */
+#define KVR_E_RANGE 2          /* span / positions / tokens out of range */
+#define KVR_E_NOMEM 3          /* device or host allocation failed */
+#define KVR_E_CUDA 4           /* CUDA runtime or kernel error */
+#define KVR_E_DEVICE_TIMEOUT 5 /* a bounded device wait ran out */
+#define KVR_E_UNSUPPORTED 6    /* shape or option this build does not handle */
+#define KVR_E_POISONED 7       /* cache was left inconsistent by an earlier CUDA error */
+
+typedef enum { KVR_DTYPE_F32 = 0, KVR_DTYPE_BF16 = 1 } kvr_dtype;
+
+/* Selection policies of Table 1.  All pick from the pool D = [s_end, n). */
+typedef enum {
+  KVR_POLICY_EDITLOCAL = 0,  /* the K positions immediately after the span */
+  KVR_POLICY_STRUCTURAL = 1, /* delimiter tokens, nearest to the span first */
+  KVR_POLICY_ATTENTION = 2,  /* top-K stale-cache attention from the span queries */
+  KVR_POLICY_CACHEBLEND = 3, /* top-K layer-1 (0-indexed) K/V deviation */
+  KVR_POLICY_RANDOM = 4      /* uniform K-subset, seeded */
+} kvr_policy;
+
+/* Llama-style decoder shape (RMSNorm, rotate-half RoPE, GQA, SwiGLU). */
+typedef struct {
+  int32_t vocab, d_model, n_layers, n_heads, n_kv_heads, head_dim, ffn;
+  int32_t qkv_bias;    /* 1: q/k/v projections carry a bias */
+  int32_t dtype;       /* kvr_dtype of weights, GEMM operands and the KV cache */
+  int32_t delim_id;    /* structural delimiter token id */
+  double rope_theta;   /* RoPE base */
+  double rms_eps;      /* RMSNorm epsilon */
+  int32_t max_context; /* longest context a cache of this model may hold */
+  int32_t max_rows;    /* rows per layer pass (prefill is chunked to this); >= 64 */
+} kvr_model_config;
+
+/* Host weights in canonical layout and the model dtype (fp32, or bf16 as
+ * uint16 bit patterns).  Matrices are row-major [out_features][in_features]:
+ * wq [H*dh][d], wk/wv [G*dh][d], wo [d][H*dh], wg/wu [ffn][d], wd [d][ffn],
+ * embed/lm_head [vocab][d]; norms [d]; biases [H*dh] / [G*dh] (NULL without
+ * qkv_bias).  Per-layer fields are arrays of n_layers pointers.  The library
+ * copies everything; the caller keeps ownership. */
+typedef struct {
+  const void *embed, *final_norm, *lm_head;
+  const void *const *attn_norm, *const *wq, *const *wk, *const *wv, *const *wo;
+  const void *const *bq, *const *bk, *const *bv;
+  const void *const *mlp_norm, *const *wg, *const *wu, *const *wd;
+} kvr_weights;
+
+typedef struct kvr_model kvr_model;
+typedef struct kvr_cache kvr_cache;
+
+/* Optional device allocator (e.g. PyTorch's caching allocator).  Must be set
+ * before the first kvr_model_create; NULL functions restore cudaMalloc/cudaFree. */
+typedef void *(*kvr_alloc_fn)(size_t bytes, void *ctx);
+typedef void (*kvr_free_fn)(void *ptr, void *ctx);
+kvr_status kvr_set_allocator(kvr_alloc_fn alloc, kvr_free_fn free_fn, void *ctx);
+
+/* Create a model on the current CUDA device.  weights == NULL: seeded random
+ * init, generated on the device: tensor t draws from SplitMix64 stream
+ * s_t = out(seed, t), element i (canonical row-major index) from
+ * r = out(s_t, i), where out(s, i) = mix(s + (i+1) * 0x9E3779B97F4A7C15);
+ * the four 16-bit lanes of r are summed, centred and scaled in double to
+ * std 0.02, rounded to fp32 and then to the model dtype; norms are 1.  Tensor
+ * ids: embed 0, lm_head 1, layer l: 8 + 16 l + {wq 0, wk 1, wv 2, wo 3, wg 4,
+ * wu 5, wd 6, bq 7, bk 8, bv 9}.  Errors: KVR_E_INVAL (config),
+ * KVR_E_UNSUPPORTED (shape), KVR_E_NOMEM. */
+kvr_status kvr_model_create(const kvr_model_config *config, const kvr_weights *weights,
+                            uint64_t seed, kvr_model **out);
+void kvr_model_free(kvr_model *model);
+
+/* Launch all device work of `model` (and its caches) on `cuda_stream`
+ * (a cudaStream_t; NULL = legacy default stream). */
+kvr_status kvr_model_set_stream(kvr_model *model, void *cuda_stream);
+
+/* Block until the model's stream is idle; reports device-side timeouts. */
+kvr_status kvr_synchronize(kvr_model *model);
+
+/* Full prefill K(C) (Sec. 3: the oracle target; Table 4's baseline).
+ * tokens: host int32[n], 0 <= id < vocab, 1 <= n <= max_context.  The new
+ * cache owns a device copy of the tokens and paged K/V for every layer. */
+kvr_status kvr_prefill(kvr_model *model, const int32_t *tokens, int32_t n, kvr_cache **out);
+void kvr_cache_free(kvr_cache *cache);
+
+/* Select A (Table 1; Sec. 3 "Cost accounting": selector work is outside K).
+ * The edit [edit_start, edit_start+edit_len) with host new_tokens[edit_len]
+ * is applied to a private copy of the context, not to the cache; the
+ * ATTENTION and CACHEBLEND policies run their model passes against the stale
+ * cache and leave it bit-identical.  positions_out: host int32[K], receives
+ * *count_out ascending positions in [edit_end, n).  *count_out == K except
+ * for STRUCTURAL when the pool holds fewer delimiters, and when the pool is
+ * smaller than K.  Ties go to the lowest position.  Errors: KVR_E_RANGE. */
+kvr_status kvr_select(kvr_model *model, const kvr_cache *cache, kvr_policy policy, int32_t K,
+                      int32_t edit_start, int32_t edit_len, const int32_t *new_tokens,
+                      uint64_t seed, int32_t *positions_out, int32_t *count_out);
+
+/* Repair in place (operator R, Sec. 3 "The repair interface", Eq. 1):
+ * write new_tokens into [edit_start, edit_start+edit_len) of the cached
+ * context, then recompute P = S u positions through every layer; all rows of
+ * P get fresh K/V at a layer before any of them attends there, every entry
+ * outside P is left unchanged.  positions: host int32[n_positions], strictly
+ * increasing, in [edit_end, n).  edit_len may be 0 (recompute positions
+ * only).  |P| <= max_rows.  Errors: KVR_E_RANGE (span, positions, token ids),
+ * KVR_E_UNSUPPORTED (|P| > max_rows). */
+kvr_status kvr_repair(kvr_cache *cache, const int32_t *new_tokens, int32_t edit_start,
+                      int32_t edit_len, const int32_t *positions, int32_t n_positions);
+
+/* One repair request of a batch: a cache, its edits and the union of the
+ * selected positions.  Edits must not overlap; positions must not fall in
+ * any edit span. */
+typedef struct {
+  kvr_cache *cache;
+  int32_t n_edits;
+  const int32_t *edit_start; /* [n_edits] */
+  const int32_t *edit_len;   /* [n_edits] */
+  const int32_t *new_tokens; /* concatenated, sum(edit_len) ids */
+  const int32_t *positions;  /* [n_positions], strictly increasing */
+  int32_t n_positions;
+} kvr_repair_req;
+
+/* Several documents, several edits each (beyond the paper's single edit;
+ * P_doc = sorted union of all spans and positions), recomputed in one
+ * layer-major pass over all rows of all requests.  All caches belong to
+ * `model`.  Sum of |P_doc| <= max_rows. */
+kvr_status kvr_repair_batch(kvr_model *model, const kvr_repair_req *reqs, int32_t n_reqs);
+
+/* Fresh-query logits (Sec. 3: the fresh query is never cached and is
+ * recomputed for scoring).  The m query tokens (1 <= m <= 64) take positions
+ * n..n+m-1 and attend to the cache; the document's K/V are not modified.
+ * logits_out: host float[vocab], the logits of the last query row. */
+kvr_status kvr_logits(kvr_model *model, const kvr_cache *cache, const int32_t *query, int32_t m,
+                      float *logits_out);
+
+/* ---- inspection (tests, benchmarks) ---- */
+
+/* Number of cached positions n. */
+int32_t kvr_cache_len(const kvr_cache *cache);
+
+/* Copy the cached context's tokens into host int32[n]. */
+kvr_status kvr_cache_tokens(const kvr_cache *cache, int32_t *tokens_out);
+
+/* Read K and V of the given positions for layers [layer_begin, layer_end)
+ * into host float arrays laid out [n_pos][layer_end-layer_begin][n_kv_heads]
+ * [head_dim] (bf16 entries are widened exactly). */
+kvr_status kvr_cache_read(const kvr_cache *cache, const int32_t *positions, int32_t n_pos,
+                          int32_t layer_begin, int32_t layer_end, float *k_out, float *v_out);
+
+/* Read one weight tensor back in canonical layout and model dtype into host
+ * memory of `bytes` bytes.  name: "embed", "lm_head", "final_norm", or per
+ * layer "wq","wk","wv","wo","wg","wu","wd","bq","bk","bv","attn_norm",
+ * "mlp_norm".  Norms and biases are returned in the model dtype too. */
+kvr_status kvr_model_read_tensor(const kvr_model *model, const char *name, int32_t layer,
+                                 void *out, size_t bytes);
+
+/* Per-kernel-class device timing with CUDA events around each launch group.
+ * enable != 0 turns it on for later calls; kvr_profile_read returns, for
+ * up to `cap` classes, the accumulated milliseconds and launch counts since
+ * the last reset, and writes the class names (NUL-separated) into `names`.
+ * Returns the number of classes via *n_out. */
+kvr_status kvr_profile_enable(kvr_model *model, int32_t enable);
+kvr_status kvr_profile_reset(kvr_model *model);
+kvr_status kvr_profile_read(kvr_model *model, int32_t cap, double *ms_out, int64_t *launches_out,
+                            int64_t *bytes_out, char *names, int32_t names_cap, int32_t *n_out);
+
+/* Number of library kernels launched so far on this model. */
+int64_t kvr_launch_count(const kvr_model *model);
+
+/* Message of the calling thread's last failure ("" if none). */
+const char *kvr_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* KVREPAIR_H */

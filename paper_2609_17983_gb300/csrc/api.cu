@@ -1,0 +1,1118 @@
+// api.cu -- the C ABI of libkvrepair and its host-side orchestration.
+//
+// Every entry point validates its arguments on the host, then enqueues the
+// layer-major pass of the repair operator R (Sec. 3, Eq. 1) on the model's
+// stream: embedding gather of the rows, then per layer RMSNorm -> QKV GEMM ->
+// RoPE at the original positions + K/V scatter of all rows -> scattered-query
+// attention -> O GEMM (+residual) -> RMSNorm -> gate/up GEMM -> SwiGLU ->
+// down GEMM (+residual).
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "kvr_internal.cuh"
+
+using namespace kvr;
+
+namespace {
+
+thread_local std::string g_err;
+
+kvr_status fail(kvr_status code, const char *fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  g_err = buf;
+  return code;
+}
+
+kvr_alloc_fn g_alloc = nullptr;
+kvr_free_fn g_free = nullptr;
+void *g_alloc_ctx = nullptr;
+
+#define CUDA_TRY(expr)                                                                   \
+  do {                                                                                   \
+    cudaError_t e__ = (expr);                                                            \
+    if (e__ != cudaSuccess)                                                              \
+      return fail(e__ == cudaErrorMemoryAllocation ? KVR_E_NOMEM : KVR_E_CUDA, "%s: %s", \
+                  #expr, cudaGetErrorString(e__));                                       \
+  } while (0)
+
+#define KVR_TRY(expr)           \
+  do {                          \
+    kvr_status s__ = (expr);    \
+    if (s__ != KVR_OK) return s__; \
+  } while (0)
+
+kvr_status launch_check(kvr_model *m, int kernels) {
+  m->launches += kernels;
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return fail(KVR_E_CUDA, "kernel launch: %s", cudaGetErrorString(e));
+  return KVR_OK;
+}
+
+// ------------------------------------------------------------ profiling
+
+enum ProfId {
+  P_EMBED, P_NORM, P_GEMM_QKV, P_ROPE, P_ATTN, P_GEMM_O, P_GEMM_GU, P_SWIGLU, P_GEMM_DOWN,
+  P_LMHEAD, P_SELECT, P_NCLASS
+};
+const char *kProfNames[P_NCLASS] = {"embed",  "rmsnorm",  "gemm_qkv",  "rope_scatter",
+                                    "attention", "gemm_o", "gemm_gu",   "swiglu",
+                                    "gemm_down", "lm_head", "select"};
+
+struct Prof {
+  kvr_model *m;
+  int cls;
+  int64_t bytes;
+  cudaEvent_t a = nullptr, b = nullptr;
+  Prof(kvr_model *mm, int c, int64_t by) : m(mm), cls(c), bytes(by) {
+    if (!m->prof) return;
+    cudaEventCreate(&a);
+    cudaEventCreate(&b);
+    cudaEventRecord(a, m->stream);
+  }
+  ~Prof() {
+    if (!m->prof || !a) return;
+    cudaEventRecord(b, m->stream);
+    m->prof_pending.push_back({cls, {a, b}});
+    m->prof_classes[cls].launches += 1;
+    m->prof_classes[cls].bytes += bytes;
+  }
+};
+
+void prof_collect(kvr_model *m) {
+  for (auto &p : m->prof_pending) {
+    float ms = 0.f;
+    cudaEventSynchronize(p.second.second);
+    cudaEventElapsedTime(&ms, p.second.first, p.second.second);
+    m->prof_classes[p.first].ms += ms;
+    cudaEventDestroy(p.second.first);
+    cudaEventDestroy(p.second.second);
+  }
+  m->prof_pending.clear();
+}
+
+// ------------------------------------------------------------ staging
+
+// Copy host int32 data to device through the model's pinned staging buffer.
+kvr_status stage_h2d(kvr_model *m, int32_t *dst_dev, const int32_t *src, size_t count) {
+  if (count == 0) return KVR_OK;
+  if (count > m->stage_cap) return fail(KVR_E_UNSUPPORTED, "staging overflow (%zu)", count);
+  CUDA_TRY(cudaEventSynchronize(m->stage_ev));
+  memcpy(m->stage_h, src, count * sizeof(int32_t));
+  CUDA_TRY(cudaMemcpyAsync(dst_dev, m->stage_h, count * sizeof(int32_t), cudaMemcpyHostToDevice,
+                           m->stream));
+  CUDA_TRY(cudaEventRecord(m->stage_ev, m->stream));
+  return KVR_OK;
+}
+
+// ------------------------------------------------------------ GEMM dispatch
+
+kvr_status gemm(kvr_model *m, int cls, const void *X, const void *W, const float *bias, float *Y,
+                int M, int N, int K, int accumulate) {
+  const Dims &dm = m->dims;
+  Prof pr(m, cls, (int64_t)N * K * (int64_t)dm.es());
+  GemmArgs g{X, W, bias, Y, M, N, K, K, N, dm.dtype, accumulate};
+  launch_gemm_simt(g, m->stream);
+  return launch_check(m, 1);
+}
+
+// ------------------------------------------------------------ the pass
+
+struct Rows {
+  int M = 0;
+  const int32_t *pos = nullptr;              // device [M]
+  const int32_t *tokens = nullptr;           // device tokens of a single document
+  const int32_t *const *doc_tokens = nullptr;  // device [docs] (batch)
+  const int32_t *rowdoc = nullptr;           // device [M] (batch)
+  const KVView *views = nullptr;             // device [docs] (batch)
+  KVView single{};
+  int max_pos = 0;                           // largest position among the rows
+};
+
+kvr_status embed(kvr_model *m, const Rows &r) {
+  Prof pr(m, P_EMBED, (int64_t)r.M * m->dims.d * (int64_t)m->dims.es());
+  launch_embed_rows(m->embed, m->dims.dtype, r.tokens, r.doc_tokens, r.rowdoc, r.pos, r.M,
+                    m->dims.d, m->h, m->stream);
+  return launch_check(m, 1);
+}
+
+kvr_status norm(kvr_model *m, const float *g, int M) {
+  Prof pr(m, P_NORM, (int64_t)M * m->dims.d * 4);
+  launch_rmsnorm(m->h, g, M, m->dims.d, m->dims.eps, m->a, m->dims.dtype, m->stream);
+  return launch_check(m, 1);
+}
+
+// QKV projection, RoPE, and (write_kv) the K/V scatter of layer l.
+kvr_status layer_qkv(kvr_model *m, const Rows &r, int l, bool write_kv) {
+  const Dims &dm = m->dims;
+  const LayerW &w = m->layers[l];
+  KVR_TRY(norm(m, w.attn_norm, r.M));
+  KVR_TRY(gemm(m, P_GEMM_QKV, m->a, w.wqkv, w.bqkv, m->qkv, r.M, dm.Nqkv(), dm.d, 0));
+  {
+    Prof pr(m, P_ROPE, (int64_t)r.M * dm.Nqkv() * 4);
+    launch_rope_scatter(m->qkv, m->rope, r.pos, r.M, dm, l, r.views, r.rowdoc, r.single, m->q,
+                        write_kv, m->stream);
+    KVR_TRY(launch_check(m, 1));
+  }
+  return KVR_OK;
+}
+
+// Attention, O projection, MLP of layer l (after layer_qkv).
+kvr_status layer_rest(kvr_model *m, const Rows &r, int l) {
+  const Dims &dm = m->dims;
+  const LayerW &w = m->layers[l];
+  {
+    int64_t kv_bytes = (int64_t)(r.max_pos + 1) * dm.G * dm.dh * 2 * (int64_t)dm.es();
+    Prof pr(m, P_ATTN, kv_bytes);
+    launch_attention_simt(m->q, r.pos, r.M, dm, l, r.views, r.rowdoc, r.single, m->attn,
+                          m->stream);
+    KVR_TRY(launch_check(m, 1));
+  }
+  KVR_TRY(gemm(m, P_GEMM_O, m->attn, w.wo, nullptr, m->h, r.M, dm.d, dm.H * dm.dh, 1));
+  KVR_TRY(norm(m, w.mlp_norm, r.M));
+  KVR_TRY(gemm(m, P_GEMM_GU, m->a, w.wgu, nullptr, m->gu, r.M, 2 * dm.F, dm.d, 0));
+  {
+    Prof pr(m, P_SWIGLU, (int64_t)r.M * dm.F * 12);
+    launch_swiglu(m->gu, r.M, dm.F, m->act, dm.dtype, m->stream);
+    KVR_TRY(launch_check(m, 1));
+  }
+  KVR_TRY(gemm(m, P_GEMM_DOWN, m->act, w.wd, nullptr, m->h, r.M, dm.d, dm.F, 1));
+  return KVR_OK;
+}
+
+// Operator R over rows r: every layer, K/V of all rows written before any of
+// them attends at that layer.
+kvr_status run_pass(kvr_model *m, const Rows &r) {
+  if (r.M <= 0) return KVR_OK;
+  KVR_TRY(embed(m, r));
+  for (int l = 0; l < m->dims.L; ++l) {
+    KVR_TRY(layer_qkv(m, r, l, true));
+    KVR_TRY(layer_rest(m, r, l));
+  }
+  return KVR_OK;
+}
+
+kvr_status sync_model(kvr_model *m) {
+  cudaError_t e = cudaStreamSynchronize(m->stream);
+  if (e != cudaSuccess) return fail(KVR_E_CUDA, "device error: %s", cudaGetErrorString(e));
+  int flag = 0;
+  e = cudaMemcpy(&flag, m->dev_flag, sizeof(int), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return fail(KVR_E_CUDA, "device error: %s", cudaGetErrorString(e));
+  if (flag) {
+    cudaMemset(m->dev_flag, 0, sizeof(int));
+    return fail(KVR_E_DEVICE_TIMEOUT, "a bounded device wait ran out (code %d)", flag);
+  }
+  return KVR_OK;
+}
+
+kvr_status use_device(const kvr_model *m) {
+  CUDA_TRY(cudaSetDevice(m->device));
+  return KVR_OK;
+}
+
+// ------------------------------------------------------------ weights
+
+struct Region {
+  size_t off, bytes;
+};
+
+double weight_scale() { return 0.02 / std::sqrt((65536.0 * 65536.0 - 1.0) / 3.0); }
+
+uint64_t host_mix64(uint64_t z) {
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+uint64_t stream_out(uint64_t seed, uint64_t i) {
+  return host_mix64(seed + (i + 1) * 0x9E3779B97F4A7C15ull);
+}
+
+enum Tid { T_EMBED = 0, T_LMHEAD = 1 };
+int layer_tid(int l, int k) { return 8 + 16 * l + k; }
+enum LayerTid { LT_WQ = 0, LT_WK, LT_WV, LT_WO, LT_WG, LT_WU, LT_WD, LT_BQ, LT_BK, LT_BV };
+
+float bf16_bits_to_f32(uint16_t b) {
+  uint32_t u = (uint32_t)b << 16;
+  float f;
+  memcpy(&f, &u, 4);
+  return f;
+}
+uint16_t f32_to_bf16_bits(float f) {
+  uint32_t u;
+  memcpy(&u, &f, 4);
+  return (uint16_t)((u + 0x7FFFu + ((u >> 16) & 1u)) >> 16);
+}
+
+// Host vector in model dtype -> fp32 device vector.
+kvr_status upload_f32(kvr_model *m, float *dst, const void *src, size_t n) {
+  std::vector<float> tmp(n);
+  for (size_t i = 0; i < n; ++i)
+    tmp[i] = m->dims.dtype == KVR_DTYPE_BF16 ? bf16_bits_to_f32(((const uint16_t *)src)[i])
+                                             : ((const float *)src)[i];
+  CUDA_TRY(cudaMemcpy(dst, tmp.data(), n * 4, cudaMemcpyHostToDevice));
+  return KVR_OK;
+}
+
+kvr_status upload_rows(kvr_model *m, void *dst, const void *src, size_t rows, size_t cols,
+                       size_t row_off) {
+  size_t es = m->dims.es();
+  CUDA_TRY(cudaMemcpy((char *)dst + row_off * cols * es, src, rows * cols * es,
+                      cudaMemcpyHostToDevice));
+  return KVR_OK;
+}
+
+// gate (inter=1) or up (inter=2) rows into the interleaved wgu.
+kvr_status upload_gu(kvr_model *m, void *wgu, const void *src, int inter) {
+  const Dims &dm = m->dims;
+  size_t es = dm.es(), row = (size_t)dm.d * es;
+  for (int b = 0; b < dm.F / GU_BLOCK; ++b) {
+    size_t drow = (size_t)b * 2 * GU_BLOCK + (inter == 2 ? GU_BLOCK : 0);
+    CUDA_TRY(cudaMemcpy((char *)wgu + drow * row, (const char *)src + (size_t)b * GU_BLOCK * row,
+                        GU_BLOCK * row, cudaMemcpyHostToDevice));
+  }
+  return KVR_OK;
+}
+
+bool valid_config(const kvr_model_config *c, std::string &why) {
+  if (c->vocab < 2 || c->d_model < 1 || c->n_layers < 1 || c->n_heads < 1 || c->n_kv_heads < 1 ||
+      c->ffn < 1) {
+    why = "non-positive dimension";
+    return false;
+  }
+  if (c->n_heads % c->n_kv_heads) {
+    why = "n_heads must be a multiple of n_kv_heads";
+    return false;
+  }
+  if (c->dtype != KVR_DTYPE_F32 && c->dtype != KVR_DTYPE_BF16) {
+    why = "dtype must be KVR_DTYPE_F32 or KVR_DTYPE_BF16";
+    return false;
+  }
+  if (c->max_context < 1 || c->max_rows < 64) {
+    why = "max_context >= 1 and max_rows >= 64 required";
+    return false;
+  }
+  if (!(c->rope_theta > 0) || !(c->rms_eps >= 0)) {
+    why = "rope_theta > 0 and rms_eps >= 0 required";
+    return false;
+  }
+  return true;
+}
+
+}  // namespace
+
+// ======================================================================== ABI
+
+namespace kvr {
+void *dev_alloc(size_t bytes) {
+  if (bytes == 0) bytes = 16;
+  if (g_alloc) return g_alloc(bytes, g_alloc_ctx);
+  void *p = nullptr;
+  if (cudaMalloc(&p, bytes) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  return p;
+}
+void dev_free(void *p) {
+  if (!p) return;
+  if (g_free)
+    g_free(p, g_alloc_ctx);
+  else
+    cudaFree(p);
+}
+}  // namespace kvr
+
+extern "C" {
+
+const char *kvr_last_error(void) { return g_err.c_str(); }
+
+kvr_status kvr_set_allocator(kvr_alloc_fn alloc, kvr_free_fn free_fn, void *ctx) {
+  if ((alloc == nullptr) != (free_fn == nullptr))
+    return fail(KVR_E_INVAL, "allocator and free function must be set together");
+  g_alloc = alloc;
+  g_free = free_fn;
+  g_alloc_ctx = ctx;
+  return KVR_OK;
+}
+
+void kvr_model_free(kvr_model *m) {
+  if (!m) return;
+  cudaSetDevice(m->device);
+  cudaStreamSynchronize(m->stream);
+  prof_collect(m);
+  dev_free(m->weight_block);
+  dev_free(m->ws_block);
+  dev_free(m->rope);
+  dev_free(m->dev_flag);
+  if (m->stage_h) cudaFreeHost(m->stage_h);
+  if (m->stage_ev) cudaEventDestroy(m->stage_ev);
+  delete m;
+}
+
+kvr_status kvr_model_create(const kvr_model_config *cfg, const kvr_weights *wts, uint64_t seed,
+                            kvr_model **out) {
+  if (!cfg || !out) return fail(KVR_E_INVAL, "NULL argument");
+  *out = nullptr;
+  std::string why;
+  if (!valid_config(cfg, why)) return fail(KVR_E_INVAL, "invalid config: %s", why.c_str());
+  if (cfg->head_dim != 64 && cfg->head_dim != 128)
+    return fail(KVR_E_UNSUPPORTED, "head_dim must be 64 or 128");
+  if (cfg->ffn % GU_BLOCK) return fail(KVR_E_UNSUPPORTED, "ffn must be a multiple of 16");
+  if (cfg->max_context > 16384) return fail(KVR_E_UNSUPPORTED, "max_context above 16384");
+
+  kvr_model *m = new kvr_model();
+  Dims &dm = m->dims;
+  dm = Dims{cfg->vocab, cfg->d_model, cfg->n_layers, cfg->n_heads, cfg->n_kv_heads,
+            cfg->head_dim, cfg->ffn, cfg->qkv_bias ? 1 : 0, cfg->dtype, cfg->delim_id,
+            cfg->rope_theta, cfg->rms_eps, cfg->max_context, cfg->max_rows};
+  cudaGetDevice(&m->device);
+  cudaDeviceGetAttribute(&m->num_sms, cudaDevAttrMultiProcessorCount, m->device);
+  m->prof_classes.resize(P_NCLASS);
+  for (int i = 0; i < P_NCLASS; ++i) m->prof_classes[i].name = kProfNames[i];
+
+  auto bail = [&](kvr_status s) {
+    kvr_model_free(m);
+    return s;
+  };
+
+  // ---- weight block layout
+  size_t es = dm.es(), d = dm.d, V = dm.V, F = dm.F, Nq = dm.Nqkv(), HD = (size_t)dm.H * dm.dh;
+  auto al = [](size_t x) { return (x + 255) / 256 * 256; };
+  size_t off = 0;
+  size_t o_embed = off;
+  off += al(V * d * es);
+  size_t o_lm = off;
+  off += al(V * d * es);
+  size_t o_fn = off;
+  off += al(d * 4);
+  std::vector<size_t> lo(dm.L);
+  size_t per_layer = al(Nq * d * es) + al(Nq * 4) + al(d * HD * es) + al(2 * F * d * es) +
+                     al(d * F * es) + 2 * al(d * 4);
+  for (int l = 0; l < dm.L; ++l) {
+    lo[l] = off;
+    off += per_layer;
+  }
+  m->weight_bytes = off;
+  m->weight_block = dev_alloc(off);
+  if (!m->weight_block) return bail(fail(KVR_E_NOMEM, "weights: %zu bytes", off));
+  char *wb = (char *)m->weight_block;
+  m->embed = wb + o_embed;
+  m->lm_head = wb + o_lm;
+  m->final_norm = (float *)(wb + o_fn);
+  m->layers.resize(dm.L);
+  for (int l = 0; l < dm.L; ++l) {
+    char *p = wb + lo[l];
+    LayerW &w = m->layers[l];
+    w.wqkv = p;
+    p += al(Nq * d * es);
+    w.bqkv = (float *)p;
+    p += al(Nq * 4);
+    w.wo = p;
+    p += al(d * HD * es);
+    w.wgu = p;
+    p += al(2 * F * d * es);
+    w.wd = p;
+    p += al(d * F * es);
+    w.attn_norm = (float *)p;
+    p += al(d * 4);
+    w.mlp_norm = (float *)p;
+    if (!dm.qkv_bias) w.bqkv = nullptr;
+  }
+
+  cudaStream_t s = 0;
+  if (!wts) {
+    double sc = weight_scale();
+    auto init = [&](void *dst, bool f32, int tid, int64_t rows, int64_t cols, int64_t row_off,
+                    int inter) {
+      launch_init_tensor(dst, dm.dtype, f32, stream_out(seed, (uint64_t)tid), sc, rows, cols,
+                         row_off, inter, s);
+    };
+    init(m->embed, false, T_EMBED, V, d, 0, 0);
+    init(m->lm_head, false, T_LMHEAD, V, d, 0, 0);
+    launch_fill_f32(m->final_norm, 1.f, d, s);
+    for (int l = 0; l < dm.L; ++l) {
+      LayerW &w = m->layers[l];
+      init(w.wqkv, false, layer_tid(l, LT_WQ), HD, d, 0, 0);
+      init(w.wqkv, false, layer_tid(l, LT_WK), (int64_t)dm.G * dm.dh, d, HD, 0);
+      init(w.wqkv, false, layer_tid(l, LT_WV), (int64_t)dm.G * dm.dh, d,
+           HD + (int64_t)dm.G * dm.dh, 0);
+      if (dm.qkv_bias) {
+        init(w.bqkv, true, layer_tid(l, LT_BQ), 1, HD, 0, 0);
+        init((float *)w.bqkv + HD, true, layer_tid(l, LT_BK), 1, (int64_t)dm.G * dm.dh, 0, 0);
+        init((float *)w.bqkv + HD + dm.G * dm.dh, true, layer_tid(l, LT_BV), 1,
+             (int64_t)dm.G * dm.dh, 0, 0);
+      }
+      init(w.wo, false, layer_tid(l, LT_WO), d, HD, 0, 0);
+      init(w.wgu, false, layer_tid(l, LT_WG), F, d, 0, 1);
+      init(w.wgu, false, layer_tid(l, LT_WU), F, d, 0, 2);
+      init(w.wd, false, layer_tid(l, LT_WD), d, F, 0, 0);
+      launch_fill_f32(w.attn_norm, 1.f, d, s);
+      launch_fill_f32(w.mlp_norm, 1.f, d, s);
+    }
+    cudaError_t e = cudaGetLastError();
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess)
+      return bail(fail(KVR_E_CUDA, "weight init: %s", cudaGetErrorString(e)));
+  } else {
+    if (!wts->embed || !wts->lm_head || !wts->final_norm || !wts->wq || !wts->wk || !wts->wv ||
+        !wts->wo || !wts->wg || !wts->wu || !wts->wd || !wts->attn_norm || !wts->mlp_norm ||
+        (dm.qkv_bias && (!wts->bq || !wts->bk || !wts->bv)))
+      return bail(fail(KVR_E_INVAL, "missing weight pointer"));
+    kvr_status st = KVR_OK;
+#define UP(x)                  \
+  do {                         \
+    st = (x);                  \
+    if (st) return bail(st);   \
+  } while (0)
+    UP(upload_rows(m, m->embed, wts->embed, V, d, 0));
+    UP(upload_rows(m, m->lm_head, wts->lm_head, V, d, 0));
+    UP(upload_f32(m, m->final_norm, wts->final_norm, d));
+    size_t GD = (size_t)dm.G * dm.dh;
+    for (int l = 0; l < dm.L; ++l) {
+      LayerW &w = m->layers[l];
+      if (!wts->wq[l] || !wts->wk[l] || !wts->wv[l] || !wts->wo[l] || !wts->wg[l] ||
+          !wts->wu[l] || !wts->wd[l] || !wts->attn_norm[l] || !wts->mlp_norm[l])
+        return bail(fail(KVR_E_INVAL, "missing weight pointer in layer %d", l));
+      UP(upload_rows(m, w.wqkv, wts->wq[l], HD, d, 0));
+      UP(upload_rows(m, w.wqkv, wts->wk[l], GD, d, HD));
+      UP(upload_rows(m, w.wqkv, wts->wv[l], GD, d, HD + GD));
+      if (dm.qkv_bias) {
+        UP(upload_f32(m, w.bqkv, wts->bq[l], HD));
+        UP(upload_f32(m, w.bqkv + HD, wts->bk[l], GD));
+        UP(upload_f32(m, w.bqkv + HD + GD, wts->bv[l], GD));
+      }
+      UP(upload_rows(m, w.wo, wts->wo[l], d, HD, 0));
+      UP(upload_gu(m, w.wgu, wts->wg[l], 1));
+      UP(upload_gu(m, w.wgu, wts->wu[l], 2));
+      UP(upload_rows(m, w.wd, wts->wd[l], d, F, 0));
+      UP(upload_f32(m, w.attn_norm, wts->attn_norm[l], d));
+      UP(upload_f32(m, w.mlp_norm, wts->mlp_norm[l], d));
+    }
+#undef UP
+  }
+
+  // ---- RoPE table: cos/sin of pos * theta^(-2i/dh), angles in double
+  {
+    int half = dm.dh / 2, P = dm.max_ctx + KVR_QUERY_RESERVE;
+    std::vector<float2> t((size_t)P * half);
+    for (int p = 0; p < P; ++p)
+      for (int i = 0; i < half; ++i) {
+        double ang = (double)p * std::pow(dm.theta, -2.0 * i / dm.dh);
+        t[(size_t)p * half + i] = make_float2((float)std::cos(ang), (float)std::sin(ang));
+      }
+    m->rope = (float2 *)dev_alloc(t.size() * sizeof(float2));
+    if (!m->rope) return bail(fail(KVR_E_NOMEM, "rope table"));
+    if (cudaMemcpy(m->rope, t.data(), t.size() * sizeof(float2), cudaMemcpyHostToDevice))
+      return bail(fail(KVR_E_CUDA, "rope table upload"));
+  }
+
+  // ---- workspace
+  {
+    size_t R = dm.max_rows, P = dm.max_ctx + KVR_QUERY_RESERVE;
+    size_t sz[] = {R * 4,          R * 4,          R * d * 4,        R * d * es,  R * Nq * 4,
+                   R * HD * 4,     R * HD * es,    R * 2 * F * 4,    R * F * es,  V * 4,
+                   P * 4,          P * 8,          P * 4,            256};
+    size_t tot = 0;
+    for (size_t x : sz) tot += al(x);
+    m->ws_block = dev_alloc(tot);
+    if (!m->ws_block) return bail(fail(KVR_E_NOMEM, "workspace: %zu bytes", tot));
+    char *p = (char *)m->ws_block;
+    void *ptrs[14];
+    for (int i = 0; i < 14; ++i) {
+      ptrs[i] = p;
+      p += al(sz[i]);
+    }
+    m->pos_d = (int32_t *)ptrs[0];
+    m->rowdoc_d = (int32_t *)ptrs[1];
+    m->h = (float *)ptrs[2];
+    m->a = ptrs[3];
+    m->qkv = (float *)ptrs[4];
+    m->q = (float *)ptrs[5];
+    m->attn = ptrs[6];
+    m->gu = (float *)ptrs[7];
+    m->act = ptrs[8];
+    m->logits = (float *)ptrs[9];
+    m->scores = (float *)ptrs[10];
+    m->keys = (unsigned long long *)ptrs[11];
+    m->sel_out = (int32_t *)ptrs[12];
+    m->sel_count = (int32_t *)ptrs[13];
+    m->dev_flag = (int *)dev_alloc(256);
+    if (!m->dev_flag) return bail(fail(KVR_E_NOMEM, "flag"));
+    cudaMemset(m->dev_flag, 0, 256);
+    m->stage_cap = std::max<size_t>(R * 2, P) + 4096;
+    if (cudaMallocHost(&m->stage_h, m->stage_cap * sizeof(int32_t)) != cudaSuccess)
+      return bail(fail(KVR_E_NOMEM, "pinned staging"));
+    cudaEventCreateWithFlags(&m->stage_ev, cudaEventDisableTiming);
+    cudaEventRecord(m->stage_ev, 0);
+  }
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return bail(fail(KVR_E_CUDA, "create: %s", cudaGetErrorString(e)));
+  *out = m;
+  return KVR_OK;
+}
+
+kvr_status kvr_model_set_stream(kvr_model *m, void *stream) {
+  if (!m) return fail(KVR_E_INVAL, "NULL model");
+  m->stream = (cudaStream_t)stream;
+  return KVR_OK;
+}
+
+kvr_status kvr_synchronize(kvr_model *m) {
+  if (!m) return fail(KVR_E_INVAL, "NULL model");
+  KVR_TRY(use_device(m));
+  return sync_model(m);
+}
+
+int64_t kvr_launch_count(const kvr_model *m) { return m ? m->launches : 0; }
+
+void kvr_cache_free(kvr_cache *c) {
+  if (!c) return;
+  cudaSetDevice(c->model->device);
+  cudaStreamSynchronize(c->model->stream);
+  dev_free(c->pages);
+  dev_free(c->table);
+  dev_free(c->tokens_d);
+  delete c;
+}
+
+int32_t kvr_cache_len(const kvr_cache *c) { return c ? c->n : -1; }
+
+kvr_status kvr_prefill(kvr_model *m, const int32_t *tokens, int32_t n, kvr_cache **out) {
+  if (!m || !tokens || !out) return fail(KVR_E_INVAL, "NULL argument");
+  *out = nullptr;
+  const Dims &dm = m->dims;
+  if (n < 1 || n > dm.max_ctx) return fail(KVR_E_RANGE, "n=%d outside [1, %d]", n, dm.max_ctx);
+  for (int i = 0; i < n; ++i)
+    if (tokens[i] < 0 || tokens[i] >= dm.V)
+      return fail(KVR_E_RANGE, "token %d at position %d outside [0, %d)", tokens[i], i, dm.V);
+  KVR_TRY(use_device(m));
+  kvr_cache *c = new kvr_cache();
+  c->model = m;
+  c->n = n;
+  c->cap = (n + KVR_QUERY_RESERVE + KVR_PAGE - 1) / KVR_PAGE * KVR_PAGE;
+  c->n_pages = c->cap / KVR_PAGE;
+  size_t page_bytes = dm.page_elems() * dm.es();
+  c->pages = dev_alloc((size_t)c->n_pages * page_bytes);
+  c->table = (int32_t *)dev_alloc((size_t)c->n_pages * 4);
+  c->tokens_d = (int32_t *)dev_alloc((size_t)c->cap * 4);
+  if (!c->pages || !c->table || !c->tokens_d) {
+    kvr_cache_free(c);
+    return fail(KVR_E_NOMEM, "cache of %d pages", c->n_pages);
+  }
+  c->tokens_h.assign(tokens, tokens + n);
+  std::vector<int32_t> tab(c->n_pages);
+  for (int i = 0; i < c->n_pages; ++i) tab[i] = i;
+  kvr_status st = stage_h2d(m, c->table, tab.data(), tab.size());
+  if (!st) st = stage_h2d(m, c->tokens_d, tokens, n);
+  Rows r;
+  r.tokens = c->tokens_d;
+  r.single = c->view();
+  std::vector<int32_t> pos;
+  for (int c0 = 0; c0 < n && !st; c0 += dm.max_rows) {
+    int M = std::min(dm.max_rows, n - c0);
+    pos.resize(M);
+    for (int i = 0; i < M; ++i) pos[i] = c0 + i;
+    st = stage_h2d(m, m->pos_d, pos.data(), M);
+    if (st) break;
+    r.M = M;
+    r.pos = m->pos_d;
+    r.max_pos = c0 + M - 1;
+    st = run_pass(m, r);
+  }
+  if (st) {
+    cudaStreamSynchronize(m->stream);
+    kvr_cache_free(c);
+    return st;
+  }
+  *out = c;
+  return KVR_OK;
+}
+
+kvr_status kvr_repair(kvr_cache *c, const int32_t *new_tokens, int32_t edit_start,
+                      int32_t edit_len, const int32_t *positions, int32_t n_positions) {
+  if (!c) return fail(KVR_E_INVAL, "NULL cache");
+  if (c->poisoned) return fail(KVR_E_POISONED, "cache poisoned by an earlier CUDA error");
+  kvr_model *m = c->model;
+  const Dims &dm = m->dims;
+  if (edit_len < 0 || n_positions < 0) return fail(KVR_E_RANGE, "negative length");
+  if (edit_len > 0 && !new_tokens) return fail(KVR_E_INVAL, "NULL new_tokens");
+  if (n_positions > 0 && !positions) return fail(KVR_E_INVAL, "NULL positions");
+  int s_end = edit_start + edit_len;
+  if (edit_start < 0 || s_end > c->n)
+    return fail(KVR_E_RANGE, "edit span [%d, %d) outside [0, %d)", edit_start, s_end, c->n);
+  for (int i = 0; i < edit_len; ++i)
+    if (new_tokens[i] < 0 || new_tokens[i] >= dm.V)
+      return fail(KVR_E_RANGE, "new token %d outside [0, %d)", new_tokens[i], dm.V);
+  for (int i = 0; i < n_positions; ++i) {
+    if (positions[i] < s_end || positions[i] >= c->n)
+      return fail(KVR_E_RANGE, "position %d outside [%d, %d)", positions[i], s_end, c->n);
+    if (i && positions[i] <= positions[i - 1])
+      return fail(KVR_E_RANGE, "positions not strictly increasing at %d", i);
+  }
+  int M = edit_len + n_positions;
+  if (M > dm.max_rows) return fail(KVR_E_UNSUPPORTED, "|P|=%d above max_rows", M);
+  KVR_TRY(use_device(m));
+  if (M == 0) return KVR_OK;
+  // a1: apply the edit
+  std::vector<int32_t> P(M);
+  for (int i = 0; i < edit_len; ++i) {
+    c->tokens_h[edit_start + i] = new_tokens[i];
+    P[i] = edit_start + i;
+  }
+  for (int i = 0; i < n_positions; ++i) P[edit_len + i] = positions[i];
+  kvr_status st = KVR_OK;
+  if (edit_len) st = stage_h2d(m, c->tokens_d + edit_start, new_tokens, edit_len);
+  if (!st) st = stage_h2d(m, m->pos_d, P.data(), M);
+  if (!st) {
+    Rows r;
+    r.M = M;
+    r.pos = m->pos_d;
+    r.tokens = c->tokens_d;
+    r.single = c->view();
+    r.max_pos = P[M - 1];
+    st = run_pass(m, r);
+  }
+  if (st == KVR_E_CUDA) c->poisoned = true;
+  return st;
+}
+
+kvr_status kvr_repair_batch(kvr_model *m, const kvr_repair_req *reqs, int32_t n_reqs) {
+  if (!m || (n_reqs > 0 && !reqs)) return fail(KVR_E_INVAL, "NULL argument");
+  if (n_reqs < 0 || n_reqs > 256) return fail(KVR_E_RANGE, "n_reqs=%d outside [0, 256]", n_reqs);
+  const Dims &dm = m->dims;
+  std::vector<int32_t> P, rowdoc;
+  int max_pos = 0;
+  // validate everything before touching any cache
+  for (int r = 0; r < n_reqs; ++r) {
+    const kvr_repair_req &q = reqs[r];
+    if (!q.cache || q.cache->model != m) return fail(KVR_E_INVAL, "request %d: bad cache", r);
+    if (q.cache->poisoned) return fail(KVR_E_POISONED, "request %d: cache poisoned", r);
+    for (int s = 0; s < r; ++s)
+      if (reqs[s].cache == q.cache) return fail(KVR_E_INVAL, "cache repeated in a batch");
+    if (q.n_edits < 0 || q.n_positions < 0) return fail(KVR_E_RANGE, "request %d: negative", r);
+    std::vector<char> inP(q.cache->n, 0);
+    int tk = 0;
+    for (int e = 0; e < q.n_edits; ++e) {
+      int s0 = q.edit_start[e], L = q.edit_len[e];
+      if (L < 0 || s0 < 0 || s0 + L > q.cache->n)
+        return fail(KVR_E_RANGE, "request %d edit %d outside the context", r, e);
+      for (int i = 0; i < L; ++i) {
+        if (inP[s0 + i]) return fail(KVR_E_RANGE, "request %d: edits overlap", r);
+        inP[s0 + i] = 1;
+        int t = q.new_tokens[tk + i];
+        if (t < 0 || t >= dm.V) return fail(KVR_E_RANGE, "request %d: token out of range", r);
+      }
+      tk += L;
+    }
+    for (int i = 0; i < q.n_positions; ++i) {
+      int p = q.positions[i];
+      if (p < 0 || p >= q.cache->n || (i && p <= q.positions[i - 1]))
+        return fail(KVR_E_RANGE, "request %d: positions invalid at %d", r, i);
+      if (inP[p]) return fail(KVR_E_RANGE, "request %d: position %d inside an edit", r, p);
+      inP[p] = 2;
+    }
+    for (int p = 0; p < q.cache->n; ++p)
+      if (inP[p]) {
+        P.push_back(p);
+        rowdoc.push_back(r);
+        max_pos = std::max(max_pos, p);
+      }
+  }
+  int M = (int)P.size();
+  if (M > dm.max_rows) return fail(KVR_E_UNSUPPORTED, "sum |P|=%d above max_rows", M);
+  KVR_TRY(use_device(m));
+  if (M == 0) return KVR_OK;
+  // apply the edits
+  for (int r = 0; r < n_reqs; ++r) {
+    const kvr_repair_req &q = reqs[r];
+    int tk = 0;
+    for (int e = 0; e < q.n_edits; ++e) {
+      int s0 = q.edit_start[e], L = q.edit_len[e];
+      for (int i = 0; i < L; ++i) q.cache->tokens_h[s0 + i] = q.new_tokens[tk + i];
+      if (L) KVR_TRY(stage_h2d(m, q.cache->tokens_d + s0, q.new_tokens + tk, L));
+      tk += L;
+    }
+  }
+  // device tables: views and token pointers of the documents
+  std::vector<KVView> views(n_reqs);
+  std::vector<const int32_t *> toks(n_reqs);
+  for (int r = 0; r < n_reqs; ++r) {
+    views[r] = reqs[r].cache->view();
+    toks[r] = reqs[r].cache->tokens_d;
+  }
+  size_t vb = n_reqs * sizeof(KVView), tb = n_reqs * sizeof(void *);
+  char *tab = (char *)dev_alloc(vb + tb + 64);
+  if (!tab) return fail(KVR_E_NOMEM, "batch tables");
+  kvr_status st = KVR_OK;
+  if (cudaMemcpyAsync(tab, views.data(), vb, cudaMemcpyHostToDevice, m->stream) ||
+      cudaMemcpyAsync(tab + vb, toks.data(), tb, cudaMemcpyHostToDevice, m->stream))
+    st = fail(KVR_E_CUDA, "batch table upload");
+  if (!st) st = stage_h2d(m, m->pos_d, P.data(), M);
+  if (!st) {
+    // rowdoc goes through a second staging round
+    st = stage_h2d(m, m->rowdoc_d, rowdoc.data(), M);
+  }
+  if (!st) {
+    Rows r;
+    r.M = M;
+    r.pos = m->pos_d;
+    r.rowdoc = m->rowdoc_d;
+    r.views = (const KVView *)tab;
+    r.doc_tokens = (const int32_t *const *)(tab + vb);
+    r.max_pos = max_pos;
+    st = run_pass(m, r);
+  }
+  cudaStreamSynchronize(m->stream);
+  dev_free(tab);
+  if (st == KVR_E_CUDA)
+    for (int r = 0; r < n_reqs; ++r) reqs[r].cache->poisoned = true;
+  return st;
+}
+
+kvr_status kvr_logits(kvr_model *m, const kvr_cache *c, const int32_t *query, int32_t qm,
+                      float *logits_out) {
+  if (!m || !c || !query || !logits_out) return fail(KVR_E_INVAL, "NULL argument");
+  if (c->model != m) return fail(KVR_E_INVAL, "cache of another model");
+  if (c->poisoned) return fail(KVR_E_POISONED, "cache poisoned");
+  const Dims &dm = m->dims;
+  if (qm < 1 || qm > KVR_QUERY_RESERVE || c->n + qm > c->cap)
+    return fail(KVR_E_RANGE, "query length %d outside [1, %d]", qm, KVR_QUERY_RESERVE);
+  for (int i = 0; i < qm; ++i)
+    if (query[i] < 0 || query[i] >= dm.V) return fail(KVR_E_RANGE, "query token out of range");
+  KVR_TRY(use_device(m));
+  std::vector<int32_t> P(qm);
+  for (int i = 0; i < qm; ++i) P[i] = c->n + i;
+  KVR_TRY(stage_h2d(m, c->tokens_d + c->n, query, qm));
+  KVR_TRY(stage_h2d(m, m->pos_d, P.data(), qm));
+  Rows r;
+  r.M = qm;
+  r.pos = m->pos_d;
+  r.tokens = c->tokens_d;
+  r.single = c->view();
+  r.max_pos = c->n + qm - 1;
+  KVR_TRY(run_pass(m, r));
+  // final RMSNorm of the last row, lm_head
+  {
+    Prof pr(m, P_NORM, (int64_t)dm.d * 4);
+    launch_rmsnorm(m->h + (size_t)(qm - 1) * dm.d, m->final_norm, 1, dm.d, dm.eps, m->a,
+                   dm.dtype, m->stream);
+    KVR_TRY(launch_check(m, 1));
+  }
+  KVR_TRY(gemm(m, P_LMHEAD, m->a, m->lm_head, nullptr, m->logits, 1, dm.V, dm.d, 0));
+  CUDA_TRY(cudaMemcpyAsync(logits_out, m->logits, (size_t)dm.V * 4, cudaMemcpyDeviceToHost,
+                           m->stream));
+  return sync_model(m);
+}
+
+kvr_status kvr_select(kvr_model *m, const kvr_cache *c, kvr_policy policy, int32_t K,
+                      int32_t edit_start, int32_t edit_len, const int32_t *new_tokens,
+                      uint64_t seed, int32_t *positions_out, int32_t *count_out) {
+  if (!m || !c || !count_out || (K > 0 && !positions_out))
+    return fail(KVR_E_INVAL, "NULL argument");
+  if (c->model != m) return fail(KVR_E_INVAL, "cache of another model");
+  if (c->poisoned) return fail(KVR_E_POISONED, "cache poisoned");
+  const Dims &dm = m->dims;
+  if (K < 0) return fail(KVR_E_RANGE, "K < 0");
+  if (edit_len < 0 || edit_start < 0 || edit_start + edit_len > c->n)
+    return fail(KVR_E_RANGE, "edit span outside the context");
+  if (edit_len > 0 && !new_tokens) return fail(KVR_E_INVAL, "NULL new_tokens");
+  for (int i = 0; i < edit_len; ++i)
+    if (new_tokens[i] < 0 || new_tokens[i] >= dm.V)
+      return fail(KVR_E_RANGE, "new token out of range");
+  if (policy < KVR_POLICY_EDITLOCAL || policy > KVR_POLICY_RANDOM)
+    return fail(KVR_E_INVAL, "unknown policy %d", (int)policy);
+  KVR_TRY(use_device(m));
+  int n = c->n, s_end = edit_start + edit_len;
+  *count_out = 0;
+  if (n - s_end <= 0 || K == 0) return KVR_OK;
+  // the edited context, private to this call
+  int32_t *toks = (int32_t *)dev_alloc((size_t)c->cap * 4);
+  if (!toks) return fail(KVR_E_NOMEM, "token scratch");
+  kvr_status st = KVR_OK;
+  if (cudaMemcpyAsync(toks, c->tokens_d, (size_t)n * 4, cudaMemcpyDeviceToDevice, m->stream))
+    st = fail(KVR_E_CUDA, "token copy");
+  if (!st && edit_len) st = stage_h2d(m, toks + edit_start, new_tokens, edit_len);
+  int topk_k = K;
+  void *save = nullptr;
+  float *probs = nullptr;
+  if (!st && (policy == KVR_POLICY_EDITLOCAL || policy == KVR_POLICY_STRUCTURAL ||
+              policy == KVR_POLICY_RANDOM)) {
+    Prof pr(m, P_SELECT, 0);
+    launch_scores_simple(policy, toks, n, s_end, dm.delim, seed, m->keys, m->stream);
+    st = launch_check(m, 1);
+    if (policy == KVR_POLICY_STRUCTURAL) topk_k = -K;
+  } else if (!st && policy == KVR_POLICY_ATTENTION) {
+    if (edit_len == 0) {
+      st = fail(KVR_E_RANGE, "attention policy needs a non-empty span");
+    } else if (edit_len > dm.max_rows) {
+      st = fail(KVR_E_UNSUPPORTED, "span above max_rows");
+    } else {
+      // span rows through every layer, fresh K/V written in place (saved and
+      // restored), probabilities of the span queries over the stale pool keys
+      std::vector<int32_t> P(edit_len);
+      for (int i = 0; i < edit_len; ++i) P[i] = edit_start + i;
+      size_t save_bytes = (size_t)edit_len * dm.L * 2 * dm.G * dm.dh * dm.es();
+      save = dev_alloc(save_bytes);
+      probs = (float *)dev_alloc((size_t)edit_len * dm.H * (n - s_end) * 4);
+      if (!save || !probs) st = fail(KVR_E_NOMEM, "selector scratch");
+      if (!st) st = stage_h2d(m, m->pos_d, P.data(), edit_len);
+      if (!st) {
+        Rows r;
+        r.M = edit_len;
+        r.pos = m->pos_d;
+        r.tokens = toks;
+        r.single = c->view();
+        r.max_pos = s_end - 1;
+        launch_rows_copy(r.single, dm.dtype, r.pos, edit_len, 0, dm.L, save, true, m->stream);
+        launch_fill_f32(m->scores, 0.f, (size_t)n, m->stream);
+        st = launch_check(m, 2);
+        if (!st) st = embed(m, r);
+        for (int l = 0; l < dm.L && !st; ++l) {
+          st = layer_qkv(m, r, l, true);
+          if (!st) {
+            Prof pr(m, P_SELECT, 0);
+            launch_attn_select_scores(m->q, edit_len, dm, l, r.single, s_end, n, probs, m->scores,
+                                      m->stream);
+            st = launch_check(m, 2);
+          }
+          if (!st) st = layer_rest(m, r, l);
+        }
+        launch_rows_copy(r.single, dm.dtype, r.pos, edit_len, 0, dm.L, save, false, m->stream);
+        if (!st) st = launch_check(m, 1);
+        if (!st) {
+          launch_float_keys(m->scores, n, s_end, m->keys, m->stream);
+          st = launch_check(m, 1);
+        }
+      }
+    }
+  } else if (!st && policy == KVR_POLICY_CACHEBLEND) {
+    if (dm.L < 2) {
+      st = fail(KVR_E_UNSUPPORTED, "cacheblend needs >= 2 layers");
+    } else if (edit_len == 0) {
+      st = fail(KVR_E_RANGE, "cacheblend policy needs a non-empty span");
+    } else if (edit_len > dm.max_rows) {
+      st = fail(KVR_E_UNSUPPORTED, "span above max_rows");
+    } else {
+      std::vector<int32_t> P(edit_len);
+      for (int i = 0; i < edit_len; ++i) P[i] = edit_start + i;
+      save = dev_alloc((size_t)edit_len * 2 * dm.G * dm.dh * dm.es());
+      if (!save) st = fail(KVR_E_NOMEM, "selector scratch");
+      Rows r;
+      r.tokens = toks;
+      r.single = c->view();
+      if (!st) st = stage_h2d(m, m->pos_d, P.data(), edit_len);
+      if (!st) {
+        // refresh the span's layer-0 K/V (saved and restored afterwards)
+        r.M = edit_len;
+        r.pos = m->pos_d;
+        r.max_pos = s_end - 1;
+        launch_rows_copy(r.single, dm.dtype, r.pos, edit_len, 0, 1, save, true, m->stream);
+        launch_fill_f32(m->scores, 0.f, (size_t)n, m->stream);
+        st = launch_check(m, 2);
+        if (!st) st = embed(m, r);
+        if (!st) st = layer_qkv(m, r, 0, true);
+      }
+      // layer 0 for every pool row (their layer-0 K/V depend on their token
+      // alone and are left as cached), then layer-1 K/V projection
+      std::vector<int32_t> D;
+      for (int c0 = s_end; c0 < n && !st; c0 += dm.max_rows) {
+        int M = std::min(dm.max_rows, n - c0);
+        D.resize(M);
+        for (int i = 0; i < M; ++i) D[i] = c0 + i;
+        st = stage_h2d(m, m->pos_d, D.data(), M);
+        if (st) break;
+        r.M = M;
+        r.pos = m->pos_d;
+        r.max_pos = c0 + M - 1;
+        st = embed(m, r);
+        if (!st) st = layer_qkv(m, r, 0, false);
+        if (!st) st = layer_rest(m, r, 0);
+        if (!st) st = layer_qkv(m, r, 1, false);
+        if (!st) {
+          Prof pr(m, P_SELECT, 0);
+          launch_kv_deviation(m->qkv, m->rope, r.pos, M, dm, r.single, m->scores, m->stream);
+          st = launch_check(m, 1);
+        }
+      }
+      if (save) {
+        kvr_status s2 = stage_h2d(m, m->pos_d, P.data(), edit_len);
+        if (!s2) {
+          launch_rows_copy(r.single, dm.dtype, m->pos_d, edit_len, 0, 1, save, false, m->stream);
+          s2 = launch_check(m, 1);
+        }
+        if (!st) st = s2;
+      }
+      if (!st) {
+        launch_float_keys(m->scores, n, s_end, m->keys, m->stream);
+        st = launch_check(m, 1);
+      }
+    }
+  }
+  if (!st) {
+    Prof pr(m, P_SELECT, 0);
+    launch_topk(m->keys, n, s_end, topk_k, m->sel_out, m->sel_count, m->stream);
+    st = launch_check(m, 1);
+  }
+  int32_t cnt = 0;
+  if (!st && (cudaMemcpyAsync(&cnt, m->sel_count, 4, cudaMemcpyDeviceToHost, m->stream) ||
+              cudaStreamSynchronize(m->stream)))
+    st = fail(KVR_E_CUDA, "select readback");
+  if (!st && cnt > 0 &&
+      (cudaMemcpyAsync(positions_out, m->sel_out, (size_t)cnt * 4, cudaMemcpyDeviceToHost,
+                       m->stream) ||
+       cudaStreamSynchronize(m->stream)))
+    st = fail(KVR_E_CUDA, "select readback");
+  if (!st) st = sync_model(m);
+  cudaStreamSynchronize(m->stream);
+  dev_free(toks);
+  dev_free(save);
+  dev_free(probs);
+  if (!st) *count_out = cnt;
+  return st;
+}
+
+kvr_status kvr_cache_tokens(const kvr_cache *c, int32_t *out) {
+  if (!c || !out) return fail(KVR_E_INVAL, "NULL argument");
+  memcpy(out, c->tokens_h.data(), (size_t)c->n * 4);
+  return KVR_OK;
+}
+
+kvr_status kvr_cache_read(const kvr_cache *c, const int32_t *positions, int32_t n_pos,
+                          int32_t l0, int32_t l1, float *k_out, float *v_out) {
+  if (!c || (n_pos > 0 && (!positions || !k_out || !v_out)))
+    return fail(KVR_E_INVAL, "NULL argument");
+  kvr_model *m = c->model;
+  const Dims &dm = m->dims;
+  if (l0 < 0 || l1 > dm.L || l0 > l1 || n_pos < 0) return fail(KVR_E_RANGE, "layer range");
+  for (int i = 0; i < n_pos; ++i)
+    if (positions[i] < 0 || positions[i] >= c->cap) return fail(KVR_E_RANGE, "position");
+  if (n_pos == 0 || l0 == l1) return KVR_OK;
+  KVR_TRY(use_device(m));
+  size_t elems = (size_t)n_pos * (l1 - l0) * dm.G * dm.dh;
+  int32_t *pd = (int32_t *)dev_alloc((size_t)n_pos * 4);
+  float *kd = (float *)dev_alloc(elems * 4), *vd = (float *)dev_alloc(elems * 4);
+  kvr_status st = KVR_OK;
+  if (!pd || !kd || !vd) st = fail(KVR_E_NOMEM, "readback buffers");
+  if (!st && cudaMemcpyAsync(pd, positions, (size_t)n_pos * 4, cudaMemcpyHostToDevice, m->stream))
+    st = fail(KVR_E_CUDA, "positions upload");
+  if (!st) {
+    launch_cache_gather(c->view(), dm.dtype, pd, n_pos, l0, l1, dm.G, dm.dh, kd, vd, m->stream);
+    st = launch_check(m, 1);
+  }
+  if (!st && (cudaMemcpyAsync(k_out, kd, elems * 4, cudaMemcpyDeviceToHost, m->stream) ||
+              cudaMemcpyAsync(v_out, vd, elems * 4, cudaMemcpyDeviceToHost, m->stream)))
+    st = fail(KVR_E_CUDA, "readback");
+  if (!st) st = sync_model(m);
+  cudaStreamSynchronize(m->stream);
+  dev_free(pd);
+  dev_free(kd);
+  dev_free(vd);
+  return st;
+}
+
+kvr_status kvr_model_read_tensor(const kvr_model *m, const char *name, int32_t layer, void *out,
+                                 size_t bytes) {
+  if (!m || !name || !out) return fail(KVR_E_INVAL, "NULL argument");
+  const Dims &dm = m->dims;
+  size_t es = dm.es(), d = dm.d, HD = (size_t)dm.H * dm.dh, GD = (size_t)dm.G * dm.dh;
+  std::string nm(name);
+  bool per_layer = !(nm == "embed" || nm == "lm_head" || nm == "final_norm");
+  if (per_layer && (layer < 0 || layer >= dm.L)) return fail(KVR_E_RANGE, "layer");
+  KVR_TRY(use_device(m));
+  const LayerW *w = per_layer ? &m->layers[layer] : nullptr;
+  auto need = [&](size_t b) { return bytes < b ? fail(KVR_E_RANGE, "need %zu bytes", b) : KVR_OK; };
+  auto rows_out = [&](const void *src, size_t rows, size_t cols, size_t row_off) -> kvr_status {
+    KVR_TRY(need(rows * cols * es));
+    CUDA_TRY(cudaMemcpy(out, (const char *)src + row_off * cols * es, rows * cols * es,
+                        cudaMemcpyDeviceToHost));
+    return KVR_OK;
+  };
+  auto vec_out = [&](const float *src, size_t n) -> kvr_status {
+    KVR_TRY(need(n * es));
+    std::vector<float> t(n);
+    CUDA_TRY(cudaMemcpy(t.data(), src, n * 4, cudaMemcpyDeviceToHost));
+    for (size_t i = 0; i < n; ++i) {
+      if (es == 2)
+        ((uint16_t *)out)[i] = f32_to_bf16_bits(t[i]);
+      else
+        ((float *)out)[i] = t[i];
+    }
+    return KVR_OK;
+  };
+  if (nm == "embed") return rows_out(m->embed, dm.V, d, 0);
+  if (nm == "lm_head") return rows_out(m->lm_head, dm.V, d, 0);
+  if (nm == "final_norm") return vec_out(m->final_norm, d);
+  if (nm == "wq") return rows_out(w->wqkv, HD, d, 0);
+  if (nm == "wk") return rows_out(w->wqkv, GD, d, HD);
+  if (nm == "wv") return rows_out(w->wqkv, GD, d, HD + GD);
+  if (nm == "wo") return rows_out(w->wo, d, HD, 0);
+  if (nm == "wd") return rows_out(w->wd, d, dm.F, 0);
+  if (nm == "attn_norm") return vec_out(w->attn_norm, d);
+  if (nm == "mlp_norm") return vec_out(w->mlp_norm, d);
+  if (nm == "bq" || nm == "bk" || nm == "bv") {
+    if (!dm.qkv_bias) return fail(KVR_E_INVAL, "model has no QKV bias");
+    size_t o = nm == "bq" ? 0 : (nm == "bk" ? HD : HD + GD);
+    return vec_out(w->bqkv + o, nm == "bq" ? HD : GD);
+  }
+  if (nm == "wg" || nm == "wu") {
+    KVR_TRY(need((size_t)dm.F * d * es));
+    size_t row = d * es;
+    for (int b = 0; b < dm.F / GU_BLOCK; ++b) {
+      size_t srow = (size_t)b * 2 * GU_BLOCK + (nm == "wu" ? GU_BLOCK : 0);
+      CUDA_TRY(cudaMemcpy((char *)out + (size_t)b * GU_BLOCK * row,
+                          (const char *)w->wgu + srow * row, GU_BLOCK * row,
+                          cudaMemcpyDeviceToHost));
+    }
+    return KVR_OK;
+  }
+  return fail(KVR_E_INVAL, "unknown tensor '%s'", name);
+}
+
+kvr_status kvr_profile_enable(kvr_model *m, int32_t enable) {
+  if (!m) return fail(KVR_E_INVAL, "NULL model");
+  m->prof = enable != 0;
+  return KVR_OK;
+}
+
+kvr_status kvr_profile_reset(kvr_model *m) {
+  if (!m) return fail(KVR_E_INVAL, "NULL model");
+  prof_collect(m);
+  for (auto &c : m->prof_classes) {
+    c.ms = 0;
+    c.launches = 0;
+    c.bytes = 0;
+  }
+  return KVR_OK;
+}
+
+kvr_status kvr_profile_read(kvr_model *m, int32_t cap, double *ms, int64_t *launches,
+                            int64_t *bytes, char *names, int32_t names_cap, int32_t *n_out) {
+  if (!m || !n_out) return fail(KVR_E_INVAL, "NULL argument");
+  prof_collect(m);
+  int n = (int)m->prof_classes.size();
+  *n_out = n;
+  int w = 0;
+  for (int i = 0; i < n && i < cap; ++i) {
+    if (ms) ms[i] = m->prof_classes[i].ms;
+    if (launches) launches[i] = m->prof_classes[i].launches;
+    if (bytes) bytes[i] = m->prof_classes[i].bytes;
+    if (names) {
+      const std::string &s = m->prof_classes[i].name;
+      if (w + (int)s.size() + 1 <= names_cap) {
+        memcpy(names + w, s.c_str(), s.size() + 1);
+        w += (int)s.size() + 1;
+      }
+    }
+  }
+  return KVR_OK;
+}
+
+}  // extern "C"

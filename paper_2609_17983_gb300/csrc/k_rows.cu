@@ -1,0 +1,280 @@
+// k_rows.cu -- per-row kernels of the repair pass: seeded weight init,
+// embedding gather, RMSNorm, RoPE + K/V scatter into the paged cache,
+// SwiGLU, and cache row readback / save / restore.
+#include "kvr_internal.cuh"
+
+namespace kvr {
+
+namespace {
+
+constexpr uint64_t GAMMA = 0x9E3779B97F4A7C15ull;
+
+__device__ __forceinline__ uint64_t mix64(uint64_t z) {
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+template <typename T>
+__device__ __forceinline__ float ld(const T *p, size_t i);
+template <>
+__device__ __forceinline__ float ld<float>(const float *p, size_t i) { return p[i]; }
+template <>
+__device__ __forceinline__ float ld<__nv_bfloat16>(const __nv_bfloat16 *p, size_t i) {
+  return __bfloat162float(p[i]);
+}
+
+template <typename T>
+__device__ __forceinline__ void st(T *p, size_t i, float v);
+template <>
+__device__ __forceinline__ void st<float>(float *p, size_t i, float v) { p[i] = v; }
+template <>
+__device__ __forceinline__ void st<__nv_bfloat16>(__nv_bfloat16 *p, size_t i, float v) {
+  p[i] = __float2bfloat16_rn(v);
+}
+
+// One element of the seeded weight definition (SplitMix64 stream, Irwin-Hall
+// sum of four 16-bit lanes, scaled in double, rounded to fp32).
+__device__ __forceinline__ float init_value(uint64_t tseed, int64_t e, double scale) {
+  uint64_t r = mix64(tseed + (uint64_t)(e + 1) * GAMMA);
+  int s = (int)(r & 0xFFFF) + (int)((r >> 16) & 0xFFFF) + (int)((r >> 32) & 0xFFFF) +
+          (int)(r >> 48);
+  double x = (double)(s - 2 * 65535) * scale;
+  return __double2float_rn(x);
+}
+
+__global__ void k_init_tensor(void *dst, int dtype, int out_f32, uint64_t tseed, double scale,
+                              int64_t rows, int64_t cols, int64_t row_off, int inter) {
+  int64_t total = rows * cols;
+  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    float f = init_value(tseed, e, scale);
+    int64_t r = e / cols, c = e % cols;
+    int64_t dr = inter == 0 ? row_off + r
+                            : (r / GU_BLOCK) * (2 * GU_BLOCK) + (inter == 2 ? GU_BLOCK : 0) +
+                                  r % GU_BLOCK;
+    size_t o = (size_t)(dr * cols + c);
+    if (dtype == KVR_DTYPE_BF16) {
+      __nv_bfloat16 b = __float2bfloat16_rn(f);
+      if (out_f32)
+        ((float *)dst)[o] = __bfloat162float(b);
+      else
+        ((__nv_bfloat16 *)dst)[o] = b;
+    } else {
+      ((float *)dst)[o] = f;
+    }
+  }
+}
+
+__global__ void k_fill_f32(float *dst, float v, size_t n) {
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n;
+       i += (size_t)gridDim.x * blockDim.x)
+    dst[i] = v;
+}
+
+template <typename T>
+__global__ void k_embed_rows(const T *embed, const int32_t *tokens,
+                             const int32_t *const *doc_tokens, const int32_t *rowdoc,
+                             const int32_t *pos, int d, float *h) {
+  int i = blockIdx.x;
+  const int32_t *tk = doc_tokens ? doc_tokens[rowdoc[i]] : tokens;
+  size_t base = (size_t)tk[pos[i]] * d;
+  for (int c = threadIdx.x; c < d; c += blockDim.x) h[(size_t)i * d + c] = ld(embed, base + c);
+}
+
+template <typename T>
+__global__ void k_rmsnorm(const float *h, const float *g, int d, float eps, T *out) {
+  int i = blockIdx.x;
+  const float *x = h + (size_t)i * d;
+  float ss = 0.f;
+  for (int c = threadIdx.x; c < d; c += blockDim.x) ss += x[c] * x[c];
+  __shared__ float red[32];
+  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    float t = threadIdx.x < (blockDim.x >> 5) ? red[threadIdx.x] : 0.f;
+    for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+    if (threadIdx.x == 0) red[0] = t;
+  }
+  __syncthreads();
+  float r = 1.0f / sqrtf(red[0] / (float)d + eps);
+  for (int c = threadIdx.x; c < d; c += blockDim.x) st(out, (size_t)i * d + c, x[c] * r * g[c]);
+}
+
+// grid (M, H + 2G), block dh/2: rotate q and k heads at the row's position;
+// q -> q_out fp32, k and v -> cache (if write_kv).
+template <typename T>
+__global__ void k_rope_scatter(const float *qkv, const float2 *rope, const int32_t *pos, int H,
+                               int G, int dh, int layer, const KVView *views,
+                               const int32_t *rowdoc, KVView single, float *q_out, int write_kv) {
+  int i = blockIdx.x, hh = blockIdx.y, t = threadIdx.x, half = dh >> 1;
+  int Nqkv = (H + 2 * G) * dh;
+  int p = pos[i];
+  const float *x = qkv + (size_t)i * Nqkv + (size_t)hh * dh;
+  float x1 = x[t], x2 = x[t + half];
+  if (hh < H + G) {
+    float2 cs = rope[(size_t)p * half + t];
+    float r1 = x1 * cs.x - x2 * cs.y;
+    float r2 = x2 * cs.x + x1 * cs.y;
+    x1 = r1;
+    x2 = r2;
+  }
+  if (hh < H) {
+    float *qo = q_out + (size_t)i * H * dh + (size_t)hh * dh;
+    qo[t] = x1;
+    qo[t + half] = x2;
+    return;
+  }
+  if (!write_kv) return;
+  KVView v = views ? views[rowdoc[i]] : single;
+  int kv = hh < H + G ? 0 : 1;
+  int g = hh - H - kv * G;
+  T *c = (T *)v.pages;
+  size_t o = v.offset(layer, kv, g, p);
+  st(c, o + t, x1);
+  st(c, o + t + half, x2);
+}
+
+template <typename T>
+__global__ void k_swiglu(const float *gu, int M, int F, T *act) {
+  size_t total = (size_t)M * F;
+  for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < total;
+       e += (size_t)gridDim.x * blockDim.x) {
+    size_t m = e / F;
+    int f = (int)(e % F);
+    size_t base = m * 2 * F + (size_t)(f / GU_BLOCK) * 2 * GU_BLOCK + f % GU_BLOCK;
+    float g = gu[base], u = gu[base + GU_BLOCK];
+    st(act, e, g / (1.0f + expf(-g)) * u);
+  }
+}
+
+template <typename T>
+__global__ void k_cache_gather(KVView v, const int32_t *pos, int n_pos, int l0, int nl, int G,
+                               int dh, float *k_out, float *v_out) {
+  size_t total = (size_t)n_pos * nl * G * dh;
+  const T *c = (const T *)v.pages;
+  for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < total;
+       e += (size_t)gridDim.x * blockDim.x) {
+    int i = (int)(e % dh);
+    size_t r = e / dh;
+    int g = (int)(r % G);
+    r /= G;
+    int l = (int)(r % nl);
+    int p = (int)(r / nl);
+    k_out[e] = ld(c, v.offset(l0 + l, 0, g, pos[p]) + i);
+    v_out[e] = ld(c, v.offset(l0 + l, 1, g, pos[p]) + i);
+  }
+}
+
+// buf layout [n_pos][nl][2][G][dh] in the cache dtype
+template <typename T>
+__global__ void k_rows_copy(KVView v, const int32_t *pos, int n_pos, int l0, int nl, T *buf,
+                            int to_buf) {
+  int G = v.G, dh = v.dh;
+  size_t total = (size_t)n_pos * nl * 2 * G * dh;
+  T *c = (T *)v.pages;
+  for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < total;
+       e += (size_t)gridDim.x * blockDim.x) {
+    int i = (int)(e % dh);
+    size_t r = e / dh;
+    int g = (int)(r % G);
+    r /= G;
+    int kv = (int)(r % 2);
+    r /= 2;
+    int l = (int)(r % nl);
+    int p = (int)(r / nl);
+    size_t o = v.offset(l0 + l, kv, g, pos[p]) + i;
+    if (to_buf)
+      buf[e] = c[o];
+    else
+      c[o] = buf[e];
+  }
+}
+
+int grid_for(size_t n, int block) {
+  size_t g = (n + block - 1) / block;
+  return (int)(g > 65535 * 8 ? 65535 * 8 : (g == 0 ? 1 : g));
+}
+
+}  // namespace
+
+void launch_init_tensor(void *dst, int dtype, bool out_f32, uint64_t tseed, double scale,
+                        int64_t rows, int64_t cols, int64_t row_off, int interleave,
+                        cudaStream_t s) {
+  size_t n = (size_t)(rows * cols);
+  k_init_tensor<<<grid_for(n, 256), 256, 0, s>>>(dst, dtype, out_f32 ? 1 : 0, tseed, scale, rows,
+                                                  cols, row_off, interleave);
+}
+
+void launch_fill_f32(float *dst, float v, size_t n, cudaStream_t s) {
+  k_fill_f32<<<grid_for(n, 256), 256, 0, s>>>(dst, v, n);
+}
+
+void launch_embed_rows(const void *embed, int dtype, const int32_t *tokens,
+                       const int32_t *const *doc_tokens, const int32_t *rowdoc,
+                       const int32_t *pos, int M, int d, float *h, cudaStream_t s) {
+  if (M <= 0) return;
+  if (dtype == KVR_DTYPE_BF16)
+    k_embed_rows<<<M, 256, 0, s>>>((const __nv_bfloat16 *)embed, tokens, doc_tokens, rowdoc, pos,
+                                   d, h);
+  else
+    k_embed_rows<<<M, 256, 0, s>>>((const float *)embed, tokens, doc_tokens, rowdoc, pos, d, h);
+}
+
+void launch_rmsnorm(const float *h, const float *g, int M, int d, double eps, void *out,
+                    int out_dtype, cudaStream_t s) {
+  if (M <= 0) return;
+  if (out_dtype == KVR_DTYPE_BF16)
+    k_rmsnorm<<<M, 256, 0, s>>>(h, g, d, (float)eps, (__nv_bfloat16 *)out);
+  else
+    k_rmsnorm<<<M, 256, 0, s>>>(h, g, d, (float)eps, (float *)out);
+}
+
+void launch_rope_scatter(const float *qkv, const float2 *rope, const int32_t *pos, int M,
+                         const Dims &dm, int layer, const KVView *views, const int32_t *rowdoc,
+                         KVView single, float *q_out, bool write_kv, cudaStream_t s) {
+  if (M <= 0) return;
+  dim3 grid(M, dm.H + 2 * dm.G);
+  if (dm.dtype == KVR_DTYPE_BF16)
+    k_rope_scatter<__nv_bfloat16><<<grid, dm.dh / 2, 0, s>>>(
+        qkv, rope, pos, dm.H, dm.G, dm.dh, layer, views, rowdoc, single, q_out, write_kv);
+  else
+    k_rope_scatter<float><<<grid, dm.dh / 2, 0, s>>>(qkv, rope, pos, dm.H, dm.G, dm.dh, layer,
+                                                     views, rowdoc, single, q_out, write_kv);
+}
+
+void launch_swiglu(const float *gu, int M, int F, void *act, int dtype, cudaStream_t s) {
+  if (M <= 0) return;
+  size_t n = (size_t)M * F;
+  if (dtype == KVR_DTYPE_BF16)
+    k_swiglu<<<grid_for(n, 256), 256, 0, s>>>(gu, M, F, (__nv_bfloat16 *)act);
+  else
+    k_swiglu<<<grid_for(n, 256), 256, 0, s>>>(gu, M, F, (float *)act);
+}
+
+void launch_cache_gather(KVView v, int dtype, const int32_t *pos, int n_pos, int l0, int l1,
+                         int G, int dh, float *k_out, float *v_out, cudaStream_t s) {
+  size_t n = (size_t)n_pos * (l1 - l0) * G * dh;
+  if (n == 0) return;
+  if (dtype == KVR_DTYPE_BF16)
+    k_cache_gather<__nv_bfloat16><<<grid_for(n, 256), 256, 0, s>>>(v, pos, n_pos, l0, l1 - l0, G,
+                                                                    dh, k_out, v_out);
+  else
+    k_cache_gather<float><<<grid_for(n, 256), 256, 0, s>>>(v, pos, n_pos, l0, l1 - l0, G, dh,
+                                                            k_out, v_out);
+}
+
+void launch_rows_copy(KVView v, int dtype, const int32_t *pos, int n_pos, int l0, int l1,
+                      void *buf, bool to_buf, cudaStream_t s) {
+  size_t n = (size_t)n_pos * (l1 - l0) * 2 * v.G * v.dh;
+  if (n == 0) return;
+  if (dtype == KVR_DTYPE_BF16)
+    k_rows_copy<<<grid_for(n, 256), 256, 0, s>>>(v, pos, n_pos, l0, l1 - l0,
+                                                  (__nv_bfloat16 *)buf, to_buf ? 1 : 0);
+  else
+    k_rows_copy<<<grid_for(n, 256), 256, 0, s>>>(v, pos, n_pos, l0, l1 - l0, (float *)buf,
+                                                  to_buf ? 1 : 0);
+}
+
+}  // namespace kvr

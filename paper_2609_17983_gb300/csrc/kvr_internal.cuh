@@ -1,0 +1,187 @@
+// kvr_internal.cuh -- internal declarations of libkvrepair (not installed).
+//
+// Device data layout (HBM):
+//   weights  one allocation; per layer
+//              wqkv [(H+2G)*dh][d]   rows: q heads, then k heads, then v heads
+//              bqkv fp32 [(H+2G)*dh] (QKV-bias models only)
+//              wo   [d][H*dh]
+//              wgu  [2F][d]          gate/up rows interleaved in blocks of 16:
+//                                    rows 32b..32b+15 = gate 16b..16b+15,
+//                                    rows 32b+16..32b+31 = up 16b..16b+15
+//              wd   [d][F]
+//              attn_norm, mlp_norm fp32 [d]
+//            embed [V][d], lm_head [V][d], final_norm fp32 [d]
+//   KV cache paged: page = KVR_PAGE positions of every layer,
+//            [page][layer][k|v][kv head][slot][dh] in the model dtype;
+//            a block table maps logical page -> physical page.
+//   activations (per model workspace, max_rows R): residual h fp32 [R][d],
+//            normed rows a [R][d], qkv fp32 [R][Nqkv], q fp32 [R][H*dh],
+//            attention output [R][H*dh], gate/up fp32 [R][2F], act [R][F].
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <cstdint>
+#include <string>
+#include <vector>
+
+#include "../../include/kvrepair.h"
+
+namespace kvr {
+
+constexpr int KVR_PAGE = 64;          // positions per KV page
+constexpr int KVR_QUERY_RESERVE = 64; // positions past n reserved for fresh queries
+constexpr int GU_BLOCK = 16;          // gate/up interleave block (rows)
+
+struct Dims {
+  int V, d, L, H, G, dh, F;
+  int qkv_bias, dtype, delim;
+  double theta, eps;
+  int max_ctx, max_rows;
+  int Nqkv() const { return (H + 2 * G) * dh; }
+  size_t es() const { return dtype == KVR_DTYPE_BF16 ? 2 : 4; }
+  // elements of one KV page (all layers, k and v)
+  size_t page_elems() const { return (size_t)L * 2 * G * KVR_PAGE * dh; }
+};
+
+struct LayerW {
+  void *wqkv, *wo, *wgu, *wd;
+  float *bqkv, *attn_norm, *mlp_norm;
+};
+
+// Device view of one document's paged cache (passed by value to kernels).
+struct KVView {
+  void *pages;              // pool base
+  const int32_t *table;     // logical page -> physical page
+  int L, G, dh;             // shape
+  __host__ __device__ size_t offset(int layer, int kv, int g, int pos) const {
+    size_t page = (size_t)table[pos / KVR_PAGE];
+    return ((((page * L + layer) * 2 + kv) * G + g) * KVR_PAGE + (pos % KVR_PAGE)) * dh;
+  }
+};
+
+// Internal error state of one kernel-class timer.
+struct ProfClass {
+  std::string name;
+  double ms = 0;
+  int64_t launches = 0;
+  int64_t bytes = 0;
+};
+
+}  // namespace kvr
+
+struct kvr_model {
+  kvr::Dims dims{};
+  void *weight_block = nullptr;
+  size_t weight_bytes = 0;
+  void *embed = nullptr, *lm_head = nullptr;
+  float *final_norm = nullptr;
+  std::vector<kvr::LayerW> layers;
+  float2 *rope = nullptr;  // [max_ctx + reserve][dh/2] (cos, sin), fp32 from fp64 angles
+  cudaStream_t stream = nullptr;
+  int device = 0;
+  int num_sms = 0;
+  // workspace
+  void *ws_block = nullptr;
+  int32_t *pos_d = nullptr;  // [R] positions of the rows of a pass
+  int32_t *rowdoc_d = nullptr;  // [R] batch: document of each row
+  float *h = nullptr, *qkv = nullptr, *q = nullptr, *gu = nullptr, *logits = nullptr;
+  void *a = nullptr, *attn = nullptr, *act = nullptr;
+  float *scores = nullptr;     // [max_ctx + reserve] selector scores
+  unsigned long long *keys = nullptr;  // [max_ctx + reserve] top-K keys
+  int32_t *sel_out = nullptr;  // [max_ctx] selected positions
+  int32_t *sel_count = nullptr;
+  void *save = nullptr;        // stale rows saved by read-only selector passes
+  size_t save_bytes = 0;
+  int *dev_flag = nullptr;     // device error flag (bounded waits)
+  // pinned staging for host->device argument copies
+  int32_t *stage_h = nullptr;
+  int32_t *stage_d = nullptr;
+  size_t stage_cap = 0;
+  cudaEvent_t stage_ev = nullptr;
+  // profiling
+  bool prof = false;
+  std::vector<kvr::ProfClass> prof_classes;
+  std::vector<std::pair<int, std::pair<cudaEvent_t, cudaEvent_t>>> prof_pending;
+  int64_t launches = 0;
+};
+
+struct kvr_cache {
+  kvr_model *model = nullptr;
+  int n = 0, cap = 0, n_pages = 0;
+  void *pages = nullptr;
+  int32_t *table = nullptr;   // device [n_pages]
+  int32_t *tokens_d = nullptr;  // device [cap]
+  std::vector<int32_t> tokens_h;
+  bool poisoned = false;
+  kvr::KVView view() const {
+    return kvr::KVView{pages, table, model->dims.L, model->dims.G, model->dims.dh};
+  }
+};
+
+namespace kvr {
+
+// ---- allocation (allocator hook) ----
+void *dev_alloc(size_t bytes);
+void dev_free(void *p);
+
+// ---- kernels: weights ----
+// Fill rows of a device tensor from the seeded generator.  Element (r, c) of
+// the canonical [rows][cols] tensor is generated and stored at
+// dst[map(r) * cols + c] with map(r) = row_off + r (interleave == 0) or the
+// gate/up interleave (interleave == 1: gate, 2: up).  out_f32: store as fp32
+// (value first rounded to the model dtype).
+void launch_init_tensor(void *dst, int dtype, bool out_f32, uint64_t tensor_seed, double scale,
+                        int64_t rows, int64_t cols, int64_t row_off, int interleave,
+                        cudaStream_t s);
+void launch_fill_f32(float *dst, float v, size_t n, cudaStream_t s);
+
+// ---- kernels: row ops ----
+void launch_embed_rows(const void *embed, int dtype, const int32_t *tokens,
+                       const int32_t *const *doc_tokens, const int32_t *rowdoc,
+                       const int32_t *pos, int M, int d, float *h, cudaStream_t s);
+void launch_rmsnorm(const float *h, const float *g, int M, int d, double eps, void *out,
+                    int out_dtype, cudaStream_t s);
+void launch_rope_scatter(const float *qkv, const float2 *rope, const int32_t *pos, int M,
+                         const Dims &dm, int layer, const KVView *views, const int32_t *rowdoc,
+                         KVView single, float *q_out, bool write_kv, cudaStream_t s);
+void launch_swiglu(const float *gu, int M, int F, void *act, int dtype, cudaStream_t s);
+void launch_cache_gather(KVView v, int dtype, const int32_t *pos, int n_pos, int l0, int l1,
+                         int G, int dh, float *k_out, float *v_out, cudaStream_t s);
+void launch_rows_copy(KVView v, int dtype, const int32_t *pos, int n_pos, int l0, int l1,
+                      void *buf, bool to_buf, cudaStream_t s);
+
+// ---- kernels: GEMM  Y[M][N] (+)= X[M][K] W[N][K]^T (+ bias) ----
+struct GemmArgs {
+  const void *X;
+  const void *W;
+  const float *bias;
+  float *Y;
+  int M, N, K;
+  int ldx, ldy;
+  int dtype;       // operands: KVR_DTYPE_F32 or KVR_DTYPE_BF16
+  int accumulate;  // 1: Y += result
+};
+void launch_gemm_simt(const GemmArgs &g, cudaStream_t s);
+
+// ---- kernels: attention ----
+// o[i] = softmax(q_i K[0..pos_i]^T / sqrt(dh)) V[0..pos_i] for every row i,
+// GQA head h -> kv head h / (H/G).  q fp32 [M][H*dh]; out [M][H*dh] in dtype.
+void launch_attention_simt(const float *q, const int32_t *pos, int M, const Dims &dm, int layer,
+                           const KVView *views, const int32_t *rowdoc, KVView single, void *out,
+                           cudaStream_t s);
+
+// ---- kernels: selectors ----
+void launch_scores_simple(int policy, const int32_t *tokens, int n, int s_end, int delim,
+                          uint64_t seed, unsigned long long *keys, cudaStream_t s);
+void launch_attn_select_scores(const float *q, int S, const Dims &dm, int layer, KVView v,
+                               int s_end, int n, float *probs_ws, float *scores, cudaStream_t s);
+void launch_kv_deviation(const float *qkv, const float2 *rope, const int32_t *pos, int M,
+                         const Dims &dm, KVView v, float *scores, cudaStream_t s);
+void launch_float_keys(const float *scores, int n, int s_end, unsigned long long *keys,
+                       cudaStream_t s);
+void launch_topk(const unsigned long long *keys, int n, int s_end, int K, int32_t *out,
+                 int32_t *count, cudaStream_t s);
+
+}  // namespace kvr

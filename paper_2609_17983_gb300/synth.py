@@ -29,6 +29,7 @@ random token ids (the delimiter id excluded from the fill).
 from __future__ import annotations
 
 import math
+import os
 
 import numpy as np
 
@@ -118,21 +119,62 @@ def normal_values(model_seed: int, tid: int, idx: np.ndarray, dtype: str,
                   std: float = WEIGHT_STD) -> np.ndarray:
     """Weight values at element indices idx of tensor tid (see module doc)."""
     r = stream_out(tensor_seed(model_seed, tid), idx)
+    return _lanes_to_values(r, dtype, std)
+
+
+def _lanes_to_values(r: np.ndarray, dtype: str, std: float) -> np.ndarray:
+    """Irwin-Hall(4) of the 16-bit lanes of r, centred, scaled, rounded (in place on r)."""
     m16 = np.uint64(0xFFFF)
-    s = ((r & m16) + ((r >> np.uint64(16)) & m16) + ((r >> np.uint64(32)) & m16)
-         + (r >> np.uint64(48))).astype(np.int64)
-    x = (s - LANE_MEAN_SUM).astype(np.float64) * weight_scale(std)
-    f = x.astype(np.float32)
+    t = np.empty_like(r)
+    s = np.bitwise_and(r, m16)
+    for sh in (16, 32):
+        np.right_shift(r, np.uint64(sh), out=t)
+        np.bitwise_and(t, m16, out=t)
+        s += t
+    np.right_shift(r, np.uint64(48), out=t)
+    s += t
+    x = s.view(np.int64)
+    x -= LANE_MEAN_SUM
+    f = (x.astype(np.float64) * weight_scale(std)).astype(np.float32)
     return f32_to_bf16_bits(f) if dtype == "bf16" else f
 
 
+def _contiguous_values(tseed: int, start: int, count: int, dtype: str, std: float) -> np.ndarray:
+    """Values of elements start..start+count-1 of the stream tseed."""
+    z = np.arange(start + 1, start + count + 1, dtype=np.uint64)
+    t = np.empty_like(z)
+    with np.errstate(over="ignore"):
+        z *= GAMMA
+        z += np.uint64(tseed)
+        np.right_shift(z, np.uint64(30), out=t)
+        z ^= t
+        z *= _M1
+        np.right_shift(z, np.uint64(27), out=t)
+        z ^= t
+        z *= _M2
+        np.right_shift(z, np.uint64(31), out=t)
+        z ^= t
+    return _lanes_to_values(z, dtype, std)
+
+
 def tensor(model_seed: int, tid: int, shape, dtype: str, std: float = WEIGHT_STD,
-           chunk: int = 1 << 24) -> np.ndarray:
+           chunk: int = 1 << 21) -> np.ndarray:
     n = int(np.prod(shape))
     out = np.empty(n, np.uint16 if dtype == "bf16" else np.float32)
-    for b in range(0, n, chunk):
+    tseed = tensor_seed(model_seed, tid)
+
+    def fill(b):
         e = min(n, b + chunk)
-        out[b:e] = normal_values(model_seed, tid, np.arange(b, e, dtype=np.uint64), dtype, std)
+        out[b:e] = _contiguous_values(tseed, b, e - b, dtype, std)
+
+    starts = range(0, n, chunk)
+    if n > 4 * chunk:
+        from concurrent.futures import ThreadPoolExecutor
+        with ThreadPoolExecutor(max_workers=min(16, os.cpu_count() or 1)) as ex:
+            list(ex.map(fill, starts))
+    else:
+        for b in starts:
+            fill(b)
     return out.reshape(shape)
 
 

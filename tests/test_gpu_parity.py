@@ -1,0 +1,328 @@
+"""GPU-versus-oracle parity through the C ABI (libkvrepair) on seeded inputs.
+
+Tolerances: max|gpu - ref| / max|ref| <= 1e-4 for the fp32 model and <= 2e-2
+for bf16 models, per layer, for K and V over the rows compared, and for the
+logits.  Selected position sets must be identical except where the oracle's
+scores of the swapped positions lie within a tie band of the K-th score
+(exact ties for editlocal/structural/random).
+"""
+import numpy as np
+import pytest
+
+import oracle
+from paper_2609_17983_gb300 import synth
+
+try:  # collected everywhere; loaded (and required) only when the tests run
+    from paper_2609_17983_gb300 import kvrepair as kv
+except ImportError as _e:  # pragma: no cover
+    kv, _IMPORT_ERROR = None, _e
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(autouse=True)
+def _library_loaded():
+    if kv is None:
+        raise _IMPORT_ERROR
+
+TOL = {"fp32": 1e-4, "bf16": 2e-2}
+
+
+def rel(a, b):
+    return float(np.abs(np.asarray(a, np.float64) - b).max() / max(np.abs(b).max(), 1e-30))
+
+
+def cmp_rows(cache, ref: oracle.Cache, rows, tol, L=None):
+    """GPU cache rows vs oracle cache rows, per layer, K and V separately."""
+    rows = np.asarray(rows)
+    k, v = cache.read(rows)
+    L = k.shape[1] if L is None else L
+    worst = 0.0
+    for l in range(L):
+        rk, rv = ref.k[l, rows], ref.v[l, rows]
+        ek, ev = rel(k[:, l], rk), rel(v[:, l], rv)
+        worst = max(worst, ek, ev)
+        assert ek <= tol and ev <= tol, (l, ek, ev)
+    return worst
+
+
+def check_selection(gpu_sel, ref_sel, ref_scores, band):
+    gpu_sel, ref_sel = list(map(int, gpu_sel)), list(map(int, ref_sel))
+    assert len(gpu_sel) == len(ref_sel)
+    if gpu_sel == ref_sel:
+        return
+    kth = min(ref_scores[j] for j in ref_sel)
+    for j in set(gpu_sel) - set(ref_sel):
+        assert ref_scores[j] >= kth - band, (j, ref_scores[j], kth)
+    for j in set(ref_sel) - set(gpu_sel):
+        assert ref_scores[j] <= kth + band, (j, ref_scores[j], kth)
+
+
+# ------------------------------------------------------------------ fixtures
+
+def tiny_setup(dtype="fp32", **over):
+    w = synth.workload("tiny")
+    cfg = synth.preset("tiny", dtype=dtype, **over)
+    W = synth.weights(cfg, 0)
+    return cfg, W, w["doc"], w["edit_start"], w["new_tokens"]
+
+
+@pytest.fixture(scope="module")
+def tiny():
+    cfg, W, doc, s, new = tiny_setup()
+    model = kv.Model(cfg, W, max_context=1024, max_rows=512)
+    ref_stale = oracle.prefill(cfg, W, doc)
+    yield dict(cfg=cfg, W=W, doc=doc, s=s, new=new, model=model, ref_stale=ref_stale)
+    model.close()
+
+
+# --------------------------------------------------------------- generator
+
+@pytest.mark.parametrize("dtype,bias", [("fp32", False), ("bf16", True)])
+def test_device_weight_generator_matches_host(dtype, bias):
+    cfg = synth.preset("tiny", dtype=dtype, qkv_bias=bias)
+    W = synth.weights(cfg, 7)
+    model = kv.Model(cfg, None, seed=7, max_context=256, max_rows=64)
+    names = ["wq", "wk", "wv", "wo", "wg", "wu", "wd", "attn_norm", "mlp_norm"]
+    if bias:
+        names += ["bq", "bk", "bv"]
+    for l in range(cfg["n_layers"]):
+        for nm in names:
+            assert np.array_equal(model.read_tensor(nm, l), W["layers"][l][nm]), (l, nm)
+    for nm in ("embed", "lm_head", "final_norm"):
+        assert np.array_equal(model.read_tensor(nm), W[nm]), nm
+    model.close()
+
+
+# ------------------------------------------------------------ forward / R
+
+def test_prefill_parity_fp32(tiny):
+    cache = tiny["model"].prefill(tiny["doc"])
+    cmp_rows(cache, tiny["ref_stale"], np.arange(len(tiny["doc"])), TOL["fp32"])
+    assert np.array_equal(cache.tokens(), tiny["doc"])
+
+
+@pytest.mark.parametrize("K", [0, 32, 308])
+def test_repair_parity_fp32(tiny, K):
+    cfg, W, doc, s, new, model = (tiny[k] for k in ("cfg", "W", "doc", "s", "new", "model"))
+    cache = model.prefill(doc)
+    n = len(doc)
+    before_k, before_v = cache.read(np.arange(n))
+    A = np.arange(s + len(new), s + len(new) + K)
+    cache.repair(new, s, A)
+    ref = oracle.repair(cfg, W, tiny["ref_stale"], new, s, A)
+    P = oracle.repaired_set(s, len(new), A)
+    cmp_rows(cache, ref, P, TOL["fp32"])
+    # every entry outside P is bit-identical to the stale cache
+    after_k, after_v = cache.read(np.arange(n))
+    mask = np.ones(n, bool)
+    mask[P] = False
+    assert np.array_equal(after_k[mask], before_k[mask])
+    assert np.array_equal(after_v[mask], before_v[mask])
+    assert np.array_equal(cache.tokens(), oracle.apply_edit(doc, s, new))
+
+
+def test_repair_scattered_positions_fp32(tiny):
+    cfg, W, doc, s, new, model = (tiny[k] for k in ("cfg", "W", "doc", "s", "new", "model"))
+    cache = model.prefill(doc)
+    A = np.array([204, 205, 230, 231, 300, 401, 402, 511])
+    cache.repair(new, s, A)
+    ref = oracle.repair(cfg, W, tiny["ref_stale"], new, s, A)
+    cmp_rows(cache, ref, oracle.repaired_set(s, len(new), A), TOL["fp32"])
+
+
+def test_endpoint_identity_gpu(tiny):
+    # Eq. 1: repair with the full suffix equals a prefill of C'
+    doc, s, new, model = tiny["doc"], tiny["s"], tiny["new"], tiny["model"]
+    cache = model.prefill(doc)
+    cache.repair(new, s, np.arange(s + len(new), len(doc)))
+    fresh = model.prefill(oracle.apply_edit(doc, s, new))
+    rows = np.arange(len(doc))
+    k1, v1 = cache.read(rows)
+    k2, v2 = fresh.read(rows)
+    assert rel(k1, k2) <= TOL["fp32"] and rel(v1, v2) <= TOL["fp32"]
+
+
+def test_noop_edit_and_idempotence_gpu(tiny):
+    doc, s, model = tiny["doc"], tiny["s"], tiny["model"]
+    cache = model.prefill(doc)
+    rows = np.arange(len(doc))
+    k0, v0 = cache.read(rows)
+    cache.repair(doc[s:s + 4], s, [])
+    k1, v1 = cache.read(rows)
+    assert rel(k1, k0) <= TOL["fp32"] and rel(v1, v0) <= TOL["fp32"]
+    A = np.arange(s + 4, s + 36)
+    cache.repair(tiny["new"], s, A)
+    k2, v2 = cache.read(rows)
+    cache.repair(tiny["new"], s, A)
+    k3, v3 = cache.read(rows)
+    assert np.array_equal(k2, k3) and np.array_equal(v2, v3)
+
+
+def test_logits_parity_fp32(tiny):
+    cfg, W, doc, model = tiny["cfg"], tiny["W"], tiny["doc"], tiny["model"]
+    cache = model.prefill(doc)
+    q = synth.fill_tokens(5, 8, cfg["vocab"], cfg["delim_id"])
+    lg = model.logits(cache, q)
+    ref = oracle.logits(cfg, W, tiny["ref_stale"], q)
+    assert rel(lg, ref) <= TOL["fp32"]
+    # the document's cache is untouched by the fresh query
+    k, v = cache.read(np.arange(len(doc)))
+    k2, v2 = model.prefill(doc).read(np.arange(len(doc)))
+    assert np.array_equal(k, k2) and np.array_equal(v, v2)
+
+
+# --------------------------------------------------------------- selectors
+
+@pytest.mark.parametrize("policy,K,seed", [("editlocal", 32, 0), ("random", 32, 0),
+                                           ("random", 32, 3), ("random", 308, 4),
+                                           ("editlocal", 400, 0)])
+def test_select_closed_form_exact(tiny, policy, K, seed):
+    cfg, W, doc, s, new, model = (tiny[k] for k in ("cfg", "W", "doc", "s", "new", "model"))
+    cache = model.prefill(doc)
+    got = model.select(cache, policy, K, s, new, seed)
+    ref = oracle.select(cfg, W, tiny["ref_stale"], policy, K, s, new, seed)
+    assert got.tolist() == ref.tolist()
+
+
+def test_select_structural_exact():
+    cfg = synth.preset("tiny")
+    W = synth.weights(cfg, 0)
+    doc = synth.document(5, 700, cfg["vocab"], cfg["delim_id"], delim_gap=(40, 80))
+    model = kv.Model(cfg, W, max_context=1024, max_rows=512)
+    cache = model.prefill(doc)
+    s = 300
+    new = synth.edit_tokens(6, doc[s:s + 10], cfg["vocab"], cfg["delim_id"])
+    ref_cache = oracle.empty_cache(cfg, len(doc))
+    ref_cache.tokens[:] = doc
+    for K in (3, 32):
+        got = model.select(cache, "structural", K, s, new)
+        ref = oracle.select(cfg, W, ref_cache, "structural", K, s, new)
+        assert got.tolist() == ref.tolist()
+    model.close()
+
+
+@pytest.mark.parametrize("policy", ["attention", "cacheblend"])
+def test_select_model_policies_parity(tiny, policy):
+    cfg, W, doc, s, new, model = (tiny[k] for k in ("cfg", "W", "doc", "s", "new", "model"))
+    cache = model.prefill(doc)
+    rows = np.arange(len(doc))
+    k0, v0 = cache.read(rows)
+    got = model.select(cache, policy, 32, s, new)
+    sc, D = oracle.scores(cfg, W, tiny["ref_stale"], policy, s, new)
+    ref = oracle.topk(sc, D, 32)
+    check_selection(got, ref, sc, 1e-4 * np.abs(sc[D]).max())
+    # observably read-only
+    k1, v1 = cache.read(rows)
+    assert np.array_equal(k0, k1) and np.array_equal(v0, v1)
+    assert np.array_equal(cache.tokens(), doc)
+
+
+# ------------------------------------------------------------------ batch
+
+def test_repair_batch_parity_fp32():
+    cfg = synth.preset("tiny")
+    W = synth.weights(cfg, 0)
+    model = kv.Model(cfg, W, max_context=1024, max_rows=512)
+    docs = [synth.document(20 + i, 400 + 37 * i, cfg["vocab"]) for i in range(3)]
+    caches = [model.prefill(d) for d in docs]
+    reqs, refs = [], []
+    for i, (d, c) in enumerate(zip(docs, caches)):
+        edits = [(50 + 10 * i, synth.edit_tokens(30 + i, d[50 + 10 * i:54 + 10 * i], cfg["vocab"])),
+                 (200, synth.edit_tokens(40 + i, d[200:203], cfg["vocab"]))]
+        A = np.concatenate([np.arange(54 + 10 * i, 70 + 10 * i), np.arange(203, 220)])
+        reqs.append((c, edits, A))
+        stale = oracle.prefill(cfg, W, d)
+        toks = d.copy()
+        P = list(A)
+        for st, nt in edits:
+            toks[st:st + len(nt)] = nt
+            P += list(range(st, st + len(nt)))
+        P = np.array(sorted(P))
+        ref = stale.copy()
+        ref.tokens = toks
+        oracle.recompute(cfg, W, ref, toks, P)
+        refs.append((ref, P))
+    model.repair_batch(reqs)
+    for c, (ref, P) in zip(caches, refs):
+        cmp_rows(c, ref, P, TOL["fp32"])
+    model.close()
+
+
+# ------------------------------------------------------------ error paths
+
+def test_range_errors_leave_cache_unchanged(tiny):
+    doc, s, new, model = tiny["doc"], tiny["s"], tiny["new"], tiny["model"]
+    cache = model.prefill(doc)
+    rows = np.arange(len(doc))
+    k0, v0 = cache.read(rows)
+    bad = [(new, s, [s + 2]),              # position inside the span
+           (new, s, [300, 299]),           # not increasing
+           (new, s, [len(doc)]),           # beyond n
+           (new, len(doc) - 2, []),        # span beyond n
+           ([5000], s, [])]                # token outside the vocab
+    for nt, st, A in bad:
+        with pytest.raises(kv.KvrError) as e:
+            cache.repair(nt, st, A)
+        assert e.value.code == 2
+    k1, v1 = cache.read(rows)
+    assert np.array_equal(k0, k1) and np.array_equal(v0, v1)
+    assert np.array_equal(cache.tokens(), doc)
+
+
+# ------------------------------------------------------- bf16 and 8B shapes
+
+def test_tiny_bf16_parity():
+    cfg, W, doc, s, new = tiny_setup("bf16", qkv_bias=True)
+    model = kv.Model(cfg, W, max_context=1024, max_rows=512)
+    cache = model.prefill(doc)
+    stale = oracle.prefill(cfg, W, doc)
+    cmp_rows(cache, stale, np.arange(len(doc)), TOL["bf16"])
+    A = np.arange(s + 4, s + 36)
+    cache.repair(new, s, A)
+    ref = oracle.repair(cfg, W, stale, new, s, A)
+    cmp_rows(cache, ref, oracle.repaired_set(s, 4, A), TOL["bf16"])
+    q = synth.fill_tokens(5, 8, cfg["vocab"], cfg["delim_id"])
+    assert rel(model.logits(cache, q), oracle.logits(cfg, W, ref, q)) <= TOL["bf16"]
+    model.close()
+
+
+def compact_inputs(cfg, seed, docs, vocab_sample):
+    """Oracle inputs for a large-vocab model: only the embedding rows of the
+    tokens used and the lm_head rows of a vocabulary sample (same seeded
+    values as the device generator), with tokens remapped into the table."""
+    W = synth.weights(cfg, seed, embed=False, lm_head=False)
+    used = np.unique(np.concatenate(docs))
+    W["embed"] = synth.rows(seed, synth.TID_EMBED, used, cfg["d_model"], cfg["dtype"])
+    W["lm_head"] = synth.rows(seed, synth.TID_LM_HEAD, vocab_sample, cfg["d_model"], cfg["dtype"])
+    remap = {int(t): i for i, t in enumerate(used)}
+    ocfg = dict(cfg, vocab=max(len(used), len(vocab_sample)))
+    if len(used) < ocfg["vocab"]:
+        pad = np.zeros((ocfg["vocab"] - len(used), cfg["d_model"]), W["embed"].dtype)
+        W["embed"] = np.concatenate([W["embed"], pad])
+    if len(vocab_sample) < ocfg["vocab"]:
+        pad = np.zeros((ocfg["vocab"] - len(vocab_sample), cfg["d_model"]), W["lm_head"].dtype)
+        W["lm_head"] = np.concatenate([W["lm_head"], pad])
+    return ocfg, W, [np.array([remap[int(t)] for t in d], np.int32) for d in docs]
+
+
+@pytest.mark.parametrize("shape", ["llama8b", "qwen7b"])
+def test_8b_shape_two_layer_parity(shape):
+    cfg = synth.preset(shape, n_layers=2)
+    n, s, L, K = 200, 90, 6, 32
+    doc = synth.document(1, n, cfg["vocab"])
+    new = synth.edit_tokens(2, doc[s:s + L], cfg["vocab"])
+    query = synth.fill_tokens(9, 4, cfg["vocab"], 13)
+    vs = np.sort(np.unique(np.concatenate([synth.fill_tokens(3, 512, cfg["vocab"], 13),
+                                           [0, cfg["vocab"] - 1]])))
+    model = kv.Model(cfg, None, seed=0, max_context=512, max_rows=256)
+    cache = model.prefill(doc)
+    A = np.arange(s + L, s + L + K)
+    cache.repair(new, s, A)
+    lg = model.logits(cache, query)
+    ocfg, W, (odoc, onew, oq) = compact_inputs(cfg, 0, [doc, new, query], vs)
+    ref = oracle.repair(ocfg, W, oracle.prefill(ocfg, W, odoc), onew, s, A)
+    cmp_rows(cache, ref, np.arange(n), TOL["bf16"])
+    rl = oracle.logits(ocfg, W, ref, oq)[:len(vs)]
+    assert rel(lg[vs], rl) <= TOL["bf16"]
+    model.close()
