@@ -192,6 +192,16 @@ kvr_status kvr_cache_read(const kvr_cache *cache, const int32_t *positions, int3
 kvr_status kvr_model_read_tensor(const kvr_model *model, const char *name, int32_t layer,
                                  void *out, size_t bytes);
 
+/* One projection of the model through the library's GEMM kernels (the
+ * operator's a5/a7/a8 contractions, exposed for kernel tests):
+ * y[M][N] = x[M][K] . W^T, x host [M][K] in the model dtype, y host float.
+ * name "wqkv" (N = (H+2G)*dh: q, k, v rows, bias added), "wo", "wd",
+ * "lm_head", or "wgu", which returns the fused SwiGLU activation
+ * silu(x Wg^T) * (x Wu^T) [M][ffn] (rounded to the model dtype).  1 <= M <=
+ * max_rows.  Synchronous. */
+kvr_status kvr_linear(kvr_model *model, const char *name, int32_t layer, const void *x, int32_t M,
+                      float *y);
+
 /* Per-kernel-class device timing with CUDA events around each launch group.
  * enable != 0 turns it on for later calls; kvr_profile_read returns, for
  * up to `cap` classes, the accumulated milliseconds and launch counts since

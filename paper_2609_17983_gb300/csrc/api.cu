@@ -7,6 +7,7 @@
 // attention -> O GEMM (+residual) -> RMSNorm -> gate/up GEMM -> SwiGLU ->
 // down GEMM (+residual).
 #include <cmath>
+#include <cstdlib>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
@@ -115,11 +116,27 @@ kvr_status stage_h2d(kvr_model *m, int32_t *dst_dev, const int32_t *src, size_t 
 
 // ------------------------------------------------------------ GEMM dispatch
 
-kvr_status gemm(kvr_model *m, int cls, const void *X, const void *W, const float *bias, float *Y,
-                int M, int N, int K, int accumulate) {
+// Y (+)= X W^T through the tensor-core kernel when the weight has a TMA
+// descriptor, else the FFMA kernel.  epi selects the epilogue; for SwiGLU
+// the FFMA path writes gate/up to m->gu and runs the SwiGLU kernel.
+kvr_status gemm(kvr_model *m, int cls, const void *X, const void *W, const CUtensorMap *tm,
+                const float *bias, float *Y, int M, int N, int K, int epi) {
   const Dims &dm = m->dims;
   Prof pr(m, cls, (int64_t)N * K * (int64_t)dm.es());
-  GemmArgs g{X, W, bias, Y, M, N, K, K, N, dm.dtype, accumulate};
+  if (tm && m->use_tc) {
+    GemmArgs g{X, W, bias, Y, M, N, K, K, N, dm.dtype, epi == GEMM_EPI_ACCUM};
+    cudaError_t e = launch_gemm_tc(g, *tm, epi, epi == GEMM_EPI_SWIGLU ? m->act : nullptr,
+                                   N / 2, m->tcw, m->stream);
+    if (e != cudaSuccess) return fail(KVR_E_CUDA, "tensor-core GEMM: %s", cudaGetErrorString(e));
+    return launch_check(m, 1);
+  }
+  if (epi == GEMM_EPI_SWIGLU) {
+    GemmArgs g{X, W, nullptr, m->gu, M, N, K, K, N, dm.dtype, 0};
+    launch_gemm_simt(g, m->stream);
+    launch_swiglu(m->gu, M, N / 2, m->act, dm.dtype, m->stream);
+    return launch_check(m, 2);
+  }
+  GemmArgs g{X, W, bias, Y, M, N, K, K, N, dm.dtype, epi == GEMM_EPI_ACCUM};
   launch_gemm_simt(g, m->stream);
   return launch_check(m, 1);
 }
@@ -155,7 +172,8 @@ kvr_status layer_qkv(kvr_model *m, const Rows &r, int l, bool write_kv) {
   const Dims &dm = m->dims;
   const LayerW &w = m->layers[l];
   KVR_TRY(norm(m, w.attn_norm, r.M));
-  KVR_TRY(gemm(m, P_GEMM_QKV, m->a, w.wqkv, w.bqkv, m->qkv, r.M, dm.Nqkv(), dm.d, 0));
+  KVR_TRY(gemm(m, P_GEMM_QKV, m->a, w.wqkv, w.tc_qkv ? &w.tm_qkv : nullptr, w.bqkv, m->qkv, r.M,
+               dm.Nqkv(), dm.d, GEMM_EPI_STORE));
   {
     Prof pr(m, P_ROPE, (int64_t)r.M * dm.Nqkv() * 4);
     launch_rope_scatter(m->qkv, m->rope, r.pos, r.M, dm, l, r.views, r.rowdoc, r.single, m->q,
@@ -176,15 +194,13 @@ kvr_status layer_rest(kvr_model *m, const Rows &r, int l) {
                           m->stream);
     KVR_TRY(launch_check(m, 1));
   }
-  KVR_TRY(gemm(m, P_GEMM_O, m->attn, w.wo, nullptr, m->h, r.M, dm.d, dm.H * dm.dh, 1));
+  KVR_TRY(gemm(m, P_GEMM_O, m->attn, w.wo, w.tc_o ? &w.tm_o : nullptr, nullptr, m->h, r.M, dm.d,
+               dm.H * dm.dh, GEMM_EPI_ACCUM));
   KVR_TRY(norm(m, w.mlp_norm, r.M));
-  KVR_TRY(gemm(m, P_GEMM_GU, m->a, w.wgu, nullptr, m->gu, r.M, 2 * dm.F, dm.d, 0));
-  {
-    Prof pr(m, P_SWIGLU, (int64_t)r.M * dm.F * 12);
-    launch_swiglu(m->gu, r.M, dm.F, m->act, dm.dtype, m->stream);
-    KVR_TRY(launch_check(m, 1));
-  }
-  KVR_TRY(gemm(m, P_GEMM_DOWN, m->act, w.wd, nullptr, m->h, r.M, dm.d, dm.F, 1));
+  KVR_TRY(gemm(m, P_GEMM_GU, m->a, w.wgu, w.tc_gu ? &w.tm_gu : nullptr, nullptr, nullptr, r.M,
+               2 * dm.F, dm.d, GEMM_EPI_SWIGLU));
+  KVR_TRY(gemm(m, P_GEMM_DOWN, m->act, w.wd, w.tc_d ? &w.tm_d : nullptr, nullptr, m->h, r.M, dm.d,
+               dm.F, GEMM_EPI_ACCUM));
   return KVR_OK;
 }
 
@@ -208,6 +224,7 @@ kvr_status sync_model(kvr_model *m) {
   if (e != cudaSuccess) return fail(KVR_E_CUDA, "device error: %s", cudaGetErrorString(e));
   if (flag) {
     cudaMemset(m->dev_flag, 0, sizeof(int));
+    if (m->tcw.counters) cudaMemset(m->tcw.counters, 0, (size_t)m->tcw.max_tiles * sizeof(int));
     return fail(KVR_E_DEVICE_TIMEOUT, "a bounded device wait ran out (code %d)", flag);
   }
   return KVR_OK;
@@ -352,6 +369,8 @@ void kvr_model_free(kvr_model *m) {
   dev_free(m->ws_block);
   dev_free(m->rope);
   dev_free(m->dev_flag);
+  dev_free(m->tcw.partials);
+  dev_free(m->tcw.counters);
   if (m->stage_h) cudaFreeHost(m->stage_h);
   if (m->stage_ev) cudaEventDestroy(m->stage_ev);
   delete m;
@@ -552,6 +571,29 @@ kvr_status kvr_model_create(const kvr_model_config *cfg, const kvr_weights *wts,
       return bail(fail(KVR_E_NOMEM, "pinned staging"));
     cudaEventCreateWithFlags(&m->stage_ev, cudaEventDisableTiming);
     cudaEventRecord(m->stage_ev, 0);
+  }
+  // ---- tensor-core GEMM: workspace and weight TMA descriptors
+  if (dm.dtype == KVR_DTYPE_BF16) {
+    const char *env = getenv("KVR_DISABLE_TC");
+    m->use_tc = !(env && env[0] == '1');
+    m->tcw.num_sms = m->num_sms;
+    m->tcw.max_tiles = 1 << 16;
+    m->tcw.dev_flag = m->dev_flag;
+    m->tcw.partials = (float *)dev_alloc(gemm_tc_ws_bytes(m->num_sms));
+    m->tcw.counters = (int *)dev_alloc((size_t)m->tcw.max_tiles * sizeof(int));
+    if (!m->tcw.partials || !m->tcw.counters) return bail(fail(KVR_E_NOMEM, "GEMM workspace"));
+    cudaMemset(m->tcw.counters, 0, (size_t)m->tcw.max_tiles * sizeof(int));
+    auto mk = [&](CUtensorMap *tm, const void *w, int N, int K) {
+      return gemm_tc_supported(N, K) && make_tmap_bf16(tm, w, N, K, 128);
+    };
+    for (int l = 0; l < dm.L; ++l) {
+      LayerW &w = m->layers[l];
+      w.tc_qkv = mk(&w.tm_qkv, w.wqkv, dm.Nqkv(), dm.d);
+      w.tc_o = mk(&w.tm_o, w.wo, dm.d, dm.H * dm.dh);
+      w.tc_gu = mk(&w.tm_gu, w.wgu, 2 * dm.F, dm.d);
+      w.tc_d = mk(&w.tm_d, w.wd, dm.d, dm.F);
+    }
+    m->tc_lm = mk(&m->tm_lm, m->lm_head, dm.V, dm.d);
   }
   cudaError_t e = cudaDeviceSynchronize();
   if (e != cudaSuccess) return bail(fail(KVR_E_CUDA, "create: %s", cudaGetErrorString(e)));
@@ -806,7 +848,8 @@ kvr_status kvr_logits(kvr_model *m, const kvr_cache *c, const int32_t *query, in
                    dm.dtype, m->stream);
     KVR_TRY(launch_check(m, 1));
   }
-  KVR_TRY(gemm(m, P_LMHEAD, m->a, m->lm_head, nullptr, m->logits, 1, dm.V, dm.d, 0));
+  KVR_TRY(gemm(m, P_LMHEAD, m->a, m->lm_head, m->tc_lm ? &m->tm_lm : nullptr, nullptr, m->logits,
+               1, dm.V, dm.d, GEMM_EPI_STORE));
   CUDA_TRY(cudaMemcpyAsync(logits_out, m->logits, (size_t)dm.V * 4, cudaMemcpyDeviceToHost,
                            m->stream));
   return sync_model(m);
@@ -1074,6 +1117,62 @@ kvr_status kvr_model_read_tensor(const kvr_model *m, const char *name, int32_t l
     return KVR_OK;
   }
   return fail(KVR_E_INVAL, "unknown tensor '%s'", name);
+}
+
+kvr_status kvr_linear(kvr_model *m, const char *name, int32_t layer, const void *x, int32_t M,
+                      float *y) {
+  if (!m || !name || !x || !y) return fail(KVR_E_INVAL, "NULL argument");
+  const Dims &dm = m->dims;
+  if (M < 1 || M > dm.max_rows) return fail(KVR_E_RANGE, "M=%d outside [1, max_rows]", M);
+  std::string nm(name);
+  bool per_layer = nm != "lm_head";
+  if (per_layer && (layer < 0 || layer >= dm.L)) return fail(KVR_E_RANGE, "layer");
+  const LayerW *w = per_layer ? &m->layers[layer] : nullptr;
+  const void *W = nullptr;
+  const CUtensorMap *tm = nullptr;
+  const float *bias = nullptr;
+  int N = 0, K = 0, epi = GEMM_EPI_STORE, cls = P_GEMM_QKV;
+  if (nm == "wqkv") {
+    W = w->wqkv, tm = w->tc_qkv ? &w->tm_qkv : nullptr, bias = w->bqkv, N = dm.Nqkv(), K = dm.d;
+  } else if (nm == "wo") {
+    W = w->wo, tm = w->tc_o ? &w->tm_o : nullptr, N = dm.d, K = dm.H * dm.dh, cls = P_GEMM_O;
+  } else if (nm == "wd") {
+    W = w->wd, tm = w->tc_d ? &w->tm_d : nullptr, N = dm.d, K = dm.F, cls = P_GEMM_DOWN;
+  } else if (nm == "wgu") {
+    W = w->wgu, tm = w->tc_gu ? &w->tm_gu : nullptr, N = 2 * dm.F, K = dm.d;
+    epi = GEMM_EPI_SWIGLU, cls = P_GEMM_GU;
+  } else if (nm == "lm_head") {
+    W = m->lm_head, tm = m->tc_lm ? &m->tm_lm : nullptr, N = dm.V, K = dm.d, cls = P_LMHEAD;
+  } else {
+    return fail(KVR_E_INVAL, "unknown projection '%s'", name);
+  }
+  KVR_TRY(use_device(m));
+  size_t es = dm.es(), xb = (size_t)M * K * es;
+  size_t yn = epi == GEMM_EPI_SWIGLU ? (size_t)M * dm.F : (size_t)M * N;
+  void *xd = dev_alloc(xb);
+  float *yd = (float *)dev_alloc(yn * 4);
+  kvr_status st = KVR_OK;
+  if (!xd || !yd) st = fail(KVR_E_NOMEM, "linear buffers");
+  if (!st && cudaMemcpyAsync(xd, x, xb, cudaMemcpyHostToDevice, m->stream))
+    st = fail(KVR_E_CUDA, "x upload");
+  if (!st) st = gemm(m, cls, xd, W, tm, bias, yd, M, N, K, epi);
+  if (!st && epi == GEMM_EPI_SWIGLU) {
+    // act is in the model dtype: widen on the host
+    std::vector<uint8_t> tmp(yn * es);
+    if (cudaMemcpyAsync(tmp.data(), m->act, yn * es, cudaMemcpyDeviceToHost, m->stream) ||
+        cudaStreamSynchronize(m->stream))
+      st = fail(KVR_E_CUDA, "readback");
+    for (size_t i = 0; !st && i < yn; ++i)
+      y[i] = es == 2 ? bf16_bits_to_f32(((uint16_t *)tmp.data())[i]) : ((float *)tmp.data())[i];
+  } else if (!st) {
+    if (cudaMemcpyAsync(y, yd, yn * 4, cudaMemcpyDeviceToHost, m->stream))
+      st = fail(KVR_E_CUDA, "readback");
+  }
+  if (!st) st = sync_model(m);
+  cudaStreamSynchronize(m->stream);
+  dev_free(xd);
+  dev_free(yd);
+  return st;
 }
 
 kvr_status kvr_profile_enable(kvr_model *m, int32_t enable) {

@@ -1,0 +1,495 @@
+// k_gemm_tc.cu -- bf16 tensor-core GEMM for sm_103a: tcgen05.mma with TMEM
+// accumulators, operands staged by TMA into 128B-swizzled shared memory.
+//
+//   Y[M][N] (+)= X[M][K] . W[N][K]^T     (bf16 operands, fp32 accumulate)
+//
+// Swap-AB: the weight W is the MMA's A operand (128 output features per tile
+// = UMMA M), the M activation rows are its N dimension (BN <= 256 per tile),
+// so a repair pass of ~40 rows still runs 128-row tensor-core tiles and the
+// kernel streams W once from HBM.
+//
+// Work decomposition: persistent stream-K.  The units (feature tile, token
+// tile, 64-wide K block) are linearised feature-tile-major and split into
+// `grid` contiguous, equal ranges, one per CTA (grid <= #SMs), so every SM
+// streams the same number of weight bytes whatever the GEMM shape.  A tile
+// covered by several CTAs is reduced by the last CTA to finish it (atomic
+// arrival counter): each part is written to a per-CTA fp32 slot and the last
+// arriver sums the parts in CTA order, so the result is deterministic.  No CTA
+// ever waits for another.
+//
+// Warp roles (192 threads): warp 0 issues TMA loads (one elected lane), warp 1
+// issues tcgen05.mma (one elected lane), warps 2-5 drain TMEM and run the
+// epilogue.  Accumulators are double-buffered in TMEM so the MMA warp starts
+// the next segment while the epilogue drains the previous one.
+//
+// Every mbarrier wait is bounded: a wait that runs out sets the device error
+// flag and an abort flag in shared memory; all roles then stop issuing work,
+// wait (bounded) for their copies and MMAs in flight, free TMEM and return.
+#include <cuda.h>
+
+#include "kvr_internal.cuh"
+
+namespace kvr {
+namespace {
+
+constexpr int BM = 128;             // output features per tile (UMMA M)
+constexpr int BK = 64;              // K per stage: one 128-byte swizzle atom of bf16
+constexpr int UK = 16;              // K per tcgen05.mma kind::f16
+constexpr int NTHREADS = 192;
+constexpr uint64_t WAIT_NS = 2000000000ull;  // a wait longer than 2 s is a fault
+constexpr int A_BYTES = BM * BK * 2;  // 16 KB
+
+struct TcParams {
+  int M, N, K;
+  int BN, n_tiles, m_tiles, KB;
+  long long total;
+  int grid, stages;
+  uint32_t tmem_cols;  // columns of one accumulator buffer
+  float *Y;
+  int ldy;
+  const float *bias;
+  int epi;
+  void *out2;  // SwiGLU output (bf16 [M][N/2])
+  int ld2;
+  float *ws;        // [grid][2][BN][128] fp32 partial tiles
+  int *counters;    // [n_tiles * m_tiles] arrival counters (self-resetting)
+  int *dev_flag;
+};
+
+// ------------------------------------------------------------ PTX wrappers
+
+__device__ __forceinline__ uint32_t su32(const void *p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t *b, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(su32(b)), "r"(count));
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint64_t *b, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(su32(b)),
+               "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t *b) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(b)) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try(uint64_t *b, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(su32(b)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+__device__ __forceinline__ uint64_t gtime_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+// Bounded wait for the phase of parity `parity` to complete.  Gives up after
+// WAIT_NS (setting the abort flag and dev_flag |= code), or as soon as another
+// role has aborted when honor_abort is set.
+__device__ __forceinline__ bool mbar_wait(uint64_t *b, uint32_t parity, volatile int *abort_f,
+                                          int *dev_flag, int code, bool honor_abort = true) {
+  if (mbar_try(b, parity)) return true;
+  uint64_t t0 = gtime_ns();
+  for (uint32_t it = 0;; ++it) {
+    if (mbar_try(b, parity)) return true;
+    if ((it & 63) == 63) {
+      if (honor_abort && *abort_f) return false;
+      if (gtime_ns() - t0 > WAIT_NS) {
+        *abort_f = 1;
+        atomicOr(dev_flag, code ? code : 16);
+        return false;
+      }
+    }
+  }
+}
+
+__device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, uint64_t *bar,
+                                            int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3}], [%4];" ::"r"(su32(dst)),
+      "l"((uint64_t)map), "r"(x), "r"(y), "r"(su32(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap *map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)map) : "memory");
+}
+
+// Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, rows of
+// 128 bytes, 8-row swizzle atoms 1024 bytes apart (SBO).
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  uint64_t d = (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)1 << 16;             // leading-dimension byte offset (unused here)
+  d |= (uint64_t)(1024 >> 4) << 32;   // stride-dimension byte offset
+  d |= (uint64_t)1 << 46;             // descriptor version
+  d |= (uint64_t)2 << 61;             // 128-byte swizzle
+  return d;
+}
+
+// Instruction descriptor, kind::f16: bf16 A and B (K-major), fp32 D, M x N.
+__device__ __forceinline__ uint32_t idesc_bf16(int m, int n) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) |
+         ((uint32_t)(m >> 4) << 24);
+}
+
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
+                                         uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+__device__ __forceinline__ void mma_commit(uint64_t *bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+          su32(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float *v) {
+  uint32_t r[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+      "%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+        "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+__device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+
+// ------------------------------------------------------------ work split
+
+__device__ __forceinline__ long long range_start(long long i, long long total, int grid) {
+  return i * total / grid;
+}
+// CTA whose range holds unit u
+__device__ __forceinline__ int cta_of(long long u, long long total, int grid) {
+  return (int)(((u + 1) * grid - 1) / total);
+}
+
+// Epilogue for output element (row t of X / Y, feature n of W), all lanes of
+// the warp call it together (SwiGLU exchanges lanes).
+__device__ __forceinline__ void epilogue(const TcParams &p, int t, int n, float v, bool valid) {
+  if (p.epi == GEMM_EPI_SWIGLU) {
+    // rows 32b..32b+15 are gate, 32b+16..32b+31 up of features 16b..16b+15;
+    // lane = n % 32
+    float u = __shfl_down_sync(0xffffffffu, v, 16);
+    int r = n & 31;
+    if (valid && r < 16) {
+      float g = v;
+      float a = g / (1.0f + expf(-g)) * u;
+      ((__nv_bfloat16 *)p.out2)[(size_t)t * p.ld2 + (n >> 5) * 16 + r] = __float2bfloat16_rn(a);
+    }
+    return;
+  }
+  if (!valid) return;
+  float *y = p.Y + (size_t)t * p.ldy + n;
+  if (p.epi == GEMM_EPI_ACCUM)
+    *y += v;
+  else
+    *y = v + (p.bias ? p.bias[n] : 0.f);
+}
+
+__global__ void __launch_bounds__(NTHREADS, 1)
+    k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX,
+              const TcParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t full_bar[8], empty_bar[8], accf_bar[2], acce_bar[2],
+      drain_bar;
+  __shared__ uint32_t tmem_slot;
+  __shared__ int abort_f;
+  __shared__ int last_f;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int S = p.stages;
+  const uint32_t base = (su32(smem_raw) + 1023u) & ~1023u;
+  const uint32_t stage_bytes = A_BYTES + (uint32_t)p.BN * 128u;
+  const long long u0 = range_start(blockIdx.x, p.total, p.grid);
+  const long long u1 = range_start(blockIdx.x + 1, p.total, p.grid);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(&full_bar[s], 1);
+      mbar_init(&empty_bar[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&accf_bar[b], 1);
+      mbar_init(&acce_bar[b], 128);
+    }
+    mbar_init(&drain_bar, 1);
+    abort_f = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 0) {
+    if (lane == 0) {
+      tma_prefetch_desc(&tmW);
+      tma_prefetch_desc(&tmX);
+    }
+    __syncwarp();
+    uint32_t ncols = 2 * p.tmem_cols;
+    asm volatile(
+        "tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+            su32(&tmem_slot)),
+        "r"(ncols)
+        : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = tmem_slot;
+  volatile int *abort_v = &abort_f;
+
+  if (warp == 0) {
+    // ---------------------------------------------------------------- TMA
+    if (lane == 0) {
+      uint32_t it = 0;
+      for (long long u = u0; u < u1; ++u) {
+        int s = (int)(it % S);
+        uint32_t ph = (it / S) & 1u;
+        if (!mbar_wait(&empty_bar[s], ph ^ 1u, abort_v, p.dev_flag, 1)) break;
+        long long tl = u / p.KB;
+        int kb = (int)(u % p.KB);
+        int ntile = (int)(tl / p.m_tiles), mtile = (int)(tl % p.m_tiles);
+        uint32_t sa = base + (uint32_t)s * stage_bytes;
+        mbar_expect_tx(&full_bar[s], stage_bytes);
+        tma_load_2d((void *)__cvta_shared_to_generic(sa), &tmW, &full_bar[s], kb * BK,
+                    ntile * BM);
+        tma_load_2d((void *)__cvta_shared_to_generic(sa + A_BYTES), &tmX, &full_bar[s],
+                    kb * BK, mtile * p.BN);
+        ++it;
+      }
+      // copies in flight complete before the CTA may exit
+      uint32_t n_issued = it;
+      for (uint32_t j = n_issued > (uint32_t)S ? n_issued - S : 0; j < n_issued; ++j)
+        mbar_wait(&full_bar[j % S], (j / S) & 1u, abort_v, p.dev_flag, 0, false);
+    }
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- MMA
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16(BM, p.BN);
+      uint32_t it = 0, seg = 0;
+      bool ok = true;
+      for (long long a = u0; a < u1 && ok;) {
+        long long tl = a / p.KB;
+        long long b = (tl + 1) * p.KB < u1 ? (tl + 1) * p.KB : u1;
+        uint32_t buf = seg & 1u, use = seg >> 1;
+        if (!mbar_wait(&acce_bar[buf], (use & 1u) ^ 1u, abort_v, p.dev_flag, 2)) break;
+        tc_fence_after();
+        uint32_t d = tmem_base + buf * p.tmem_cols;
+        for (long long u = a; u < b; ++u) {
+          int s = (int)(it % S);
+          uint32_t ph = (it / S) & 1u;
+          if (!mbar_wait(&full_bar[s], ph, abort_v, p.dev_flag, 4)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          uint32_t sa = base + (uint32_t)s * stage_bytes;
+          uint64_t da = sw128_desc(sa), db = sw128_desc(sa + A_BYTES);
+#pragma unroll
+          for (int k = 0; k < BK / UK; ++k)
+            mma_bf16(d, da + (uint64_t)(k * UK * 2 / 16), db + (uint64_t)(k * UK * 2 / 16), idesc,
+                     (u > a || k > 0) ? 1u : 0u);
+          mma_commit(&empty_bar[s]);
+          ++it;
+        }
+        if (ok) mma_commit(&accf_bar[buf]);
+        ++seg;
+        a = b;
+      }
+      // all MMAs issued by this thread complete before TMEM is freed
+      mma_commit(&drain_bar);
+      mbar_wait(&drain_bar, 0, abort_v, p.dev_flag, 0, false);
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int q = warp & 3;  // TMEM lane quarter of this warp
+    const int f = q * 32 + lane;
+    const int et = threadIdx.x - 64;  // 0..127
+    uint32_t seg = 0;
+    for (long long a = u0; a < u1;) {
+      long long tl = a / p.KB;
+      long long b = (tl + 1) * p.KB < u1 ? (tl + 1) * p.KB : u1;
+      uint32_t buf = seg & 1u, use = seg >> 1;
+      if (!mbar_wait(&accf_bar[buf], use & 1u, abort_v, p.dev_flag, 8)) break;
+      tc_fence_after();
+      int ntile = (int)(tl / p.m_tiles), mtile = (int)(tl % p.m_tiles);
+      int t0 = mtile * p.BN;
+      int mv = min(p.BN, p.M - t0);
+      int n = ntile * BM + f;
+      long long tile_u0 = tl * p.KB;
+      int i_first = cta_of(tile_u0, p.total, p.grid);
+      int i_last = cta_of(tile_u0 + p.KB - 1, p.total, p.grid);
+      int parts = i_last - i_first + 1;
+      uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + buf * p.tmem_cols;
+      if (parts == 1) {
+        for (int c = 0; c < mv; c += 16) {
+          float v[16];
+          tmem_ld16(taddr + c, v);
+#pragma unroll
+          for (int j = 0; j < 16; ++j) epilogue(p, t0 + c + j, n, v[j], c + j < mv);
+        }
+      } else {
+        int slot = range_start(blockIdx.x, p.total, p.grid) >= tile_u0 ? 0 : 1;
+        float *w = p.ws + ((size_t)blockIdx.x * 2 + slot) * p.BN * BM;
+        for (int c = 0; c < mv; c += 16) {
+          float v[16];
+          tmem_ld16(taddr + c, v);
+#pragma unroll
+          for (int j = 0; j < 16; ++j)
+            if (c + j < mv) w[(size_t)(c + j) * BM + f] = v[j];
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(&acce_bar[buf]);
+      if (parts > 1) {
+        __threadfence();
+        epi_bar();
+        if (et == 0) last_f = atomicAdd(&p.counters[tl], 1) == parts - 1;
+        epi_bar();
+        if (last_f) {
+          __threadfence();
+          for (int t = 0; t < mv; ++t) {
+            float v = 0.f;
+            for (int i = i_first; i <= i_last; ++i) {
+              int sl = range_start(i, p.total, p.grid) >= tile_u0 ? 0 : 1;
+              v += __ldcg(p.ws + (((size_t)i * 2 + sl) * p.BN + t) * BM + f);
+            }
+            epilogue(p, t0 + t, n, v, true);
+          }
+          if (et == 0) p.counters[tl] = 0;
+        }
+        epi_bar();
+      }
+      ++seg;
+      a = b;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 0) {
+    uint32_t ncols = 2 * p.tmem_cols;
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
+                 "r"(ncols)
+                 : "memory");
+  }
+}
+
+// ------------------------------------------------------------ host side
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                                  const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                                  const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    cudaDriverEntryPointQueryResult q;
+    void *f = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = (EncodeTiledFn)f;
+  }
+  return fn;
+}
+
+}  // namespace
+
+bool make_tmap_bf16(CUtensorMap *map, const void *ptr, int rows, int cols, int box_rows) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn || ((uintptr_t)ptr & 15) || (cols * 2) % 16 || box_rows > 256 || box_rows < 1)
+    return false;
+  cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
+  cuuint32_t box[2] = {BK, (cuuint32_t)box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), dims,
+                  strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+bool gemm_tc_supported(int N, int K) { return N % BM == 0 && K % BK == 0 && N > 0 && K > 0; }
+
+int gemm_tc_bn(int M) {
+  if (M > 256) return 256;
+  int bn = (M + 15) / 16 * 16;
+  return bn < 16 ? 16 : bn;
+}
+
+size_t gemm_tc_ws_bytes(int num_sms) { return (size_t)num_sms * 2 * 256 * BM * sizeof(float); }
+
+cudaError_t launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, void *out2,
+                           int ld2, const TcWorkspace &ws, cudaStream_t s) {
+  if (g.M <= 0) return cudaSuccess;
+  TcParams p{};
+  p.M = g.M;
+  p.N = g.N;
+  p.K = g.K;
+  p.BN = gemm_tc_bn(g.M);
+  p.n_tiles = g.N / BM;
+  p.m_tiles = (g.M + p.BN - 1) / p.BN;
+  p.KB = g.K / BK;
+  p.total = (long long)p.n_tiles * p.m_tiles * p.KB;
+  p.grid = (int)(p.total < ws.num_sms ? p.total : ws.num_sms);
+  uint32_t stage_bytes = A_BYTES + (uint32_t)p.BN * 128u;
+  int smem_budget = 227 * 1024 - 1024 - 256;
+  p.stages = smem_budget / (int)stage_bytes;
+  if (p.stages > 8) p.stages = 8;
+  if (p.stages < 2) return cudaErrorInvalidValue;
+  uint32_t cols = 32;
+  while (cols < (uint32_t)p.BN) cols <<= 1;
+  p.tmem_cols = cols;
+  p.Y = g.Y;
+  p.ldy = g.ldy;
+  p.bias = g.bias;
+  p.epi = epi;
+  p.out2 = out2;
+  p.ld2 = ld2;
+  p.ws = ws.partials;
+  p.counters = ws.counters;
+  p.dev_flag = ws.dev_flag;
+  if ((long long)p.n_tiles * p.m_tiles > ws.max_tiles) return cudaErrorInvalidValue;
+  CUtensorMap tmX;
+  if (!make_tmap_bf16(&tmX, g.X, g.M, g.K, p.BN)) return cudaErrorInvalidValue;
+  size_t smem = 1024 + (size_t)p.stages * stage_bytes;
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaFuncSetAttribute(k_gemm_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
+    attr_set = true;
+  }
+  k_gemm_tc<<<p.grid, NTHREADS, smem, s>>>(tmW, tmX, p);
+  return cudaGetLastError();
+}
+
+}  // namespace kvr

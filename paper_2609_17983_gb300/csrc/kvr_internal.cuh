@@ -19,6 +19,7 @@
 //            attention output [R][H*dh], gate/up fp32 [R][2F], act [R][F].
 #pragma once
 
+#include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -48,6 +49,9 @@ struct Dims {
 struct LayerW {
   void *wqkv, *wo, *wgu, *wd;
   float *bqkv, *attn_norm, *mlp_norm;
+  // TMA descriptors of the weights (bf16 models, tensor-core GEMM shapes)
+  CUtensorMap tm_qkv, tm_o, tm_gu, tm_d;
+  bool tc_qkv, tc_o, tc_gu, tc_d;
 };
 
 // Device view of one document's paged cache (passed by value to kernels).
@@ -61,7 +65,16 @@ struct KVView {
   }
 };
 
-// Internal error state of one kernel-class timer.
+// Scratch of the tensor-core GEMM (split-tile partials, arrival counters).
+struct TcWorkspace {
+  float *partials;  // gemm_tc_ws_bytes(num_sms)
+  int *counters;    // max_tiles zeroed ints
+  int *dev_flag;
+  int num_sms;
+  long long max_tiles;
+};
+
+// Accumulated device time of one kernel class.
 struct ProfClass {
   std::string name;
   double ms = 0;
@@ -79,6 +92,10 @@ struct kvr_model {
   float *final_norm = nullptr;
   std::vector<kvr::LayerW> layers;
   float2 *rope = nullptr;  // [max_ctx + reserve][dh/2] (cos, sin), fp32 from fp64 angles
+  CUtensorMap tm_lm;
+  bool tc_lm = false;
+  kvr::TcWorkspace tcw{};
+  bool use_tc = true;  // tensor-core GEMM for bf16 shapes it takes
   cudaStream_t stream = nullptr;
   int device = 0;
   int num_sms = 0;
@@ -164,6 +181,17 @@ struct GemmArgs {
   int accumulate;  // 1: Y += result
 };
 void launch_gemm_simt(const GemmArgs &g, cudaStream_t s);
+
+// Tensor-core GEMM (bf16, N % 128 == 0, K % 64 == 0).  Epilogues:
+enum { GEMM_EPI_STORE = 0, GEMM_EPI_ACCUM = 1, GEMM_EPI_SWIGLU = 2 };
+bool make_tmap_bf16(CUtensorMap *map, const void *ptr, int rows, int cols, int box_rows);
+bool gemm_tc_supported(int N, int K);
+int gemm_tc_bn(int M);
+size_t gemm_tc_ws_bytes(int num_sms);
+// GEMM_EPI_SWIGLU: W rows interleaved gate/up in blocks of 16; writes
+// out2[t][f] = bf16(silu(gate) * up), f < N/2, row stride ld2.
+cudaError_t launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, void *out2,
+                           int ld2, const TcWorkspace &ws, cudaStream_t s);
 
 // ---- kernels: attention ----
 // o[i] = softmax(q_i K[0..pos_i]^T / sqrt(dh)) V[0..pos_i] for every row i,

@@ -86,6 +86,7 @@ _sigs = {
     "kvr_profile_reset": ([_P], _I32),
     "kvr_profile_read": ([_P, _I32, _P, _P, _P, _P, _I32, _P], _I32),
     "kvr_launch_count": ([_P], ctypes.c_int64),
+    "kvr_linear": ([_P, ctypes.c_char_p, _I32, _P, _I32, _P], _I32),
 }
 for _name, (_args, _res) in _sigs.items():
     _f = getattr(_lib, _name)
@@ -237,6 +238,14 @@ def kvr_model_read_tensor(model, name: str, layer: int, shape, dtype) -> np.ndar
     out = np.zeros(shape, dtype)
     _check(_lib.kvr_model_read_tensor(model, name.encode(), layer, out.ctypes.data, out.nbytes))
     return out
+
+
+def kvr_linear(model, name: str, layer: int, x: np.ndarray, n_out: int) -> np.ndarray:
+    x = np.ascontiguousarray(x)
+    y = np.zeros((x.shape[0], n_out), np.float32)
+    _check(_lib.kvr_linear(model, name.encode(), layer, x.ctypes.data, x.shape[0],
+                           y.ctypes.data))
+    return y
 
 
 def kvr_profile_enable(model, enable: bool = True):
