@@ -125,9 +125,9 @@ kvr_status gemm(kvr_model *m, int cls, const void *X, const void *W, const CUten
   Prof pr(m, cls, (int64_t)N * K * (int64_t)dm.es());
   if (tm && m->use_tc) {
     GemmArgs g{X, W, bias, Y, M, N, K, K, N, dm.dtype, epi == GEMM_EPI_ACCUM};
-    cudaError_t e = launch_gemm_tc(g, *tm, epi, epi == GEMM_EPI_SWIGLU ? m->act : nullptr,
+    const char *e = launch_gemm_tc(g, *tm, epi, epi == GEMM_EPI_SWIGLU ? m->act : nullptr,
                                    N / 2, m->tcw, m->stream);
-    if (e != cudaSuccess) return fail(KVR_E_CUDA, "tensor-core GEMM: %s", cudaGetErrorString(e));
+    if (e) return fail(KVR_E_CUDA, "tensor-core GEMM (M=%d N=%d K=%d): %s", M, N, K, e);
     return launch_check(m, 1);
   }
   if (epi == GEMM_EPI_SWIGLU) {
@@ -891,6 +891,7 @@ kvr_status kvr_select(kvr_model *m, const kvr_cache *c, kvr_policy policy, int32
     Prof pr(m, P_SELECT, 0);
     launch_scores_simple(policy, toks, n, s_end, dm.delim, seed, m->keys, m->stream);
     st = launch_check(m, 1);
+    if (st) st = fail(KVR_E_CUDA, "selector scores: %s", kvr_last_error());
     if (policy == KVR_POLICY_STRUCTURAL) topk_k = -K;
   } else if (!st && policy == KVR_POLICY_ATTENTION) {
     if (edit_len == 0) {
@@ -1001,8 +1002,8 @@ kvr_status kvr_select(kvr_model *m, const kvr_cache *c, kvr_policy policy, int32
   }
   if (!st) {
     Prof pr(m, P_SELECT, 0);
-    launch_topk(m->keys, n, s_end, topk_k, m->sel_out, m->sel_count, m->stream);
-    st = launch_check(m, 1);
+    const char *e = launch_topk(m->keys, n, s_end, topk_k, m->sel_out, m->sel_count, m->stream);
+    st = e ? fail(KVR_E_CUDA, "top-K over %d candidates: %s", n - s_end, e) : launch_check(m, 1);
   }
   int32_t cnt = 0;
   if (!st && (cudaMemcpyAsync(&cnt, m->sel_count, 4, cudaMemcpyDeviceToHost, m->stream) ||

@@ -42,6 +42,7 @@ constexpr int A_BYTES = BM * BK * 2;  // 16 KB
 struct TcParams {
   int M, N, K;
   int BN, n_tiles, m_tiles, KB;
+  int brows;  // rows of the activation TMA box: min(BN, M)
   long long total;
   int grid, stages;
   uint32_t tmem_cols;  // columns of one accumulator buffer
@@ -230,6 +231,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
   const int S = p.stages;
   const uint32_t base = (su32(smem_raw) + 1023u) & ~1023u;
   const uint32_t stage_bytes = A_BYTES + (uint32_t)p.BN * 128u;
+  const uint32_t tx_bytes = A_BYTES + (uint32_t)p.brows * 128u;
   const long long u0 = range_start(blockIdx.x, p.total, p.grid);
   const long long u1 = range_start(blockIdx.x + 1, p.total, p.grid);
 
@@ -278,7 +280,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         int kb = (int)(u % p.KB);
         int ntile = (int)(tl / p.m_tiles), mtile = (int)(tl % p.m_tiles);
         uint32_t sa = base + (uint32_t)s * stage_bytes;
-        mbar_expect_tx(&full_bar[s], stage_bytes);
+        mbar_expect_tx(&full_bar[s], tx_bytes);
         tma_load_2d((void *)__cvta_shared_to_generic(sa), &tmW, &full_bar[s], kb * BK,
                     ntile * BM);
         tma_load_2d((void *)__cvta_shared_to_generic(sa + A_BYTES), &tmX, &full_bar[s],
@@ -449,9 +451,9 @@ int gemm_tc_bn(int M) {
 
 size_t gemm_tc_ws_bytes(int num_sms) { return (size_t)num_sms * 2 * 256 * BM * sizeof(float); }
 
-cudaError_t launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, void *out2,
+const char *launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, void *out2,
                            int ld2, const TcWorkspace &ws, cudaStream_t s) {
-  if (g.M <= 0) return cudaSuccess;
+  if (g.M <= 0) return nullptr;
   TcParams p{};
   p.M = g.M;
   p.N = g.N;
@@ -460,13 +462,31 @@ cudaError_t launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, v
   p.n_tiles = g.N / BM;
   p.m_tiles = (g.M + p.BN - 1) / p.BN;
   p.KB = g.K / BK;
+  // A box may not be taller than the tensor: a single short token tile loads
+  // just its M rows (the MMA's extra columns are never stored).
+  p.brows = p.BN < g.M ? p.BN : g.M;
   p.total = (long long)p.n_tiles * p.m_tiles * p.KB;
   p.grid = (int)(p.total < ws.num_sms ? p.total : ws.num_sms);
+  // dynamic shared memory allowed for this kernel (opt-in limit minus static)
+  static int max_dyn = -1;
+  if (max_dyn < 0) {
+    int dev = 0, optin = 0;
+    cudaFuncAttributes fa{};
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+    if (cudaFuncGetAttributes(&fa, k_gemm_tc) != cudaSuccess) return "kernel attributes";
+    max_dyn = optin - (int)fa.sharedSizeBytes;
+    if (cudaFuncSetAttribute(k_gemm_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, max_dyn) !=
+        cudaSuccess) {
+      max_dyn = -1;
+      return "cannot raise the dynamic shared memory limit";
+    }
+  }
   uint32_t stage_bytes = A_BYTES + (uint32_t)p.BN * 128u;
-  int smem_budget = 227 * 1024 - 1024 - 256;
+  int smem_budget = max_dyn - 1024;
   p.stages = smem_budget / (int)stage_bytes;
   if (p.stages > 8) p.stages = 8;
-  if (p.stages < 2) return cudaErrorInvalidValue;
+  if (p.stages < 2) return "token tile too large for shared memory";
   uint32_t cols = 32;
   while (cols < (uint32_t)p.BN) cols <<= 1;
   p.tmem_cols = cols;
@@ -479,17 +499,13 @@ cudaError_t launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, v
   p.ws = ws.partials;
   p.counters = ws.counters;
   p.dev_flag = ws.dev_flag;
-  if ((long long)p.n_tiles * p.m_tiles > ws.max_tiles) return cudaErrorInvalidValue;
+  if ((long long)p.n_tiles * p.m_tiles > ws.max_tiles) return "more tiles than counters";
   CUtensorMap tmX;
-  if (!make_tmap_bf16(&tmX, g.X, g.M, g.K, p.BN)) return cudaErrorInvalidValue;
+  if (!make_tmap_bf16(&tmX, g.X, g.M, g.K, p.brows)) return "activation TMA descriptor rejected";
   size_t smem = 1024 + (size_t)p.stages * stage_bytes;
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaFuncSetAttribute(k_gemm_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
-    attr_set = true;
-  }
   k_gemm_tc<<<p.grid, NTHREADS, smem, s>>>(tmW, tmX, p);
-  return cudaGetLastError();
+  cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? nullptr : cudaGetErrorString(e);
 }
 
 }  // namespace kvr

@@ -282,8 +282,9 @@ void launch_float_keys(const float *scores, int n, int s_end, unsigned long long
 
 // Top-K over c = n - s_end candidates (c <= 16384).  nonzero_only is
 // encoded in the sign of K: K < 0 means "only nonzero keys are eligible".
-void launch_topk(const unsigned long long *keys, int n, int s_end, int K, int32_t *out,
-                 int32_t *count, cudaStream_t s) {
+// Returns nullptr on success, else what failed.
+const char *launch_topk(const unsigned long long *keys, int n, int s_end, int K, int32_t *out,
+                        int32_t *count, cudaStream_t s) {
   int c = n - s_end;
   int nonzero_only = K < 0 ? 1 : 0;
   if (K < 0) K = -K;
@@ -291,8 +292,14 @@ void launch_topk(const unsigned long long *keys, int n, int s_end, int K, int32_
   int P = 1;
   while (P < c) P <<= 1;
   size_t smem = (size_t)P * (sizeof(unsigned long long) + sizeof(int));
-  cudaFuncSetAttribute(k_topk, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (smem >= 32 * 1024) {  // the default 48 KB limit also covers static shared memory
+    cudaError_t e = cudaFuncSetAttribute(k_topk, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return cudaGetErrorString(e);
+  }
   k_topk<<<1, 1024, smem, s>>>(keys, c, s_end, K, nonzero_only, out, count);
+  cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? nullptr : cudaGetErrorString(e);
 }
 
 void launch_attn_select_scores(const float *q, int S, const Dims &dm, int layer, KVView v,

@@ -190,7 +190,8 @@ int gemm_tc_bn(int M);
 size_t gemm_tc_ws_bytes(int num_sms);
 // GEMM_EPI_SWIGLU: W rows interleaved gate/up in blocks of 16; writes
 // out2[t][f] = bf16(silu(gate) * up), f < N/2, row stride ld2.
-cudaError_t launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, void *out2,
+// Returns nullptr on success, else what went wrong.
+const char *launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, void *out2,
                            int ld2, const TcWorkspace &ws, cudaStream_t s);
 
 // ---- kernels: attention ----
@@ -209,7 +210,7 @@ void launch_kv_deviation(const float *qkv, const float2 *rope, const int32_t *po
                          const Dims &dm, KVView v, float *scores, cudaStream_t s);
 void launch_float_keys(const float *scores, int n, int s_end, unsigned long long *keys,
                        cudaStream_t s);
-void launch_topk(const unsigned long long *keys, int n, int s_end, int K, int32_t *out,
-                 int32_t *count, cudaStream_t s);
+const char *launch_topk(const unsigned long long *keys, int n, int s_end, int K, int32_t *out,
+                        int32_t *count, cudaStream_t s);
 
 }  // namespace kvr

@@ -326,3 +326,23 @@ def test_8b_shape_two_layer_parity(shape):
     rl = oracle.logits(ocfg, W, ref, oq)[:len(vs)]
     assert rel(lg[vs], rl) <= TOL["bf16"]
     model.close()
+
+
+@pytest.mark.parametrize("n", [5000, 8192])
+def test_select_long_context_exact(n):
+    # the top-K at the largest pools (up to max_context candidates)
+    cfg = synth.preset("tiny")
+    W = synth.weights(cfg, 0)
+    model = kv.Model(cfg, W, max_context=8192, max_rows=4096)
+    doc = synth.document(7, n, cfg["vocab"], cfg["delim_id"], delim_gap=(40, 80))
+    cache = model.prefill(doc)
+    s = n // 2
+    new = synth.edit_tokens(8, doc[s:s + 8], cfg["vocab"], cfg["delim_id"])
+    ref_cache = oracle.empty_cache(cfg, n)
+    ref_cache.tokens[:] = doc
+    for policy, K, seed in [("editlocal", 32, 0), ("structural", 32, 0), ("random", 64, 2),
+                            ("editlocal", n, 0)]:
+        got = model.select(cache, policy, K, s, new, seed)
+        ref = oracle.select(cfg, W, ref_cache, policy, K, s, new, seed)
+        assert got.tolist() == ref.tolist(), policy
+    model.close()
