@@ -174,11 +174,15 @@ def main():
     ap.add_argument("--prefill-steps", type=int, default=3)
     ap.add_argument("--oracle-layers", type=int, default=4)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--layers", type=int, default=None,
+                    help="decoder layers (default: the model's 32); fewer only for profiling")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
 
     from paper_2609_17983_gb300 import synth
     cfg = synth.preset(WORKLOAD)
+    if args.layers:
+        cfg["n_layers"] = args.layers
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
 

@@ -152,7 +152,44 @@ struct Rows {
   const KVView *views = nullptr;             // device [docs] (batch)
   KVView single{};
   int max_pos = 0;                           // largest position among the rows
+  const int4 *blocks = nullptr;              // attention query blocks (device)
+  int n_blocks = 0, n_splits = 1;
 };
+
+bool use_tc_attention(const kvr_model *m) {
+  return m->dims.dtype == KVR_DTYPE_BF16 && (m->dims.dh == 64 || m->dims.dh == 128);
+}
+
+// Query blocks for the tensor-core attention: consecutive rows of one
+// document (rows of a document are in ascending position order), at most
+// rows_per_block rows; and a key split count giving about two CTAs per SM.
+kvr_status plan_attention(kvr_model *m, Rows &r, const int32_t *pos, const int32_t *rowdoc) {
+  if (!use_tc_attention(m) || r.M <= 0) return KVR_OK;
+  const Dims &dm = m->dims;
+  const int qb = attn_tc_rows_per_block(dm.H / dm.G);
+  std::vector<int32_t> b;
+  int max_chunks = 0;
+  for (int i = 0; i < r.M;) {
+    int doc = rowdoc ? rowdoc[i] : 0;
+    int j = i;
+    while (j < r.M && j - i < qb && (rowdoc ? rowdoc[j] : 0) == doc) ++j;
+    int kmax = pos[j - 1];
+    b.insert(b.end(), {i, j - i, kmax, doc});
+    max_chunks = std::max(max_chunks, kmax / KVR_PAGE + 1);
+    i = j;
+  }
+  int nb = (int)b.size() / 4;
+  if (nb > m->max_blocks) return fail(KVR_E_UNSUPPORTED, "too many attention blocks (%d)", nb);
+  int target = 2 * m->num_sms;
+  int splits = std::max(1, (target + nb * dm.G - 1) / (nb * dm.G));
+  splits = std::min(splits, max_chunks);
+  while (splits > 1 && attn_tc_ws_floats(splits, nb, dm.G, dm.dh) > m->attn_ws_floats) --splits;
+  KVR_TRY(stage_h2d(m, (int32_t *)m->blocks_d, b.data(), b.size()));
+  r.blocks = m->blocks_d;
+  r.n_blocks = nb;
+  r.n_splits = splits;
+  return KVR_OK;
+}
 
 kvr_status embed(kvr_model *m, const Rows &r) {
   Prof pr(m, P_EMBED, (int64_t)r.M * m->dims.d * (int64_t)m->dims.es());
@@ -190,9 +227,17 @@ kvr_status layer_rest(kvr_model *m, const Rows &r, int l) {
   {
     int64_t kv_bytes = (int64_t)(r.max_pos + 1) * dm.G * dm.dh * 2 * (int64_t)dm.es();
     Prof pr(m, P_ATTN, kv_bytes);
-    launch_attention_simt(m->q, r.pos, r.M, dm, l, r.views, r.rowdoc, r.single, m->attn,
-                          m->stream);
-    KVR_TRY(launch_check(m, 1));
+    if (use_tc_attention(m)) {
+      const char *e = launch_attention_tc(m->q, r.pos, r.blocks, r.n_blocks, r.n_splits, dm, l,
+                                          r.views, r.single, m->attn_ws_o, m->attn_ws_ml,
+                                          m->attn, m->stream);
+      if (e) return fail(KVR_E_CUDA, "attention: %s", e);
+      KVR_TRY(launch_check(m, r.n_splits > 1 ? 2 : 1));
+    } else {
+      launch_attention_simt(m->q, r.pos, r.M, dm, l, r.views, r.rowdoc, r.single, m->attn,
+                            m->stream);
+      KVR_TRY(launch_check(m, 1));
+    }
   }
   KVR_TRY(gemm(m, P_GEMM_O, m->attn, w.wo, w.tc_o ? &w.tm_o : nullptr, nullptr, m->h, r.M, dm.d,
                dm.H * dm.dh, GEMM_EPI_ACCUM));
@@ -371,6 +416,9 @@ void kvr_model_free(kvr_model *m) {
   dev_free(m->dev_flag);
   dev_free(m->tcw.partials);
   dev_free(m->tcw.counters);
+  dev_free(m->blocks_d);
+  dev_free(m->attn_ws_o);
+  dev_free(m->attn_ws_ml);
   if (m->stage_h) cudaFreeHost(m->stage_h);
   if (m->stage_ev) cudaEventDestroy(m->stage_ev);
   delete m;
@@ -566,7 +614,7 @@ kvr_status kvr_model_create(const kvr_model_config *cfg, const kvr_weights *wts,
     m->dev_flag = (int *)dev_alloc(256);
     if (!m->dev_flag) return bail(fail(KVR_E_NOMEM, "flag"));
     cudaMemset(m->dev_flag, 0, 256);
-    m->stage_cap = std::max<size_t>(R * 2, P) + 4096;
+    m->stage_cap = std::max<size_t>(R * 4, P) + 4096;
     if (cudaMallocHost(&m->stage_h, m->stage_cap * sizeof(int32_t)) != cudaSuccess)
       return bail(fail(KVR_E_NOMEM, "pinned staging"));
     cudaEventCreateWithFlags(&m->stage_ev, cudaEventDisableTiming);
@@ -594,6 +642,15 @@ kvr_status kvr_model_create(const kvr_model_config *cfg, const kvr_weights *wts,
       w.tc_d = mk(&w.tm_d, w.wd, dm.d, dm.F);
     }
     m->tc_lm = mk(&m->tm_lm, m->lm_head, dm.V, dm.d);
+  }
+  if (use_tc_attention(m)) {
+    m->max_blocks = dm.max_rows + 256;
+    m->attn_ws_floats = (size_t)16 << 20;  // 64 MB of split-KV partials
+    m->blocks_d = (int4 *)dev_alloc((size_t)m->max_blocks * sizeof(int4));
+    m->attn_ws_o = (float *)dev_alloc(m->attn_ws_floats * sizeof(float));
+    m->attn_ws_ml = (float2 *)dev_alloc(m->attn_ws_floats / dm.dh * sizeof(float2));
+    if (!m->blocks_d || !m->attn_ws_o || !m->attn_ws_ml)
+      return bail(fail(KVR_E_NOMEM, "attention workspace"));
   }
   cudaError_t e = cudaDeviceSynchronize();
   if (e != cudaSuccess) return bail(fail(KVR_E_CUDA, "create: %s", cudaGetErrorString(e)));
@@ -650,6 +707,12 @@ kvr_status kvr_prefill(kvr_model *m, const int32_t *tokens, int32_t n, kvr_cache
     return fail(KVR_E_NOMEM, "cache of %d pages", c->n_pages);
   }
   c->tokens_h.assign(tokens, tokens + n);
+  // zeroed pages: slots never written hold finite values (masked keys meet
+  // probability 0, and 0 * NaN would not vanish)
+  if (cudaMemsetAsync(c->pages, 0, (size_t)c->n_pages * page_bytes, m->stream)) {
+    kvr_cache_free(c);
+    return fail(KVR_E_CUDA, "cache clear");
+  }
   std::vector<int32_t> tab(c->n_pages);
   for (int i = 0; i < c->n_pages; ++i) tab[i] = i;
   kvr_status st = stage_h2d(m, c->table, tab.data(), tab.size());
@@ -667,7 +730,8 @@ kvr_status kvr_prefill(kvr_model *m, const int32_t *tokens, int32_t n, kvr_cache
     r.M = M;
     r.pos = m->pos_d;
     r.max_pos = c0 + M - 1;
-    st = run_pass(m, r);
+    st = plan_attention(m, r, pos.data(), nullptr);
+    if (!st) st = run_pass(m, r);
   }
   if (st) {
     cudaStreamSynchronize(m->stream);
@@ -720,7 +784,8 @@ kvr_status kvr_repair(kvr_cache *c, const int32_t *new_tokens, int32_t edit_star
     r.tokens = c->tokens_d;
     r.single = c->view();
     r.max_pos = P[M - 1];
-    st = run_pass(m, r);
+    st = plan_attention(m, r, P.data(), nullptr);
+    if (!st) st = run_pass(m, r);
   }
   if (st == KVR_E_CUDA) c->poisoned = true;
   return st;
@@ -810,7 +875,8 @@ kvr_status kvr_repair_batch(kvr_model *m, const kvr_repair_req *reqs, int32_t n_
     r.views = (const KVView *)tab;
     r.doc_tokens = (const int32_t *const *)(tab + vb);
     r.max_pos = max_pos;
-    st = run_pass(m, r);
+    st = plan_attention(m, r, P.data(), rowdoc.data());
+    if (!st) st = run_pass(m, r);
   }
   cudaStreamSynchronize(m->stream);
   dev_free(tab);
@@ -840,6 +906,7 @@ kvr_status kvr_logits(kvr_model *m, const kvr_cache *c, const int32_t *query, in
   r.tokens = c->tokens_d;
   r.single = c->view();
   r.max_pos = c->n + qm - 1;
+  KVR_TRY(plan_attention(m, r, P.data(), nullptr));
   KVR_TRY(run_pass(m, r));
   // final RMSNorm of the last row, lm_head
   {
@@ -915,9 +982,10 @@ kvr_status kvr_select(kvr_model *m, const kvr_cache *c, kvr_policy policy, int32
         r.tokens = toks;
         r.single = c->view();
         r.max_pos = s_end - 1;
+        st = plan_attention(m, r, P.data(), nullptr);
         launch_rows_copy(r.single, dm.dtype, r.pos, edit_len, 0, dm.L, save, true, m->stream);
         launch_fill_f32(m->scores, 0.f, (size_t)n, m->stream);
-        st = launch_check(m, 2);
+        if (!st) st = launch_check(m, 2);
         if (!st) st = embed(m, r);
         for (int l = 0; l < dm.L && !st; ++l) {
           st = layer_qkv(m, r, l, true);
@@ -976,7 +1044,8 @@ kvr_status kvr_select(kvr_model *m, const kvr_cache *c, kvr_policy policy, int32
         r.M = M;
         r.pos = m->pos_d;
         r.max_pos = c0 + M - 1;
-        st = embed(m, r);
+        st = plan_attention(m, r, D.data(), nullptr);
+        if (!st) st = embed(m, r);
         if (!st) st = layer_qkv(m, r, 0, false);
         if (!st) st = layer_rest(m, r, 0);
         if (!st) st = layer_qkv(m, r, 1, false);

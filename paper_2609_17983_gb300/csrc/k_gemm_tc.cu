@@ -194,27 +194,41 @@ __device__ __forceinline__ int cta_of(long long u, long long total, int grid) {
   return (int)(((u + 1) * grid - 1) / total);
 }
 
-// Epilogue for output element (row t of X / Y, feature n of W), all lanes of
-// the warp call it together (SwiGLU exchanges lanes).
-__device__ __forceinline__ void epilogue(const TcParams &p, int t, int n, float v, bool valid) {
+// Epilogue for 16 consecutive rows t0..t0+15 of Y (the first `cnt` valid) at
+// feature n of W.  All lanes of the warp call it together (SwiGLU exchanges
+// lanes); every load is issued before any dependent use, so the chunk costs
+// one L2 round trip, not sixteen.
+__device__ __forceinline__ void epilogue16(const TcParams &p, int t0, int n, const float *v,
+                                           int cnt) {
   if (p.epi == GEMM_EPI_SWIGLU) {
-    // rows 32b..32b+15 are gate, 32b+16..32b+31 up of features 16b..16b+15;
-    // lane = n % 32
-    float u = __shfl_down_sync(0xffffffffu, v, 16);
+    // rows 32b..32b+15 of W are gate, 32b+16..32b+31 up, of features
+    // 16b..16b+15; lane = n % 32
     int r = n & 31;
-    if (valid && r < 16) {
-      float g = v;
-      float a = g / (1.0f + expf(-g)) * u;
-      ((__nv_bfloat16 *)p.out2)[(size_t)t * p.ld2 + (n >> 5) * 16 + r] = __float2bfloat16_rn(a);
+    __nv_bfloat16 *out = (__nv_bfloat16 *)p.out2 + (n >> 5) * 16 + r;
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      float u = __shfl_down_sync(0xffffffffu, v[j], 16);
+      if (j < cnt && r < 16) {
+        float g = v[j];
+        out[(size_t)(t0 + j) * p.ld2] = __float2bfloat16_rn(g / (1.0f + expf(-g)) * u);
+      }
     }
     return;
   }
-  if (!valid) return;
-  float *y = p.Y + (size_t)t * p.ldy + n;
-  if (p.epi == GEMM_EPI_ACCUM)
-    *y += v;
-  else
-    *y = v + (p.bias ? p.bias[n] : 0.f);
+  float *y = p.Y + (size_t)t0 * p.ldy + n;
+  if (p.epi == GEMM_EPI_ACCUM) {
+    float old[16];
+#pragma unroll
+    for (int j = 0; j < 16; ++j) old[j] = j < cnt ? y[(size_t)j * p.ldy] : 0.f;
+#pragma unroll
+    for (int j = 0; j < 16; ++j)
+      if (j < cnt) y[(size_t)j * p.ldy] = old[j] + v[j];
+    return;
+  }
+  float b = p.bias ? p.bias[n] : 0.f;
+#pragma unroll
+  for (int j = 0; j < 16; ++j)
+    if (j < cnt) y[(size_t)j * p.ldy] = v[j] + b;
 }
 
 __global__ void __launch_bounds__(NTHREADS, 1)
@@ -355,8 +369,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         for (int c = 0; c < mv; c += 16) {
           float v[16];
           tmem_ld16(taddr + c, v);
-#pragma unroll
-          for (int j = 0; j < 16; ++j) epilogue(p, t0 + c + j, n, v[j], c + j < mv);
+          epilogue16(p, t0 + c, n, v, mv - c);
         }
       } else {
         int slot = range_start(blockIdx.x, p.total, p.grid) >= tile_u0 ? 0 : 1;
@@ -378,13 +391,20 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         epi_bar();
         if (last_f) {
           __threadfence();
-          for (int t = 0; t < mv; ++t) {
-            float v = 0.f;
+          for (int c = 0; c < mv; c += 16) {
+            float v[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) v[j] = 0.f;
             for (int i = i_first; i <= i_last; ++i) {
               int sl = range_start(i, p.total, p.grid) >= tile_u0 ? 0 : 1;
-              v += __ldcg(p.ws + (((size_t)i * 2 + sl) * p.BN + t) * BM + f);
+              const float *src = p.ws + (((size_t)i * 2 + sl) * p.BN + c) * BM + f;
+              float x[16];
+#pragma unroll
+              for (int j = 0; j < 16; ++j) x[j] = c + j < mv ? __ldcg(src + (size_t)j * BM) : 0.f;
+#pragma unroll
+              for (int j = 0; j < 16; ++j) v[j] += x[j];
             }
-            epilogue(p, t0 + t, n, v, true);
+            epilogue16(p, t0 + c, n, v, mv - c);
           }
           if (et == 0) p.counters[tl] = 0;
         }

@@ -95,6 +95,11 @@ struct kvr_model {
   CUtensorMap tm_lm;
   bool tc_lm = false;
   kvr::TcWorkspace tcw{};
+  int4 *blocks_d = nullptr;      // attention query blocks of the current pass
+  int max_blocks = 0;
+  float *attn_ws_o = nullptr;    // split-KV partials
+  float2 *attn_ws_ml = nullptr;
+  size_t attn_ws_floats = 0;
   bool use_tc = true;  // tensor-core GEMM for bf16 shapes it takes
   cudaStream_t stream = nullptr;
   int device = 0;
@@ -200,6 +205,18 @@ const char *launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, v
 void launch_attention_simt(const float *q, const int32_t *pos, int M, const Dims &dm, int layer,
                            const KVView *views, const int32_t *rowdoc, KVView single, void *out,
                            cudaStream_t s);
+
+// Tensor-core attention (bf16 cache, head_dim 64 or 128).  blocks: device
+// int4 (row0, nrows, kmax, doc) per query block (rows of one document, at
+// most attn_tc_rows_per_block(grp) rows, kmax = largest position); the
+// keys 0..kmax of each block are split into n_splits ranges of 64-key
+// chunks (ws_o/ws_ml hold the partials when n_splits > 1).
+int attn_tc_rows_per_block(int grp);
+size_t attn_tc_ws_floats(int n_splits, int n_blocks, int G, int dh);
+const char *launch_attention_tc(const float *q, const int32_t *pos, const int4 *blocks,
+                                int n_blocks, int n_splits, const Dims &dm, int layer,
+                                const KVView *views, KVView single, float *ws_o, float2 *ws_ml,
+                                void *out, cudaStream_t s);
 
 // ---- kernels: selectors ----
 void launch_scores_simple(int policy, const int32_t *tokens, int n, int s_end, int delim,
