@@ -202,6 +202,24 @@ kvr_status kvr_model_read_tensor(const kvr_model *model, const char *name, int32
 kvr_status kvr_linear(kvr_model *model, const char *name, int32_t layer, const void *x, int32_t M,
                       float *y);
 
+/* kvr_linear without any allocation during the call.  The paper has no
+ * counterpart; this serves callers that must not allocate device memory at
+ * call time (a serving loop under a memory budget reserved up front, code
+ * that cannot take the device-wide synchronisation cudaMalloc/cudaFree may
+ * imply, hosts whose allocator belongs to another framework).  x: DEVICE
+ * bf16 [M][K], y: DEVICE float [M][N], both owned by the caller; name
+ * "wqkv", "wo", "wd" or "lm_head" of a bf16 model on the tensor-core GEMM;
+ * 1 <= M <= 64, otherwise KVR_E_UNSUPPORTED.  The GEMM's scratch (partial
+ * tiles, arrival counters) is a fixed ~10.5 MB device array that every GPU
+ * loading the library holds until exit; the first call on a device looks up
+ * its address (make that call before any stream capture).  All calls share
+ * the array: calls whose GPU work overlaps race and give wrong results.
+ * Asynchronous on the model's stream; kvr_synchronize reports device
+ * timeouts.  Allocates nothing: no cudaMalloc, cudaFree or allocating
+ * library call. */
+kvr_status kvr_linear_noalloc(kvr_model *model, const char *name, int32_t layer, const void *x,
+                              int32_t M, float *y);
+
 /* Per-kernel-class device timing with CUDA events around each launch group.
  * enable != 0 turns it on for later calls; kvr_profile_read returns, for
  * up to `cap` classes, the accumulated milliseconds and launch counts since

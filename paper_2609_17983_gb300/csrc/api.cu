@@ -373,6 +373,8 @@ bool valid_config(const kvr_model_config *c, std::string &why) {
 // ======================================================================== ABI
 
 namespace kvr {
+void set_last_error(const char *msg) { g_err = msg; }
+
 void *dev_alloc(size_t bytes) {
   if (bytes == 0) bytes = 16;
   if (g_alloc) return g_alloc(bytes, g_alloc_ctx);

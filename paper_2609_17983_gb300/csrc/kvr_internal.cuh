@@ -144,6 +144,9 @@ struct kvr_cache {
 
 namespace kvr {
 
+// Message returned by kvr_last_error() on the calling thread.
+void set_last_error(const char *msg);
+
 // ---- allocation (allocator hook) ----
 void *dev_alloc(size_t bytes);
 void dev_free(void *p);

@@ -87,6 +87,7 @@ _sigs = {
     "kvr_profile_read": ([_P, _I32, _P, _P, _P, _P, _I32, _P], _I32),
     "kvr_launch_count": ([_P], ctypes.c_int64),
     "kvr_linear": ([_P, ctypes.c_char_p, _I32, _P, _I32, _P], _I32),
+    "kvr_linear_noalloc": ([_P, ctypes.c_char_p, _I32, _P, _I32, _P], _I32),
 }
 for _name, (_args, _res) in _sigs.items():
     _f = getattr(_lib, _name)
@@ -246,6 +247,12 @@ def kvr_linear(model, name: str, layer: int, x: np.ndarray, n_out: int) -> np.nd
     _check(_lib.kvr_linear(model, name.encode(), layer, x.ctypes.data, x.shape[0],
                            y.ctypes.data))
     return y
+
+
+def kvr_linear_noalloc(model, name: str, layer: int, x_dev_ptr: int, M: int, y_dev_ptr: int):
+    """x_dev_ptr, y_dev_ptr: device addresses owned by the caller (e.g.
+    torch tensors' data_ptr()); asynchronous on the model's stream."""
+    _check(_lib.kvr_linear_noalloc(model, name.encode(), layer, x_dev_ptr, M, y_dev_ptr))
 
 
 def kvr_profile_enable(model, enable: bool = True):
