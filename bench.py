@@ -210,7 +210,10 @@ def main():
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     from paper_2609_17983_gb300 import kvrepair as kv
 
-    stream = torch.cuda.current_stream()
+    # a stream of our own: the library captures the repair pass as a CUDA graph
+    # (the legacy default stream cannot be captured)
+    stream = torch.cuda.Stream()
+    torch.cuda.set_stream(stream)
     model = kv.Model(cfg, None, seed=0, max_context=8192, max_rows=4096)
     model.set_stream(stream.cuda_stream)
     doc, new = edit_inputs(cfg)

@@ -119,14 +119,21 @@ kvr_status stage_h2d(kvr_model *m, int32_t *dst_dev, const int32_t *src, size_t 
 // Y (+)= X W^T through the tensor-core kernel when the weight has a TMA
 // descriptor, else the FFMA kernel.  epi selects the epilogue; for SwiGLU
 // the FFMA path writes gate/up to m->gu and runs the SwiGLU kernel.
+// Bytes of the next GEMM's weights each CTA prefetches into L2 while a
+// few-row GEMM drains (the gap before the next GEMM would leave HBM idle).
+constexpr long long PREFETCH_BYTES_PER_CTA = 256 << 10;
+
 kvr_status gemm(kvr_model *m, int cls, const void *X, const void *W, const CUtensorMap *tm,
-                const float *bias, float *Y, int M, int N, int K, int epi) {
+                const float *bias, float *Y, int M, int N, int K, int epi,
+                const CUtensorMap *next_tm = nullptr, int next_N = 0, int next_K = 0) {
   const Dims &dm = m->dims;
   Prof pr(m, cls, (int64_t)N * K * (int64_t)dm.es());
   if (tm && m->use_tc) {
     GemmArgs g{X, W, bias, Y, M, N, K, K, N, dm.dtype, epi == GEMM_EPI_ACCUM};
+    TcNext nx{next_tm, M, next_N, next_K, PREFETCH_BYTES_PER_CTA};
+    bool pf = next_tm && m->prefetch && M <= 256;
     const char *e = launch_gemm_tc(g, *tm, epi, epi == GEMM_EPI_SWIGLU ? m->act : nullptr,
-                                   N / 2, m->tcw, m->stream);
+                                   N / 2, m->tcw, m->stream, pf ? &nx : nullptr);
     if (e) return fail(KVR_E_CUDA, "tensor-core GEMM (M=%d N=%d K=%d): %s", M, N, K, e);
     return launch_check(m, 1);
   }
@@ -182,7 +189,7 @@ kvr_status plan_attention(kvr_model *m, Rows &r, const int32_t *pos, const int32
   if (nb > m->max_blocks) return fail(KVR_E_UNSUPPORTED, "too many attention blocks (%d)", nb);
   int target = 2 * m->num_sms;
   int splits = std::max(1, (target + nb * dm.G - 1) / (nb * dm.G));
-  splits = std::min(splits, max_chunks);
+  splits = std::min(std::min(splits, max_chunks), 64);  // the combine merges <= 64 splits
   while (splits > 1 && attn_tc_ws_floats(splits, nb, dm.G, dm.dh) > m->attn_ws_floats) --splits;
   KVR_TRY(stage_h2d(m, (int32_t *)m->blocks_d, b.data(), b.size()));
   r.blocks = m->blocks_d;
@@ -210,7 +217,7 @@ kvr_status layer_qkv(kvr_model *m, const Rows &r, int l, bool write_kv) {
   const LayerW &w = m->layers[l];
   KVR_TRY(norm(m, w.attn_norm, r.M));
   KVR_TRY(gemm(m, P_GEMM_QKV, m->a, w.wqkv, w.tc_qkv ? &w.tm_qkv : nullptr, w.bqkv, m->qkv, r.M,
-               dm.Nqkv(), dm.d, GEMM_EPI_STORE));
+               dm.Nqkv(), dm.d, GEMM_EPI_STORE, w.tc_o ? &w.tm_o : nullptr, dm.d, dm.H * dm.dh));
   {
     Prof pr(m, P_ROPE, (int64_t)r.M * dm.Nqkv() * 4);
     launch_rope_scatter(m->qkv, m->rope, r.pos, r.M, dm, l, r.views, r.rowdoc, r.single, m->q,
@@ -239,13 +246,14 @@ kvr_status layer_rest(kvr_model *m, const Rows &r, int l) {
       KVR_TRY(launch_check(m, 1));
     }
   }
+  const LayerW *wn = l + 1 < dm.L ? &m->layers[l + 1] : nullptr;
   KVR_TRY(gemm(m, P_GEMM_O, m->attn, w.wo, w.tc_o ? &w.tm_o : nullptr, nullptr, m->h, r.M, dm.d,
-               dm.H * dm.dh, GEMM_EPI_ACCUM));
+               dm.H * dm.dh, GEMM_EPI_ACCUM, w.tc_gu ? &w.tm_gu : nullptr, 2 * dm.F, dm.d));
   KVR_TRY(norm(m, w.mlp_norm, r.M));
   KVR_TRY(gemm(m, P_GEMM_GU, m->a, w.wgu, w.tc_gu ? &w.tm_gu : nullptr, nullptr, nullptr, r.M,
-               2 * dm.F, dm.d, GEMM_EPI_SWIGLU));
+               2 * dm.F, dm.d, GEMM_EPI_SWIGLU, w.tc_d ? &w.tm_d : nullptr, dm.d, dm.F));
   KVR_TRY(gemm(m, P_GEMM_DOWN, m->act, w.wd, w.tc_d ? &w.tm_d : nullptr, nullptr, m->h, r.M, dm.d,
-               dm.F, GEMM_EPI_ACCUM));
+               dm.F, GEMM_EPI_ACCUM, wn && wn->tc_qkv ? &wn->tm_qkv : nullptr, dm.Nqkv(), dm.d));
   return KVR_OK;
 }
 
@@ -258,6 +266,41 @@ kvr_status run_pass(kvr_model *m, const Rows &r) {
     KVR_TRY(layer_qkv(m, r, l, true));
     KVR_TRY(layer_rest(m, r, l));
   }
+  return KVR_OK;
+}
+
+// The repair pass through a CUDA graph: the launch sequence of a pass
+// depends only on the cache, the row count and the attention block/split
+// plan (positions, tokens and block contents are read from device memory),
+// so it is captured once per such key and replayed.  Only on a stream that
+// can be captured (not the legacy default stream) and with profiling off.
+kvr_status run_pass_graph(kvr_model *m, kvr_cache *c, const Rows &r) {
+  if (!m->use_graphs || m->prof || m->stream == nullptr) return run_pass(m, r);
+  for (auto &g : c->graphs)
+    if (g.M == r.M && g.nb == r.n_blocks && g.ns == r.n_splits) {
+      cudaError_t e = cudaGraphLaunch(g.exec, m->stream);
+      if (e != cudaSuccess) return fail(KVR_E_CUDA, "graph launch: %s", cudaGetErrorString(e));
+      m->launches += g.kernels;
+      return KVR_OK;
+    }
+  int64_t l0 = m->launches;
+  cudaError_t e = cudaStreamBeginCapture(m->stream, cudaStreamCaptureModeThreadLocal);
+  if (e != cudaSuccess) return fail(KVR_E_CUDA, "begin capture: %s", cudaGetErrorString(e));
+  kvr_status st = run_pass(m, r);
+  cudaGraph_t graph = nullptr;
+  e = cudaStreamEndCapture(m->stream, &graph);
+  if (st || e != cudaSuccess) {
+    if (graph) cudaGraphDestroy(graph);
+    cudaGetLastError();
+    return st ? st : fail(KVR_E_CUDA, "end capture: %s", cudaGetErrorString(e));
+  }
+  cudaGraphExec_t exec = nullptr;
+  e = cudaGraphInstantiate(&exec, graph, 0);
+  cudaGraphDestroy(graph);
+  if (e != cudaSuccess) return fail(KVR_E_CUDA, "graph instantiate: %s", cudaGetErrorString(e));
+  c->graphs.push_back({r.M, r.n_blocks, r.n_splits, m->launches - l0, exec});
+  e = cudaGraphLaunch(exec, m->stream);
+  if (e != cudaSuccess) return fail(KVR_E_CUDA, "graph launch: %s", cudaGetErrorString(e));
   return KVR_OK;
 }
 
@@ -434,6 +477,8 @@ kvr_status kvr_model_create(const kvr_model_config *cfg, const kvr_weights *wts,
   if (!valid_config(cfg, why)) return fail(KVR_E_INVAL, "invalid config: %s", why.c_str());
   if (cfg->head_dim != 64 && cfg->head_dim != 128)
     return fail(KVR_E_UNSUPPORTED, "head_dim must be 64 or 128");
+  if (cfg->d_model % 4 || cfg->d_model > 8192)
+    return fail(KVR_E_UNSUPPORTED, "d_model must be a multiple of 4 and at most 8192");
   if (cfg->ffn % GU_BLOCK) return fail(KVR_E_UNSUPPORTED, "ffn must be a multiple of 16");
   if (cfg->max_context > 16384) return fail(KVR_E_UNSUPPORTED, "max_context above 16384");
 
@@ -443,6 +488,10 @@ kvr_status kvr_model_create(const kvr_model_config *cfg, const kvr_weights *wts,
             cfg->head_dim, cfg->ffn, cfg->qkv_bias ? 1 : 0, cfg->dtype, cfg->delim_id,
             cfg->rope_theta, cfg->rms_eps, cfg->max_context, cfg->max_rows};
   cudaGetDevice(&m->device);
+  {
+    const char *g = getenv("KVR_DISABLE_GRAPHS");
+    m->use_graphs = !(g && g[0] == '1');
+  }
   cudaDeviceGetAttribute(&m->num_sms, cudaDevAttrMultiProcessorCount, m->device);
   m->prof_classes.resize(P_NCLASS);
   for (int i = 0; i < P_NCLASS; ++i) m->prof_classes[i].name = kProfNames[i];
@@ -626,6 +675,8 @@ kvr_status kvr_model_create(const kvr_model_config *cfg, const kvr_weights *wts,
   if (dm.dtype == KVR_DTYPE_BF16) {
     const char *env = getenv("KVR_DISABLE_TC");
     m->use_tc = !(env && env[0] == '1');
+    const char *pf = getenv("KVR_DISABLE_PREFETCH");
+    m->prefetch = !(pf && pf[0] == '1');
     m->tcw.num_sms = m->num_sms;
     m->tcw.max_tiles = 1 << 16;
     m->tcw.dev_flag = m->dev_flag;
@@ -678,6 +729,7 @@ void kvr_cache_free(kvr_cache *c) {
   if (!c) return;
   cudaSetDevice(c->model->device);
   cudaStreamSynchronize(c->model->stream);
+  for (auto &g : c->graphs) cudaGraphExecDestroy(g.exec);
   dev_free(c->pages);
   dev_free(c->table);
   dev_free(c->tokens_d);
@@ -787,7 +839,7 @@ kvr_status kvr_repair(kvr_cache *c, const int32_t *new_tokens, int32_t edit_star
     r.single = c->view();
     r.max_pos = P[M - 1];
     st = plan_attention(m, r, P.data(), nullptr);
-    if (!st) st = run_pass(m, r);
+    if (!st) st = run_pass_graph(m, c, r);
   }
   if (st == KVR_E_CUDA) c->poisoned = true;
   return st;

@@ -279,38 +279,55 @@ __global__ void __launch_bounds__(NW * 32, 2) k_attn_tc(const AttnTcParams p) {
 }
 
 // Merge the key splits of every (block, kv head, query vector), split order.
+// One warp per query vector: lane s reads split s's (max, sum), the weights
+// are reduced across the warp, then the partial outputs are gathered eight
+// splits at a time with all loads in flight together.
 template <int DH>
 __global__ void __launch_bounds__(256) k_attn_combine(const AttnTcParams p) {
   const int warp = (blockIdx.x * 8) + (threadIdx.x >> 5), lane = threadIdx.x & 31;
-  const int per_bg = MAXQ;
-  const int total = p.n_blocks * p.G * per_bg;
+  const int total = p.n_blocks * p.G * MAXQ;
   if (warp >= total) return;
-  const int v = warp % per_bg, bg = warp / per_bg;
+  const int v = warp % MAXQ, bg = warp / MAXQ;
   const int g = bg % p.G, blk = bg / p.G;
   const int4 bd = p.blocks[blk];
   const int mq = bd.y * p.grp;
   if (v >= mq) return;
   const int n_chunks = bd.z / CHUNK + 1;
   const int cps = (n_chunks + p.n_splits - 1) / p.n_splits;
-  float mstar = -INFINITY;
-  for (int s = 0; s * cps < n_chunks; ++s) {
-    float2 ml = p.ws_ml[(((size_t)s * p.n_blocks + blk) * p.G + g) * MAXQ + v];
-    if (ml.y > 0.f) mstar = fmaxf(mstar, ml.x);
-  }
+  const int ns = (n_chunks + cps - 1) / cps;  // non-empty splits
+  const size_t stride = (size_t)p.n_blocks * p.G;  // between splits, in (block, head) units
+  const size_t base = (size_t)blk * p.G + g;
+  // (max, sum) of up to 64 splits, two per lane
+  float2 ml0 = lane < ns ? p.ws_ml[(base + lane * stride) * MAXQ + v] : make_float2(-INFINITY, 0.f);
+  float2 ml1 = lane + 32 < ns ? p.ws_ml[(base + (lane + 32) * stride) * MAXQ + v]
+                              : make_float2(-INFINITY, 0.f);
+  float mx = fmaxf(ml0.y > 0.f ? ml0.x : -INFINITY, ml1.y > 0.f ? ml1.x : -INFINITY);
+  for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  const float w0 = ml0.y > 0.f ? exp2f(ml0.x - mx) : 0.f;
+  const float w1 = ml1.y > 0.f ? exp2f(ml1.x - mx) : 0.f;
+  float l = w0 * ml0.y + w1 * ml1.y;
+  for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
   constexpr int VPL = DH / 32;
   float acc[VPL];
 #pragma unroll
   for (int i = 0; i < VPL; ++i) acc[i] = 0.f;
-  float l = 0.f;
-  for (int s = 0; s * cps < n_chunks; ++s) {
-    size_t bs = ((size_t)s * p.n_blocks + blk) * p.G + g;
-    float2 ml = p.ws_ml[bs * MAXQ + v];
-    if (!(ml.y > 0.f)) continue;
-    float w = exp2f(ml.x - mstar);
-    l += w * ml.y;
-    const float *src = p.ws_o + (bs * MAXQ + v) * DH + lane * VPL;
+  const float *src = p.ws_o + (base * MAXQ + v) * DH + lane * VPL;
+  const size_t sstride = stride * MAXQ * DH;
+  for (int s0 = 0; s0 < ns; s0 += 8) {
+    float x[8][VPL];
 #pragma unroll
-    for (int i = 0; i < VPL; ++i) acc[i] += w * src[i];
+    for (int j = 0; j < 8; ++j)
+#pragma unroll
+      for (int i = 0; i < VPL; ++i) x[j][i] = s0 + j < ns ? src[(s0 + j) * sstride + i] : 0.f;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      int sj = s0 + j;
+      float w = __shfl_sync(0xffffffffu, sj < 32 ? w0 : w1, sj & 31);
+      if (sj < ns) {
+#pragma unroll
+        for (int i = 0; i < VPL; ++i) acc[i] += w * x[j][i];
+      }
+    }
   }
   const float inv = l > 0.f ? 1.f / l : 0.f;
   const int r = bd.x + v / p.grp, hh = g * p.grp + v % p.grp;

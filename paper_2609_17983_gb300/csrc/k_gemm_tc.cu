@@ -55,6 +55,10 @@ struct TcParams {
   float *ws;        // [grid][2][BN][128] fp32 partial tiles
   int *counters;    // [n_tiles * m_tiles] arrival counters (self-resetting)
   int *dev_flag;
+  // L2 prefetch of the next GEMM's weights: CTA i prefetches the first
+  // pf_units units of its own range in the next GEMM's stream-K split
+  long long next_total;
+  int next_KB, next_m_tiles, next_grid, pf_units;
 };
 
 // ------------------------------------------------------------ PTX wrappers
@@ -122,6 +126,13 @@ __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, u
       " [%0], [%1, {%2, %3}], [%4];" ::"r"(su32(dst)),
       "l"((uint64_t)map), "r"(x), "r"(y), "r"(su32(bar))
       : "memory");
+}
+
+__device__ __forceinline__ void tma_prefetch_l2(const CUtensorMap *map, int x, int y) {
+  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
+                   (uint64_t)map),
+               "r"(x), "r"(y)
+               : "memory");
 }
 
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap *map) {
@@ -233,7 +244,7 @@ __device__ __forceinline__ void epilogue16(const TcParams &p, int t0, int n, con
 
 __global__ void __launch_bounds__(NTHREADS, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX,
-              const TcParams p) {
+              const __grid_constant__ CUtensorMap tmNext, const TcParams p) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[8], empty_bar[8], accf_bar[2], acce_bar[2],
       drain_bar;
@@ -300,6 +311,16 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         tma_load_2d((void *)__cvta_shared_to_generic(sa + A_BYTES), &tmX, &full_bar[s],
                     kb * BK, mtile * p.BN);
         ++it;
+      }
+      // warm L2 with the start of this CTA's share of the next GEMM's weights
+      if (p.pf_units > 0 && (int)blockIdx.x < p.next_grid && !*abort_v) {
+        long long nu0 = range_start(blockIdx.x, p.next_total, p.next_grid);
+        long long nu1 = range_start(blockIdx.x + 1, p.next_total, p.next_grid);
+        if (nu1 > nu0 + p.pf_units) nu1 = nu0 + p.pf_units;
+        for (long long u = nu0; u < nu1; ++u) {
+          long long tl = u / p.next_KB;
+          tma_prefetch_l2(&tmNext, (int)(u % p.next_KB) * BK, (int)(tl / p.next_m_tiles) * BM);
+        }
       }
       // copies in flight complete before the CTA may exit
       uint32_t n_issued = it;
@@ -391,20 +412,23 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         epi_bar();
         if (last_f) {
           __threadfence();
-          for (int c = 0; c < mv; c += 16) {
-            float v[16];
+          // 48 rows of one part per round trip: all their loads are in flight
+          for (int c = 0; c < mv; c += 48) {
+            float v[48];
 #pragma unroll
-            for (int j = 0; j < 16; ++j) v[j] = 0.f;
+            for (int j = 0; j < 48; ++j) v[j] = 0.f;
             for (int i = i_first; i <= i_last; ++i) {
               int sl = range_start(i, p.total, p.grid) >= tile_u0 ? 0 : 1;
               const float *src = p.ws + (((size_t)i * 2 + sl) * p.BN + c) * BM + f;
-              float x[16];
+              float x[48];
 #pragma unroll
-              for (int j = 0; j < 16; ++j) x[j] = c + j < mv ? __ldcg(src + (size_t)j * BM) : 0.f;
+              for (int j = 0; j < 48; ++j) x[j] = c + j < mv ? __ldcg(src + (size_t)j * BM) : 0.f;
 #pragma unroll
-              for (int j = 0; j < 16; ++j) v[j] += x[j];
+              for (int j = 0; j < 48; ++j) v[j] += x[j];
             }
-            epilogue16(p, t0 + c, n, v, mv - c);
+#pragma unroll
+            for (int q16 = 0; q16 < 3; ++q16)
+              if (c + 16 * q16 < mv) epilogue16(p, t0 + c + 16 * q16, n, v + 16 * q16, mv - c - 16 * q16);
           }
           if (et == 0) p.counters[tl] = 0;
         }
@@ -472,7 +496,7 @@ int gemm_tc_bn(int M) {
 size_t gemm_tc_ws_bytes(int num_sms) { return (size_t)num_sms * 2 * 256 * BM * sizeof(float); }
 
 const char *launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, void *out2,
-                           int ld2, const TcWorkspace &ws, cudaStream_t s) {
+                           int ld2, const TcWorkspace &ws, cudaStream_t s, const TcNext *next) {
   if (g.M <= 0) return nullptr;
   TcParams p{};
   p.M = g.M;
@@ -522,8 +546,19 @@ const char *launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, v
   if ((long long)p.n_tiles * p.m_tiles > ws.max_tiles) return "more tiles than counters";
   CUtensorMap tmX;
   if (!make_tmap_bf16(&tmX, g.X, g.M, g.K, p.brows)) return "activation TMA descriptor rejected";
+  const CUtensorMap *tmN = &tmW;
+  if (next && next->tm && next->bytes_per_cta > 0) {
+    int nbn = gemm_tc_bn(next->M);
+    long long nm = (next->M + nbn - 1) / nbn;
+    p.next_KB = next->K / BK;
+    p.next_m_tiles = (int)nm;
+    p.next_total = (long long)(next->N / BM) * nm * p.next_KB;
+    p.next_grid = (int)(p.next_total < ws.num_sms ? p.next_total : ws.num_sms);
+    p.pf_units = (int)(next->bytes_per_cta / A_BYTES);
+    tmN = next->tm;
+  }
   size_t smem = 1024 + (size_t)p.stages * stage_bytes;
-  k_gemm_tc<<<p.grid, NTHREADS, smem, s>>>(tmW, tmX, p);
+  k_gemm_tc<<<p.grid, NTHREADS, smem, s>>>(tmW, tmX, *tmN, p);
   cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? nullptr : cudaGetErrorString(e);
 }

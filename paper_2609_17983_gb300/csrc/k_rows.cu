@@ -82,24 +82,45 @@ __global__ void k_embed_rows(const T *embed, const int32_t *tokens,
   for (int c = threadIdx.x; c < d; c += blockDim.x) h[(size_t)i * d + c] = ld(embed, base + c);
 }
 
+// One block of 256 threads per row; the row (d <= 8192, d % 4 == 0) is
+// loaded once into registers with every load issued before the first use.
 template <typename T>
-__global__ void k_rmsnorm(const float *h, const float *g, int d, float eps, T *out) {
+__global__ void __launch_bounds__(256) k_rmsnorm(const float *h, const float *g, int d, float eps,
+                                                 T *out) {
+  constexpr int NV = 8;  // float4 per thread: 8 * 4 * 256 = 8192 elements
   int i = blockIdx.x;
-  const float *x = h + (size_t)i * d;
+  const float4 *x = (const float4 *)(h + (size_t)i * d);
+  const int nq = d >> 2;
+  float4 v[NV];
   float ss = 0.f;
-  for (int c = threadIdx.x; c < d; c += blockDim.x) ss += x[c] * x[c];
-  __shared__ float red[32];
+#pragma unroll
+  for (int k = 0; k < NV; ++k) {
+    int q = k * 256 + threadIdx.x;
+    v[k] = q < nq ? x[q] : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+#pragma unroll
+  for (int k = 0; k < NV; ++k) ss += v[k].x * v[k].x + v[k].y * v[k].y + v[k].z * v[k].z + v[k].w * v[k].w;
+  __shared__ float red[8];
   for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
   if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
   __syncthreads();
-  if (threadIdx.x < 32) {
-    float t = threadIdx.x < (blockDim.x >> 5) ? red[threadIdx.x] : 0.f;
-    for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
-    if (threadIdx.x == 0) red[0] = t;
+  float tot = 0.f;
+#pragma unroll
+  for (int w = 0; w < 8; ++w) tot += red[w];
+  float r = 1.0f / sqrtf(tot / (float)d + eps);
+  const float4 *gg = (const float4 *)g;
+#pragma unroll
+  for (int k = 0; k < NV; ++k) {
+    int q = k * 256 + threadIdx.x;
+    if (q < nq) {
+      float4 w = gg[q];
+      size_t o = (size_t)i * d + 4 * q;
+      st(out, o, v[k].x * r * w.x);
+      st(out, o + 1, v[k].y * r * w.y);
+      st(out, o + 2, v[k].z * r * w.z);
+      st(out, o + 3, v[k].w * r * w.w);
+    }
   }
-  __syncthreads();
-  float r = 1.0f / sqrtf(red[0] / (float)d + eps);
-  for (int c = threadIdx.x; c < d; c += blockDim.x) st(out, (size_t)i * d + c, x[c] * r * g[c]);
 }
 
 // grid (M, H + 2G), block dh/2: rotate q and k heads at the row's position;

@@ -101,6 +101,8 @@ struct kvr_model {
   float2 *attn_ws_ml = nullptr;
   size_t attn_ws_floats = 0;
   bool use_tc = true;  // tensor-core GEMM for bf16 shapes it takes
+  bool prefetch = true;  // L2 prefetch of the next GEMM's weights
+  bool use_graphs = true;  // CUDA graphs for repeated repair passes
   cudaStream_t stream = nullptr;
   int device = 0;
   int num_sms = 0;
@@ -137,6 +139,12 @@ struct kvr_cache {
   int32_t *tokens_d = nullptr;  // device [cap]
   std::vector<int32_t> tokens_h;
   bool poisoned = false;
+  struct Graph {
+    int M, nb, ns;
+    int64_t kernels;
+    cudaGraphExec_t exec;
+  };
+  std::vector<Graph> graphs;  // captured repair passes of this cache
   kvr::KVView view() const {
     return kvr::KVView{pages, table, model->dims.L, model->dims.G, model->dims.dh};
   }
@@ -198,9 +206,17 @@ int gemm_tc_bn(int M);
 size_t gemm_tc_ws_bytes(int num_sms);
 // GEMM_EPI_SWIGLU: W rows interleaved gate/up in blocks of 16; writes
 // out2[t][f] = bf16(silu(gate) * up), f < N/2, row stride ld2.
+// The GEMM that follows in the stream: while this one drains, each CTA
+// prefetches into L2 up to bytes_per_cta of its share of next's weights.
+struct TcNext {
+  const CUtensorMap *tm;
+  int M, N, K;
+  long long bytes_per_cta;
+};
 // Returns nullptr on success, else what went wrong.
 const char *launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, void *out2,
-                           int ld2, const TcWorkspace &ws, cudaStream_t s);
+                           int ld2, const TcWorkspace &ws, cudaStream_t s,
+                           const TcNext *next = nullptr);
 
 // ---- kernels: attention ----
 // o[i] = softmax(q_i K[0..pos_i]^T / sqrt(dh)) V[0..pos_i] for every row i,

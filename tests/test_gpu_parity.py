@@ -346,3 +346,31 @@ def test_select_long_context_exact(n):
         ref = oracle.select(cfg, W, ref_cache, policy, K, s, new, seed)
         assert got.tolist() == ref.tolist(), policy
     model.close()
+
+
+def test_graph_replay_matches_eager():
+    # repair passes captured as a CUDA graph (model on a non-default stream)
+    # give bit-identical caches to eager launches, on the first (capturing)
+    # call and on replays with different positions of the same shape
+    import torch
+    cfg = synth.preset("llama8b", n_layers=2)
+    n, s, L = 600, 300, 8
+    doc = synth.document(1, n, cfg["vocab"])
+    new = synth.edit_tokens(2, doc[s:s + L], cfg["vocab"])
+    eager = kv.Model(cfg, None, seed=0, max_context=1024, max_rows=256)
+    graph = kv.Model(cfg, None, seed=0, max_context=1024, max_rows=256)
+    st = torch.cuda.Stream()
+    graph.set_stream(st.cuda_stream)
+    ce, cg = eager.prefill(doc), graph.prefill(doc)
+    graph.synchronize()
+    rows = np.arange(n)
+    for A in (np.arange(s + L, s + L + 32), np.arange(s + L + 5, s + L + 37),
+              np.arange(s + L + 5, s + L + 37)):
+        ce.repair(new, s, A)
+        cg.repair(new, s, A)
+        graph.synchronize()
+        k1, v1 = ce.read(rows)
+        k2, v2 = cg.read(rows)
+        assert np.array_equal(k1, k2) and np.array_equal(v1, v2)
+    eager.close()
+    graph.close()
