@@ -416,6 +416,8 @@ bool valid_config(const kvr_model_config *c, std::string &why) {
 // ======================================================================== ABI
 
 namespace kvr {
+bool g_pdl = true;
+
 void set_last_error(const char *msg) { g_err = msg; }
 
 void *dev_alloc(size_t bytes) {
@@ -491,6 +493,8 @@ kvr_status kvr_model_create(const kvr_model_config *cfg, const kvr_weights *wts,
   {
     const char *g = getenv("KVR_DISABLE_GRAPHS");
     m->use_graphs = !(g && g[0] == '1');
+    const char *pd = getenv("KVR_DISABLE_PDL");
+    g_pdl = !(pd && pd[0] == '1');
   }
   cudaDeviceGetAttribute(&m->num_sms, cudaDevAttrMultiProcessorCount, m->device);
   m->prof_classes.resize(P_NCLASS);

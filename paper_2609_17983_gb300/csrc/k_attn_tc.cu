@@ -100,6 +100,8 @@ __global__ void __launch_bounds__(NW * 32, 2) k_attn_tc(const AttnTcParams p) {
   uint8_t *sV = sK + 2 * TILE;                 // 2 x CHUNK x DH
   __shared__ int spos[MAXQ];
 
+  pdl_trigger();
+  pdl_wait();
   const int split = blockIdx.x, g = blockIdx.y, blk = blockIdx.z;
   const int4 bd = p.blocks[blk];
   const int row0 = bd.x, nrows = bd.y, kmax = bd.z;
@@ -284,6 +286,8 @@ __global__ void __launch_bounds__(NW * 32, 2) k_attn_tc(const AttnTcParams p) {
 // splits at a time with all loads in flight together.
 template <int DH>
 __global__ void __launch_bounds__(256) k_attn_combine(const AttnTcParams p) {
+  pdl_trigger();
+  pdl_wait();
   const int warp = (blockIdx.x * 8) + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   const int total = p.n_blocks * p.G * MAXQ;
   if (warp >= total) return;
@@ -347,10 +351,10 @@ const char *run(const AttnTcParams &p, cudaStream_t s) {
     set = true;
   }
   dim3 grid(p.n_splits, p.G, p.n_blocks);
-  k_attn_tc<DH><<<grid, NW * 32, smem, s>>>(p);
+  launch_pdl(k_attn_tc<DH>, grid, NW * 32, smem, s, p);
   if (p.n_splits > 1) {
     int warps = p.n_blocks * p.G * MAXQ;
-    k_attn_combine<DH><<<(warps + 7) / 8, 256, 0, s>>>(p);
+    launch_pdl(k_attn_combine<DH>, (warps + 7) / 8, 256, 0, s, p);
   }
   cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? nullptr : cudaGetErrorString(e);

@@ -247,11 +247,12 @@ __global__ void __launch_bounds__(NTHREADS, 1)
               const __grid_constant__ CUtensorMap tmNext, const TcParams p) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[8], empty_bar[8], accf_bar[2], acce_bar[2],
-      drain_bar;
+      drain_bar, fix_bar;
   __shared__ uint32_t tmem_slot;
   __shared__ int abort_f;
   __shared__ int last_f;
 
+  pdl_trigger();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int S = p.stages;
   const uint32_t base = (su32(smem_raw) + 1023u) & ~1023u;
@@ -270,6 +271,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       mbar_init(&acce_bar[b], 128);
     }
     mbar_init(&drain_bar, 1);
+    mbar_init(&fix_bar, 1);
     abort_f = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -296,21 +298,71 @@ __global__ void __launch_bounds__(NTHREADS, 1)
   if (warp == 0) {
     // ---------------------------------------------------------------- TMA
     if (lane == 0) {
-      uint32_t it = 0;
-      for (long long u = u0; u < u1; ++u) {
-        int s = (int)(it % S);
-        uint32_t ph = (it / S) & 1u;
+      // incremental walk over (feature tile, token tile, K block) and stages
+      long long tl0 = u0 / p.KB;
+      int kb = (int)(u0 - tl0 * p.KB);
+      int ntile = (int)(tl0 / p.m_tiles), mtile = (int)(tl0 - (long long)ntile * p.m_tiles);
+      int s = 0;
+      uint32_t ph = 0, it = 0;
+      // The weights never depend on the previous kernel: their tiles for the
+      // first stages are requested before waiting for it (PDL), the
+      // activation tiles of those stages right after.
+      {
+        const long long npre = (u1 - u0) < S ? (u1 - u0) : S;
+        int kb2 = kb, nt2 = ntile;
+        int mt2 = mtile;
+        for (long long j = 0; j < npre; ++j) {
+          uint32_t sa = base + (uint32_t)j * stage_bytes;
+          mbar_expect_tx(&full_bar[j], tx_bytes);
+          tma_load_2d((void *)__cvta_shared_to_generic(sa), &tmW, &full_bar[j], kb2 * BK,
+                      nt2 * BM);
+          if (++kb2 == p.KB) {
+            kb2 = 0;
+            if (++mt2 == p.m_tiles) {
+              mt2 = 0;
+              ++nt2;
+            }
+          }
+        }
+        pdl_wait();
+        for (long long j = 0; j < npre; ++j) {
+          uint32_t sa = base + (uint32_t)j * stage_bytes;
+          tma_load_2d((void *)__cvta_shared_to_generic(sa + A_BYTES), &tmX, &full_bar[j],
+                      kb * BK, mtile * p.BN);
+          ++it;
+          if (++s == S) {
+            s = 0;
+            ph ^= 1u;
+          }
+          if (++kb == p.KB) {
+            kb = 0;
+            if (++mtile == p.m_tiles) {
+              mtile = 0;
+              ++ntile;
+            }
+          }
+        }
+      }
+      for (long long u = u0 + it; u < u1; ++u) {
         if (!mbar_wait(&empty_bar[s], ph ^ 1u, abort_v, p.dev_flag, 1)) break;
-        long long tl = u / p.KB;
-        int kb = (int)(u % p.KB);
-        int ntile = (int)(tl / p.m_tiles), mtile = (int)(tl % p.m_tiles);
         uint32_t sa = base + (uint32_t)s * stage_bytes;
         mbar_expect_tx(&full_bar[s], tx_bytes);
         tma_load_2d((void *)__cvta_shared_to_generic(sa), &tmW, &full_bar[s], kb * BK,
                     ntile * BM);
-        tma_load_2d((void *)__cvta_shared_to_generic(sa + A_BYTES), &tmX, &full_bar[s],
-                    kb * BK, mtile * p.BN);
+        tma_load_2d((void *)__cvta_shared_to_generic(sa + A_BYTES), &tmX, &full_bar[s], kb * BK,
+                    mtile * p.BN);
         ++it;
+        if (++s == S) {
+          s = 0;
+          ph ^= 1u;
+        }
+        if (++kb == p.KB) {
+          kb = 0;
+          if (++mtile == p.m_tiles) {
+            mtile = 0;
+            ++ntile;
+          }
+        }
       }
       // warm L2 with the start of this CTA's share of the next GEMM's weights
       if (p.pf_units > 0 && (int)blockIdx.x < p.next_grid && !*abort_v) {
@@ -331,7 +383,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     // ---------------------------------------------------------------- MMA
     if (lane == 0) {
       const uint32_t idesc = idesc_bf16(BM, p.BN);
-      uint32_t it = 0, seg = 0;
+      uint32_t seg = 0, ph = 0;
+      int s = 0;
       bool ok = true;
       for (long long a = u0; a < u1 && ok;) {
         long long tl = a / p.KB;
@@ -341,8 +394,6 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         tc_fence_after();
         uint32_t d = tmem_base + buf * p.tmem_cols;
         for (long long u = a; u < b; ++u) {
-          int s = (int)(it % S);
-          uint32_t ph = (it / S) & 1u;
           if (!mbar_wait(&full_bar[s], ph, abort_v, p.dev_flag, 4)) {
             ok = false;
             break;
@@ -355,7 +406,10 @@ __global__ void __launch_bounds__(NTHREADS, 1)
             mma_bf16(d, da + (uint64_t)(k * UK * 2 / 16), db + (uint64_t)(k * UK * 2 / 16), idesc,
                      (u > a || k > 0) ? 1u : 0u);
           mma_commit(&empty_bar[s]);
-          ++it;
+          if (++s == S) {
+            s = 0;
+            ph ^= 1u;
+          }
         }
         if (ok) mma_commit(&accf_bar[buf]);
         ++seg;
@@ -367,10 +421,11 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     }
   } else {
     // ------------------------------------------------------------ epilogue
+    pdl_wait();  // outputs, partials and counters may still be in use upstream
     const int q = warp & 3;  // TMEM lane quarter of this warp
     const int f = q * 32 + lane;
     const int et = threadIdx.x - 64;  // 0..127
-    uint32_t seg = 0;
+    uint32_t seg = 0, fix_phase = 0;
     for (long long a = u0; a < u1;) {
       long long tl = a / p.KB;
       long long b = (tl + 1) * p.KB < u1 ? (tl + 1) * p.KB : u1;
@@ -412,6 +467,41 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         epi_bar();
         if (last_f) {
           __threadfence();
+          const uint32_t part_bytes = (uint32_t)mv * BM * 4u;
+          if (b == u1 && (uint32_t)parts * (uint32_t)p.BN * BM * 4u <= (uint32_t)S * stage_bytes) {
+            // Final segment of this CTA: every pipeline stage is free.  One
+            // thread fetches all parts with bulk copies into shared memory,
+            // then the warps sum them in part order.
+            if (et == 0) {
+              asm volatile("fence.proxy.async.global;" ::: "memory");
+              mbar_expect_tx(&fix_bar, part_bytes * parts);
+              for (int i = i_first; i <= i_last; ++i) {
+                int sl = range_start(i, p.total, p.grid) >= tile_u0 ? 0 : 1;
+                const float *src = p.ws + ((size_t)i * 2 + sl) * p.BN * BM;
+                uint32_t dst = base + (uint32_t)(i - i_first) * (uint32_t)p.BN * BM * 4u;
+                asm volatile(
+                    "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], "
+                    "%2, [%3];" ::"r"(dst),
+                    "l"(src), "r"(part_bytes), "r"(su32(&fix_bar))
+                    : "memory");
+              }
+            }
+            mbar_wait(&fix_bar, fix_phase, abort_v, p.dev_flag, 32);
+            fix_phase ^= 1u;
+            const float *sp = (const float *)__cvta_shared_to_generic(base);
+            for (int c = 0; c < mv; c += 16) {
+              float v[16];
+#pragma unroll
+              for (int j = 0; j < 16; ++j) v[j] = 0.f;
+              for (int i = 0; i < parts; ++i) {
+                const float *q = sp + ((size_t)i * p.BN + c) * BM + f;
+#pragma unroll
+                for (int j = 0; j < 16; ++j)
+                  if (c + j < mv) v[j] += q[(size_t)j * BM];
+              }
+              epilogue16(p, t0 + c, n, v, mv - c);
+            }
+          } else {
           // 48 rows of one part per round trip: all their loads are in flight
           for (int c = 0; c < mv; c += 48) {
             float v[48];
@@ -429,6 +519,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
 #pragma unroll
             for (int q16 = 0; q16 < 3; ++q16)
               if (c + 16 * q16 < mv) epilogue16(p, t0 + c + 16 * q16, n, v + 16 * q16, mv - c - 16 * q16);
+          }
           }
           if (et == 0) p.counters[tl] = 0;
         }
@@ -530,6 +621,9 @@ const char *launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, v
   int smem_budget = max_dyn - 1024;
   p.stages = smem_budget / (int)stage_bytes;
   if (p.stages > 8) p.stages = 8;
+  // few-row tiles: 4 stages keep HBM streaming (as fast as 8 when measured)
+  // and leave room on the SM for the next kernel's CTA during the tail
+  if (p.BN <= 64 && p.stages > 4) p.stages = 4;
   if (p.stages < 2) return "token tile too large for shared memory";
   uint32_t cols = 32;
   while (cols < (uint32_t)p.BN) cols <<= 1;
@@ -558,7 +652,7 @@ const char *launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, v
     tmN = next->tm;
   }
   size_t smem = 1024 + (size_t)p.stages * stage_bytes;
-  k_gemm_tc<<<p.grid, NTHREADS, smem, s>>>(tmW, tmX, *tmN, p);
+  launch_pdl(k_gemm_tc, p.grid, NTHREADS, smem, s, tmW, tmX, *tmN, p);
   cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? nullptr : cudaGetErrorString(e);
 }

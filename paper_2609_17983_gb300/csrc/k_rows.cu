@@ -76,6 +76,8 @@ template <typename T>
 __global__ void k_embed_rows(const T *embed, const int32_t *tokens,
                              const int32_t *const *doc_tokens, const int32_t *rowdoc,
                              const int32_t *pos, int d, float *h) {
+  pdl_trigger();
+  pdl_wait();
   int i = blockIdx.x;
   const int32_t *tk = doc_tokens ? doc_tokens[rowdoc[i]] : tokens;
   size_t base = (size_t)tk[pos[i]] * d;
@@ -88,6 +90,8 @@ template <typename T>
 __global__ void __launch_bounds__(256) k_rmsnorm(const float *h, const float *g, int d, float eps,
                                                  T *out) {
   constexpr int NV = 8;  // float4 per thread: 8 * 4 * 256 = 8192 elements
+  pdl_trigger();
+  pdl_wait();
   int i = blockIdx.x;
   const float4 *x = (const float4 *)(h + (size_t)i * d);
   const int nq = d >> 2;
@@ -129,6 +133,8 @@ template <typename T>
 __global__ void k_rope_scatter(const float *qkv, const float2 *rope, const int32_t *pos, int H,
                                int G, int dh, int layer, const KVView *views,
                                const int32_t *rowdoc, KVView single, float *q_out, int write_kv) {
+  pdl_trigger();
+  pdl_wait();
   int i = blockIdx.x, hh = blockIdx.y, t = threadIdx.x, half = dh >> 1;
   int Nqkv = (H + 2 * G) * dh;
   int p = pos[i];
@@ -237,19 +243,21 @@ void launch_embed_rows(const void *embed, int dtype, const int32_t *tokens,
                        const int32_t *pos, int M, int d, float *h, cudaStream_t s) {
   if (M <= 0) return;
   if (dtype == KVR_DTYPE_BF16)
-    k_embed_rows<<<M, 256, 0, s>>>((const __nv_bfloat16 *)embed, tokens, doc_tokens, rowdoc, pos,
-                                   d, h);
+    launch_pdl(k_embed_rows<__nv_bfloat16>, M, 256, 0, s, (const __nv_bfloat16 *)embed, tokens,
+               doc_tokens, rowdoc, pos, d, h);
   else
-    k_embed_rows<<<M, 256, 0, s>>>((const float *)embed, tokens, doc_tokens, rowdoc, pos, d, h);
+    launch_pdl(k_embed_rows<float>, M, 256, 0, s, (const float *)embed, tokens, doc_tokens,
+               rowdoc, pos, d, h);
 }
 
 void launch_rmsnorm(const float *h, const float *g, int M, int d, double eps, void *out,
                     int out_dtype, cudaStream_t s) {
   if (M <= 0) return;
   if (out_dtype == KVR_DTYPE_BF16)
-    k_rmsnorm<<<M, 256, 0, s>>>(h, g, d, (float)eps, (__nv_bfloat16 *)out);
+    launch_pdl(k_rmsnorm<__nv_bfloat16>, M, 256, 0, s, h, g, d, (float)eps,
+               (__nv_bfloat16 *)out);
   else
-    k_rmsnorm<<<M, 256, 0, s>>>(h, g, d, (float)eps, (float *)out);
+    launch_pdl(k_rmsnorm<float>, M, 256, 0, s, h, g, d, (float)eps, (float *)out);
 }
 
 void launch_rope_scatter(const float *qkv, const float2 *rope, const int32_t *pos, int M,
@@ -257,12 +265,13 @@ void launch_rope_scatter(const float *qkv, const float2 *rope, const int32_t *po
                          KVView single, float *q_out, bool write_kv, cudaStream_t s) {
   if (M <= 0) return;
   dim3 grid(M, dm.H + 2 * dm.G);
+  int wk = write_kv ? 1 : 0;
   if (dm.dtype == KVR_DTYPE_BF16)
-    k_rope_scatter<__nv_bfloat16><<<grid, dm.dh / 2, 0, s>>>(
-        qkv, rope, pos, dm.H, dm.G, dm.dh, layer, views, rowdoc, single, q_out, write_kv);
+    launch_pdl(k_rope_scatter<__nv_bfloat16>, grid, dm.dh / 2, 0, s, qkv, rope, pos, dm.H, dm.G,
+               dm.dh, layer, views, rowdoc, single, q_out, wk);
   else
-    k_rope_scatter<float><<<grid, dm.dh / 2, 0, s>>>(qkv, rope, pos, dm.H, dm.G, dm.dh, layer,
-                                                     views, rowdoc, single, q_out, write_kv);
+    launch_pdl(k_rope_scatter<float>, grid, dm.dh / 2, 0, s, qkv, rope, pos, dm.H, dm.G, dm.dh,
+               layer, views, rowdoc, single, q_out, wk);
 }
 
 void launch_swiglu(const float *gu, int M, int F, void *act, int dtype, cudaStream_t s) {

@@ -152,6 +152,36 @@ struct kvr_cache {
 
 namespace kvr {
 
+// ---- programmatic dependent launch (PDL) ----
+// Kernels of a pass are launched with programmatic stream serialisation: a
+// kernel may start while its predecessor drains.  Every such kernel calls
+// pdl_trigger() on entry (its own successor may then be scheduled) and
+// pdl_wait() before it touches anything its predecessors write; pdl_wait()
+// returns once the predecessor grid has completed and its memory is visible.
+// Without the launch attribute both are no-ops.
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+extern bool g_pdl;  // launch with the PDL attribute (KVR_DISABLE_PDL=1 turns it off)
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t s, Args... args) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = g_pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
 // Message returned by kvr_last_error() on the calling thread.
 void set_last_error(const char *msg);
 
