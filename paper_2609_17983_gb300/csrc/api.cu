@@ -160,7 +160,7 @@ struct Rows {
   KVView single{};
   int max_pos = 0;                           // largest position among the rows
   const int4 *blocks = nullptr;              // attention query blocks (device)
-  int n_blocks = 0, n_splits = 1;
+  int n_blocks = 0, n_splits = 1, max_block_rows = 0;
 };
 
 bool use_tc_attention(const kvr_model *m) {
@@ -175,19 +175,20 @@ kvr_status plan_attention(kvr_model *m, Rows &r, const int32_t *pos, const int32
   const Dims &dm = m->dims;
   const int qb = attn_tc_rows_per_block(dm.H / dm.G);
   std::vector<int32_t> b;
-  int max_chunks = 0;
+  int max_chunks = 0, max_rows = 0;
   for (int i = 0; i < r.M;) {
     int doc = rowdoc ? rowdoc[i] : 0;
     int j = i;
     while (j < r.M && j - i < qb && (rowdoc ? rowdoc[j] : 0) == doc) ++j;
     int kmax = pos[j - 1];
+    max_rows = std::max(max_rows, j - i);
     b.insert(b.end(), {i, j - i, kmax, doc});
     max_chunks = std::max(max_chunks, kmax / KVR_PAGE + 1);
     i = j;
   }
   int nb = (int)b.size() / 4;
   if (nb > m->max_blocks) return fail(KVR_E_UNSUPPORTED, "too many attention blocks (%d)", nb);
-  int target = 2 * m->num_sms;
+  int target = m->num_sms;  // one CTA per SM (128 KB of shared memory each)
   int splits = std::max(1, (target + nb * dm.G - 1) / (nb * dm.G));
   splits = std::min(std::min(splits, max_chunks), 64);  // the combine merges <= 64 splits
   while (splits > 1 && attn_tc_ws_floats(splits, nb, dm.G, dm.dh) > m->attn_ws_floats) --splits;
@@ -195,6 +196,7 @@ kvr_status plan_attention(kvr_model *m, Rows &r, const int32_t *pos, const int32
   r.blocks = m->blocks_d;
   r.n_blocks = nb;
   r.n_splits = splits;
+  r.max_block_rows = max_rows;
   return KVR_OK;
 }
 
@@ -221,7 +223,9 @@ kvr_status layer_qkv(kvr_model *m, const Rows &r, int l, bool write_kv) {
   {
     Prof pr(m, P_ROPE, (int64_t)r.M * dm.Nqkv() * 4);
     launch_rope_scatter(m->qkv, m->rope, r.pos, r.M, dm, l, r.views, r.rowdoc, r.single, m->q,
-                        write_kv, m->stream);
+                        use_tc_attention(m) ? m->qb : nullptr,
+                        (float)(1.4426950408889634 / std::sqrt((double)dm.dh)), write_kv,
+                        m->stream);
     KVR_TRY(launch_check(m, 1));
   }
   return KVR_OK;
@@ -235,9 +239,9 @@ kvr_status layer_rest(kvr_model *m, const Rows &r, int l) {
     int64_t kv_bytes = (int64_t)(r.max_pos + 1) * dm.G * dm.dh * 2 * (int64_t)dm.es();
     Prof pr(m, P_ATTN, kv_bytes);
     if (use_tc_attention(m)) {
-      const char *e = launch_attention_tc(m->q, r.pos, r.blocks, r.n_blocks, r.n_splits, dm, l,
-                                          r.views, r.single, m->attn_ws_o, m->attn_ws_ml,
-                                          m->attn, m->stream);
+      const char *e = launch_attention_tc(m->qb, r.pos, r.blocks, r.n_blocks, r.max_block_rows,
+                                          r.n_splits, dm, l, r.views, r.single, m->attn_ws_o,
+                                          m->attn_ws_ml, m->attn, m->stream);
       if (e) return fail(KVR_E_CUDA, "attention: %s", e);
       KVR_TRY(launch_check(m, r.n_splits > 1 ? 2 : 1));
     } else {
@@ -641,14 +645,14 @@ kvr_status kvr_model_create(const kvr_model_config *cfg, const kvr_weights *wts,
     size_t R = dm.max_rows, P = dm.max_ctx + KVR_QUERY_RESERVE;
     size_t sz[] = {R * 4,          R * 4,          R * d * 4,        R * d * es,  R * Nq * 4,
                    R * HD * 4,     R * HD * es,    R * 2 * F * 4,    R * F * es,  V * 4,
-                   P * 4,          P * 8,          P * 4,            256};
+                   P * 4,          P * 8,          P * 4,            256,         R * HD * 2};
     size_t tot = 0;
     for (size_t x : sz) tot += al(x);
     m->ws_block = dev_alloc(tot);
     if (!m->ws_block) return bail(fail(KVR_E_NOMEM, "workspace: %zu bytes", tot));
     char *p = (char *)m->ws_block;
-    void *ptrs[14];
-    for (int i = 0; i < 14; ++i) {
+    void *ptrs[15];
+    for (int i = 0; i < 15; ++i) {
       ptrs[i] = p;
       p += al(sz[i]);
     }
@@ -666,6 +670,7 @@ kvr_status kvr_model_create(const kvr_model_config *cfg, const kvr_weights *wts,
     m->keys = (unsigned long long *)ptrs[11];
     m->sel_out = (int32_t *)ptrs[12];
     m->sel_count = (int32_t *)ptrs[13];
+    m->qb = ptrs[14];
     m->dev_flag = (int *)dev_alloc(256);
     if (!m->dev_flag) return bail(fail(KVR_E_NOMEM, "flag"));
     cudaMemset(m->dev_flag, 0, 256);

@@ -3,7 +3,8 @@
 // and unsplit for prefill-size passes.
 //
 // A CTA owns one query block -- consecutive rows of one document, times the
-// grp = H/G query heads that share KV head g, at most 128 query vectors -- and
+// grp = H/G query heads that share KV head g, at most 192 query vectors, one
+// warp per 16 -- and
 // a contiguous range of 64-key chunks (one KV page each).  It streams the K
 // and V pages of its range through double-buffered cp.async into XOR-swizzled
 // shared memory, computes S = Q K^T and O += P V with mma.sync m16n8k16 (bf16
@@ -23,13 +24,12 @@ namespace kvr {
 namespace {
 
 constexpr int CHUNK = KVR_PAGE;  // keys per chunk = one page
-constexpr int MAXQ = 128;        // query vectors per CTA (8 warps x 16)
-constexpr int NW = 8;
+constexpr int MAXW = 12;         // warps per CTA, 16 query vectors each
+constexpr int MAXQ = MAXW * 16;  // query vectors per CTA
 
 struct AttnTcParams {
-  const float *q;  // [M][H*dh] fp32, post-RoPE
+  const __nv_bfloat16 *q;  // [M][H*dh] post-RoPE, pre-scaled by log2(e)/sqrt(dh)
   int H, G, grp;
-  float qscale;  // log2(e) / sqrt(dh)
   const int32_t *pos;
   const int4 *blocks;  // (row0, nrows, kmax, doc)
   int layer;
@@ -89,7 +89,7 @@ __device__ __forceinline__ uint32_t swz(int r, int c) {
 }
 
 template <int DH>
-__global__ void __launch_bounds__(NW * 32, 2) k_attn_tc(const AttnTcParams p) {
+__global__ void __launch_bounds__(MAXW * 32, 1) k_attn_tc(const AttnTcParams p) {
   constexpr int NCH = DH / 8;        // 16-byte chunks per row
   constexpr int KT = DH / 16;        // k-steps of QK^T
   constexpr int OT = DH / 8;         // n-tiles of O
@@ -112,13 +112,14 @@ __global__ void __launch_bounds__(NW * 32, 2) k_attn_tc(const AttnTcParams p) {
   const int c0 = split * cps, c1 = min(n_chunks, c0 + cps);
   if (c0 >= c1) return;  // empty split: the combine skips it
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int nthr = blockDim.x, nq = blockDim.x >> 1;  // query vectors of this launch
   const __nv_bfloat16 *cache = (const __nv_bfloat16 *)kv.pages;
 
   auto load_chunk = [&](int c, int buf) {
     const __nv_bfloat16 *kp = cache + kv.offset(p.layer, 0, g, c * CHUNK);
     const __nv_bfloat16 *vp = cache + kv.offset(p.layer, 1, g, c * CHUNK);
     uint32_t kb = su32(sK + buf * TILE), vb = su32(sV + buf * TILE);
-    for (int e = tid; e < CHUNK * NCH; e += NW * 32) {
+    for (int e = tid; e < CHUNK * NCH; e += nthr) {
       int r = e / NCH, ch = e % NCH;
       cp_async16(kb + swz<DH>(r, ch), kp + r * DH + ch * 8);
       cp_async16(vb + swz<DH>(r, ch), vp + r * DH + ch * 8);
@@ -126,23 +127,22 @@ __global__ void __launch_bounds__(NW * 32, 2) k_attn_tc(const AttnTcParams p) {
     cp_commit();
   };
 
-  load_chunk(c0, 0);
-  // Q block -> bf16, scaled, swizzled; positions per query vector
-  for (int e = tid; e < MAXQ * NCH; e += NW * 32) {
-    int v = e / NCH, ch = e % NCH;
-    uint4 w = make_uint4(0, 0, 0, 0);
-    if (v < mq) {
-      int r = row0 + v / p.grp, hh = g * p.grp + v % p.grp;
-      const float4 *src = (const float4 *)(p.q + ((size_t)r * p.H + hh) * DH + ch * 8);
-      float4 x = src[0], y = src[1];
-      w.x = pack_bf16(x.x * p.qscale, x.y * p.qscale);
-      w.y = pack_bf16(x.z * p.qscale, x.w * p.qscale);
-      w.z = pack_bf16(y.x * p.qscale, y.y * p.qscale);
-      w.w = pack_bf16(y.z * p.qscale, y.w * p.qscale);
+  // Q block (bf16, already scaled) straight into swizzled shared memory,
+  // committed with the first chunk
+  {
+    const uint32_t qb = su32(sQ);
+    for (int e = tid; e < nq * NCH; e += nthr) {
+      int v = e / NCH, ch = e % NCH;
+      if (v < mq) {
+        int r = row0 + v / p.grp, hh = g * p.grp + v % p.grp;
+        cp_async16(qb + swz<DH>(v, ch), p.q + ((size_t)r * p.H + hh) * DH + ch * 8);
+      } else {
+        *(uint4 *)(sQ + swz<DH>(v, ch)) = make_uint4(0, 0, 0, 0);
+      }
     }
-    *(uint4 *)(sQ + swz<DH>(v, ch)) = w;
   }
-  for (int v = tid; v < MAXQ; v += NW * 32) spos[v] = v < mq ? p.pos[row0 + v / p.grp] : -1;
+  load_chunk(c0, 0);
+  for (int v = tid; v < nq; v += nthr) spos[v] = v < mq ? p.pos[row0 + v / p.grp] : -1;
 
   const bool active = warp * 16 < mq;
   const int v0 = warp * 16 + (lane >> 2), v1 = v0 + 8;
@@ -266,7 +266,7 @@ __global__ void __launch_bounds__(NW * 32, 2) k_attn_tc(const AttnTcParams p) {
   } else {
     // ws index: split-major, then (block, kv head) pair, then query vector
     const size_t bs = ((size_t)split * p.n_blocks + blk) * p.G + g;
-    float *wo = p.ws_o + bs * MAXQ * DH;
+    float *wo = p.ws_o + bs * MAXQ * DH;  // per (split, block, head): MAXQ x DH
 #pragma unroll
     for (int nt = 0; nt < OT; ++nt) {
       int d = 8 * nt + dcol;
@@ -341,8 +341,9 @@ __global__ void __launch_bounds__(256) k_attn_combine(const AttnTcParams p) {
 }
 
 template <int DH>
-const char *run(const AttnTcParams &p, cudaStream_t s) {
+const char *run(const AttnTcParams &p, int max_mq, cudaStream_t s) {
   constexpr int smem = MAXQ * DH * 2 + 4 * CHUNK * DH * 2;
+  const int warps = (max_mq + 15) / 16;
   static bool set = false;
   if (!set) {
     cudaError_t e = cudaFuncSetAttribute(k_attn_tc<DH>,
@@ -351,7 +352,7 @@ const char *run(const AttnTcParams &p, cudaStream_t s) {
     set = true;
   }
   dim3 grid(p.n_splits, p.G, p.n_blocks);
-  launch_pdl(k_attn_tc<DH>, grid, NW * 32, smem, s, p);
+  launch_pdl(k_attn_tc<DH>, grid, warps * 32, smem, s, p);
   if (p.n_splits > 1) {
     int warps = p.n_blocks * p.G * MAXQ;
     launch_pdl(k_attn_combine<DH>, (warps + 7) / 8, 256, 0, s, p);
@@ -368,17 +369,16 @@ size_t attn_tc_ws_floats(int n_splits, int n_blocks, int G, int dh) {
   return (size_t)n_splits * n_blocks * G * MAXQ * dh;
 }
 
-const char *launch_attention_tc(const float *q, const int32_t *pos, const int4 *blocks,
-                                int n_blocks, int n_splits, const Dims &dm, int layer,
-                                const KVView *views, KVView single, float *ws_o, float2 *ws_ml,
-                                void *out, cudaStream_t s) {
+const char *launch_attention_tc(const void *q, const int32_t *pos, const int4 *blocks,
+                                int n_blocks, int max_rows_per_block, int n_splits, const Dims &dm,
+                                int layer, const KVView *views, KVView single, float *ws_o,
+                                float2 *ws_ml, void *out, cudaStream_t s) {
   if (n_blocks <= 0) return nullptr;
   AttnTcParams p{};
-  p.q = q;
+  p.q = (const __nv_bfloat16 *)q;
   p.H = dm.H;
   p.G = dm.G;
   p.grp = dm.H / dm.G;
-  p.qscale = (float)(1.4426950408889634 / sqrt((double)dm.dh));
   p.pos = pos;
   p.blocks = blocks;
   p.layer = layer;
@@ -389,8 +389,9 @@ const char *launch_attention_tc(const float *q, const int32_t *pos, const int4 *
   p.ws_ml = ws_ml;
   p.n_blocks = n_blocks;
   p.out = (__nv_bfloat16 *)out;
-  if (dm.dh == 128) return run<128>(p, s);
-  if (dm.dh == 64) return run<64>(p, s);
+  const int max_mq = max_rows_per_block * p.grp;
+  if (dm.dh == 128) return run<128>(p, max_mq, s);
+  if (dm.dh == 64) return run<64>(p, max_mq, s);
   return "head_dim not supported";
 }
 

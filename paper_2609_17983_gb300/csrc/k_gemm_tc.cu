@@ -621,9 +621,6 @@ const char *launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, v
   int smem_budget = max_dyn - 1024;
   p.stages = smem_budget / (int)stage_bytes;
   if (p.stages > 8) p.stages = 8;
-  // few-row tiles: 4 stages keep HBM streaming (as fast as 8 when measured)
-  // and leave room on the SM for the next kernel's CTA during the tail
-  if (p.BN <= 64 && p.stages > 4) p.stages = 4;
   if (p.stages < 2) return "token tile too large for shared memory";
   uint32_t cols = 32;
   while (cols < (uint32_t)p.BN) cols <<= 1;

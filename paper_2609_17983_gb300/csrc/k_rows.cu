@@ -132,7 +132,8 @@ __global__ void __launch_bounds__(256) k_rmsnorm(const float *h, const float *g,
 template <typename T>
 __global__ void k_rope_scatter(const float *qkv, const float2 *rope, const int32_t *pos, int H,
                                int G, int dh, int layer, const KVView *views,
-                               const int32_t *rowdoc, KVView single, float *q_out, int write_kv) {
+                               const int32_t *rowdoc, KVView single, float *q_out,
+                               __nv_bfloat16 *qb_out, float qscale, int write_kv) {
   pdl_trigger();
   pdl_wait();
   int i = blockIdx.x, hh = blockIdx.y, t = threadIdx.x, half = dh >> 1;
@@ -151,6 +152,11 @@ __global__ void k_rope_scatter(const float *qkv, const float2 *rope, const int32
     float *qo = q_out + (size_t)i * H * dh + (size_t)hh * dh;
     qo[t] = x1;
     qo[t + half] = x2;
+    if (qb_out) {
+      __nv_bfloat16 *qb = qb_out + (size_t)i * H * dh + (size_t)hh * dh;
+      qb[t] = __float2bfloat16_rn(x1 * qscale);
+      qb[t + half] = __float2bfloat16_rn(x2 * qscale);
+    }
     return;
   }
   if (!write_kv) return;
@@ -262,16 +268,17 @@ void launch_rmsnorm(const float *h, const float *g, int M, int d, double eps, vo
 
 void launch_rope_scatter(const float *qkv, const float2 *rope, const int32_t *pos, int M,
                          const Dims &dm, int layer, const KVView *views, const int32_t *rowdoc,
-                         KVView single, float *q_out, bool write_kv, cudaStream_t s) {
+                         KVView single, float *q_out, void *qb_out, float qscale, bool write_kv,
+                         cudaStream_t s) {
   if (M <= 0) return;
   dim3 grid(M, dm.H + 2 * dm.G);
   int wk = write_kv ? 1 : 0;
   if (dm.dtype == KVR_DTYPE_BF16)
     launch_pdl(k_rope_scatter<__nv_bfloat16>, grid, dm.dh / 2, 0, s, qkv, rope, pos, dm.H, dm.G,
-               dm.dh, layer, views, rowdoc, single, q_out, wk);
+               dm.dh, layer, views, rowdoc, single, q_out, (__nv_bfloat16 *)qb_out, qscale, wk);
   else
     launch_pdl(k_rope_scatter<float>, grid, dm.dh / 2, 0, s, qkv, rope, pos, dm.H, dm.G, dm.dh,
-               layer, views, rowdoc, single, q_out, wk);
+               layer, views, rowdoc, single, q_out, (__nv_bfloat16 *)qb_out, qscale, wk);
 }
 
 void launch_swiglu(const float *gu, int M, int F, void *act, int dtype, cudaStream_t s) {

@@ -111,6 +111,7 @@ struct kvr_model {
   int32_t *pos_d = nullptr;  // [R] positions of the rows of a pass
   int32_t *rowdoc_d = nullptr;  // [R] batch: document of each row
   float *h = nullptr, *qkv = nullptr, *q = nullptr, *gu = nullptr, *logits = nullptr;
+  void *qb = nullptr;  // bf16 scaled q for the tensor-core attention
   void *a = nullptr, *attn = nullptr, *act = nullptr;
   float *scores = nullptr;     // [max_ctx + reserve] selector scores
   unsigned long long *keys = nullptr;  // [max_ctx + reserve] top-K keys
@@ -206,9 +207,11 @@ void launch_embed_rows(const void *embed, int dtype, const int32_t *tokens,
                        const int32_t *pos, int M, int d, float *h, cudaStream_t s);
 void launch_rmsnorm(const float *h, const float *g, int M, int d, double eps, void *out,
                     int out_dtype, cudaStream_t s);
+// q_out: fp32 rotated q; qb_out (optional): bf16 rotated q times qscale.
 void launch_rope_scatter(const float *qkv, const float2 *rope, const int32_t *pos, int M,
                          const Dims &dm, int layer, const KVView *views, const int32_t *rowdoc,
-                         KVView single, float *q_out, bool write_kv, cudaStream_t s);
+                         KVView single, float *q_out, void *qb_out, float qscale, bool write_kv,
+                         cudaStream_t s);
 void launch_swiglu(const float *gu, int M, int F, void *act, int dtype, cudaStream_t s);
 void launch_cache_gather(KVView v, int dtype, const int32_t *pos, int n_pos, int l0, int l1,
                          int G, int dh, float *k_out, float *v_out, cudaStream_t s);
@@ -262,10 +265,11 @@ void launch_attention_simt(const float *q, const int32_t *pos, int M, const Dims
 // chunks (ws_o/ws_ml hold the partials when n_splits > 1).
 int attn_tc_rows_per_block(int grp);
 size_t attn_tc_ws_floats(int n_splits, int n_blocks, int G, int dh);
-const char *launch_attention_tc(const float *q, const int32_t *pos, const int4 *blocks,
-                                int n_blocks, int n_splits, const Dims &dm, int layer,
-                                const KVView *views, KVView single, float *ws_o, float2 *ws_ml,
-                                void *out, cudaStream_t s);
+// q: bf16 [M][H*dh], rotated and scaled by log2(e)/sqrt(dh).
+const char *launch_attention_tc(const void *q, const int32_t *pos, const int4 *blocks,
+                                int n_blocks, int max_rows_per_block, int n_splits, const Dims &dm,
+                                int layer, const KVView *views, KVView single, float *ws_o,
+                                float2 *ws_ml, void *out, cudaStream_t s);
 
 // ---- kernels: selectors ----
 void launch_scores_simple(int policy, const int32_t *tokens, int n, int s_end, int delim,
