@@ -374,3 +374,24 @@ def test_graph_replay_matches_eager():
         assert np.array_equal(k1, k2) and np.array_equal(v1, v2)
     eager.close()
     graph.close()
+
+
+@pytest.mark.parametrize("shape,policy", [("qwen7b", "attention"), ("mistral7b", "cacheblend"),
+                                          ("llama8b", "attention")])
+def test_8b_shape_model_selectors_parity(shape, policy):
+    # the two model-based selectors at the paper's model shapes (2 layers,
+    # a pool of ~200 positions: several tiles and a ragged tail)
+    cfg = synth.preset(shape, n_layers=2)
+    n, s, L, K = 320, 100, 6, 32
+    doc = synth.document(4, n, cfg["vocab"], cfg["delim_id"])
+    new = synth.edit_tokens(5, doc[s:s + L], cfg["vocab"], cfg["delim_id"])
+    vs = np.array([0, 1], np.int64)
+    model = kv.Model(cfg, None, seed=0, max_context=512, max_rows=256)
+    cache = model.prefill(doc)
+    got = model.select(cache, policy, K, s, new)
+    ocfg, W, (odoc, onew) = compact_inputs(cfg, 0, [doc, new], vs)
+    stale = oracle.prefill(ocfg, W, odoc)
+    sc, D = oracle.scores(ocfg, W, stale, policy, s, onew)
+    ref = oracle.topk(sc, D, K)
+    check_selection(got, ref, sc, 2e-2 * np.abs(sc[D]).max())
+    model.close()
