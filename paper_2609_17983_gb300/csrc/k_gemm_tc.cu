@@ -17,6 +17,14 @@
 // arriver sums the parts in CTA order, so the result is deterministic.  No CTA
 // ever waits for another.
 //
+// Few-row GEMMs whose tiles cannot fill the GPU (e.g. O with 32 tiles) run
+// in cluster split-K mode instead: the P CTAs of a thread-block cluster
+// share one tile, each owning K/P of it; at the end each stages its partial
+// tile in shared memory and, after a cluster barrier, sums its share of the
+// rows over all P partials through distributed shared memory (rank order,
+// deterministic) and applies the epilogue.  No global partials, fences or
+// atomics on the tail.
+//
 // Warp roles (192 threads): warp 0 issues TMA loads (one elected lane), warp 1
 // issues tcgen05.mma (one elected lane), warps 2-5 drain TMEM and run the
 // epilogue.  Accumulators are double-buffered in TMEM so the MMA warp starts
@@ -25,6 +33,8 @@
 // Every mbarrier wait is bounded: a wait that runs out sets the device error
 // flag and an abort flag in shared memory; all roles then stop issuing work,
 // wait (bounded) for their copies and MMAs in flight, free TMEM and return.
+#include <cooperative_groups.h>
+#include <cstdlib>
 #include <cuda.h>
 
 #include "kvr_internal.cuh"
@@ -56,9 +66,10 @@ struct TcParams {
   int *counters;    // [n_tiles * m_tiles] arrival counters (self-resetting)
   int *dev_flag;
   // L2 prefetch of the next GEMM's weights: CTA i prefetches the first
-  // pf_units units of its own range in the next GEMM's stream-K split
+  // pf_units units of its own range in the next GEMM's split
   long long next_total;
-  int next_KB, next_m_tiles, next_grid, pf_units;
+  int next_KB, next_m_tiles, next_grid, pf_units, next_cluster;
+  int cluster;  // > 1: cluster split-K with this many CTAs per tile
 };
 
 // ------------------------------------------------------------ PTX wrappers
@@ -200,6 +211,19 @@ __device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: 
 __device__ __forceinline__ long long range_start(long long i, long long total, int grid) {
   return i * total / grid;
 }
+// Units [a, b) of CTA i: stream-K ranges, or K/P of tile i/P in cluster mode
+__device__ __forceinline__ void unit_range(long long i, long long total, int grid, int KB,
+                                           int cluster, long long &a, long long &b) {
+  if (cluster > 1) {
+    long long tile = i / cluster, r = i % cluster;
+    a = tile * KB + r * KB / cluster;
+    b = tile * KB + (r + 1) * KB / cluster;
+  } else {
+    a = range_start(i, total, grid);
+    b = range_start(i + 1, total, grid);
+  }
+}
+
 // CTA whose range holds unit u
 __device__ __forceinline__ int cta_of(long long u, long long total, int grid) {
   return (int)(((u + 1) * grid - 1) / total);
@@ -247,7 +271,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
               const __grid_constant__ CUtensorMap tmNext, const TcParams p) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[8], empty_bar[8], accf_bar[2], acce_bar[2],
-      drain_bar, fix_bar;
+      drain_bar;
   __shared__ uint32_t tmem_slot;
   __shared__ int abort_f;
   __shared__ int last_f;
@@ -258,8 +282,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
   const uint32_t base = (su32(smem_raw) + 1023u) & ~1023u;
   const uint32_t stage_bytes = A_BYTES + (uint32_t)p.BN * 128u;
   const uint32_t tx_bytes = A_BYTES + (uint32_t)p.brows * 128u;
-  const long long u0 = range_start(blockIdx.x, p.total, p.grid);
-  const long long u1 = range_start(blockIdx.x + 1, p.total, p.grid);
+  long long u0, u1;
+  unit_range(blockIdx.x, p.total, p.grid, p.KB, p.cluster, u0, u1);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
@@ -271,7 +295,6 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       mbar_init(&acce_bar[b], 128);
     }
     mbar_init(&drain_bar, 1);
-    mbar_init(&fix_bar, 1);
     abort_f = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -366,8 +389,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       }
       // warm L2 with the start of this CTA's share of the next GEMM's weights
       if (p.pf_units > 0 && (int)blockIdx.x < p.next_grid && !*abort_v) {
-        long long nu0 = range_start(blockIdx.x, p.next_total, p.next_grid);
-        long long nu1 = range_start(blockIdx.x + 1, p.next_total, p.next_grid);
+        long long nu0, nu1;
+        unit_range(blockIdx.x, p.next_total, p.next_grid, p.next_KB, p.next_cluster, nu0, nu1);
         if (nu1 > nu0 + p.pf_units) nu1 = nu0 + p.pf_units;
         for (long long u = nu0; u < nu1; ++u) {
           long long tl = u / p.next_KB;
@@ -425,8 +448,26 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     const int q = warp & 3;  // TMEM lane quarter of this warp
     const int f = q * 32 + lane;
     const int et = threadIdx.x - 64;  // 0..127
-    uint32_t seg = 0, fix_phase = 0;
-    for (long long a = u0; a < u1;) {
+    uint32_t seg = 0;
+    if (p.cluster > 1) {
+      // stage this CTA's partial tile [mv][128] in shared memory (the
+      // pipeline stages are free: every TMA load was consumed by the MMAs)
+      if (mbar_wait(&accf_bar[0], 0, abort_v, p.dev_flag, 8)) {
+        tc_fence_after();
+        const int mv = min(p.BN, p.M);
+        float *sp = (float *)__cvta_shared_to_generic(base);
+        uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16);
+        for (int c = 0; c < mv; c += 16) {
+          float v[16];
+          tmem_ld16(taddr + c, v);
+#pragma unroll
+          for (int j = 0; j < 16; ++j)
+            if (c + j < mv) sp[(c + j) * BM + f] = v[j];
+        }
+      }
+      tc_fence_before();
+    }
+    for (long long a = u0; a < u1 && p.cluster <= 1;) {
       long long tl = a / p.KB;
       long long b = (tl + 1) * p.KB < u1 ? (tl + 1) * p.KB : u1;
       uint32_t buf = seg & 1u, use = seg >> 1;
@@ -467,41 +508,6 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         epi_bar();
         if (last_f) {
           __threadfence();
-          const uint32_t part_bytes = (uint32_t)mv * BM * 4u;
-          if (b == u1 && (uint32_t)parts * (uint32_t)p.BN * BM * 4u <= (uint32_t)S * stage_bytes) {
-            // Final segment of this CTA: every pipeline stage is free.  One
-            // thread fetches all parts with bulk copies into shared memory,
-            // then the warps sum them in part order.
-            if (et == 0) {
-              asm volatile("fence.proxy.async.global;" ::: "memory");
-              mbar_expect_tx(&fix_bar, part_bytes * parts);
-              for (int i = i_first; i <= i_last; ++i) {
-                int sl = range_start(i, p.total, p.grid) >= tile_u0 ? 0 : 1;
-                const float *src = p.ws + ((size_t)i * 2 + sl) * p.BN * BM;
-                uint32_t dst = base + (uint32_t)(i - i_first) * (uint32_t)p.BN * BM * 4u;
-                asm volatile(
-                    "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], "
-                    "%2, [%3];" ::"r"(dst),
-                    "l"(src), "r"(part_bytes), "r"(su32(&fix_bar))
-                    : "memory");
-              }
-            }
-            mbar_wait(&fix_bar, fix_phase, abort_v, p.dev_flag, 32);
-            fix_phase ^= 1u;
-            const float *sp = (const float *)__cvta_shared_to_generic(base);
-            for (int c = 0; c < mv; c += 16) {
-              float v[16];
-#pragma unroll
-              for (int j = 0; j < 16; ++j) v[j] = 0.f;
-              for (int i = 0; i < parts; ++i) {
-                const float *q = sp + ((size_t)i * p.BN + c) * BM + f;
-#pragma unroll
-                for (int j = 0; j < 16; ++j)
-                  if (c + j < mv) v[j] += q[(size_t)j * BM];
-              }
-              epilogue16(p, t0 + c, n, v, mv - c);
-            }
-          } else {
           // 48 rows of one part per round trip: all their loads are in flight
           for (int c = 0; c < mv; c += 48) {
             float v[48];
@@ -520,7 +526,6 @@ __global__ void __launch_bounds__(NTHREADS, 1)
             for (int q16 = 0; q16 < 3; ++q16)
               if (c + 16 * q16 < mv) epilogue16(p, t0 + c + 16 * q16, n, v + 16 * q16, mv - c - 16 * q16);
           }
-          }
           if (et == 0) p.counters[tl] = 0;
         }
         epi_bar();
@@ -531,6 +536,32 @@ __global__ void __launch_bounds__(NTHREADS, 1)
   }
   tc_fence_before();
   __syncthreads();
+  if (p.cluster > 1) {
+    // every CTA of the cluster reaches both barriers, on every path
+    cooperative_groups::cluster_group cl = cooperative_groups::this_cluster();
+    cl.sync();  // all partials staged
+    if (warp >= 2) {
+      const int P = p.cluster, rank = (int)cl.block_rank();
+      const int mv = min(p.BN, p.M);
+      const int r0 = rank * mv / P, r1 = (rank + 1) * mv / P;
+      const int f = (warp & 3) * 32 + lane;
+      const int n = (int)(blockIdx.x / P) * BM + f;
+      float *local = (float *)__cvta_shared_to_generic(base);
+      for (int c = r0; c < r1; c += 16) {
+        float v[16];
+#pragma unroll
+        for (int j = 0; j < 16; ++j) v[j] = 0.f;
+        for (int qr = 0; qr < P; ++qr) {
+          const float *rp = cl.map_shared_rank(local, qr);
+#pragma unroll
+          for (int j = 0; j < 16; ++j)
+            if (c + j < r1) v[j] += rp[(c + j) * BM + f];
+        }
+        epilogue16(p, c, n, v, r1 - c);
+      }
+    }
+    cl.sync();  // peers have finished reading this CTA's shared memory
+  }
   tc_fence_after();
   if (warp == 0) {
     uint32_t ncols = 2 * p.tmem_cols;
@@ -577,6 +608,51 @@ bool make_tmap_bf16(CUtensorMap *map, const void *ptr, int rows, int cols, int b
 }
 
 bool gemm_tc_supported(int N, int K) { return N % BM == 0 && K % BK == 0 && N > 0 && K > 0; }
+
+namespace {
+// Cluster split-K width for a few-row GEMM whose n_tiles cannot fill the
+// SMs: the largest P <= 8 with n_tiles * P <= #SMs, used when it covers at
+// least 3/4 of the SMs and all clusters fit in one wave; else 0 (stream-K).
+int choose_cluster(int M, int N, int num_sms, size_t smem) {
+  static const bool off = [] {
+    const char *e = getenv("KVR_DISABLE_CLUSTER_SPLITK");
+    return e && e[0] == '1';
+  }();
+  if (off || M > 64) return 0;
+  int T = N / BM;
+  int P = num_sms / T;
+  if (P > 8) P = 8;
+  if (P < 2 || T * P * 4 < num_sms * 3) return 0;
+  static int cache_p[16] = {0}, cache_ok[16] = {0};
+  static size_t cache_smem[16] = {0};
+  for (int i = 0; i < 16; ++i)
+    if (cache_p[i] == P && cache_smem[i] == smem) return cache_ok[i] >= T ? P : 0;
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(T * P);
+  cfg.blockDim = dim3(NTHREADS);
+  cfg.dynamicSmemBytes = smem;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeClusterDimension;
+  at[0].val.clusterDim.x = P;
+  at[0].val.clusterDim.y = 1;
+  at[0].val.clusterDim.z = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  int nc = 0;
+  if (cudaOccupancyMaxActiveClusters(&nc, (void *)k_gemm_tc, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    nc = 0;
+  }
+  for (int i = 0; i < 16; ++i)
+    if (cache_p[i] == 0) {
+      cache_p[i] = P;
+      cache_smem[i] = smem;
+      cache_ok[i] = nc;
+      break;
+    }
+  return nc >= T ? P : 0;
+}
+}  // namespace
 
 int gemm_tc_bn(int M) {
   if (M > 256) return 256;
@@ -637,6 +713,9 @@ const char *launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, v
   if ((long long)p.n_tiles * p.m_tiles > ws.max_tiles) return "more tiles than counters";
   CUtensorMap tmX;
   if (!make_tmap_bf16(&tmX, g.X, g.M, g.K, p.brows)) return "activation TMA descriptor rejected";
+  size_t smem = 1024 + (size_t)p.stages * stage_bytes;
+  p.cluster = p.m_tiles == 1 ? choose_cluster(g.M, g.N, ws.num_sms, smem) : 0;
+  if (p.cluster > 1) p.grid = p.n_tiles * p.cluster;
   const CUtensorMap *tmN = &tmW;
   if (next && next->tm && next->bytes_per_cta > 0) {
     int nbn = gemm_tc_bn(next->M);
@@ -645,11 +724,33 @@ const char *launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, v
     p.next_m_tiles = (int)nm;
     p.next_total = (long long)(next->N / BM) * nm * p.next_KB;
     p.next_grid = (int)(p.next_total < ws.num_sms ? p.next_total : ws.num_sms);
+    p.next_cluster = nm == 1 ? choose_cluster(next->M, next->N, ws.num_sms, smem) : 0;
+    if (p.next_cluster > 1) p.next_grid = (next->N / BM) * p.next_cluster;
     p.pf_units = (int)(next->bytes_per_cta / A_BYTES);
     tmN = next->tm;
   }
-  size_t smem = 1024 + (size_t)p.stages * stage_bytes;
-  launch_pdl(k_gemm_tc, p.grid, NTHREADS, smem, s, tmW, tmX, *tmN, p);
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(p.grid);
+  cfg.blockDim = dim3(NTHREADS);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute at[2];
+  int na = 0;
+  if (g_pdl) {
+    at[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[na].val.programmaticStreamSerializationAllowed = 1;
+    ++na;
+  }
+  if (p.cluster > 1) {
+    at[na].id = cudaLaunchAttributeClusterDimension;
+    at[na].val.clusterDim.x = p.cluster;
+    at[na].val.clusterDim.y = 1;
+    at[na].val.clusterDim.z = 1;
+    ++na;
+  }
+  cfg.attrs = at;
+  cfg.numAttrs = na;
+  cudaLaunchKernelEx(&cfg, k_gemm_tc, tmW, tmX, *tmN, p);
   cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? nullptr : cudaGetErrorString(e);
 }
