@@ -17,7 +17,8 @@
  *   - Token, position and output arrays are HOST pointers (int32 / float),
  *     owned by the caller and only read/written during the call.
  *   - Model and cache handles are owned by the library and freed with
- *     kvr_model_free / kvr_cache_free.  A cache must be freed before its model.
+ *     kvr_model_free / kvr_cache_free.  kvr_model_free also frees every
+ *     cache of the model still live; their handles are invalid afterwards.
  *   - Device work is enqueued on the model's stream (kvr_model_set_stream;
  *     default: the legacy default stream).  Calls that return data to the host
  *     (kvr_select, kvr_logits, kvr_cache_read*) synchronise that stream;
@@ -59,7 +60,12 @@ typedef enum {
   KVR_POLICY_STRUCTURAL = 1, /* delimiter tokens, nearest to the span first */
   KVR_POLICY_ATTENTION = 2,  /* top-K stale-cache attention from the span queries */
   KVR_POLICY_CACHEBLEND = 3, /* top-K layer-1 (0-indexed) K/V deviation */
-  KVR_POLICY_RANDOM = 4      /* uniform K-subset, seeded */
+  KVR_POLICY_RANDOM = 4,     /* uniform K-subset, seeded */
+  /* EditLocal@boundary (Sec. 5.2): the positions from the span end through
+   * the next document boundary (the first delimiter token at or after
+   * edit_end, inclusive; the end of the context if there is none), with no
+   * selector forward; K caps the window. */
+  KVR_POLICY_EDITLOCAL_BOUNDARY = 5
 } kvr_policy;
 
 /* Llama-style decoder shape (RMSNorm, rotate-half RoPE, GQA, SwiGLU). */
@@ -163,6 +169,29 @@ typedef struct {
  * layer-major pass over all rows of all requests.  All caches belong to
  * `model`.  Sum of |P_doc| <= max_rows. */
 kvr_status kvr_repair_batch(kvr_model *model, const kvr_repair_req *reqs, int32_t n_reqs);
+
+/* Transplant (Sec. 3, "Transplant is not recomputation"): copy the K/V of
+ * every layer, and the token, at the given positions from `src` into `dst`
+ * -- e.g. from a fresh prefill of the edited context into the stale cache.
+ * A diagnostic operator: it needs the oracle cache, so it is not a repair.
+ * Both caches belong to one model and hold the same number of positions;
+ * positions: host int32[n_positions], strictly increasing, in [0, n).
+ * Asynchronous on the model's stream.  Errors: KVR_E_INVAL, KVR_E_RANGE. */
+kvr_status kvr_transplant(kvr_cache *dst, const kvr_cache *src, const int32_t *positions,
+                          int32_t n_positions);
+
+/* Teacher-forced answer log-probability for the margin of Eq. 2: the prompt
+ * (m_prompt >= 1 tokens) and the answer (m_answer >= 1 tokens) follow the
+ * cached context at positions n.., the answer fed one token behind (teacher
+ * forcing); *mean_logprob_out = (1/m_answer) sum_i log p(answer_i | context,
+ * prompt, answer_<i) under the cache's K/V, length-averaged as Eq. 2
+ * prescribes.  The document's K/V are not modified.  m_prompt + m_answer - 1
+ * <= 64.  The margin m_x of a cache state is the difference of this value for
+ * a_new and a_old; MR (Eq. 2) follows from m of the repaired, stale and
+ * oracle caches. */
+kvr_status kvr_answer_logprob(kvr_model *model, const kvr_cache *cache, const int32_t *prompt,
+                              int32_t m_prompt, const int32_t *answer, int32_t m_answer,
+                              double *mean_logprob_out);
 
 /* Fresh-query logits (Sec. 3: the fresh query is never cached and is
  * recomputed for scoring).  The m query tokens (1 <= m <= 64) take positions

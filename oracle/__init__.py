@@ -23,6 +23,9 @@ Pin status (what each function is checked against, in tests/test_oracle_*.py):
                           invariance, split-call and idempotence.
   logits               -- the same textbook decoder run over C' + query.
   editlocal/structural -- closed forms and hand-written golden cases.
+  editlocal_boundary   -- hand-written golden case.
+  logits_all / answer_logprob -- the textbook decoder run over C' + query.
+  transplant           -- identity (all positions) and no-op (none) cases.
   random               -- published SplitMix64 test vectors, uniformity.
   attention score      -- special cases: zero W_q gives uniform scores (ties ->
                           EditLocal set); the scores sum to layers*heads*|S|.
@@ -108,8 +111,10 @@ def _load():
             lib.orc_score_cacheblend.argtypes = common + [ctypes.c_int, P, ctypes.c_int,
                                                           ctypes.c_int, P]
             lib.orc_logits.argtypes = common + [ctypes.c_int, P, ctypes.c_int, P]
+            lib.orc_logits_all.argtypes = common + [ctypes.c_int, P, ctypes.c_int, P]
             for f in (lib.orc_recompute, lib.orc_recompute_token_major,
-                      lib.orc_score_attention, lib.orc_score_cacheblend, lib.orc_logits):
+                      lib.orc_score_attention, lib.orc_score_cacheblend, lib.orc_logits,
+                      lib.orc_logits_all):
                 f.restype = ctypes.c_int
             _lib = lib
     return _lib
@@ -282,9 +287,61 @@ def logits(cfg, W, cache: Cache, query) -> np.ndarray:
     return out
 
 
+def logits_all(cfg, W, cache: Cache, query) -> np.ndarray:
+    """Logits [m, vocab] of every query row (positions n..n+m-1)."""
+    lib = _load()
+    query = np.asarray(query, np.int32)
+    n, m = cache.n, int(query.shape[0])
+    work = cache.copy(cap=n + m)
+    toks = np.concatenate([cache.tokens, query]).astype(np.int32)
+    out = np.zeros((m, cfg["vocab"]), np.float64)
+    wh = _WeightsHandle(cfg, W)
+    c = _cfg_struct(cfg)
+    _check(lib.orc_logits_all(ctypes.byref(c), ctypes.byref(wh.s), work.k.ctypes.data,
+                              work.v.ctypes.data, n + m, n, toks.ctypes.data, m,
+                              out.ctypes.data), "logits_all")
+    return out
+
+
+def answer_logprob(cfg, W, cache: Cache, prompt, answer) -> float:
+    """Length-averaged teacher-forced log-probability of `answer` after the
+    cached context and `prompt` (the quantity whose a_new - a_old difference
+    is the margin m_x of Eq. 2)."""
+    prompt = np.asarray(prompt, np.int32)
+    answer = np.asarray(answer, np.int32)
+    feed = np.concatenate([prompt, answer[:-1]])
+    lg = logits_all(cfg, W, cache, feed)[len(prompt) - 1:]
+    mx = lg.max(axis=1, keepdims=True)
+    lse = mx[:, 0] + np.log(np.exp(lg - mx).sum(axis=1))
+    return float(np.mean(lg[np.arange(len(answer)), answer] - lse))
+
+
+def margin(cfg, W, cache: Cache, prompt, a_new, a_old) -> float:
+    """m_x (Eq. 2): answer log-probability of a_new minus that of a_old."""
+    return answer_logprob(cfg, W, cache, prompt, a_new) - answer_logprob(cfg, W, cache, prompt,
+                                                                          a_old)
+
+
+def margin_recovery(m_repaired: float, m_stale: float, m_oracle: float) -> float:
+    """MR (Eq. 2): (m_repaired - m_stale) / (m_oracle - m_stale), unclipped."""
+    return (m_repaired - m_stale) / (m_oracle - m_stale)
+
+
+def transplant(dst: Cache, src: Cache, positions) -> Cache:
+    """Transplant (Sec. 3): a copy of dst whose K/V of every layer and token
+    at `positions` come from src."""
+    positions = np.asarray(positions, np.int64)
+    out = dst.copy()
+    out.k[:, positions] = src.k[:, positions]
+    out.v[:, positions] = src.v[:, positions]
+    out.tokens[positions] = src.tokens[positions]
+    return out
+
+
 # ------------------------------------------------------------------ selectors
 
-POLICIES = ("editlocal", "structural", "attention", "cacheblend", "random")
+POLICIES = ("editlocal", "structural", "attention", "cacheblend", "random",
+            "editlocal_boundary")
 
 
 def pool(n: int, edit_start: int, edit_len: int) -> np.ndarray:
@@ -334,6 +391,14 @@ def scores(cfg, W, cache: Cache, policy: str, edit_start: int, new_tokens, seed:
         return {int(j): -float(j - s_end) for j in elig}, elig
     if policy == "random":
         return {int(j): splitmix64(seed ^ ((int(j) * GOLDEN) & MASK64)) for j in D}, D
+    if policy == "editlocal_boundary":
+        # Sec. 5.2: through the next document boundary (first delimiter at or
+        # after the span end, inclusive; the context end if there is none)
+        delim = cfg["delim_id"]
+        hits = [int(j) for j in D if toks[j] == delim]
+        b = hits[0] if hits else n - 1
+        elig = np.arange(s_end, b + 1, dtype=np.int64)
+        return {int(j): -float(j - s_end) for j in elig}, elig
     if policy in ("attention", "cacheblend"):
         lib = _load()
         work = cache.copy()

@@ -474,6 +474,34 @@ done:
   return rc;
 }
 
+/* Logits of every row of a fresh query: rows n..n+m-1 of `tokens` attend
+ * to the caller's copy of the cache (cap >= n+m); logits [m][vocab] =
+ * lm_head RMSNorm(h_row).  Used for teacher-forced answer scoring (Eq. 2). */
+int orc_logits_all(const orc_config *c, const orc_weights *w, float *kc, float *vc, int cap,
+                   int n, const int32_t *tokens, int m, double *logits) {
+  if (m <= 0 || n < 0 || n + m > cap) return ORC_EINVAL;
+  int d = c->d_model;
+  int64_t *pos = malloc(sizeof(int64_t) * (size_t)m);
+  double *h = malloc(sizeof(double) * (size_t)m * d);
+  double *a = malloc(sizeof(double) * (size_t)m * d);
+  int rc = ORC_OK;
+  if (!pos || !h || !a) {
+    rc = ORC_ENOMEM;
+    goto done;
+  }
+  for (int r = 0; r < m; ++r) pos[r] = n + r;
+  rc = orc_recompute(c, w, kc, vc, cap, tokens, pos, m, h);
+  if (rc) goto done;
+  for (int r = 0; r < m; ++r)
+    rmsnorm(h + (size_t)r * d, w->final_norm, c->wdtype, d, c->rms_eps, a + (size_t)r * d);
+  linear_rows(a, m, d, w->lm_head, NULL, c->wdtype, c->vocab, logits);
+done:
+  free(pos);
+  free(h);
+  free(a);
+  return rc;
+}
+
 /* Fresh-query logits (Sec. 3: the fresh query is never cached and is
  * recomputed for scoring).  The m query tokens sit at positions n..n+m-1;
  * their k, v go into the caller's copy of the cache (cap >= n+m) and never

@@ -460,6 +460,7 @@ void kvr_model_free(kvr_model *m) {
   if (!m) return;
   cudaSetDevice(m->device);
   cudaStreamSynchronize(m->stream);
+  while (!m->caches.empty()) kvr_cache_free(m->caches.back());
   prof_collect(m);
   dev_free(m->weight_block);
   dev_free(m->ws_block);
@@ -644,7 +645,8 @@ kvr_status kvr_model_create(const kvr_model_config *cfg, const kvr_weights *wts,
   {
     size_t R = dm.max_rows, P = dm.max_ctx + KVR_QUERY_RESERVE;
     size_t sz[] = {R * 4,          R * 4,          R * d * 4,        R * d * es,  R * Nq * 4,
-                   R * HD * 4,     R * HD * es,    R * 2 * F * 4,    R * F * es,  V * 4,
+                   R * HD * 4,     R * HD * es,    R * 2 * F * 4,    R * F * es,
+                   (size_t)KVR_QUERY_RESERVE * V * 4,
                    P * 4,          P * 8,          P * 4,            256,         R * HD * 2};
     size_t tot = 0;
     for (size_t x : sz) tot += al(x);
@@ -739,6 +741,12 @@ void kvr_cache_free(kvr_cache *c) {
   cudaSetDevice(c->model->device);
   cudaStreamSynchronize(c->model->stream);
   for (auto &g : c->graphs) cudaGraphExecDestroy(g.exec);
+  auto &live = c->model->caches;
+  for (size_t i = 0; i < live.size(); ++i)
+    if (live[i] == c) {
+      live.erase(live.begin() + i);
+      break;
+    }
   dev_free(c->pages);
   dev_free(c->table);
   dev_free(c->tokens_d);
@@ -758,6 +766,7 @@ kvr_status kvr_prefill(kvr_model *m, const int32_t *tokens, int32_t n, kvr_cache
   KVR_TRY(use_device(m));
   kvr_cache *c = new kvr_cache();
   c->model = m;
+  m->caches.push_back(c);
   c->n = n;
   c->cap = (n + KVR_QUERY_RESERVE + KVR_PAGE - 1) / KVR_PAGE * KVR_PAGE;
   c->n_pages = c->cap / KVR_PAGE;
@@ -1000,7 +1009,7 @@ kvr_status kvr_select(kvr_model *m, const kvr_cache *c, kvr_policy policy, int32
   for (int i = 0; i < edit_len; ++i)
     if (new_tokens[i] < 0 || new_tokens[i] >= dm.V)
       return fail(KVR_E_RANGE, "new token out of range");
-  if (policy < KVR_POLICY_EDITLOCAL || policy > KVR_POLICY_RANDOM)
+  if (policy < KVR_POLICY_EDITLOCAL || policy > KVR_POLICY_EDITLOCAL_BOUNDARY)
     return fail(KVR_E_INVAL, "unknown policy %d", (int)policy);
   KVR_TRY(use_device(m));
   int n = c->n, s_end = edit_start + edit_len;
@@ -1017,12 +1026,16 @@ kvr_status kvr_select(kvr_model *m, const kvr_cache *c, kvr_policy policy, int32
   void *save = nullptr;
   float *probs = nullptr;
   if (!st && (policy == KVR_POLICY_EDITLOCAL || policy == KVR_POLICY_STRUCTURAL ||
-              policy == KVR_POLICY_RANDOM)) {
+              policy == KVR_POLICY_RANDOM || policy == KVR_POLICY_EDITLOCAL_BOUNDARY)) {
     Prof pr(m, P_SELECT, 0);
-    launch_scores_simple(policy, toks, n, s_end, dm.delim, seed, m->keys, m->stream);
-    st = launch_check(m, 1);
-    if (st) st = fail(KVR_E_CUDA, "selector scores: %s", kvr_last_error());
-    if (policy == KVR_POLICY_STRUCTURAL) topk_k = -K;
+    int *bound = (int *)(m->sel_count + 1);
+    int init = n - 1;
+    if (policy == KVR_POLICY_EDITLOCAL_BOUNDARY) st = stage_h2d(m, bound, &init, 1);
+    if (!st) {
+      launch_scores_simple(policy, toks, n, s_end, dm.delim, seed, bound, m->keys, m->stream);
+      st = launch_check(m, policy == KVR_POLICY_EDITLOCAL_BOUNDARY ? 2 : 1);
+    }
+    if (policy == KVR_POLICY_STRUCTURAL || policy == KVR_POLICY_EDITLOCAL_BOUNDARY) topk_k = -K;
   } else if (!st && policy == KVR_POLICY_ATTENTION) {
     if (edit_len == 0) {
       st = fail(KVR_E_RANGE, "attention policy needs a non-empty span");
@@ -1153,6 +1166,86 @@ kvr_status kvr_select(kvr_model *m, const kvr_cache *c, kvr_policy policy, int32
   dev_free(probs);
   if (!st) *count_out = cnt;
   return st;
+}
+
+kvr_status kvr_transplant(kvr_cache *dst, const kvr_cache *src, const int32_t *positions,
+                          int32_t n_positions) {
+  if (!dst || !src || (n_positions > 0 && !positions)) return fail(KVR_E_INVAL, "NULL argument");
+  if (dst->model != src->model) return fail(KVR_E_INVAL, "caches of different models");
+  if (dst == src) return fail(KVR_E_INVAL, "transplant into the source cache");
+  if (dst->poisoned || src->poisoned) return fail(KVR_E_POISONED, "cache poisoned");
+  if (dst->n != src->n) return fail(KVR_E_RANGE, "caches of different lengths");
+  kvr_model *m = dst->model;
+  if (n_positions < 0 || n_positions > m->dims.max_rows)
+    return fail(KVR_E_RANGE, "n_positions outside [0, max_rows]");
+  for (int i = 0; i < n_positions; ++i)
+    if (positions[i] < 0 || positions[i] >= dst->n || (i && positions[i] <= positions[i - 1]))
+      return fail(KVR_E_RANGE, "positions must be strictly increasing in [0, n)");
+  KVR_TRY(use_device(m));
+  if (n_positions == 0) return KVR_OK;
+  for (int i = 0; i < n_positions; ++i) dst->tokens_h[positions[i]] = src->tokens_h[positions[i]];
+  KVR_TRY(stage_h2d(m, m->pos_d, positions, n_positions));
+  launch_transplant(dst->view(), src->view(), m->dims.dtype, m->pos_d, n_positions, m->stream);
+  kvr_status st = launch_check(m, 1);
+  // the token copies: one device-to-device copy per position keeps the
+  // device tokens identical to the host mirror
+  for (int i = 0; !st && i < n_positions; ++i)
+    if (cudaMemcpyAsync(dst->tokens_d + positions[i], src->tokens_d + positions[i], 4,
+                        cudaMemcpyDeviceToDevice, m->stream))
+      st = fail(KVR_E_CUDA, "token copy");
+  if (st == KVR_E_CUDA) dst->poisoned = true;
+  return st;
+}
+
+kvr_status kvr_answer_logprob(kvr_model *m, const kvr_cache *c, const int32_t *prompt,
+                              int32_t mp, const int32_t *answer, int32_t ma, double *out) {
+  if (!m || !c || !prompt || !answer || !out) return fail(KVR_E_INVAL, "NULL argument");
+  if (c->model != m) return fail(KVR_E_INVAL, "cache of another model");
+  if (c->poisoned) return fail(KVR_E_POISONED, "cache poisoned");
+  const Dims &dm = m->dims;
+  int rows = mp + ma - 1;
+  if (mp < 1 || ma < 1 || rows > KVR_QUERY_RESERVE || c->n + rows > c->cap)
+    return fail(KVR_E_RANGE, "prompt + answer - 1 must be in [1, %d]", KVR_QUERY_RESERVE);
+  std::vector<int32_t> feed(prompt, prompt + mp);
+  feed.insert(feed.end(), answer, answer + ma - 1);
+  for (int t : feed)
+    if (t < 0 || t >= dm.V) return fail(KVR_E_RANGE, "token out of range");
+  for (int i = 0; i < ma; ++i)
+    if (answer[i] < 0 || answer[i] >= dm.V) return fail(KVR_E_RANGE, "answer token out of range");
+  KVR_TRY(use_device(m));
+  std::vector<int32_t> P(rows);
+  for (int i = 0; i < rows; ++i) P[i] = c->n + i;
+  KVR_TRY(stage_h2d(m, c->tokens_d + c->n, feed.data(), rows));
+  KVR_TRY(stage_h2d(m, m->pos_d, P.data(), rows));
+  Rows r;
+  r.M = rows;
+  r.pos = m->pos_d;
+  r.tokens = c->tokens_d;
+  r.single = c->view();
+  r.max_pos = c->n + rows - 1;
+  KVR_TRY(plan_attention(m, r, P.data(), nullptr));
+  KVR_TRY(run_pass(m, r));
+  // rows mp-1 .. mp+ma-2 predict answer[0..ma-1]
+  {
+    Prof pr(m, P_NORM, (int64_t)ma * dm.d * 4);
+    launch_rmsnorm(m->h + (size_t)(mp - 1) * dm.d, m->final_norm, ma, dm.d, dm.eps, m->a,
+                   dm.dtype, m->stream);
+    KVR_TRY(launch_check(m, 1));
+  }
+  KVR_TRY(gemm(m, P_LMHEAD, m->a, m->lm_head, m->tc_lm ? &m->tm_lm : nullptr, nullptr, m->logits,
+               ma, dm.V, dm.d, GEMM_EPI_STORE));
+  // answer ids staged behind the positions in the row-document slot
+  KVR_TRY(stage_h2d(m, m->rowdoc_d, answer, ma));
+  float *lp = m->scores;  // [ma] scratch
+  launch_row_logprob(m->logits, ma, dm.V, m->rowdoc_d, lp, m->stream);
+  KVR_TRY(launch_check(m, 1));
+  std::vector<float> h(ma);
+  CUDA_TRY(cudaMemcpyAsync(h.data(), lp, (size_t)ma * 4, cudaMemcpyDeviceToHost, m->stream));
+  KVR_TRY(sync_model(m));
+  double acc = 0.0;
+  for (int i = 0; i < ma; ++i) acc += h[i];
+  *out = acc / ma;
+  return KVR_OK;
 }
 
 kvr_status kvr_cache_tokens(const kvr_cache *c, int32_t *out) {

@@ -225,6 +225,53 @@ __global__ void k_rows_copy(KVView v, const int32_t *pos, int n_pos, int l0, int
   }
 }
 
+// Transplant: copy K/V of every layer at the listed positions from one
+// document's pages into another's (same model shape).
+template <typename T>
+__global__ void k_transplant(KVView dst, KVView src, const int32_t *pos, int n_pos) {
+  const int L = dst.L, G = dst.G, dh = dst.dh;
+  size_t total = (size_t)n_pos * L * 2 * G * dh;
+  const T *s = (const T *)src.pages;
+  T *d = (T *)dst.pages;
+  for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < total;
+       e += (size_t)gridDim.x * blockDim.x) {
+    int i = (int)(e % dh);
+    size_t r = e / dh;
+    int g = (int)(r % G);
+    r /= G;
+    int kv = (int)(r % 2);
+    r /= 2;
+    int l = (int)(r % L);
+    int p = pos[r / L];
+    d[dst.offset(l, kv, g, p) + i] = s[src.offset(l, kv, g, p) + i];
+  }
+}
+
+// out[i] = logits[i][target[i]] - logsumexp(logits[i]) for each row.
+__global__ void __launch_bounds__(256) k_row_logprob(const float *logits, int V,
+                                                     const int32_t *target, float *out) {
+  const float *x = logits + (size_t)blockIdx.x * V;
+  __shared__ float red[8];
+  float mx = -INFINITY;
+  for (int j = threadIdx.x; j < V; j += 256) mx = fmaxf(mx, x[j]);
+  for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = mx;
+  __syncthreads();
+  mx = red[0];
+  for (int w = 1; w < 8; ++w) mx = fmaxf(mx, red[w]);
+  __syncthreads();
+  float sm = 0.f;
+  for (int j = threadIdx.x; j < V; j += 256) sm += expf(x[j] - mx);
+  for (int o = 16; o > 0; o >>= 1) sm += __shfl_xor_sync(0xffffffffu, sm, o);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = sm;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float t = 0.f;
+    for (int w = 0; w < 8; ++w) t += red[w];
+    out[blockIdx.x] = x[target[blockIdx.x]] - (mx + logf(t));
+  }
+}
+
 int grid_for(size_t n, int block) {
   size_t g = (n + block - 1) / block;
   return (int)(g > 65535 * 8 ? 65535 * 8 : (g == 0 ? 1 : g));
@@ -300,6 +347,21 @@ void launch_cache_gather(KVView v, int dtype, const int32_t *pos, int n_pos, int
   else
     k_cache_gather<float><<<grid_for(n, 256), 256, 0, s>>>(v, pos, n_pos, l0, l1 - l0, G, dh,
                                                             k_out, v_out);
+}
+
+void launch_transplant(KVView dst, KVView src, int dtype, const int32_t *pos, int n_pos,
+                       cudaStream_t s) {
+  size_t n = (size_t)n_pos * dst.L * 2 * dst.G * dst.dh;
+  if (n == 0) return;
+  if (dtype == KVR_DTYPE_BF16)
+    k_transplant<__nv_bfloat16><<<grid_for(n, 256), 256, 0, s>>>(dst, src, pos, n_pos);
+  else
+    k_transplant<float><<<grid_for(n, 256), 256, 0, s>>>(dst, src, pos, n_pos);
+}
+
+void launch_row_logprob(const float *logits, int rows, int V, const int32_t *target, float *out,
+                        cudaStream_t s) {
+  if (rows > 0) k_row_logprob<<<rows, 256, 0, s>>>(logits, V, target, out);
 }
 
 void launch_rows_copy(KVView v, int dtype, const int32_t *pos, int n_pos, int l0, int l1,

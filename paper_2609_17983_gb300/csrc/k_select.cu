@@ -27,8 +27,15 @@ __device__ __forceinline__ uint32_t ord_f32(float f) {
   return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
+// First delimiter position at or after s_end (n - 1 if none): the document
+// boundary of EditLocal@boundary.  *bound must hold n - 1 on entry.
+__global__ void k_first_delim(const int32_t *tokens, int n, int s_end, int delim, int *bound) {
+  for (int j = s_end + blockIdx.x * blockDim.x + threadIdx.x; j < n; j += gridDim.x * blockDim.x)
+    if (tokens[j] == delim) atomicMin(bound, j);
+}
+
 __global__ void k_scores_simple(int policy, const int32_t *tokens, int n, int s_end, int delim,
-                                uint64_t seed, unsigned long long *keys) {
+                                uint64_t seed, const int *bound, unsigned long long *keys) {
   int c = n - s_end;
   for (int t = blockIdx.x * blockDim.x + threadIdx.x; t < c; t += gridDim.x * blockDim.x) {
     int j = s_end + t;
@@ -40,6 +47,7 @@ __global__ void k_scores_simple(int policy, const int32_t *tokens, int n, int s_
       // nearest to the span first
       k = 0x100000000ull - (unsigned long long)t;
       if (policy == KVR_POLICY_STRUCTURAL && tokens[j] != delim) k = 0;
+      if (policy == KVR_POLICY_EDITLOCAL_BOUNDARY && j > *bound) k = 0;
     }
     keys[t] = k;
   }
@@ -267,10 +275,13 @@ int grid_for(int n, int block) {
 }  // namespace
 
 void launch_scores_simple(int policy, const int32_t *tokens, int n, int s_end, int delim,
-                          uint64_t seed, unsigned long long *keys, cudaStream_t s) {
+                          uint64_t seed, int *bound, unsigned long long *keys, cudaStream_t s) {
   int c = n - s_end;
   if (c <= 0) return;
-  k_scores_simple<<<grid_for(c, 256), 256, 0, s>>>(policy, tokens, n, s_end, delim, seed, keys);
+  if (policy == KVR_POLICY_EDITLOCAL_BOUNDARY)
+    k_first_delim<<<grid_for(c, 256), 256, 0, s>>>(tokens, n, s_end, delim, bound);
+  k_scores_simple<<<grid_for(c, 256), 256, 0, s>>>(policy, tokens, n, s_end, delim, seed, bound,
+                                                   keys);
 }
 
 void launch_float_keys(const float *scores, int n, int s_end, unsigned long long *keys,

@@ -84,8 +84,11 @@ struct ProfClass {
 
 }  // namespace kvr
 
+struct kvr_cache;
+
 struct kvr_model {
   kvr::Dims dims{};
+  std::vector<kvr_cache *> caches;  // live caches, freed with the model
   void *weight_block = nullptr;
   size_t weight_bytes = 0;
   void *embed = nullptr, *lm_head = nullptr;
@@ -217,6 +220,10 @@ void launch_cache_gather(KVView v, int dtype, const int32_t *pos, int n_pos, int
                          int G, int dh, float *k_out, float *v_out, cudaStream_t s);
 void launch_rows_copy(KVView v, int dtype, const int32_t *pos, int n_pos, int l0, int l1,
                       void *buf, bool to_buf, cudaStream_t s);
+void launch_transplant(KVView dst, KVView src, int dtype, const int32_t *pos, int n_pos,
+                       cudaStream_t s);
+void launch_row_logprob(const float *logits, int rows, int V, const int32_t *target, float *out,
+                        cudaStream_t s);
 
 // ---- kernels: GEMM  Y[M][N] (+)= X[M][K] W[N][K]^T (+ bias) ----
 struct GemmArgs {
@@ -272,8 +279,10 @@ const char *launch_attention_tc(const void *q, const int32_t *pos, const int4 *b
                                 float2 *ws_ml, void *out, cudaStream_t s);
 
 // ---- kernels: selectors ----
+// bound: device int holding n - 1 (EditLocal@boundary writes the first
+// delimiter position at or after s_end into it).
 void launch_scores_simple(int policy, const int32_t *tokens, int n, int s_end, int delim,
-                          uint64_t seed, unsigned long long *keys, cudaStream_t s);
+                          uint64_t seed, int *bound, unsigned long long *keys, cudaStream_t s);
 void launch_attn_select_scores(const float *q, int S, const Dims &dm, int layer, KVView v,
                                int s_end, int n, float *probs_ws, float *scores, cudaStream_t s);
 void launch_kv_deviation(const float *qkv, const float2 *rope, const int32_t *pos, int M,

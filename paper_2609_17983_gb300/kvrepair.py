@@ -12,6 +12,7 @@ from __future__ import annotations
 
 import ctypes
 import os
+import weakref
 
 import numpy as np
 
@@ -25,7 +26,8 @@ KVR_OK = 0
 ERRORS = {1: "KVR_E_INVAL", 2: "KVR_E_RANGE", 3: "KVR_E_NOMEM", 4: "KVR_E_CUDA",
           5: "KVR_E_DEVICE_TIMEOUT", 6: "KVR_E_UNSUPPORTED", 7: "KVR_E_POISONED"}
 DTYPES = {"fp32": 0, "bf16": 1}
-POLICIES = {"editlocal": 0, "structural": 1, "attention": 2, "cacheblend": 3, "random": 4}
+POLICIES = {"editlocal": 0, "structural": 1, "attention": 2, "cacheblend": 3, "random": 4,
+            "editlocal_boundary": 5}
 
 
 class KvrError(RuntimeError):
@@ -88,6 +90,8 @@ _sigs = {
     "kvr_launch_count": ([_P], ctypes.c_int64),
     "kvr_linear": ([_P, ctypes.c_char_p, _I32, _P, _I32, _P], _I32),
     "kvr_linear_noalloc": ([_P, ctypes.c_char_p, _I32, _P, _I32, _P], _I32),
+    "kvr_transplant": ([_P, _P, _P, _I32], _I32),
+    "kvr_answer_logprob": ([_P, _P, _P, _I32, _P, _I32, _P], _I32),
 }
 for _name, (_args, _res) in _sigs.items():
     _f = getattr(_lib, _name)
@@ -214,6 +218,19 @@ def kvr_logits(model, cache, query, vocab: int) -> np.ndarray:
     return out
 
 
+def kvr_transplant(dst, src, positions):
+    ps = _i32(positions)
+    _check(_lib.kvr_transplant(dst, src, _ptr(ps), ps.size))
+
+
+def kvr_answer_logprob(model, cache, prompt, answer) -> float:
+    pr, an = _i32(prompt), _i32(answer)
+    out = ctypes.c_double(0.0)
+    _check(_lib.kvr_answer_logprob(model, cache, _ptr(pr), pr.size, _ptr(an), an.size,
+                                   ctypes.byref(out)))
+    return out.value
+
+
 def kvr_cache_len(cache) -> int:
     return int(_lib.kvr_cache_len(cache))
 
@@ -319,10 +336,13 @@ class Model:
     def __init__(self, cfg: dict, weights: dict | None = None, seed: int = 0,
                  max_context: int = 8192, max_rows: int = 4096):
         self.cfg = dict(cfg)
+        self._caches = weakref.WeakSet()
         self.h = kvr_model_create(cfg, weights, seed, max_context, max_rows)
 
     def close(self):
         if getattr(self, "h", None):
+            for c in list(self._caches):  # the library frees them with the model
+                c.h = None
             kvr_model_free(self.h)
             self.h = None
 
@@ -344,6 +364,14 @@ class Model:
 
     def logits(self, cache: "Cache", query) -> np.ndarray:
         return kvr_logits(self.h, cache.h, query, self.cfg["vocab"])
+
+    def answer_logprob(self, cache: "Cache", prompt, answer) -> float:
+        return kvr_answer_logprob(self.h, cache.h, prompt, answer)
+
+    def margin(self, cache: "Cache", prompt, a_new, a_old) -> float:
+        """m_x of Eq. 2 for this cache state."""
+        return (self.answer_logprob(cache, prompt, a_new)
+                - self.answer_logprob(cache, prompt, a_old))
 
     def repair_batch(self, reqs):
         kvr_repair_batch(self.h, [(c.h, e, p) for c, e, p in reqs])
@@ -367,6 +395,7 @@ class Cache:
     def __init__(self, model: Model, handle):
         self.model = model
         self.h = handle
+        model._caches.add(self)
 
     def close(self):
         if getattr(self, "h", None):
@@ -385,6 +414,9 @@ class Cache:
 
     def tokens(self) -> np.ndarray:
         return kvr_cache_tokens(self.h)
+
+    def transplant_from(self, src: "Cache", positions):
+        kvr_transplant(self.h, src.h, positions)
 
     def read(self, positions, layer_begin: int = 0, layer_end: int | None = None):
         c = self.model.cfg

@@ -180,6 +180,10 @@ def test_mistral7b_structural_and_cacheblend():
     assert got.tolist() == oracle.select(cfg, None, ref_cache, "structural", 32, s, new).tolist()
     n_delims = int(np.sum(doc[s + len(new):] == cfg["delim_id"]))
     assert len(got) == min(32, n_delims)  # fewer when the pool holds fewer delimiters
+    for K in (32, 4096):  # EditLocal@boundary: window to the next delimiter, K caps it
+        got = m.select(cache, "editlocal_boundary", K, s, new)
+        ref = oracle.select(cfg, None, ref_cache, "editlocal_boundary", K, s, new)
+        assert got.tolist() == ref.tolist(), K
     rows = sample_rows(n, np.arange(s, s + 100), stride=19)
     k0, v0 = cache.read(rows)
     cb = m.select(cache, "cacheblend", 32, s, new)
@@ -193,6 +197,56 @@ def test_mistral7b_structural_and_cacheblend():
     assert rel(gk[:, 0], rk) <= TOL and rel(gv[:, 0], rv) <= TOL
     cache.close()
     m.close()
+
+
+def test_llama8b_margin_harness_endpoints(llama):
+    # The margin harness (Eq. 2) at the bench size, through both operators
+    # at the full-suffix endpoint.  Transplanting every row from s on gives
+    # the fresh prefill's margins exactly.  Repairing the full suffix matches
+    # them up to bf16 rounding noise, whose level comes from null controls:
+    # the same prefill of C' tiled with other row chunkings (the margins of
+    # equivalent caches spread by a few 1e-2 nats).
+    cfg, m = llama
+    w = synth.workload("llama8b")
+    doc, s, new = w["doc"], w["edit_start"], w["new_tokens"]
+    n = len(doc)
+    edited = oracle.apply_edit(doc, s, new)
+    prompt = synth.fill_tokens(51, 12, cfg["vocab"], cfg["delim_id"])
+    pairs = [(synth.fill_tokens(52 + 2 * i, 4, cfg["vocab"], cfg["delim_id"]),
+              synth.fill_tokens(53 + 2 * i, 4, cfg["vocab"], cfg["delim_id"])) for i in range(4)]
+    stale, fresh = m.prefill(doc), m.prefill(edited)
+    rep, trans = m.prefill(doc), m.prefill(doc)
+    rep.repair(new, s, np.arange(s + len(new), n))
+    trans.transplant_from(fresh, np.arange(s, n))
+    rows = sample_rows(n, [], stride=13)
+    kt, vt = trans.read(rows)
+    kf, vf = fresh.read(rows)
+    after = rows >= s
+    assert np.array_equal(kt[after], kf[after]) and np.array_equal(vt[after], vf[after])
+    assert np.array_equal(trans.tokens(), edited)
+
+    def margins(model, cache):
+        return np.array([model.margin(cache, prompt, a, b) for a, b in pairs])
+
+    mg = {k: margins(m, c) for k, c in dict(stale=stale, fresh=fresh, rep=rep,
+                                           trans=trans).items()}
+    for c in (stale, fresh, rep, trans):
+        c.close()
+    ctrl = []
+    for max_rows in (2048, 1024):
+        other = kv.Model(cfg, None, seed=0, max_context=8192, max_rows=max_rows)
+        control = other.prefill(edited)
+        ctrl.append(margins(other, control) - mg["fresh"])
+        control.close()
+        other.close()
+    noise = float(np.sqrt(np.mean(np.square(ctrl))))
+    assert all(np.all(np.isfinite(v)) for v in mg.values())
+    assert np.array_equal(mg["trans"], mg["fresh"]), mg
+    gap = float(np.sqrt(np.mean(np.square(mg["rep"] - mg["fresh"]))))
+    assert gap <= 1.5 * noise + 1e-3, (mg, noise)
+    # the edit moves the margins far beyond the noise, so MR is meaningful
+    shift = float(np.sqrt(np.mean(np.square(mg["fresh"] - mg["stale"]))))
+    assert shift >= 5 * noise, (mg, noise)
 
 
 def test_batched_repair_16x8192_matches_per_document(llama):

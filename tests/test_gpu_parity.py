@@ -196,9 +196,10 @@ def test_select_structural_exact():
     ref_cache = oracle.empty_cache(cfg, len(doc))
     ref_cache.tokens[:] = doc
     for K in (3, 32):
-        got = model.select(cache, "structural", K, s, new)
-        ref = oracle.select(cfg, W, ref_cache, "structural", K, s, new)
-        assert got.tolist() == ref.tolist()
+        for pol in ("structural", "editlocal_boundary"):
+            got = model.select(cache, pol, K, s, new)
+            ref = oracle.select(cfg, W, ref_cache, pol, K, s, new)
+            assert got.tolist() == ref.tolist(), (pol, K)
     model.close()
 
 
@@ -341,7 +342,7 @@ def test_select_long_context_exact(n):
     ref_cache = oracle.empty_cache(cfg, n)
     ref_cache.tokens[:] = doc
     for policy, K, seed in [("editlocal", 32, 0), ("structural", 32, 0), ("random", 64, 2),
-                            ("editlocal", n, 0)]:
+                            ("editlocal", n, 0), ("editlocal_boundary", 200, 0)]:
         got = model.select(cache, policy, K, s, new, seed)
         ref = oracle.select(cfg, W, ref_cache, policy, K, s, new, seed)
         assert got.tolist() == ref.tolist(), policy
@@ -395,3 +396,88 @@ def test_8b_shape_model_selectors_parity(shape, policy):
     ref = oracle.topk(sc, D, K)
     check_selection(got, ref, sc, 2e-2 * np.abs(sc[D]).max())
     model.close()
+
+
+# ------------------------------------------------------------- NEXT rows
+
+def test_transplant_gpu_exact():
+    # Transplant (Sec. 3): rows of P take the fresh cache's K/V and tokens
+    # bit for bit; every other row keeps the stale entries
+    cfg, W, doc, s, new = tiny_setup("bf16")
+    model = kv.Model(cfg, W, max_context=1024, max_rows=512)
+    stale = model.prefill(doc)
+    fresh = model.prefill(oracle.apply_edit(doc, s, new))
+    P = np.array([200, 201, 202, 203, 210, 250, 300, 511])
+    rows = np.arange(len(doc))
+    ks, vs = stale.read(rows)
+    kf, vf = fresh.read(rows)
+    stale.transplant_from(fresh, P)
+    kt, vt = stale.read(rows)
+    mask = np.isin(rows, P)
+    assert np.array_equal(kt[mask], kf[mask]) and np.array_equal(vt[mask], vf[mask])
+    assert np.array_equal(kt[~mask], ks[~mask]) and np.array_equal(vt[~mask], vs[~mask])
+    toks = doc.copy()
+    toks[P] = fresh.tokens()[P]
+    assert np.array_equal(stale.tokens(), toks)
+    model.close()
+
+
+@pytest.mark.parametrize("dtype", ["fp32", "bf16"])
+def test_answer_logprob_parity(dtype):
+    cfg, W, doc, s, new = tiny_setup(dtype)
+    model = kv.Model(cfg, W, max_context=1024, max_rows=512)
+    cache = model.prefill(doc)
+    ref_cache = oracle.prefill(cfg, W, doc)
+    prompt = synth.fill_tokens(31, 5, cfg["vocab"], cfg["delim_id"])
+    ans = synth.fill_tokens(32, 3, cfg["vocab"], cfg["delim_id"])
+    got = model.answer_logprob(cache, prompt, ans)
+    ref = oracle.answer_logprob(cfg, W, ref_cache, prompt, ans)
+    assert abs(got - ref) <= TOL[dtype] * abs(ref), (got, ref)
+    model.close()
+
+
+def test_transplant_vs_recompute_margin_harness():
+    # E4 harness on synthetic answers: the same position set through both
+    # operators, margin recovery (Eq. 2) of each, GPU against the oracle
+    cfg, W, doc, s, new = tiny_setup()
+    model = kv.Model(cfg, W, max_context=1024, max_rows=512)
+    prompt = synth.fill_tokens(41, 4, cfg["vocab"], cfg["delim_id"])
+    a_new = synth.fill_tokens(42, 2, cfg["vocab"], cfg["delim_id"])
+    a_old = synth.fill_tokens(43, 2, cfg["vocab"], cfg["delim_id"])
+    edited = oracle.apply_edit(doc, s, new)
+    A = np.array([204, 206, 215, 240, 300, 301, 420])
+    P = oracle.repaired_set(s, len(new), A)
+    # GPU
+    stale, fresh = model.prefill(doc), model.prefill(edited)
+    rep, trans = model.prefill(doc), model.prefill(doc)
+    rep.repair(new, s, A)
+    trans.transplant_from(fresh, P)
+    gm = {k: model.margin(c, prompt, a_new, a_old)
+          for k, c in dict(stale=stale, fresh=fresh, rep=rep, trans=trans).items()}
+    # oracle
+    o_stale = oracle.prefill(cfg, W, doc)
+    o_fresh = oracle.prefill(cfg, W, edited)
+    o_rep = oracle.repair(cfg, W, o_stale, new, s, A)
+    o_trans = oracle.transplant(o_stale, o_fresh, P)
+    om = {k: oracle.margin(cfg, W, c, prompt, a_new, a_old)
+          for k, c in dict(stale=o_stale, fresh=o_fresh, rep=o_rep, trans=o_trans).items()}
+    for k in gm:
+        assert abs(gm[k] - om[k]) <= 1e-3 * max(1.0, abs(om[k])), (k, gm[k], om[k])
+    for op in ("rep", "trans"):
+        g = oracle.margin_recovery(gm[op], gm["stale"], gm["fresh"])
+        o = oracle.margin_recovery(om[op], om["stale"], om["fresh"])
+        assert abs(g - o) <= 1e-2 * max(1.0, abs(o)), (op, g, o)
+    model.close()
+
+
+def test_model_free_releases_live_caches():
+    # kvr_model_free frees the caches still live; the binding's handles to
+    # them become inert, so closing them afterwards is a no-op
+    cfg, W, doc, s, new = tiny_setup()
+    model = kv.Model(cfg, W, max_context=1024, max_rows=512)
+    caches = [model.prefill(doc) for _ in range(3)]
+    caches[1].close()
+    model.close()
+    assert all(c.h is None for c in caches)
+    for c in caches:
+        c.close()

@@ -341,3 +341,53 @@ def test_cacheblend_unchanged_tokens_all_zero():
     assert np.all(sc == 0.0)
     assert oracle.select(cfg, W, stale, "cacheblend", 8, s, doc[s:s + 4]).tolist() == \
         list(range(s + 4, s + 12))
+
+
+# ------------------------------------------------------------- NEXT rows
+
+def test_editlocal_boundary_golden():
+    g = read_golden("editlocal_boundary_example.txt")
+    n, delim = int(g["n"][0]), int(g["delim_id"][0])
+    toks = np.full(n, 5, np.int32)
+    toks[[int(x) for x in g["delims"]]] = delim
+    cfg = synth.preset("tiny")
+    cache = oracle.empty_cache(cfg, n)
+    cache.tokens[:] = toks
+    for key in ("S13_2_K10", "S13_2_K4", "S34_2_K10", "S22_2_K16"):
+        s, L, K = key.split("_")
+        s, L, K = int(s[1:]), int(L), int(K[1:])
+        got = oracle.select(cfg, None, cache, "editlocal_boundary", K, s, toks[s:s + L])
+        assert got.tolist() == [int(x) for x in g[key]], key
+
+
+def test_transplant_identity_and_noop():
+    cfg, W, doc, s, new = small_workload(n=96, s=40)
+    stale = oracle.prefill(cfg, W, doc)
+    fresh = oracle.prefill(cfg, W, oracle.apply_edit(doc, s, new))
+    full = oracle.transplant(stale, fresh, np.arange(len(doc)))
+    assert np.array_equal(full.k, fresh.k) and np.array_equal(full.tokens, fresh.tokens)
+    none = oracle.transplant(stale, fresh, np.array([], np.int64))
+    assert np.array_equal(none.k, stale.k) and np.array_equal(none.tokens, stale.tokens)
+
+
+def test_answer_logprob_matches_textbook_and_mr_endpoints():
+    cfg, W, doc, s, new = small_workload(n=96, s=40)
+    prompt = synth.fill_tokens(31, 3, cfg["vocab"], cfg["delim_id"])
+    a_new = synth.fill_tokens(32, 2, cfg["vocab"], cfg["delim_id"])
+    a_old = synth.fill_tokens(33, 2, cfg["vocab"], cfg["delim_id"])
+    stale = oracle.prefill(cfg, W, doc)
+    got = oracle.answer_logprob(cfg, W, stale, prompt, a_new)
+    seq = np.concatenate([doc, prompt, a_new[:-1]])
+    lg = textbook.forward(cfg, W, seq)["logits"][len(doc) + len(prompt) - 1:]
+    ref = float(torch.log_softmax(lg, dim=-1)[torch.arange(len(a_new)),
+                                              torch.as_tensor(a_new, dtype=torch.long)].mean())
+    assert abs(got - ref) <= 1e-6 * abs(ref)
+    # MR endpoints (Eq. 2): the oracle cache recovers 1, the stale cache 0
+    fresh = oracle.prefill(cfg, W, oracle.apply_edit(doc, s, new))
+    rep = oracle.repair(cfg, W, stale, new, s, oracle.pool(len(doc), s, len(new)))
+    m_st = oracle.margin(cfg, W, stale, prompt, a_new, a_old)
+    m_or = oracle.margin(cfg, W, fresh, prompt, a_new, a_old)
+    m_rep = oracle.margin(cfg, W, rep, prompt, a_new, a_old)
+    assert m_st != m_or
+    assert oracle.margin_recovery(m_rep, m_st, m_or) == pytest.approx(1.0, abs=1e-12)
+    assert oracle.margin_recovery(m_st, m_st, m_or) == 0.0
