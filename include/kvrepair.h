@@ -259,6 +259,33 @@ kvr_status kvr_profile_reset(kvr_model *model);
 kvr_status kvr_profile_read(kvr_model *model, int32_t cap, double *ms_out, int64_t *launches_out,
                             int64_t *bytes_out, char *names, int32_t names_cap, int32_t *n_out);
 
+/* Device timeline trace (tooling; the paper has no counterpart).  Only the
+ * KVR_TRACE build of the library (libkvrepair_trace.so) records; elsewhere
+ * kvr_trace_enable with capacity > 0 returns KVR_E_UNSUPPORTED.  With
+ * capacity > 0, a device buffer of `capacity` records is attached and every
+ * CTA of the pass kernels (embedding, RMSNorm, GEMM, RoPE/scatter,
+ * attention, combine) appends one record of 16 uint64 words:
+ *   [0] kind (1 embed, 2 rmsnorm, 3 GEMM, 4 RoPE/scatter, 5 attention,
+ *       6 combine) | SM id << 8 | linear block index << 16,
+ *   [1] start, [2] return of the wait on the predecessor kernel, [3] end,
+ *   [4..11] eight marks, 0 where the kernel sets none.  GEMM, for the CTA's
+ *       last tile: first operand stage landed, all MMAs complete,
+ *       accumulator taken by the epilogue, partial tile stored, split-tile
+ *       arrival counted or partials staged across the cluster, tile reduced
+ *       and written, epilogue done, all warps done.  Attention: last key
+ *       chunk consumed.
+ *   [12..15] zero,
+ * times in ns of the device's global timer.  Records past `capacity` are
+ * dropped.  capacity == 0 detaches and frees the buffer.  The buffer is
+ * process-wide: the model that attached it last owns it, and kernels of
+ * every model on the device write to it.  kvr_trace_read synchronises the
+ * model's stream, copies up to `cap` records to host `out` (uint64[16*cap]),
+ * returns the number appended via *n_out (which may exceed what fitted),
+ * and empties the buffer.  Errors: KVR_E_INVAL, KVR_E_NOMEM,
+ * KVR_E_UNSUPPORTED. */
+kvr_status kvr_trace_enable(kvr_model *model, int32_t capacity);
+kvr_status kvr_trace_read(kvr_model *model, uint64_t *out, int32_t cap, int32_t *n_out);
+
 /* Number of library kernels launched so far on this model. */
 int64_t kvr_launch_count(const kvr_model *model);
 

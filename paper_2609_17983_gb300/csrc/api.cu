@@ -6,6 +6,7 @@
 // RoPE at the original positions + K/V scatter of all rows -> scattered-query
 // attention -> O GEMM (+residual) -> RMSNorm -> gate/up GEMM -> SwiGLU ->
 // down GEMM (+residual).
+#include <algorithm>
 #include <cmath>
 #include <cstdlib>
 #include <cstdarg>
@@ -119,21 +120,18 @@ kvr_status stage_h2d(kvr_model *m, int32_t *dst_dev, const int32_t *src, size_t 
 // Y (+)= X W^T through the tensor-core kernel when the weight has a TMA
 // descriptor, else the FFMA kernel.  epi selects the epilogue; for SwiGLU
 // the FFMA path writes gate/up to m->gu and runs the SwiGLU kernel.
-// Bytes of the next GEMM's weights each CTA prefetches into L2 while a
-// few-row GEMM drains (the gap before the next GEMM would leave HBM idle).
-constexpr long long PREFETCH_BYTES_PER_CTA = 256 << 10;
-
+// defer: split tiles of the tensor-core GEMM are left to the kernel that
+// next reads Y, which must take *defer (ws null when Y is complete).
 kvr_status gemm(kvr_model *m, int cls, const void *X, const void *W, const CUtensorMap *tm,
                 const float *bias, float *Y, int M, int N, int K, int epi,
-                const CUtensorMap *next_tm = nullptr, int next_N = 0, int next_K = 0) {
+                SplitView *defer = nullptr) {
   const Dims &dm = m->dims;
   Prof pr(m, cls, (int64_t)N * K * (int64_t)dm.es());
+  if (defer) *defer = SplitView{};
   if (tm && m->use_tc) {
     GemmArgs g{X, W, bias, Y, M, N, K, K, N, dm.dtype, epi == GEMM_EPI_ACCUM};
-    TcNext nx{next_tm, M, next_N, next_K, PREFETCH_BYTES_PER_CTA};
-    bool pf = next_tm && m->prefetch && M <= 256;
     const char *e = launch_gemm_tc(g, *tm, epi, epi == GEMM_EPI_SWIGLU ? m->act : nullptr,
-                                   N / 2, m->tcw, m->stream, pf ? &nx : nullptr);
+                                   N / 2, m->tcw, m->stream, m->defer_splits ? defer : nullptr);
     if (e) return fail(KVR_E_CUDA, "tensor-core GEMM (M=%d N=%d K=%d): %s", M, N, K, e);
     return launch_check(m, 1);
   }
@@ -202,30 +200,38 @@ kvr_status plan_attention(kvr_model *m, Rows &r, const int32_t *pos, const int32
 
 kvr_status embed(kvr_model *m, const Rows &r) {
   Prof pr(m, P_EMBED, (int64_t)r.M * m->dims.d * (int64_t)m->dims.es());
+  m->pending = SplitView{};
   launch_embed_rows(m->embed, m->dims.dtype, r.tokens, r.doc_tokens, r.rowdoc, r.pos, r.M,
                     m->dims.d, m->h, m->stream);
   return launch_check(m, 1);
 }
 
-kvr_status norm(kvr_model *m, const float *g, int M) {
+// RMSNorm of h rows row0 .. row0+M-1 into m->a, first adding the split
+// tiles a deferred GEMM left pending in h.
+kvr_status norm(kvr_model *m, const float *g, int M, int row0 = 0) {
   Prof pr(m, P_NORM, (int64_t)M * m->dims.d * 4);
-  launch_rmsnorm(m->h, g, M, m->dims.d, m->dims.eps, m->a, m->dims.dtype, m->stream);
+  launch_rmsnorm(m->h, g, row0, M, m->dims.d, m->dims.eps, m->a, m->dims.dtype, m->stream,
+                 &m->pending);
+  m->pending = SplitView{};
   return launch_check(m, 1);
 }
 
-// QKV projection, RoPE, and (write_kv) the K/V scatter of layer l.
-kvr_status layer_qkv(kvr_model *m, const Rows &r, int l, bool write_kv) {
+// QKV projection, RoPE, and (write_kv) the K/V scatter of layer l.  keep_qkv:
+// m->qkv must hold the complete projection afterwards (else split tiles of
+// the GEMM are completed by the RoPE kernel alone).
+kvr_status layer_qkv(kvr_model *m, const Rows &r, int l, bool write_kv, bool keep_qkv = false) {
   const Dims &dm = m->dims;
   const LayerW &w = m->layers[l];
   KVR_TRY(norm(m, w.attn_norm, r.M));
+  SplitView sv;
   KVR_TRY(gemm(m, P_GEMM_QKV, m->a, w.wqkv, w.tc_qkv ? &w.tm_qkv : nullptr, w.bqkv, m->qkv, r.M,
-               dm.Nqkv(), dm.d, GEMM_EPI_STORE, w.tc_o ? &w.tm_o : nullptr, dm.d, dm.H * dm.dh));
+               dm.Nqkv(), dm.d, GEMM_EPI_STORE, keep_qkv ? nullptr : &sv));
   {
     Prof pr(m, P_ROPE, (int64_t)r.M * dm.Nqkv() * 4);
     launch_rope_scatter(m->qkv, m->rope, r.pos, r.M, dm, l, r.views, r.rowdoc, r.single, m->q,
                         use_tc_attention(m) ? m->qb : nullptr,
                         (float)(1.4426950408889634 / std::sqrt((double)dm.dh)), write_kv,
-                        m->stream);
+                        m->stream, &sv);
     KVR_TRY(launch_check(m, 1));
   }
   return KVR_OK;
@@ -250,14 +256,13 @@ kvr_status layer_rest(kvr_model *m, const Rows &r, int l) {
       KVR_TRY(launch_check(m, 1));
     }
   }
-  const LayerW *wn = l + 1 < dm.L ? &m->layers[l + 1] : nullptr;
   KVR_TRY(gemm(m, P_GEMM_O, m->attn, w.wo, w.tc_o ? &w.tm_o : nullptr, nullptr, m->h, r.M, dm.d,
-               dm.H * dm.dh, GEMM_EPI_ACCUM, w.tc_gu ? &w.tm_gu : nullptr, 2 * dm.F, dm.d));
+               dm.H * dm.dh, GEMM_EPI_ACCUM, &m->pending));
   KVR_TRY(norm(m, w.mlp_norm, r.M));
   KVR_TRY(gemm(m, P_GEMM_GU, m->a, w.wgu, w.tc_gu ? &w.tm_gu : nullptr, nullptr, nullptr, r.M,
-               2 * dm.F, dm.d, GEMM_EPI_SWIGLU, w.tc_d ? &w.tm_d : nullptr, dm.d, dm.F));
+               2 * dm.F, dm.d, GEMM_EPI_SWIGLU));
   KVR_TRY(gemm(m, P_GEMM_DOWN, m->act, w.wd, w.tc_d ? &w.tm_d : nullptr, nullptr, m->h, r.M, dm.d,
-               dm.F, GEMM_EPI_ACCUM, wn && wn->tc_qkv ? &wn->tm_qkv : nullptr, dm.Nqkv(), dm.d));
+               dm.F, GEMM_EPI_ACCUM, &m->pending));
   return KVR_OK;
 }
 
@@ -456,11 +461,14 @@ kvr_status kvr_set_allocator(kvr_alloc_fn alloc, kvr_free_fn free_fn, void *ctx)
   return KVR_OK;
 }
 
+static void trace_release(kvr_model *m);
+
 void kvr_model_free(kvr_model *m) {
   if (!m) return;
   cudaSetDevice(m->device);
   cudaStreamSynchronize(m->stream);
   while (!m->caches.empty()) kvr_cache_free(m->caches.back());
+  trace_release(m);
   prof_collect(m);
   dev_free(m->weight_block);
   dev_free(m->ws_block);
@@ -498,6 +506,8 @@ kvr_status kvr_model_create(const kvr_model_config *cfg, const kvr_weights *wts,
   {
     const char *g = getenv("KVR_DISABLE_GRAPHS");
     m->use_graphs = !(g && g[0] == '1');
+    const char *df = getenv("KVR_DISABLE_DEFERRED_SPLITS");
+    m->defer_splits = !(df && df[0] == '1');
     const char *pd = getenv("KVR_DISABLE_PDL");
     g_pdl = !(pd && pd[0] == '1');
   }
@@ -686,8 +696,6 @@ kvr_status kvr_model_create(const kvr_model_config *cfg, const kvr_weights *wts,
   if (dm.dtype == KVR_DTYPE_BF16) {
     const char *env = getenv("KVR_DISABLE_TC");
     m->use_tc = !(env && env[0] == '1');
-    const char *pf = getenv("KVR_DISABLE_PREFETCH");
-    m->prefetch = !(pf && pf[0] == '1');
     m->tcw.num_sms = m->num_sms;
     m->tcw.max_tiles = 1 << 16;
     m->tcw.dev_flag = m->dev_flag;
@@ -983,8 +991,9 @@ kvr_status kvr_logits(kvr_model *m, const kvr_cache *c, const int32_t *query, in
   // final RMSNorm of the last row, lm_head
   {
     Prof pr(m, P_NORM, (int64_t)dm.d * 4);
-    launch_rmsnorm(m->h + (size_t)(qm - 1) * dm.d, m->final_norm, 1, dm.d, dm.eps, m->a,
-                   dm.dtype, m->stream);
+    launch_rmsnorm(m->h, m->final_norm, qm - 1, 1, dm.d, dm.eps, m->a, dm.dtype, m->stream,
+                   &m->pending);
+    m->pending = SplitView{};
     KVR_TRY(launch_check(m, 1));
   }
   KVR_TRY(gemm(m, P_LMHEAD, m->a, m->lm_head, m->tc_lm ? &m->tm_lm : nullptr, nullptr, m->logits,
@@ -1124,7 +1133,7 @@ kvr_status kvr_select(kvr_model *m, const kvr_cache *c, kvr_policy policy, int32
         if (!st) st = embed(m, r);
         if (!st) st = layer_qkv(m, r, 0, false);
         if (!st) st = layer_rest(m, r, 0);
-        if (!st) st = layer_qkv(m, r, 1, false);
+        if (!st) st = layer_qkv(m, r, 1, false, true);
         if (!st) {
           Prof pr(m, P_SELECT, 0);
           launch_kv_deviation(m->qkv, m->rope, r.pos, M, dm, r.single, m->scores, m->stream);
@@ -1228,8 +1237,9 @@ kvr_status kvr_answer_logprob(kvr_model *m, const kvr_cache *c, const int32_t *p
   // rows mp-1 .. mp+ma-2 predict answer[0..ma-1]
   {
     Prof pr(m, P_NORM, (int64_t)ma * dm.d * 4);
-    launch_rmsnorm(m->h + (size_t)(mp - 1) * dm.d, m->final_norm, ma, dm.d, dm.eps, m->a,
-                   dm.dtype, m->stream);
+    launch_rmsnorm(m->h, m->final_norm, mp - 1, ma, dm.d, dm.eps, m->a, dm.dtype, m->stream,
+                   &m->pending);
+    m->pending = SplitView{};
     KVR_TRY(launch_check(m, 1));
   }
   KVR_TRY(gemm(m, P_LMHEAD, m->a, m->lm_head, m->tc_lm ? &m->tm_lm : nullptr, nullptr, m->logits,
@@ -1399,6 +1409,60 @@ kvr_status kvr_linear(kvr_model *m, const char *name, int32_t layer, const void 
   dev_free(xd);
   dev_free(yd);
   return st;
+}
+
+static cudaError_t trace_attach_all(const TraceBuf &b) {
+  cudaError_t e = trace_attach_rows(b);
+  if (e == cudaSuccess) e = trace_attach_gemm(b);
+  if (e == cudaSuccess) e = trace_attach_attn(b);
+  return e;
+}
+
+static void trace_release(kvr_model *m) {
+  if (!m->trace.rec) return;
+  trace_attach_all(TraceBuf{});
+  dev_free(m->trace.rec);
+  dev_free(m->trace.count);
+  m->trace = TraceBuf{};
+}
+
+kvr_status kvr_trace_enable(kvr_model *m, int32_t capacity) {
+  if (!m || capacity < 0) return fail(KVR_E_INVAL, "NULL model or negative capacity");
+#ifndef KVR_TRACE
+  if (capacity > 0)
+    return fail(KVR_E_UNSUPPORTED, "library built without the device trace (KVR_TRACE build)");
+#endif
+  CUDA_TRY(cudaSetDevice(m->device));
+  CUDA_TRY(cudaStreamSynchronize(m->stream));
+  trace_release(m);
+  if (capacity == 0) return KVR_OK;
+  TraceBuf b;
+  b.rec = (unsigned long long *)dev_alloc((size_t)capacity * 16 * sizeof(uint64_t));
+  b.count = (unsigned int *)dev_alloc(sizeof(unsigned int));
+  b.cap = (unsigned int)capacity;
+  if (!b.rec || !b.count) {
+    dev_free(b.rec);
+    dev_free(b.count);
+    return fail(KVR_E_NOMEM, "trace buffer of %d records", capacity);
+  }
+  CUDA_TRY(cudaMemset(b.count, 0, sizeof(unsigned int)));
+  m->trace = b;
+  CUDA_TRY(trace_attach_all(b));
+  return KVR_OK;
+}
+
+kvr_status kvr_trace_read(kvr_model *m, uint64_t *out, int32_t cap, int32_t *n_out) {
+  if (!m || !n_out || (cap > 0 && !out)) return fail(KVR_E_INVAL, "NULL argument");
+  if (!m->trace.rec) return fail(KVR_E_INVAL, "no trace buffer attached");
+  CUDA_TRY(cudaSetDevice(m->device));
+  CUDA_TRY(cudaStreamSynchronize(m->stream));
+  unsigned int n = 0;
+  CUDA_TRY(cudaMemcpy(&n, m->trace.count, sizeof n, cudaMemcpyDeviceToHost));
+  *n_out = (int32_t)std::min<unsigned int>(n, 0x7fffffffu);
+  size_t k = std::min<size_t>({(size_t)n, (size_t)m->trace.cap, (size_t)std::max(cap, 0)});
+  if (k) CUDA_TRY(cudaMemcpy(out, m->trace.rec, k * 16 * sizeof(uint64_t), cudaMemcpyDeviceToHost));
+  CUDA_TRY(cudaMemset(m->trace.count, 0, sizeof(unsigned int)));
+  return KVR_OK;
 }
 
 kvr_status kvr_profile_enable(kvr_model *m, int32_t enable) {

@@ -100,8 +100,10 @@ __global__ void __launch_bounds__(MAXW * 32, 1) k_attn_tc(const AttnTcParams p) 
   uint8_t *sV = sK + 2 * TILE;                 // 2 x CHUNK x DH
   __shared__ int spos[MAXQ];
 
+  TraceScope ts(TK_ATTN);
   pdl_trigger();
   pdl_wait();
+  ts.waited();
   const int split = blockIdx.x, g = blockIdx.y, blk = blockIdx.z;
   const int4 bd = p.blocks[blk];
   const int row0 = bd.x, nrows = bd.y, kmax = bd.z;
@@ -241,6 +243,7 @@ __global__ void __launch_bounds__(MAXW * 32, 1) k_attn_tc(const AttnTcParams p) 
     }
     __syncthreads();  // buffer buf is refilled by the next iteration's prefetch
   }
+  if (threadIdx.x == 0) trace_mark(0);
   if (!active) return;
   l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
   l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
@@ -286,8 +289,10 @@ __global__ void __launch_bounds__(MAXW * 32, 1) k_attn_tc(const AttnTcParams p) 
 // splits at a time with all loads in flight together.
 template <int DH>
 __global__ void __launch_bounds__(256) k_attn_combine(const AttnTcParams p) {
+  TraceScope ts(TK_COMBINE);
   pdl_trigger();
   pdl_wait();
+  ts.waited();
   const int warp = (blockIdx.x * 8) + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   const int total = p.n_blocks * p.G * MAXQ;
   if (warp >= total) return;
@@ -394,5 +399,7 @@ const char *launch_attention_tc(const void *q, const int32_t *pos, const int4 *b
   if (dm.dh == 64) return run<64>(p, max_mq, s);
   return "head_dim not supported";
 }
+
+KVR_TRACE_ATTACH(trace_attach_attn)
 
 }  // namespace kvr

@@ -65,11 +65,8 @@ struct TcParams {
   float *ws;        // [grid][2][BN][128] fp32 partial tiles
   int *counters;    // [n_tiles * m_tiles] arrival counters (self-resetting)
   int *dev_flag;
-  // L2 prefetch of the next GEMM's weights: CTA i prefetches the first
-  // pf_units units of its own range in the next GEMM's split
-  long long next_total;
-  int next_KB, next_m_tiles, next_grid, pf_units, next_cluster;
   int cluster;  // > 1: cluster split-K with this many CTAs per tile
+  int defer;    // 1: split tiles are left as partials for the consumer
 };
 
 // ------------------------------------------------------------ PTX wrappers
@@ -139,13 +136,6 @@ __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, u
       : "memory");
 }
 
-__device__ __forceinline__ void tma_prefetch_l2(const CUtensorMap *map, int x, int y) {
-  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
-                   (uint64_t)map),
-               "r"(x), "r"(y)
-               : "memory");
-}
-
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap *map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)map) : "memory");
 }
@@ -208,9 +198,6 @@ __device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: 
 
 // ------------------------------------------------------------ work split
 
-__device__ __forceinline__ long long range_start(long long i, long long total, int grid) {
-  return i * total / grid;
-}
 // Units [a, b) of CTA i: stream-K ranges, or K/P of tile i/P in cluster mode
 __device__ __forceinline__ void unit_range(long long i, long long total, int grid, int KB,
                                            int cluster, long long &a, long long &b) {
@@ -224,10 +211,6 @@ __device__ __forceinline__ void unit_range(long long i, long long total, int gri
   }
 }
 
-// CTA whose range holds unit u
-__device__ __forceinline__ int cta_of(long long u, long long total, int grid) {
-  return (int)(((u + 1) * grid - 1) / total);
-}
 
 // Epilogue for 16 consecutive rows t0..t0+15 of Y (the first `cnt` valid) at
 // feature n of W.  All lanes of the warp call it together (SwiGLU exchanges
@@ -268,7 +251,7 @@ __device__ __forceinline__ void epilogue16(const TcParams &p, int t0, int n, con
 
 __global__ void __launch_bounds__(NTHREADS, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX,
-              const __grid_constant__ CUtensorMap tmNext, const TcParams p) {
+              const TcParams p) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[8], empty_bar[8], accf_bar[2], acce_bar[2],
       drain_bar;
@@ -276,6 +259,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
   __shared__ int abort_f;
   __shared__ int last_f;
 
+  TraceScope ts(TK_GEMM);
   pdl_trigger();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int S = p.stages;
@@ -348,6 +332,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           }
         }
         pdl_wait();
+        ts.waited();
         for (long long j = 0; j < npre; ++j) {
           uint32_t sa = base + (uint32_t)j * stage_bytes;
           tma_load_2d((void *)__cvta_shared_to_generic(sa + A_BYTES), &tmX, &full_bar[j],
@@ -388,15 +373,6 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         }
       }
       // warm L2 with the start of this CTA's share of the next GEMM's weights
-      if (p.pf_units > 0 && (int)blockIdx.x < p.next_grid && !*abort_v) {
-        long long nu0, nu1;
-        unit_range(blockIdx.x, p.next_total, p.next_grid, p.next_KB, p.next_cluster, nu0, nu1);
-        if (nu1 > nu0 + p.pf_units) nu1 = nu0 + p.pf_units;
-        for (long long u = nu0; u < nu1; ++u) {
-          long long tl = u / p.next_KB;
-          tma_prefetch_l2(&tmNext, (int)(u % p.next_KB) * BK, (int)(tl / p.next_m_tiles) * BM);
-        }
-      }
       // copies in flight complete before the CTA may exit
       uint32_t n_issued = it;
       for (uint32_t j = n_issued > (uint32_t)S ? n_issued - S : 0; j < n_issued; ++j)
@@ -421,6 +397,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
             ok = false;
             break;
           }
+          if (u == u0) trace_mark(0);
           tc_fence_after();
           uint32_t sa = base + (uint32_t)s * stage_bytes;
           uint64_t da = sw128_desc(sa), db = sw128_desc(sa + A_BYTES);
@@ -441,6 +418,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       // all MMAs issued by this thread complete before TMEM is freed
       mma_commit(&drain_bar);
       mbar_wait(&drain_bar, 0, abort_v, p.dev_flag, 0, false);
+      trace_mark(1);
     }
   } else {
     // ------------------------------------------------------------ epilogue
@@ -454,6 +432,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       // pipeline stages are free: every TMA load was consumed by the MMAs)
       if (mbar_wait(&accf_bar[0], 0, abort_v, p.dev_flag, 8)) {
         tc_fence_after();
+        if (et == 0) trace_mark(2);
         const int mv = min(p.BN, p.M);
         float *sp = (float *)__cvta_shared_to_generic(base);
         uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16);
@@ -464,6 +443,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           for (int j = 0; j < 16; ++j)
             if (c + j < mv) sp[(c + j) * BM + f] = v[j];
         }
+        if (et == 0) trace_mark(3);
       }
       tc_fence_before();
     }
@@ -473,6 +453,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       uint32_t buf = seg & 1u, use = seg >> 1;
       if (!mbar_wait(&accf_bar[buf], use & 1u, abort_v, p.dev_flag, 8)) break;
       tc_fence_after();
+      if (et == 0) trace_mark(2);
       int ntile = (int)(tl / p.m_tiles), mtile = (int)(tl % p.m_tiles);
       int t0 = mtile * p.BN;
       int mv = min(p.BN, p.M - t0);
@@ -488,6 +469,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           tmem_ld16(taddr + c, v);
           epilogue16(p, t0 + c, n, v, mv - c);
         }
+        if (et == 0) trace_mark(5);
       } else {
         int slot = range_start(blockIdx.x, p.total, p.grid) >= tile_u0 ? 0 : 1;
         float *w = p.ws + ((size_t)blockIdx.x * 2 + slot) * p.BN * BM;
@@ -501,10 +483,14 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       }
       tc_fence_before();
       mbar_arrive(&acce_bar[buf]);
-      if (parts > 1) {
+      if (parts > 1 && !p.defer) {
         __threadfence();
         epi_bar();
-        if (et == 0) last_f = atomicAdd(&p.counters[tl], 1) == parts - 1;
+        if (et == 0) {
+          trace_mark(3);
+          last_f = atomicAdd(&p.counters[tl], 1) == parts - 1;
+          trace_mark(4);
+        }
         epi_bar();
         if (last_f) {
           __threadfence();
@@ -526,20 +512,26 @@ __global__ void __launch_bounds__(NTHREADS, 1)
             for (int q16 = 0; q16 < 3; ++q16)
               if (c + 16 * q16 < mv) epilogue16(p, t0 + c + 16 * q16, n, v + 16 * q16, mv - c - 16 * q16);
           }
-          if (et == 0) p.counters[tl] = 0;
+          if (et == 0) {
+            p.counters[tl] = 0;
+            trace_mark(5);
+          }
         }
         epi_bar();
       }
       ++seg;
       a = b;
     }
+    if (et == 0) trace_mark(6);
   }
   tc_fence_before();
   __syncthreads();
+  if (threadIdx.x == 64) trace_mark(7);
   if (p.cluster > 1) {
     // every CTA of the cluster reaches both barriers, on every path
     cooperative_groups::cluster_group cl = cooperative_groups::this_cluster();
     cl.sync();  // all partials staged
+    if (threadIdx.x == 64) trace_mark(4);
     if (warp >= 2) {
       const int P = p.cluster, rank = (int)cl.block_rank();
       const int mv = min(p.BN, p.M);
@@ -559,8 +551,10 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         }
         epilogue16(p, c, n, v, r1 - c);
       }
+      if (threadIdx.x == 64) trace_mark(5);
     }
     cl.sync();  // peers have finished reading this CTA's shared memory
+    if (threadIdx.x == 64) trace_mark(6);
   }
   tc_fence_after();
   if (warp == 0) {
@@ -569,6 +563,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
                  "r"(ncols)
                  : "memory");
   }
+  ts.finish();
 }
 
 // ------------------------------------------------------------ host side
@@ -662,37 +657,44 @@ int gemm_tc_bn(int M) {
 
 size_t gemm_tc_ws_bytes(int num_sms) { return (size_t)num_sms * 2 * 256 * BM * sizeof(float); }
 
-const char *launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, void *out2,
-                           int ld2, const TcWorkspace &ws, cudaStream_t s, const TcNext *next) {
-  if (g.M <= 0) return nullptr;
-  TcParams p{};
-  p.M = g.M;
-  p.N = g.N;
-  p.K = g.K;
-  p.BN = gemm_tc_bn(g.M);
-  p.n_tiles = g.N / BM;
-  p.m_tiles = (g.M + p.BN - 1) / p.BN;
-  p.KB = g.K / BK;
-  // A box may not be taller than the tensor: a single short token tile loads
-  // just its M rows (the MMA's extra columns are never stored).
-  p.brows = p.BN < g.M ? p.BN : g.M;
-  p.total = (long long)p.n_tiles * p.m_tiles * p.KB;
-  p.grid = (int)(p.total < ws.num_sms ? p.total : ws.num_sms);
-  // dynamic shared memory allowed for this kernel (opt-in limit minus static)
+namespace {
+
+// Dynamic shared memory this kernel may use (opt-in limit minus static);
+// < 0 on failure.
+int dyn_smem_limit() {
   static int max_dyn = -1;
   if (max_dyn < 0) {
     int dev = 0, optin = 0;
     cudaFuncAttributes fa{};
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
-    if (cudaFuncGetAttributes(&fa, k_gemm_tc) != cudaSuccess) return "kernel attributes";
-    max_dyn = optin - (int)fa.sharedSizeBytes;
-    if (cudaFuncSetAttribute(k_gemm_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, max_dyn) !=
-        cudaSuccess) {
-      max_dyn = -1;
-      return "cannot raise the dynamic shared memory limit";
-    }
+    if (cudaFuncGetAttributes(&fa, k_gemm_tc) != cudaSuccess) return -1;
+    int lim = optin - (int)fa.sharedSizeBytes;
+    if (cudaFuncSetAttribute(k_gemm_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, lim) !=
+        cudaSuccess)
+      return -1;
+    max_dyn = lim;
   }
+  return max_dyn;
+}
+
+// Tiling, pipeline depth and split of an M x N x K GEMM: fills the shape
+// fields of p and the dynamic shared memory; nullptr on success.
+const char *configure(int M, int N, int K, int num_sms, bool defer, TcParams &p, size_t &smem) {
+  p.M = M;
+  p.N = N;
+  p.K = K;
+  p.BN = gemm_tc_bn(M);
+  p.n_tiles = N / BM;
+  p.m_tiles = (M + p.BN - 1) / p.BN;
+  p.KB = K / BK;
+  // A box may not be taller than the tensor: a single short token tile loads
+  // just its M rows (the MMA's extra columns are never stored).
+  p.brows = p.BN < M ? p.BN : M;
+  p.total = (long long)p.n_tiles * p.m_tiles * p.KB;
+  p.grid = (int)(p.total < num_sms ? p.total : num_sms);
+  int max_dyn = dyn_smem_limit();
+  if (max_dyn < 0) return "cannot raise the dynamic shared memory limit";
   uint32_t stage_bytes = A_BYTES + (uint32_t)p.BN * 128u;
   int smem_budget = max_dyn - 1024;
   p.stages = smem_budget / (int)stage_bytes;
@@ -701,6 +703,23 @@ const char *launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, v
   uint32_t cols = 32;
   while (cols < (uint32_t)p.BN) cols <<= 1;
   p.tmem_cols = cols;
+  smem = 1024 + (size_t)p.stages * stage_bytes;
+  p.defer = defer ? 1 : 0;
+  p.cluster = p.m_tiles == 1 && !defer ? choose_cluster(M, N, num_sms, smem) : 0;
+  if (p.cluster > 1) p.grid = p.n_tiles * p.cluster;
+  return nullptr;
+}
+
+}  // namespace
+
+const char *launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, void *out2,
+                           int ld2, const TcWorkspace &ws, cudaStream_t s, SplitView *defer) {
+  if (defer) *defer = SplitView{};
+  if (g.M <= 0) return nullptr;
+  const bool dfr = defer && epi != GEMM_EPI_SWIGLU;
+  TcParams p{};
+  size_t smem = 0;
+  if (const char *e = configure(g.M, g.N, g.K, ws.num_sms, dfr, p, smem)) return e;
   p.Y = g.Y;
   p.ldy = g.ldy;
   p.bias = g.bias;
@@ -713,22 +732,6 @@ const char *launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, v
   if ((long long)p.n_tiles * p.m_tiles > ws.max_tiles) return "more tiles than counters";
   CUtensorMap tmX;
   if (!make_tmap_bf16(&tmX, g.X, g.M, g.K, p.brows)) return "activation TMA descriptor rejected";
-  size_t smem = 1024 + (size_t)p.stages * stage_bytes;
-  p.cluster = p.m_tiles == 1 ? choose_cluster(g.M, g.N, ws.num_sms, smem) : 0;
-  if (p.cluster > 1) p.grid = p.n_tiles * p.cluster;
-  const CUtensorMap *tmN = &tmW;
-  if (next && next->tm && next->bytes_per_cta > 0) {
-    int nbn = gemm_tc_bn(next->M);
-    long long nm = (next->M + nbn - 1) / nbn;
-    p.next_KB = next->K / BK;
-    p.next_m_tiles = (int)nm;
-    p.next_total = (long long)(next->N / BM) * nm * p.next_KB;
-    p.next_grid = (int)(p.next_total < ws.num_sms ? p.next_total : ws.num_sms);
-    p.next_cluster = nm == 1 ? choose_cluster(next->M, next->N, ws.num_sms, smem) : 0;
-    if (p.next_cluster > 1) p.next_grid = (next->N / BM) * p.next_cluster;
-    p.pf_units = (int)(next->bytes_per_cta / A_BYTES);
-    tmN = next->tm;
-  }
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3(p.grid);
   cfg.blockDim = dim3(NTHREADS);
@@ -750,9 +753,27 @@ const char *launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, v
   }
   cfg.attrs = at;
   cfg.numAttrs = na;
-  cudaLaunchKernelEx(&cfg, k_gemm_tc, tmW, tmX, *tmN, p);
+  cudaLaunchKernelEx(&cfg, k_gemm_tc, tmW, tmX, p);
   cudaError_t e = cudaGetLastError();
+  if (e == cudaSuccess && dfr) {
+    // a tile is split when a range boundary falls inside it
+    bool split = false;
+    for (int i = 0; i < p.grid && !split; ++i)
+      split = range_start(i, p.total, p.grid) % p.KB != 0;
+    if (split) {
+      defer->ws = ws.partials;
+      defer->bias = epi == GEMM_EPI_STORE ? g.bias : nullptr;
+      defer->total = p.total;
+      defer->grid = p.grid;
+      defer->KB = p.KB;
+      defer->BN = p.BN;
+      defer->m_tiles = p.m_tiles;
+      defer->accum = epi == GEMM_EPI_ACCUM ? 1 : 0;
+    }
+  }
   return e == cudaSuccess ? nullptr : cudaGetErrorString(e);
 }
+
+KVR_TRACE_ATTACH(trace_attach_gemm)
 
 }  // namespace kvr

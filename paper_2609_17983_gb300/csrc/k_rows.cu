@@ -76,49 +76,72 @@ template <typename T>
 __global__ void k_embed_rows(const T *embed, const int32_t *tokens,
                              const int32_t *const *doc_tokens, const int32_t *rowdoc,
                              const int32_t *pos, int d, float *h) {
+  TraceScope ts(TK_EMBED);
   pdl_trigger();
   pdl_wait();
+  ts.waited();
   int i = blockIdx.x;
   const int32_t *tk = doc_tokens ? doc_tokens[rowdoc[i]] : tokens;
   size_t base = (size_t)tk[pos[i]] * d;
   for (int c = threadIdx.x; c < d; c += blockDim.x) h[(size_t)i * d + c] = ld(embed, base + c);
 }
 
-// One block of 256 threads per row; the row (d <= 8192, d % 4 == 0) is
-// loaded once into registers with every load issued before the first use.
-template <typename T>
-__global__ void __launch_bounds__(256) k_rmsnorm(const float *h, const float *g, int d, float eps,
-                                                 T *out) {
-  constexpr int NV = 8;  // float4 per thread: 8 * 4 * 256 = 8192 elements
+// One block of 1024 threads per row (d <= 8192, d % 4 == 0: NV = 1 float4
+// per thread up to d = 4096, else 2), each load issued before its first use.  Block i
+// normalises h row row0 + i into out row i.  With a split view, the row is
+// first completed from the GEMM's split-tile partials (their tile table is
+// built once per block in shared memory) and written back to h.
+constexpr int NORM_THREADS = 1024;
+template <typename T, int NV>
+__global__ void __launch_bounds__(NORM_THREADS) k_rmsnorm(float *h, const float *g, int row0,
+                                                          int d, float eps, T *out,
+                                                          const SplitView sv) {
+  __shared__ SplitTile tiles[64];
+  __shared__ float red[NORM_THREADS / 32];
+  TraceScope ts(TK_NORM);
   pdl_trigger();
-  pdl_wait();
-  int i = blockIdx.x;
-  const float4 *x = (const float4 *)(h + (size_t)i * d);
+  const int i = blockIdx.x, row = row0 + i;
   const int nq = d >> 2;
+  if (sv.ws && (int)threadIdx.x < (d >> 7)) {
+    const int mt = row / sv.BN;
+    tiles[threadIdx.x] = split_tile(sv, (long long)threadIdx.x * sv.m_tiles + mt);
+  }
+  pdl_wait();
+  ts.waited();
+  if (sv.ws) __syncthreads();
+  float4 *x = (float4 *)(h + (size_t)row * d);
   float4 v[NV];
   float ss = 0.f;
 #pragma unroll
   for (int k = 0; k < NV; ++k) {
-    int q = k * 256 + threadIdx.x;
-    v[k] = q < nq ? x[q] : make_float4(0.f, 0.f, 0.f, 0.f);
+    const int q = k * NORM_THREADS + threadIdx.x;
+    v[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (q < nq) {
+      v[k] = x[q];
+      if (sv.ws) {
+        const SplitTile st = tiles[q >> 5];
+        if (st.i0 != st.i1) {
+          v[k] = split_value4(sv, st, v[k], row, 4 * q);
+          x[q] = v[k];
+        }
+      }
+    }
+    ss += v[k].x * v[k].x + v[k].y * v[k].y + v[k].z * v[k].z + v[k].w * v[k].w;
   }
-#pragma unroll
-  for (int k = 0; k < NV; ++k) ss += v[k].x * v[k].x + v[k].y * v[k].y + v[k].z * v[k].z + v[k].w * v[k].w;
-  __shared__ float red[8];
   for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
   if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
   __syncthreads();
   float tot = 0.f;
 #pragma unroll
-  for (int w = 0; w < 8; ++w) tot += red[w];
-  float r = 1.0f / sqrtf(tot / (float)d + eps);
+  for (int w = 0; w < NORM_THREADS / 32; ++w) tot += red[w];
+  const float r = 1.0f / sqrtf(tot / (float)d + eps);
   const float4 *gg = (const float4 *)g;
 #pragma unroll
   for (int k = 0; k < NV; ++k) {
-    int q = k * 256 + threadIdx.x;
+    const int q = k * NORM_THREADS + threadIdx.x;
     if (q < nq) {
-      float4 w = gg[q];
-      size_t o = (size_t)i * d + 4 * q;
+      const float4 w = gg[q];
+      const size_t o = (size_t)i * d + 4 * q;
       st(out, o, v[k].x * r * w.x);
       st(out, o + 1, v[k].y * r * w.y);
       st(out, o + 2, v[k].z * r * w.z);
@@ -128,19 +151,29 @@ __global__ void __launch_bounds__(256) k_rmsnorm(const float *h, const float *g,
 }
 
 // grid (M, H + 2G), block dh/2: rotate q and k heads at the row's position;
-// q -> q_out fp32, k and v -> cache (if write_kv).
+// q -> q_out fp32, k and v -> cache (if write_kv).  With a split view the
+// projection is completed from the GEMM's split-tile partials.
 template <typename T>
 __global__ void k_rope_scatter(const float *qkv, const float2 *rope, const int32_t *pos, int H,
                                int G, int dh, int layer, const KVView *views,
                                const int32_t *rowdoc, KVView single, float *q_out,
-                               __nv_bfloat16 *qb_out, float qscale, int write_kv) {
+                               __nv_bfloat16 *qb_out, float qscale, int write_kv,
+                               const SplitView sv) {
+  TraceScope ts(TK_ROPE);
   pdl_trigger();
   pdl_wait();
+  ts.waited();
   int i = blockIdx.x, hh = blockIdx.y, t = threadIdx.x, half = dh >> 1;
   int Nqkv = (H + 2 * G) * dh;
   int p = pos[i];
   const float *x = qkv + (size_t)i * Nqkv + (size_t)hh * dh;
   float x1 = x[t], x2 = x[t + half];
+  if (sv.ws) {
+    // dh divides 128: both halves of the head lie in one feature tile
+    const SplitTile st = split_tile(sv, (long long)((hh * dh) >> 7) * sv.m_tiles + i / sv.BN);
+    x1 = split_value(sv, st, x1, i, hh * dh + t);
+    x2 = split_value(sv, st, x2, i, hh * dh + t + half);
+  }
   if (hh < H + G) {
     float2 cs = rope[(size_t)p * half + t];
     float r1 = x1 * cs.x - x2 * cs.y;
@@ -303,29 +336,34 @@ void launch_embed_rows(const void *embed, int dtype, const int32_t *tokens,
                rowdoc, pos, d, h);
 }
 
-void launch_rmsnorm(const float *h, const float *g, int M, int d, double eps, void *out,
-                    int out_dtype, cudaStream_t s) {
+void launch_rmsnorm(float *h, const float *g, int row0, int M, int d, double eps, void *out,
+                    int out_dtype, cudaStream_t s, const SplitView *sv) {
   if (M <= 0) return;
+  const SplitView v = sv ? *sv : SplitView{};
+  const bool one = d <= 4 * NORM_THREADS;
   if (out_dtype == KVR_DTYPE_BF16)
-    launch_pdl(k_rmsnorm<__nv_bfloat16>, M, 256, 0, s, h, g, d, (float)eps,
-               (__nv_bfloat16 *)out);
+    launch_pdl(one ? k_rmsnorm<__nv_bfloat16, 1> : k_rmsnorm<__nv_bfloat16, 2>, M, NORM_THREADS,
+               0, s, h, g, row0, d, (float)eps, (__nv_bfloat16 *)out, v);
   else
-    launch_pdl(k_rmsnorm<float>, M, 256, 0, s, h, g, d, (float)eps, (float *)out);
+    launch_pdl(one ? k_rmsnorm<float, 1> : k_rmsnorm<float, 2>, M, NORM_THREADS, 0, s, h, g, row0,
+               d, (float)eps, (float *)out, v);
 }
 
 void launch_rope_scatter(const float *qkv, const float2 *rope, const int32_t *pos, int M,
                          const Dims &dm, int layer, const KVView *views, const int32_t *rowdoc,
                          KVView single, float *q_out, void *qb_out, float qscale, bool write_kv,
-                         cudaStream_t s) {
+                         cudaStream_t s, const SplitView *sv) {
   if (M <= 0) return;
   dim3 grid(M, dm.H + 2 * dm.G);
   int wk = write_kv ? 1 : 0;
+  const SplitView v = sv ? *sv : SplitView{};
   if (dm.dtype == KVR_DTYPE_BF16)
     launch_pdl(k_rope_scatter<__nv_bfloat16>, grid, dm.dh / 2, 0, s, qkv, rope, pos, dm.H, dm.G,
-               dm.dh, layer, views, rowdoc, single, q_out, (__nv_bfloat16 *)qb_out, qscale, wk);
+               dm.dh, layer, views, rowdoc, single, q_out, (__nv_bfloat16 *)qb_out, qscale, wk,
+               v);
   else
     launch_pdl(k_rope_scatter<float>, grid, dm.dh / 2, 0, s, qkv, rope, pos, dm.H, dm.G, dm.dh,
-               layer, views, rowdoc, single, q_out, (__nv_bfloat16 *)qb_out, qscale, wk);
+               layer, views, rowdoc, single, q_out, (__nv_bfloat16 *)qb_out, qscale, wk, v);
 }
 
 void launch_swiglu(const float *gu, int M, int F, void *act, int dtype, cudaStream_t s) {
@@ -375,5 +413,7 @@ void launch_rows_copy(KVView v, int dtype, const int32_t *pos, int n_pos, int l0
     k_rows_copy<<<grid_for(n, 256), 256, 0, s>>>(v, pos, n_pos, l0, l1 - l0, (float *)buf,
                                                   to_buf ? 1 : 0);
 }
+
+KVR_TRACE_ATTACH(trace_attach_rows)
 
 }  // namespace kvr

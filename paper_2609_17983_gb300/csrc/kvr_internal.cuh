@@ -66,6 +66,115 @@ struct KVView {
 };
 
 // Scratch of the tensor-core GEMM (split-tile partials, arrival counters).
+// Device timeline trace buffer (see TraceScope).
+struct TraceBuf {
+  unsigned long long *rec = nullptr;
+  unsigned int *count = nullptr;
+  unsigned int cap = 0;
+};
+
+// ---- split-K tiles reduced by the consumer ----
+// The tensor-core GEMM splits its (feature tile, token tile, K block) units
+// into one contiguous stream-K range per CTA: CTA i owns units
+// [range_start(i), range_start(i + 1)).  A tile whose units all fall in one
+// CTA is written whole by that CTA.  In deferred mode a tile split over CTAs
+// i0..i1 is not reduced by the GEMM: each CTA stores its fp32 partial in the
+// workspace slot (i, s) -- s = 0 if the tile is the first of i's range, else
+// 1 -- as [BN rows][128 features], and leaves Y untouched.  The kernel that
+// next reads Y (RMSNorm, RoPE) forms the value itself: Y (accumulate) or the
+// bias (store), plus the sum of the partials in CTA order, which keeps the
+// result deterministic and takes the reduction off the GEMM's tail.
+__host__ __device__ inline long long range_start(long long i, long long total, int grid) {
+  return i * total / grid;
+}
+// CTA whose range holds unit u
+__host__ __device__ inline int cta_of(long long u, long long total, int grid) {
+  return (int)(((u + 1) * grid - 1) / total);
+}
+
+struct SplitView {
+  const float *ws = nullptr;    // null: Y is complete
+  const float *bias = nullptr;  // store mode: added to split tiles
+  long long total = 0;
+  int grid = 0, KB = 0, BN = 0, m_tiles = 0;
+  int accum = 0;  // 1: Y holds the old value the product adds to
+};
+
+// CTAs i0..i1 hold the units of tile tl; the tile is i0's slot s0 and the
+// slot 0 of every later CTA (their ranges start inside it).
+struct SplitTile {
+  int i0, i1, s0;
+};
+__device__ __forceinline__ SplitTile split_tile(const SplitView &sv, long long tl) {
+  const long long u0 = tl * sv.KB;
+  SplitTile st;
+  st.i0 = cta_of(u0, sv.total, sv.grid);
+  st.i1 = cta_of(u0 + sv.KB - 1, sv.total, sv.grid);
+  st.s0 = range_start(st.i0, sv.total, sv.grid) >= u0 ? 0 : 1;
+  return st;
+}
+
+// Sum of the partials of split tile st at element offset `off` within a slot
+// ([BN][128] fp32), in CTA order; up to 8 parts are loaded before the first
+// add, so the whole sum costs one round trip to L2.
+__device__ __forceinline__ float4 split_sum4(const SplitView &sv, const SplitTile &st, size_t off) {
+  const size_t slot = (size_t)sv.BN * 128;
+  float4 x[8];
+  x[0] = __ldcg((const float4 *)(sv.ws + ((size_t)st.i0 * 2 + st.s0) * slot + off));
+#pragma unroll
+  for (int j = 1; j < 8; ++j)
+    if (st.i0 + j <= st.i1) x[j] = __ldcg((const float4 *)(sv.ws + (size_t)(st.i0 + j) * 2 * slot + off));
+  float4 acc = x[0];
+#pragma unroll
+  for (int j = 1; j < 8; ++j)
+    if (st.i0 + j <= st.i1) {
+      acc.x += x[j].x;
+      acc.y += x[j].y;
+      acc.z += x[j].z;
+      acc.w += x[j].w;
+    }
+  for (int i = st.i0 + 8; i <= st.i1; ++i) {
+    const float4 v = __ldcg((const float4 *)(sv.ws + (size_t)i * 2 * slot + off));
+    acc.x += v.x;
+    acc.y += v.y;
+    acc.z += v.z;
+    acc.w += v.w;
+  }
+  return acc;
+}
+__device__ __forceinline__ float split_sum(const SplitView &sv, const SplitTile &st, size_t off) {
+  const size_t slot = (size_t)sv.BN * 128;
+  float x[8];
+  x[0] = __ldcg(sv.ws + ((size_t)st.i0 * 2 + st.s0) * slot + off);
+#pragma unroll
+  for (int j = 1; j < 8; ++j)
+    if (st.i0 + j <= st.i1) x[j] = __ldcg(sv.ws + (size_t)(st.i0 + j) * 2 * slot + off);
+  float acc = x[0];
+#pragma unroll
+  for (int j = 1; j < 8; ++j)
+    if (st.i0 + j <= st.i1) acc += x[j];
+  for (int i = st.i0 + 8; i <= st.i1; ++i) acc += __ldcg(sv.ws + (size_t)i * 2 * slot + off);
+  return acc;
+}
+
+// Value of Y[t][n..n+3] (n % 4 == 0, one tile) given the raw Y entries y.
+__device__ __forceinline__ float4 split_value4(const SplitView &sv, const SplitTile &st, float4 y,
+                                               int t, int n) {
+  if (!sv.ws || st.i0 == st.i1) return y;
+  const int mt = t / sv.BN;
+  const float4 acc = split_sum4(sv, st, (size_t)(t - mt * sv.BN) * 128 + (n & 127));
+  float4 b = y;
+  if (!sv.accum) b = sv.bias ? *(const float4 *)(sv.bias + n) : make_float4(0.f, 0.f, 0.f, 0.f);
+  return make_float4(b.x + acc.x, b.y + acc.y, b.z + acc.z, b.w + acc.w);
+}
+__device__ __forceinline__ float split_value(const SplitView &sv, const SplitTile &st, float y,
+                                             int t, int n) {
+  if (!sv.ws || st.i0 == st.i1) return y;
+  const int mt = t / sv.BN;
+  const float acc = split_sum(sv, st, (size_t)(t - mt * sv.BN) * 128 + (n & 127));
+  return (sv.accum ? y : (sv.bias ? sv.bias[n] : 0.f)) + acc;
+}
+
 struct TcWorkspace {
   float *partials;  // gemm_tc_ws_bytes(num_sms)
   int *counters;    // max_tiles zeroed ints
@@ -104,7 +213,6 @@ struct kvr_model {
   float2 *attn_ws_ml = nullptr;
   size_t attn_ws_floats = 0;
   bool use_tc = true;  // tensor-core GEMM for bf16 shapes it takes
-  bool prefetch = true;  // L2 prefetch of the next GEMM's weights
   bool use_graphs = true;  // CUDA graphs for repeated repair passes
   cudaStream_t stream = nullptr;
   int device = 0;
@@ -123,6 +231,9 @@ struct kvr_model {
   void *save = nullptr;        // stale rows saved by read-only selector passes
   size_t save_bytes = 0;
   int *dev_flag = nullptr;     // device error flag (bounded waits)
+  kvr::TraceBuf trace{};       // attached device timeline buffer, if any
+  kvr::SplitView pending{};    // split tiles of h not yet added (next RMSNorm adds them)
+  bool defer_splits = true;    // GEMM split tiles reduced by the consumer
   // pinned staging for host->device argument copies
   int32_t *stage_h = nullptr;
   int32_t *stage_d = nullptr;
@@ -155,6 +266,102 @@ struct kvr_cache {
 };
 
 namespace kvr {
+
+// ---- device timeline trace ----
+// With a buffer attached, thread 0 of every CTA of the pass kernels appends
+// one record of 16 words: kind | smid << 8 | linear block index << 16; the
+// time the CTA started; the time its wait on the predecessor kernel returned;
+// the time it finished; eight kernel-specific marks (0 where unset); four
+// zero words (%globaltimer, ns).  GEMM marks, each for the CTA's last tile:
+// 0 first operand stage landed, 1 all MMAs complete, 2 accumulator taken by
+// the epilogue, 3 partial tile stored, 4 split-tile arrival counted
+// (stream-K) or partials staged across the cluster, 5 tile reduced and
+// written, 6 epilogue warps done, 7 all warps done.  Attention mark: 0 last key
+// chunk consumed.  The buffer pointer lives in constant memory (one copy per
+// translation unit, set by its trace_attach_* function).  Even detached, the
+// checks lengthen each kernel's critical path, so tracing is compiled only
+// into the KVR_TRACE build of the library; elsewhere the hooks are empty.
+enum TraceKind : int { TK_EMBED = 1, TK_NORM, TK_GEMM, TK_ROPE, TK_ATTN, TK_COMBINE, TK_OTHER };
+#ifdef KVR_TRACE
+static __constant__ TraceBuf g_trace;
+
+__device__ __forceinline__ unsigned long long trace_now() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+// Stamps of thread 0's CTA, in shared memory: start, wait, marks 0..7.
+__device__ __forceinline__ unsigned long long *trace_stamps() {
+  __shared__ unsigned long long t[10];
+  return t;
+}
+
+// Kernel-specific mark i (0..7), by any one thread of the CTA.
+__device__ __forceinline__ void trace_mark(int i) {
+  if (g_trace.rec) trace_stamps()[2 + i] = trace_now();
+}
+
+struct TraceScope {
+  int kind;
+  __device__ explicit TraceScope(int k) : kind(k) {
+    if (threadIdx.x == 0 && g_trace.rec) {
+      unsigned long long *t = trace_stamps();
+      t[0] = t[1] = trace_now();
+#pragma unroll
+      for (int i = 2; i < 10; ++i) t[i] = 0;
+    }
+  }
+  __device__ void waited() {
+    if (threadIdx.x == 0 && g_trace.rec) trace_stamps()[1] = trace_now();
+  }
+  __device__ void finish() {
+    if (threadIdx.x != 0 || !g_trace.rec) return;
+    unsigned long long *t = trace_stamps();
+    if (t[0] == 0) return;
+    unsigned long long t2 = trace_now();
+    unsigned int i = atomicAdd(g_trace.count, 1u);
+    if (i < g_trace.cap) {
+      unsigned int smid;
+      asm volatile("mov.u32 %0, %%smid;" : "=r"(smid));
+      unsigned long long blk =
+          blockIdx.x +
+          (unsigned long long)gridDim.x * (blockIdx.y + (unsigned long long)gridDim.y * blockIdx.z);
+      unsigned long long *r = g_trace.rec + 16ull * i;
+      r[0] = (unsigned long long)kind | (unsigned long long)(smid & 0xff) << 8 | blk << 16;
+      r[1] = t[0];
+      r[2] = t[1];
+      r[3] = t2;
+#pragma unroll
+      for (int k = 0; k < 8; ++k) r[4 + k] = t[2 + k];
+#pragma unroll
+      for (int k = 12; k < 16; ++k) r[k] = 0;
+    }
+    t[0] = 0;
+  }
+  __device__ ~TraceScope() { finish(); }
+};
+#else
+__device__ __forceinline__ void trace_mark(int) {}
+struct TraceScope {
+  __device__ explicit TraceScope(int) {}
+  __device__ void waited() {}
+  __device__ void finish() {}
+};
+#endif
+
+#ifdef KVR_TRACE
+#define KVR_TRACE_ATTACH(fn)                                           \
+  cudaError_t fn(const kvr::TraceBuf &b) {                             \
+    return cudaMemcpyToSymbol(kvr::g_trace, &b, sizeof(kvr::TraceBuf)); \
+  }
+#else
+#define KVR_TRACE_ATTACH(fn) \
+  cudaError_t fn(const kvr::TraceBuf &) { return cudaSuccess; }
+#endif
+cudaError_t trace_attach_rows(const TraceBuf &b);
+cudaError_t trace_attach_gemm(const TraceBuf &b);
+cudaError_t trace_attach_attn(const TraceBuf &b);
 
 // ---- programmatic dependent launch (PDL) ----
 // Kernels of a pass are launched with programmatic stream serialisation: a
@@ -208,13 +415,15 @@ void launch_fill_f32(float *dst, float v, size_t n, cudaStream_t s);
 void launch_embed_rows(const void *embed, int dtype, const int32_t *tokens,
                        const int32_t *const *doc_tokens, const int32_t *rowdoc,
                        const int32_t *pos, int M, int d, float *h, cudaStream_t s);
-void launch_rmsnorm(const float *h, const float *g, int M, int d, double eps, void *out,
-                    int out_dtype, cudaStream_t s);
+// Rows row0 .. row0+M-1 of h; out row i is h row row0 + i.  With a split
+// view (rows indexed from h's base), the completed rows are written back to h.
+void launch_rmsnorm(float *h, const float *g, int row0, int M, int d, double eps, void *out,
+                    int out_dtype, cudaStream_t s, const SplitView *sv = nullptr);
 // q_out: fp32 rotated q; qb_out (optional): bf16 rotated q times qscale.
 void launch_rope_scatter(const float *qkv, const float2 *rope, const int32_t *pos, int M,
                          const Dims &dm, int layer, const KVView *views, const int32_t *rowdoc,
                          KVView single, float *q_out, void *qb_out, float qscale, bool write_kv,
-                         cudaStream_t s);
+                         cudaStream_t s, const SplitView *sv = nullptr);
 void launch_swiglu(const float *gu, int M, int F, void *act, int dtype, cudaStream_t s);
 void launch_cache_gather(KVView v, int dtype, const int32_t *pos, int n_pos, int l0, int l1,
                          int G, int dh, float *k_out, float *v_out, cudaStream_t s);
@@ -246,17 +455,12 @@ int gemm_tc_bn(int M);
 size_t gemm_tc_ws_bytes(int num_sms);
 // GEMM_EPI_SWIGLU: W rows interleaved gate/up in blocks of 16; writes
 // out2[t][f] = bf16(silu(gate) * up), f < N/2, row stride ld2.
-// The GEMM that follows in the stream: while this one drains, each CTA
-// prefetches into L2 up to bytes_per_cta of its share of next's weights.
-struct TcNext {
-  const CUtensorMap *tm;
-  int M, N, K;
-  long long bytes_per_cta;
-};
 // Returns nullptr on success, else what went wrong.
+// defer (STORE / ACCUM epilogues only): leave split tiles to the consumer
+// and describe them in *defer; defer->ws stays null when no tile was split.
 const char *launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, void *out2,
                            int ld2, const TcWorkspace &ws, cudaStream_t s,
-                           const TcNext *next = nullptr);
+                           SplitView *defer = nullptr);
 
 // ---- kernels: attention ----
 // o[i] = softmax(q_i K[0..pos_i]^T / sqrt(dh)) V[0..pos_i] for every row i,

@@ -3,8 +3,10 @@
 The functions below carry the names of the C entry points in
 ``include/kvrepair.h`` and forward to them; every step of the method runs in
 the library's CUDA kernels.  Importing this module loads
-``libkvrepair.so`` from this package directory and raises ImportError if it
-has not been built (``__graft_entry__.build()``): there is no fallback.
+``libkvrepair.so`` from this package directory (``libkvrepair_trace.so``, the
+build with the device timeline trace, when ``KVR_LIB=trace``) and raises
+ImportError if it has not been built (``__graft_entry__.build()``): there is
+no fallback.
 
 ``Model`` and ``Cache`` are thin owners of the C handles for convenience.
 """
@@ -17,7 +19,8 @@ import weakref
 import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(_HERE, "libkvrepair.so")
+LIB_PATH = os.path.join(_HERE, "libkvrepair_trace.so" if os.environ.get("KVR_LIB") == "trace"
+                        else "libkvrepair.so")
 if not os.path.exists(LIB_PATH):
     raise ImportError(f"{LIB_PATH} is missing: build it with __graft_entry__.build()")
 _lib = ctypes.CDLL(LIB_PATH)
@@ -88,6 +91,8 @@ _sigs = {
     "kvr_profile_reset": ([_P], _I32),
     "kvr_profile_read": ([_P, _I32, _P, _P, _P, _P, _I32, _P], _I32),
     "kvr_launch_count": ([_P], ctypes.c_int64),
+    "kvr_trace_enable": ([_P, _I32], _I32),
+    "kvr_trace_read": ([_P, _P, _I32, _P], _I32),
     "kvr_linear": ([_P, ctypes.c_char_p, _I32, _P, _I32, _P], _I32),
     "kvr_linear_noalloc": ([_P, ctypes.c_char_p, _I32, _P, _I32, _P], _I32),
     "kvr_transplant": ([_P, _P, _P, _I32], _I32),
@@ -294,6 +299,19 @@ def kvr_profile_read(model) -> dict:
             for i, lab in enumerate(labels)}
 
 
+def kvr_trace_enable(model, capacity: int) -> None:
+    _check(_lib.kvr_trace_enable(model, int(capacity)))
+
+
+def kvr_trace_read(model, cap: int) -> np.ndarray:
+    """Trace records as uint64 [n][16]: kind | smid << 8 | block << 16,
+    start, wait return, end, marks 0..7, zeros (ns)."""
+    out = np.zeros((max(cap, 1), 16), np.uint64)
+    n = ctypes.c_int32(0)
+    _check(_lib.kvr_trace_read(model, out.ctypes.data, int(cap), ctypes.byref(n)))
+    return out[:min(n.value, cap)].copy()
+
+
 def kvr_launch_count(model) -> int:
     return int(_lib.kvr_launch_count(model))
 
@@ -386,6 +404,14 @@ class Model:
                       mlp_norm=(d,))
         dt = np.uint16 if c["dtype"] == "bf16" else np.float32
         return kvr_model_read_tensor(self.h, name, layer, shapes[name], dt)
+
+    def trace_enable(self, capacity: int) -> None:
+        """Attach a device timeline buffer of `capacity` records (0 detaches)."""
+        self._trace_cap = int(capacity)
+        kvr_trace_enable(self.h, capacity)
+
+    def trace_read(self) -> np.ndarray:
+        return kvr_trace_read(self.h, getattr(self, "_trace_cap", 0))
 
     def launches(self) -> int:
         return kvr_launch_count(self.h)
