@@ -259,6 +259,8 @@ kvr_status layer_rest(kvr_model *m, const Rows &r, int l) {
   KVR_TRY(gemm(m, P_GEMM_O, m->attn, w.wo, w.tc_o ? &w.tm_o : nullptr, nullptr, m->h, r.M, dm.d,
                dm.H * dm.dh, GEMM_EPI_ACCUM, &m->pending));
   KVR_TRY(norm(m, w.mlp_norm, r.M));
+  // gate/up reduces its own split tiles (SwiGLU needs the complete sums; a
+  // separate reduction kernel measured slower than the in-GEMM fixup)
   KVR_TRY(gemm(m, P_GEMM_GU, m->a, w.wgu, w.tc_gu ? &w.tm_gu : nullptr, nullptr, nullptr, r.M,
                2 * dm.F, dm.d, GEMM_EPI_SWIGLU));
   KVR_TRY(gemm(m, P_GEMM_DOWN, m->act, w.wd, w.tc_d ? &w.tm_d : nullptr, nullptr, m->h, r.M, dm.d,
@@ -321,7 +323,8 @@ kvr_status sync_model(kvr_model *m) {
   if (e != cudaSuccess) return fail(KVR_E_CUDA, "device error: %s", cudaGetErrorString(e));
   if (flag) {
     cudaMemset(m->dev_flag, 0, sizeof(int));
-    if (m->tcw.counters) cudaMemset(m->tcw.counters, 0, (size_t)m->tcw.max_tiles * sizeof(int));
+    if (m->tcw.counters)
+      cudaMemset(m->tcw.counters, 0, 2 * (size_t)m->tcw.max_tiles * sizeof(int));
     return fail(KVR_E_DEVICE_TIMEOUT, "a bounded device wait ran out (code %d)", flag);
   }
   return KVR_OK;
@@ -700,9 +703,9 @@ kvr_status kvr_model_create(const kvr_model_config *cfg, const kvr_weights *wts,
     m->tcw.max_tiles = 1 << 16;
     m->tcw.dev_flag = m->dev_flag;
     m->tcw.partials = (float *)dev_alloc(gemm_tc_ws_bytes(m->num_sms));
-    m->tcw.counters = (int *)dev_alloc((size_t)m->tcw.max_tiles * sizeof(int));
+    m->tcw.counters = (int *)dev_alloc(2 * (size_t)m->tcw.max_tiles * sizeof(int));
     if (!m->tcw.partials || !m->tcw.counters) return bail(fail(KVR_E_NOMEM, "GEMM workspace"));
-    cudaMemset(m->tcw.counters, 0, (size_t)m->tcw.max_tiles * sizeof(int));
+    cudaMemset(m->tcw.counters, 0, 2 * (size_t)m->tcw.max_tiles * sizeof(int));
     auto mk = [&](CUtensorMap *tm, const void *w, int N, int K) {
       return gemm_tc_supported(N, K) && make_tmap_bf16(tm, w, N, K, 128);
     };

@@ -18,6 +18,8 @@
 // elsewhere (operator R, Sec. 3).
 #include <math.h>
 
+#include <type_traits>
+
 #include "kvr_internal.cuh"
 
 namespace kvr {
@@ -102,8 +104,11 @@ __global__ void __launch_bounds__(MAXW * 32, 1) k_attn_tc(const AttnTcParams p) 
 
   TraceScope ts(TK_ATTN);
   pdl_trigger();
-  pdl_wait();
-  ts.waited();
+  // The block table, positions and page table are written before the pass;
+  // the cache pages are final except for the pass's own rows, which the RoPE
+  // kernel writes.  So everything up to the wait may read them, and the key
+  // range of this CTA is pulled into L2 meanwhile (the RoPE writes land in
+  // the same L2 lines).
   const int split = blockIdx.x, g = blockIdx.y, blk = blockIdx.z;
   const int4 bd = p.blocks[blk];
   const int row0 = bd.x, nrows = bd.y, kmax = bd.z;
@@ -116,6 +121,13 @@ __global__ void __launch_bounds__(MAXW * 32, 1) k_attn_tc(const AttnTcParams p) 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int nthr = blockDim.x, nq = blockDim.x >> 1;  // query vectors of this launch
   const __nv_bfloat16 *cache = (const __nv_bfloat16 *)kv.pages;
+  if (tid < 2 * (c1 - c0)) {
+    const __nv_bfloat16 *pg = cache + kv.offset(p.layer, tid & 1, g, (c0 + (tid >> 1)) * CHUNK);
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(pg), "r"(TILE) : "memory");
+  }
+  for (int v = tid; v < nq; v += nthr) spos[v] = v < mq ? p.pos[row0 + v / p.grp] : -1;
+  pdl_wait();
+  ts.waited();
 
   auto load_chunk = [&](int c, int buf) {
     const __nv_bfloat16 *kp = cache + kv.offset(p.layer, 0, g, c * CHUNK);
@@ -144,7 +156,6 @@ __global__ void __launch_bounds__(MAXW * 32, 1) k_attn_tc(const AttnTcParams p) 
     }
   }
   load_chunk(c0, 0);
-  for (int v = tid; v < nq; v += nthr) spos[v] = v < mq ? p.pos[row0 + v / p.grp] : -1;
 
   const bool active = warp * 16 < mq;
   const int v0 = warp * 16 + (lane >> 2), v1 = v0 + 8;
@@ -306,6 +317,15 @@ __global__ void __launch_bounds__(256) k_attn_combine(const AttnTcParams p) {
   const int ns = (n_chunks + cps - 1) / cps;  // non-empty splits
   const size_t stride = (size_t)p.n_blocks * p.G;  // between splits, in (block, head) units
   const size_t base = (size_t)blk * p.G + g;
+  constexpr int VPL = DH / 32;
+  constexpr int NB = 24;  // splits whose partial outputs load in the first round trip
+  using VecT = typename std::conditional<VPL == 4, float4, float2>::type;
+  const VecT *src = (const VecT *)(p.ws_o + (base * MAXQ + v) * DH) + lane;
+  const size_t sstride = stride * MAXQ * DH / VPL;  // in vectors
+  VecT x[NB];
+#pragma unroll
+  for (int j = 0; j < NB; ++j)
+    if (j < ns) x[j] = __ldcg(src + j * sstride);
   // (max, sum) of up to 64 splits, two per lane
   float2 ml0 = lane < ns ? p.ws_ml[(base + lane * stride) * MAXQ + v] : make_float2(-INFINITY, 0.f);
   float2 ml1 = lane + 32 < ns ? p.ws_ml[(base + (lane + 32) * stride) * MAXQ + v]
@@ -316,27 +336,25 @@ __global__ void __launch_bounds__(256) k_attn_combine(const AttnTcParams p) {
   const float w1 = ml1.y > 0.f ? exp2f(ml1.x - mx) : 0.f;
   float l = w0 * ml0.y + w1 * ml1.y;
   for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
-  constexpr int VPL = DH / 32;
   float acc[VPL];
 #pragma unroll
   for (int i = 0; i < VPL; ++i) acc[i] = 0.f;
-  const float *src = p.ws_o + (base * MAXQ + v) * DH + lane * VPL;
-  const size_t sstride = stride * MAXQ * DH;
-  for (int s0 = 0; s0 < ns; s0 += 8) {
-    float x[8][VPL];
+  // in split order, as the partials of split j carry weight w_j
 #pragma unroll
-    for (int j = 0; j < 8; ++j)
+  for (int j = 0; j < NB; ++j) {
+    const float w = __shfl_sync(0xffffffffu, w0, j & 31);
+    if (j < ns) {
+      const float *xv = (const float *)&x[j];
 #pragma unroll
-      for (int i = 0; i < VPL; ++i) x[j][i] = s0 + j < ns ? src[(s0 + j) * sstride + i] : 0.f;
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      int sj = s0 + j;
-      float w = __shfl_sync(0xffffffffu, sj < 32 ? w0 : w1, sj & 31);
-      if (sj < ns) {
-#pragma unroll
-        for (int i = 0; i < VPL; ++i) acc[i] += w * x[j][i];
-      }
+      for (int i = 0; i < VPL; ++i) acc[i] += w * xv[i];
     }
+  }
+  for (int sj = NB; sj < ns; ++sj) {
+    const float w = __shfl_sync(0xffffffffu, sj < 32 ? w0 : w1, sj & 31);
+    const VecT y = __ldcg(src + sj * sstride);
+    const float *yv = (const float *)&y;
+#pragma unroll
+    for (int i = 0; i < VPL; ++i) acc[i] += w * yv[i];
   }
   const float inv = l > 0.f ? 1.f / l : 0.f;
   const int r = bd.x + v / p.grp, hh = g * p.grp + v % p.grp;

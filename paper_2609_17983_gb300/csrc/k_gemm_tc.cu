@@ -63,7 +63,8 @@ struct TcParams {
   void *out2;  // SwiGLU output (bf16 [M][N/2])
   int ld2;
   float *ws;        // [grid][2][BN][128] fp32 partial tiles
-  int *counters;    // [n_tiles * m_tiles] arrival counters (self-resetting)
+  int *counters;    // [2][max_tiles]: arrivals, then published parts (self-resetting)
+  long long max_tiles;
   int *dev_flag;
   int cluster;  // > 1: cluster split-K with this many CTAs per tile
   int defer;    // 1: split tiles are left as partials for the consumer
@@ -220,16 +221,20 @@ __device__ __forceinline__ void epilogue16(const TcParams &p, int t0, int n, con
                                            int cnt) {
   if (p.epi == GEMM_EPI_SWIGLU) {
     // rows 32b..32b+15 of W are gate, 32b+16..32b+31 up, of features
-    // 16b..16b+15; lane = n % 32
-    int r = n & 31;
-    __nv_bfloat16 *out = (__nv_bfloat16 *)p.out2 + (n >> 5) * 16 + r;
+    // 16b..16b+15; lane = n % 32.  Lanes r and r ^ 16 swap their values, so
+    // both hold gate and up of feature r % 16; the low half then writes the
+    // even rows and the high half the odd ones.
+    const int r = n & 31, hi = r >> 4;
+    float o[16];
 #pragma unroll
-    for (int j = 0; j < 16; ++j) {
-      float u = __shfl_down_sync(0xffffffffu, v[j], 16);
-      if (j < cnt && r < 16) {
-        float g = v[j];
-        out[(size_t)(t0 + j) * p.ld2] = __float2bfloat16_rn(g / (1.0f + expf(-g)) * u);
-      }
+    for (int j = 0; j < 16; ++j) o[j] = __shfl_xor_sync(0xffffffffu, v[j], 16);
+    __nv_bfloat16 *out = (__nv_bfloat16 *)p.out2 + (size_t)t0 * p.ld2 + (n >> 5) * 16 + (r & 15);
+#pragma unroll
+    for (int jj = 0; jj < 8; ++jj) {
+      // low lanes hold gate in v, up in o; high lanes the reverse
+      const float g = hi ? o[2 * jj + 1] : v[2 * jj], u = hi ? v[2 * jj + 1] : o[2 * jj];
+      const int j = 2 * jj + hi;
+      if (j < cnt) out[(size_t)j * p.ld2] = __float2bfloat16_rn(swiglu_bf16path(g, u));
     }
     return;
   }
@@ -470,7 +475,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           epilogue16(p, t0 + c, n, v, mv - c);
         }
         if (et == 0) trace_mark(5);
-      } else {
+      } else if (p.defer) {
+        // the consumer of Y adds this part: store it and go on
         int slot = range_start(blockIdx.x, p.total, p.grid) >= tile_u0 ? 0 : 1;
         float *w = p.ws + ((size_t)blockIdx.x * 2 + slot) * p.BN * BM;
         for (int c = 0; c < mv; c += 16) {
@@ -480,45 +486,97 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           for (int j = 0; j < 16; ++j)
             if (c + j < mv) w[(size_t)(c + j) * BM + f] = v[j];
         }
-      }
-      tc_fence_before();
-      mbar_arrive(&acce_bar[buf]);
-      if (parts > 1 && !p.defer) {
-        __threadfence();
+        if (et == 0) trace_mark(3);
+      } else {
+        // Reduced by the last CTA to arrive.  Arrival comes first: a CTA that
+        // is not last stores its part and then publishes it; the last one
+        // keeps its own part in TMEM, waits (bounded) until the others are
+        // published, and sums all parts in CTA order.
         epi_bar();
         if (et == 0) {
-          trace_mark(3);
           last_f = atomicAdd(&p.counters[tl], 1) == parts - 1;
           trace_mark(4);
         }
         epi_bar();
-        if (last_f) {
-          __threadfence();
-          // 48 rows of one part per round trip: all their loads are in flight
-          for (int c = 0; c < mv; c += 48) {
-            float v[48];
+        if (!last_f) {
+          int slot = range_start(blockIdx.x, p.total, p.grid) >= tile_u0 ? 0 : 1;
+          float *w = p.ws + ((size_t)blockIdx.x * 2 + slot) * p.BN * BM;
+          for (int c = 0; c < mv; c += 16) {
+            float v[16];
+            tmem_ld16(taddr + c, v);
 #pragma unroll
-            for (int j = 0; j < 48; ++j) v[j] = 0.f;
-            for (int i = i_first; i <= i_last; ++i) {
-              int sl = range_start(i, p.total, p.grid) >= tile_u0 ? 0 : 1;
-              const float *src = p.ws + (((size_t)i * 2 + sl) * p.BN + c) * BM + f;
-              float x[48];
-#pragma unroll
-              for (int j = 0; j < 48; ++j) x[j] = c + j < mv ? __ldcg(src + (size_t)j * BM) : 0.f;
-#pragma unroll
-              for (int j = 0; j < 48; ++j) v[j] += x[j];
-            }
-#pragma unroll
-            for (int q16 = 0; q16 < 3; ++q16)
-              if (c + 16 * q16 < mv) epilogue16(p, t0 + c + 16 * q16, n, v + 16 * q16, mv - c - 16 * q16);
+            for (int j = 0; j < 16; ++j)
+              if (c + j < mv) w[(size_t)(c + j) * BM + f] = v[j];
           }
+          __threadfence();
+          epi_bar();
           if (et == 0) {
-            p.counters[tl] = 0;
-            trace_mark(5);
+            atomicAdd(&p.counters[p.max_tiles + tl], 1);
+            trace_mark(3);
+          }
+        } else {
+          if (et == 0) {
+            volatile int *ready = p.counters + p.max_tiles + tl;
+            const uint64_t t0w = gtime_ns();
+            for (uint32_t it = 0; *ready < parts - 1; ++it)
+              if ((it & 63) == 63 && (*abort_v || gtime_ns() - t0w > WAIT_NS)) {
+                if (!*abort_v) {
+                  *abort_v = 1;
+                  atomicOr(p.dev_flag, 32);
+                }
+                break;
+              }
+          }
+          epi_bar();
+          if (!*abort_v) {
+            __threadfence();
+            // two parts and at most 48 rows: the other part in one round trip
+            const bool pre = parts == 2 && mv <= 48;
+            float other[48];
+            if (pre) {
+              const int o = (int)blockIdx.x == i_first ? i_last : i_first;
+              const int so = range_start(o, p.total, p.grid) >= tile_u0 ? 0 : 1;
+              const float *src = p.ws + ((size_t)o * 2 + so) * p.BN * BM + f;
+#pragma unroll
+              for (int j = 0; j < 48; ++j) other[j] = j < mv ? __ldcg(src + (size_t)j * BM) : 0.f;
+            }
+#pragma unroll 1
+            for (int c = 0; c < mv; c += 16) {
+              float own[16], v[16];
+              tmem_ld16(taddr + c, own);
+#pragma unroll
+              for (int j = 0; j < 16; ++j) v[j] = 0.f;
+              for (int i = i_first; i <= i_last; ++i) {
+                if (i == (int)blockIdx.x) {
+#pragma unroll
+                  for (int j = 0; j < 16; ++j) v[j] += own[j];
+                } else if (pre) {
+                  // rows c..c+15 of the preloaded part (c is 0, 16 or 32)
+#pragma unroll
+                  for (int j = 0; j < 16; ++j)
+                    v[j] += c == 0 ? other[j] : c == 16 ? other[16 + j] : other[32 + j];
+                } else {
+                  const int si = range_start(i, p.total, p.grid) >= tile_u0 ? 0 : 1;
+                  const float *src = p.ws + (((size_t)i * 2 + si) * p.BN + c) * BM + f;
+                  float x[16];
+#pragma unroll
+                  for (int j = 0; j < 16; ++j) x[j] = c + j < mv ? __ldcg(src + (size_t)j * BM) : 0.f;
+#pragma unroll
+                  for (int j = 0; j < 16; ++j) v[j] += x[j];
+                }
+              }
+              epilogue16(p, t0 + c, n, v, mv - c);
+            }
+            if (et == 0) {
+              p.counters[tl] = 0;
+              p.counters[p.max_tiles + tl] = 0;
+              trace_mark(5);
+            }
           }
         }
-        epi_bar();
       }
+      tc_fence_before();
+      mbar_arrive(&acce_bar[buf]);
       ++seg;
       a = b;
     }
@@ -716,10 +774,18 @@ const char *launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, v
                            int ld2, const TcWorkspace &ws, cudaStream_t s, SplitView *defer) {
   if (defer) *defer = SplitView{};
   if (g.M <= 0) return nullptr;
-  const bool dfr = defer && epi != GEMM_EPI_SWIGLU;
+  bool dfr = defer != nullptr && epi != GEMM_EPI_SWIGLU;
   TcParams p{};
   size_t smem = 0;
   if (const char *e = configure(g.M, g.N, g.K, ws.num_sms, dfr, p, smem)) return e;
+  if (dfr) {
+    // CTAs per tile: at most ceil(KB / (units per CTA)) + 1
+    long long per = p.total / p.grid;
+    if (per < 1 || (p.KB + per - 1) / per + 1 > SPLIT_MAX_PARTS) {
+      dfr = false;
+      if (const char *e = configure(g.M, g.N, g.K, ws.num_sms, false, p, smem)) return e;
+    }
+  }
   p.Y = g.Y;
   p.ldy = g.ldy;
   p.bias = g.bias;
@@ -728,6 +794,7 @@ const char *launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, v
   p.ld2 = ld2;
   p.ws = ws.partials;
   p.counters = ws.counters;
+  p.max_tiles = ws.max_tiles;
   p.dev_flag = ws.dev_flag;
   if ((long long)p.n_tiles * p.m_tiles > ws.max_tiles) return "more tiles than counters";
   CUtensorMap tmX;
@@ -769,6 +836,7 @@ const char *launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, v
       defer->BN = p.BN;
       defer->m_tiles = p.m_tiles;
       defer->accum = epi == GEMM_EPI_ACCUM ? 1 : 0;
+      defer->small = (p.total + 1) * (long long)p.grid < (1ll << 31) ? 1 : 0;
     }
   }
   return e == cudaSuccess ? nullptr : cudaGetErrorString(e);

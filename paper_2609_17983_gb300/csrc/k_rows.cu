@@ -152,7 +152,9 @@ __global__ void __launch_bounds__(NORM_THREADS) k_rmsnorm(float *h, const float 
 
 // grid (M, H + 2G), block dh/2: rotate q and k heads at the row's position;
 // q -> q_out fp32, k and v -> cache (if write_kv).  With a split view the
-// projection is completed from the GEMM's split-tile partials.
+// projection is completed from the GEMM's split-tile partials.  Positions,
+// the RoPE table, the page table and the bias are written before the pass,
+// so they are read before the wait on the projection.
 template <typename T>
 __global__ void k_rope_scatter(const float *qkv, const float2 *rope, const int32_t *pos, int H,
                                int G, int dh, int layer, const KVView *views,
@@ -161,23 +163,46 @@ __global__ void k_rope_scatter(const float *qkv, const float2 *rope, const int32
                                const SplitView sv) {
   TraceScope ts(TK_ROPE);
   pdl_trigger();
+  const int i = blockIdx.x, hh = blockIdx.y, t = threadIdx.x, half = dh >> 1;
+  const int Nqkv = (H + 2 * G) * dh;
+  const int n1 = hh * dh + t, n2 = n1 + half;
+  const int p = pos[i];
+  float2 cs = make_float2(1.f, 0.f);
+  if (hh < H + G) cs = rope[(size_t)p * half + t];
+  T *c = nullptr;
+  size_t o = 0;
+  if (hh >= H && write_kv) {
+    const KVView v = views ? views[rowdoc[i]] : single;
+    const int kv = hh < H + G ? 0 : 1;
+    c = (T *)v.pages;
+    o = v.offset(layer, kv, hh - H - kv * G, p);
+  }
+  // dh divides 128: both halves of the head lie in one feature tile
+  SplitTile stl{0, 0, 0};
+  float b1 = 0.f, b2 = 0.f;
+  if (sv.ws) {
+    stl = split_tile(sv, (long long)((hh * dh) >> 7) * sv.m_tiles + i / sv.BN);
+    if (sv.bias) {
+      b1 = sv.bias[n1];
+      b2 = sv.bias[n2];
+    }
+  }
+  const bool split = sv.ws && stl.i0 != stl.i1;
   pdl_wait();
   ts.waited();
-  int i = blockIdx.x, hh = blockIdx.y, t = threadIdx.x, half = dh >> 1;
-  int Nqkv = (H + 2 * G) * dh;
-  int p = pos[i];
-  const float *x = qkv + (size_t)i * Nqkv + (size_t)hh * dh;
-  float x1 = x[t], x2 = x[t + half];
-  if (sv.ws) {
-    // dh divides 128: both halves of the head lie in one feature tile
-    const SplitTile st = split_tile(sv, (long long)((hh * dh) >> 7) * sv.m_tiles + i / sv.BN);
-    x1 = split_value(sv, st, x1, i, hh * dh + t);
-    x2 = split_value(sv, st, x2, i, hh * dh + t + half);
+  float x1, x2;
+  if (split) {
+    const size_t off = (size_t)(i - (i / sv.BN) * sv.BN) * 128;
+    x1 = b1 + split_sum(sv, stl, off + (n1 & 127));
+    x2 = b2 + split_sum(sv, stl, off + (n2 & 127));
+  } else {
+    const float *x = qkv + (size_t)i * Nqkv;
+    x1 = x[n1];
+    x2 = x[n2];
   }
   if (hh < H + G) {
-    float2 cs = rope[(size_t)p * half + t];
-    float r1 = x1 * cs.x - x2 * cs.y;
-    float r2 = x2 * cs.x + x1 * cs.y;
+    const float r1 = x1 * cs.x - x2 * cs.y;
+    const float r2 = x2 * cs.x + x1 * cs.y;
     x1 = r1;
     x2 = r2;
   }
@@ -192,12 +217,7 @@ __global__ void k_rope_scatter(const float *qkv, const float2 *rope, const int32
     }
     return;
   }
-  if (!write_kv) return;
-  KVView v = views ? views[rowdoc[i]] : single;
-  int kv = hh < H + G ? 0 : 1;
-  int g = hh - H - kv * G;
-  T *c = (T *)v.pages;
-  size_t o = v.offset(layer, kv, g, p);
+  if (!c) return;
   st(c, o + t, x1);
   st(c, o + t + half, x2);
 }

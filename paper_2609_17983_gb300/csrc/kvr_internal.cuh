@@ -73,6 +73,16 @@ struct TraceBuf {
   unsigned int cap = 0;
 };
 
+// silu(g) * u for the bf16 tensor-core GEMM's fused epilogue: the logistic
+// function through tanh, sigma(g) = (1 + tanh(g / 2)) / 2, on the hardware
+// tanh approximation (one special-function op per element; its relative
+// error, below 1e-3, is far under the bf16 rounding of the result).
+__device__ __forceinline__ float swiglu_bf16path(float g, float u) {
+  float t;
+  asm("tanh.approx.f32 %0, %1;" : "=f"(t) : "f"(0.5f * g));
+  return 0.5f * g * (1.0f + t) * u;
+}
+
 // ---- split-K tiles reduced by the consumer ----
 // The tensor-core GEMM splits its (feature tile, token tile, K block) units
 // into one contiguous stream-K range per CTA: CTA i owns units
@@ -98,6 +108,7 @@ struct SplitView {
   long long total = 0;
   int grid = 0, KB = 0, BN = 0, m_tiles = 0;
   int accum = 0;  // 1: Y holds the old value the product adds to
+  int small = 0;  // 1: (total + 1) * grid < 2^31, so 32-bit index math is exact
 };
 
 // CTAs i0..i1 hold the units of tile tl; the tile is i0's slot s0 and the
@@ -106,8 +117,16 @@ struct SplitTile {
   int i0, i1, s0;
 };
 __device__ __forceinline__ SplitTile split_tile(const SplitView &sv, long long tl) {
-  const long long u0 = tl * sv.KB;
   SplitTile st;
+  if (sv.small) {
+    const unsigned u0 = (unsigned)tl * (unsigned)sv.KB, T = (unsigned)sv.total,
+                   g = (unsigned)sv.grid;
+    st.i0 = (int)(((u0 + 1) * g - 1) / T);
+    st.i1 = (int)(((u0 + sv.KB) * g - 1) / T);
+    st.s0 = (unsigned)st.i0 * T / g >= u0 ? 0 : 1;
+    return st;
+  }
+  const long long u0 = tl * sv.KB;
   st.i0 = cta_of(u0, sv.total, sv.grid);
   st.i1 = cta_of(u0 + sv.KB - 1, sv.total, sv.grid);
   st.s0 = range_start(st.i0, sv.total, sv.grid) >= u0 ? 0 : 1;
@@ -115,45 +134,39 @@ __device__ __forceinline__ SplitTile split_tile(const SplitView &sv, long long t
 }
 
 // Sum of the partials of split tile st at element offset `off` within a slot
-// ([BN][128] fp32), in CTA order; up to 8 parts are loaded before the first
-// add, so the whole sum costs one round trip to L2.
+// ([BN][128] fp32), in CTA order.  A deferred GEMM splits no tile over more
+// than SPLIT_MAX_PARTS CTAs, so the code is straight-line: every load is
+// issued before the first add and the sum costs one round trip to L2.
+constexpr int SPLIT_MAX_PARTS = 8;
 __device__ __forceinline__ float4 split_sum4(const SplitView &sv, const SplitTile &st, size_t off) {
   const size_t slot = (size_t)sv.BN * 128;
-  float4 x[8];
+  float4 x[SPLIT_MAX_PARTS];
   x[0] = __ldcg((const float4 *)(sv.ws + ((size_t)st.i0 * 2 + st.s0) * slot + off));
 #pragma unroll
-  for (int j = 1; j < 8; ++j)
+  for (int j = 1; j < SPLIT_MAX_PARTS; ++j)
     if (st.i0 + j <= st.i1) x[j] = __ldcg((const float4 *)(sv.ws + (size_t)(st.i0 + j) * 2 * slot + off));
   float4 acc = x[0];
 #pragma unroll
-  for (int j = 1; j < 8; ++j)
+  for (int j = 1; j < SPLIT_MAX_PARTS; ++j)
     if (st.i0 + j <= st.i1) {
       acc.x += x[j].x;
       acc.y += x[j].y;
       acc.z += x[j].z;
       acc.w += x[j].w;
     }
-  for (int i = st.i0 + 8; i <= st.i1; ++i) {
-    const float4 v = __ldcg((const float4 *)(sv.ws + (size_t)i * 2 * slot + off));
-    acc.x += v.x;
-    acc.y += v.y;
-    acc.z += v.z;
-    acc.w += v.w;
-  }
   return acc;
 }
 __device__ __forceinline__ float split_sum(const SplitView &sv, const SplitTile &st, size_t off) {
   const size_t slot = (size_t)sv.BN * 128;
-  float x[8];
+  float x[SPLIT_MAX_PARTS];
   x[0] = __ldcg(sv.ws + ((size_t)st.i0 * 2 + st.s0) * slot + off);
 #pragma unroll
-  for (int j = 1; j < 8; ++j)
+  for (int j = 1; j < SPLIT_MAX_PARTS; ++j)
     if (st.i0 + j <= st.i1) x[j] = __ldcg(sv.ws + (size_t)(st.i0 + j) * 2 * slot + off);
   float acc = x[0];
 #pragma unroll
-  for (int j = 1; j < 8; ++j)
+  for (int j = 1; j < SPLIT_MAX_PARTS; ++j)
     if (st.i0 + j <= st.i1) acc += x[j];
-  for (int i = st.i0 + 8; i <= st.i1; ++i) acc += __ldcg(sv.ws + (size_t)i * 2 * slot + off);
   return acc;
 }
 
@@ -177,7 +190,7 @@ __device__ __forceinline__ float split_value(const SplitView &sv, const SplitTil
 
 struct TcWorkspace {
   float *partials;  // gemm_tc_ws_bytes(num_sms)
-  int *counters;    // max_tiles zeroed ints
+  int *counters;    // 2 * max_tiles zeroed ints (arrivals, published parts)
   int *dev_flag;
   int num_sms;
   long long max_tiles;
@@ -456,8 +469,10 @@ size_t gemm_tc_ws_bytes(int num_sms);
 // GEMM_EPI_SWIGLU: W rows interleaved gate/up in blocks of 16; writes
 // out2[t][f] = bf16(silu(gate) * up), f < N/2, row stride ld2.
 // Returns nullptr on success, else what went wrong.
-// defer (STORE / ACCUM epilogues only): leave split tiles to the consumer
-// and describe them in *defer; defer->ws stays null when no tile was split.
+// defer: leave split tiles to the consumer and describe them in *defer
+// (ws stays null when no tile was split, or when a tile would span more
+// than SPLIT_MAX_PARTS CTAs: then the GEMM reduces them itself).  Not for
+// the SwiGLU epilogue, which needs complete sums.
 const char *launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, void *out2,
                            int ld2, const TcWorkspace &ws, cudaStream_t s,
                            SplitView *defer = nullptr);

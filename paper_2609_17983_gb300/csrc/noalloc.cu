@@ -101,7 +101,7 @@ extern "C" kvr_status kvr_linear_noalloc(kvr_model *m, const char *name, int32_t
                    "kvr_linear_noalloc: name must be wqkv, wo, wd or lm_head");
   }
   if (!tm) return na_fail(KVR_E_UNSUPPORTED, "kvr_linear_noalloc: shape not on tensor cores");
-  if ((long long)(N / 128) > NOALLOC_COUNTERS)
+  if ((long long)(N / 128) > NOALLOC_COUNTERS / 2)
     return na_fail(KVR_E_UNSUPPORTED, "kvr_linear_noalloc: more output tiles than counters");
   if (cudaSetDevice(m->device) != cudaSuccess)
     return na_fail(KVR_E_CUDA, "kvr_linear_noalloc: cudaSetDevice");
@@ -113,7 +113,7 @@ extern "C" kvr_status kvr_linear_noalloc(kvr_model *m, const char *name, int32_t
   ws.counters = (int *)((unsigned char *)scratch + NOALLOC_PARTIAL_BYTES);
   ws.dev_flag = m->dev_flag;  // reported by kvr_synchronize
   ws.num_sms = m->num_sms < NOALLOC_MAX_CTAS ? m->num_sms : NOALLOC_MAX_CTAS;
-  ws.max_tiles = NOALLOC_COUNTERS;
+  ws.max_tiles = NOALLOC_COUNTERS / 2;  // arrivals, then published parts
   // the counters must start at zero: clear whatever an earlier call left
   if (cudaMemsetAsync(ws.counters, 0, NOALLOC_COUNTER_BYTES, m->stream) != cudaSuccess)
     return na_fail(KVR_E_CUDA, "kvr_linear_noalloc: counter clear");
