@@ -165,6 +165,24 @@ def run_reference(args, cfg, rank):
 
 # ------------------------------------------------------------- GPU arm
 
+# DRAM bytes (read + write) of one gate/up GEMM launch at this workload's shape
+# (40 x 28672 x 4096), from one ncu capture of that launch; reported only while the
+# GEMM kernel's source is the one the capture was taken on.
+GU_TRAFFIC_BYTES = 238599936 + 6328832
+GU_TRAFFIC_SOURCE_SHA256 = "31d14821e988d082de436734649e38d73bfbd3236e950b4ba1138c9dc6d67a60"
+
+
+def gemm_source_sha256() -> str:
+    import hashlib
+    h = hashlib.sha256()
+    here = os.path.join(os.path.dirname(os.path.abspath(__file__)), "paper_2609_17983_gb300",
+                        "csrc")
+    for f in ("k_gemm_tc.cu", "kvr_internal.cuh"):
+        with open(os.path.join(here, f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -264,6 +282,8 @@ def main():
     peak, peak_kind = load_peaks()
     achieved = d["bytes"] / d["launches"] / (d["ms"] / d["launches"] / 1e3) / 1e9
     all_w = sum(v["bytes"] for v in gemms.values())
+    traffic = (GU_TRAFFIC_BYTES if dom == "gemm_gu" and cfg["n_layers"] == 32
+               and gemm_source_sha256() == GU_TRAFFIC_SOURCE_SHA256 else None)
     all_ms = sum(v["ms"] for v in gemms.values())
 
     # e2e through the public API: host inputs in, repaired rows out
@@ -311,7 +331,7 @@ def main():
                "e2e": {"value": world * M / e2e_s, "unit": "positions/s",
                        "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
                "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peak,
-                            "unit": "GB/s", "frac": achieved / peak, "traffic": None,
+                            "unit": "GB/s", "frac": achieved / peak, "traffic": traffic,
                             "peak_kind": peak_kind,
                             "all_gemms_gbs": all_w / (all_ms / 1e3) / 1e9},
                "kernel_ms_per_step": {k: v["ms"] / args.steps for k, v in prof.items()

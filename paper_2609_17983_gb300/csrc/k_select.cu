@@ -59,82 +59,138 @@ __global__ void k_float_keys(const float *scores, int n, int s_end, unsigned lon
     keys[t] = (unsigned long long)ord_f32(scores[s_end + t]) + 1ull;
 }
 
-__device__ __forceinline__ bool better(unsigned long long ka, int ia, unsigned long long kb,
-                                       int ib) {
-  return ka > kb || (ka == kb && ia < ib);
+// Top-K of c (key, index) pairs, one CTA of TOPK_THREADS: key descending, ties to
+// the lowest index, the chosen indices written ascending.  Instead of a sort,
+// the K-th key T is found by an MSB-first radix select (8 bits per pass, a
+// shared-memory histogram of the keys that still match the prefix); then
+// every key above T is taken, and of the keys equal to T the lowest-indexed
+// ones until K are taken.  Thread i owns the contiguous keys [i*E, (i+1)*E),
+// so a block-wide scan of per-thread counts writes the output in index order.
+constexpr int TOPK_THREADS = 1024;
+
+__device__ __forceinline__ int block_excl_scan(int x, int *tmp) {
+  // tmp: TOPK_THREADS / 32 ints
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  int v = x;
+  for (int o = 1; o < 32; o <<= 1) {
+    int y = __shfl_up_sync(0xffffffffu, v, o);
+    if (lane >= o) v += y;
+  }
+  if (lane == 31) tmp[warp] = v;
+  __syncthreads();
+  if (warp == 0) {
+    int w = lane < TOPK_THREADS / 32 ? tmp[lane] : 0;
+    for (int o = 1; o < 32; o <<= 1) {
+      int y = __shfl_up_sync(0xffffffffu, w, o);
+      if (lane >= o) w += y;
+    }
+    if (lane < TOPK_THREADS / 32) tmp[lane] = w;
+  }
+  __syncthreads();
+  const int before = (warp ? tmp[warp - 1] : 0) + v - x;
+  __syncthreads();
+  return before;
 }
 
-// Single CTA bitonic sort of (key, index) pairs in shared memory.
-__global__ void __launch_bounds__(1024)
+__global__ void __launch_bounds__(TOPK_THREADS)
     k_topk(const unsigned long long *keys, int c, int s_end, int K, int nonzero_only,
            int32_t *out, int32_t *count) {
-  extern __shared__ unsigned char smem[];
-  int P = 1;
-  while (P < c) P <<= 1;
-  unsigned long long *sk = (unsigned long long *)smem;
-  int *si = (int *)(sk + P);
-  __shared__ int n_elig;
-  if (threadIdx.x == 0) n_elig = 0;
+  extern __shared__ unsigned long long sk[];  // c keys
+  __shared__ int hist[256];
+  __shared__ int scan_tmp[TOPK_THREADS / 32];
+  __shared__ int s_elig, s_bin, s_above;
+  const int tid = threadIdx.x;
+  const int E = (c + TOPK_THREADS - 1) / TOPK_THREADS;
+  const int t0 = min(c, tid * E), t1 = min(c, t0 + E);
+  if (tid == 0) s_elig = 0;
   __syncthreads();
   int local = 0;
-  for (int t = threadIdx.x; t < P; t += blockDim.x) {
-    if (t < c) {
-      sk[t] = keys[t];
-      si[t] = t;
-      local += (!nonzero_only || keys[t] != 0ull) ? 1 : 0;
-    } else {
-      sk[t] = 0ull;
-      si[t] = 0x7FFFFFFF;
-    }
+  for (int t = tid; t < c; t += TOPK_THREADS) {
+    const unsigned long long k = keys[t];
+    sk[t] = k;
+    local += (!nonzero_only || k != 0ull) ? 1 : 0;
   }
-  atomicAdd(&n_elig, local);
+  local += __shfl_xor_sync(0xffffffffu, local, 16);
+  local += __shfl_xor_sync(0xffffffffu, local, 8);
+  local += __shfl_xor_sync(0xffffffffu, local, 4);
+  local += __shfl_xor_sync(0xffffffffu, local, 2);
+  local += __shfl_xor_sync(0xffffffffu, local, 1);
+  if ((tid & 31) == 0) atomicAdd(&s_elig, local);
   __syncthreads();
-  for (int k = 2; k <= P; k <<= 1) {
-    for (int j = k >> 1; j > 0; j >>= 1) {
-      for (int t = threadIdx.x; t < P; t += blockDim.x) {
-        int u = t ^ j;
-        if (u > t) {
-          bool up = (t & k) == 0;
-          bool sw = up ? better(sk[u], si[u], sk[t], si[t]) : better(sk[t], si[t], sk[u], si[u]);
-          if (sw) {
-            unsigned long long tk = sk[t];
-            sk[t] = sk[u];
-            sk[u] = tk;
-            int ti = si[t];
-            si[t] = si[u];
-            si[u] = ti;
-          }
-        }
-      }
-      __syncthreads();
+  const int cnt = min(K, s_elig);
+  // radix select: prefix/mask of T, need = how many keys equal to the prefix
+  // (so far) are still to be taken
+  unsigned long long pref = 0ull, mask = 0ull;
+  int need = cnt;
+  for (int d = 56; d >= 0 && need > 0; d -= 8) {
+    for (int i = tid; i < 256; i += TOPK_THREADS) hist[i] = 0;
+    __syncthreads();
+    for (int t = t0; t < t1; ++t) {
+      const unsigned long long k = sk[t];
+      if ((k & mask) == pref) atomicAdd(&hist[(int)(k >> d) & 255], 1);
     }
-  }
-  int cnt = min(K, n_elig);
-  // chosen indices ascending: sort the first cnt indices (ascending) in place
-  int Q = 1;
-  while (Q < cnt) Q <<= 1;
-  for (int t = threadIdx.x; t < Q; t += blockDim.x)
-    if (t >= cnt) si[t] = 0x7FFFFFFF;
-  __syncthreads();
-  for (int k = 2; k <= Q; k <<= 1) {
-    for (int j = k >> 1; j > 0; j >>= 1) {
-      for (int t = threadIdx.x; t < Q; t += blockDim.x) {
-        int u = t ^ j;
-        if (u > t) {
-          bool up = (t & k) == 0;
-          bool sw = up ? si[t] > si[u] : si[t] < si[u];
-          if (sw) {
-            int ti = si[t];
-            si[t] = si[u];
-            si[u] = ti;
-          }
-        }
+    __syncthreads();
+    if (tid < 32) {
+      // suffix sums over bins 255..0, 8 bins per lane (lane 0 holds 255..248)
+      int loc[8], sum = 0;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        loc[j] = hist[255 - (tid * 8 + j)];
+        sum += loc[j];
       }
-      __syncthreads();
+      int incl = sum;
+      for (int o = 1; o < 32; o <<= 1) {
+        int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (tid >= o) incl += y;
+      }
+      int acc = incl - sum;  // keys in bins above this lane's first bin
+      int found = -1, above = 0;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        if (found < 0 && acc + loc[j] >= need) {
+          found = 255 - (tid * 8 + j);
+          above = acc;
+        }
+        acc += loc[j];
+      }
+      const unsigned ball = __ballot_sync(0xffffffffu, found >= 0);
+      const int src = __ffs(ball) - 1;  // first lane (highest bins) that found it
+      const int bin = __shfl_sync(0xffffffffu, found, src);
+      const int ab = __shfl_sync(0xffffffffu, above, src);
+      if (tid == 0) {
+        s_bin = bin;
+        s_above = ab;
+      }
     }
+    __syncthreads();
+    pref |= (unsigned long long)s_bin << d;
+    mask |= 0xFFull << d;
+    need -= s_above;
+    __syncthreads();
   }
-  for (int t = threadIdx.x; t < cnt; t += blockDim.x) out[t] = s_end + si[t];
-  if (threadIdx.x == 0) *count = cnt;
+  // T = pref (when cnt > 0): take keys > T, and the first `need` keys == T
+  int gt = 0, eq = 0;
+  if (cnt > 0)
+    for (int t = t0; t < t1; ++t) {
+      const unsigned long long k = sk[t];
+      gt += k > pref ? 1 : 0;
+      eq += k == pref ? 1 : 0;
+    }
+  const int eq_before = block_excl_scan(eq, scan_tmp);
+  int take_eq = cnt > 0 ? min(eq, max(0, need - eq_before)) : 0;
+  const int sel = gt + take_eq;
+  int pos = block_excl_scan(sel, scan_tmp);
+  if (cnt > 0)
+    for (int t = t0; t < t1; ++t) {
+      const unsigned long long k = sk[t];
+      bool take = k > pref;
+      if (!take && k == pref && take_eq > 0) {
+        take = true;
+        --take_eq;
+      }
+      if (take) out[pos++] = s_end + t;
+    }
+  if (tid == 0) *count = cnt;
 }
 
 // Attention selector, one layer: block (span row r, query head hh) writes the
@@ -300,15 +356,13 @@ const char *launch_topk(const unsigned long long *keys, int n, int s_end, int K,
   int nonzero_only = K < 0 ? 1 : 0;
   if (K < 0) K = -K;
   if (c < 0) c = 0;
-  int P = 1;
-  while (P < c) P <<= 1;
-  size_t smem = (size_t)P * (sizeof(unsigned long long) + sizeof(int));
+  size_t smem = (size_t)c * sizeof(unsigned long long);
   if (smem >= 32 * 1024) {  // the default 48 KB limit also covers static shared memory
     cudaError_t e = cudaFuncSetAttribute(k_topk, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
     if (e != cudaSuccess) return cudaGetErrorString(e);
   }
-  k_topk<<<1, 1024, smem, s>>>(keys, c, s_end, K, nonzero_only, out, count);
+  k_topk<<<1, TOPK_THREADS, smem, s>>>(keys, c, s_end, K, nonzero_only, out, count);
   cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? nullptr : cudaGetErrorString(e);
 }
