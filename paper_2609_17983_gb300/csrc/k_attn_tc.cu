@@ -294,20 +294,23 @@ __global__ void __launch_bounds__(MAXW * 32, 1) k_attn_tc(const AttnTcParams p) 
   }
 }
 
-// Merge the key splits of every (block, kv head, query vector), split order.
-// One warp per query vector: lane s reads split s's (max, sum), the weights
-// are reduced across the warp, then the partial outputs are gathered eight
-// splits at a time with all loads in flight together.
+// Merge the key splits of every (block, kv head, query vector), in split
+// order.  Two warps per query vector, each owning half of head_dim: lane s
+// reads split s's (max, sum), the weights are reduced across the warp, and
+// the partial outputs of up to NB splits load in one round trip with few
+// registers (so the next GEMM's CTAs can be resident, and stream their first
+// weight tiles, while this kernel runs).
 template <int DH>
 __global__ void __launch_bounds__(256) k_attn_combine(const AttnTcParams p) {
   TraceScope ts(TK_COMBINE);
   pdl_trigger();
   pdl_wait();
   ts.waited();
-  const int warp = (blockIdx.x * 8) + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  const int gw = (blockIdx.x * 8) + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  const int half = gw & 1, wv = gw >> 1;
   const int total = p.n_blocks * p.G * MAXQ;
-  if (warp >= total) return;
-  const int v = warp % MAXQ, bg = warp / MAXQ;
+  if (wv >= total) return;
+  const int v = wv % MAXQ, bg = wv / MAXQ;
   const int g = bg % p.G, blk = bg / p.G;
   const int4 bd = p.blocks[blk];
   const int mq = bd.y * p.grp;
@@ -317,10 +320,10 @@ __global__ void __launch_bounds__(256) k_attn_combine(const AttnTcParams p) {
   const int ns = (n_chunks + cps - 1) / cps;  // non-empty splits
   const size_t stride = (size_t)p.n_blocks * p.G;  // between splits, in (block, head) units
   const size_t base = (size_t)blk * p.G + g;
-  constexpr int VPL = DH / 32;
-  constexpr int NB = 24;  // splits whose partial outputs load in the first round trip
-  using VecT = typename std::conditional<VPL == 4, float4, float2>::type;
-  const VecT *src = (const VecT *)(p.ws_o + (base * MAXQ + v) * DH) + lane;
+  constexpr int VPL = DH / 64;  // floats per lane
+  constexpr int NB = 24;        // splits whose partial outputs load in the first round trip
+  using VecT = typename std::conditional<VPL == 2, float2, float>::type;
+  const VecT *src = (const VecT *)(p.ws_o + (base * MAXQ + v) * DH + half * (DH / 2)) + lane;
   const size_t sstride = stride * MAXQ * DH / VPL;  // in vectors
   VecT x[NB];
 #pragma unroll
@@ -358,9 +361,11 @@ __global__ void __launch_bounds__(256) k_attn_combine(const AttnTcParams p) {
   }
   const float inv = l > 0.f ? 1.f / l : 0.f;
   const int r = bd.x + v / p.grp, hh = g * p.grp + v % p.grp;
-  __nv_bfloat16 *dst = p.out + ((size_t)r * p.H + hh) * DH + lane * VPL;
-#pragma unroll
-  for (int i = 0; i < VPL; i += 2) *(uint32_t *)(dst + i) = pack_bf16(acc[i] * inv, acc[i + 1] * inv);
+  __nv_bfloat16 *dst = p.out + ((size_t)r * p.H + hh) * DH + half * (DH / 2) + lane * VPL;
+  if constexpr (VPL == 2)
+    *(uint32_t *)dst = pack_bf16(acc[0] * inv, acc[1] * inv);
+  else
+    *dst = __float2bfloat16_rn(acc[0] * inv);
 }
 
 template <int DH>
@@ -377,7 +382,7 @@ const char *run(const AttnTcParams &p, int max_mq, cudaStream_t s) {
   dim3 grid(p.n_splits, p.G, p.n_blocks);
   launch_pdl(k_attn_tc<DH>, grid, warps * 32, smem, s, p);
   if (p.n_splits > 1) {
-    int warps = p.n_blocks * p.G * MAXQ;
+    int warps = 2 * p.n_blocks * p.G * MAXQ;
     launch_pdl(k_attn_combine<DH>, (warps + 7) / 8, 256, 0, s, p);
   }
   cudaError_t e = cudaGetLastError();

@@ -508,7 +508,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
             for (int j = 0; j < 16; ++j)
               if (c + j < mv) w[(size_t)(c + j) * BM + f] = v[j];
           }
-          __threadfence();
+          asm volatile("fence.acq_rel.gpu;" ::: "memory");  // release the part
           epi_bar();
           if (et == 0) {
             atomicAdd(&p.counters[p.max_tiles + tl], 1);
@@ -529,7 +529,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           }
           epi_bar();
           if (!*abort_v) {
-            __threadfence();
+            asm volatile("fence.acq_rel.gpu;" ::: "memory");  // acquire the parts
             // two parts and at most 48 rows: the other part in one round trip
             const bool pre = parts == 2 && mv <= 48;
             float other[48];
