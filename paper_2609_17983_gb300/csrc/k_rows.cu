@@ -106,6 +106,13 @@ __global__ void __launch_bounds__(NORM_THREADS) k_rmsnorm(float *h, const float 
     const int mt = row / sv.BN;
     tiles[threadIdx.x] = split_tile(sv, (long long)threadIdx.x * sv.m_tiles + mt);
   }
+  // the gains are weights: read them before waiting on the residual's producer
+  float4 gw[NV];
+#pragma unroll
+  for (int k = 0; k < NV; ++k) {
+    const int q = k * NORM_THREADS + threadIdx.x;
+    gw[k] = q < nq ? ((const float4 *)g)[q] : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
   pdl_wait();
   ts.waited();
   if (sv.ws) __syncthreads();
@@ -135,12 +142,11 @@ __global__ void __launch_bounds__(NORM_THREADS) k_rmsnorm(float *h, const float 
 #pragma unroll
   for (int w = 0; w < NORM_THREADS / 32; ++w) tot += red[w];
   const float r = 1.0f / sqrtf(tot / (float)d + eps);
-  const float4 *gg = (const float4 *)g;
 #pragma unroll
   for (int k = 0; k < NV; ++k) {
     const int q = k * NORM_THREADS + threadIdx.x;
     if (q < nq) {
-      const float4 w = gg[q];
+      const float4 w = gw[k];
       const size_t o = (size_t)i * d + 4 * q;
       st(out, o, v[k].x * r * w.x);
       st(out, o + 1, v[k].y * r * w.y);
