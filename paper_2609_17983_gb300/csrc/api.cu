@@ -159,6 +159,8 @@ struct Rows {
   int max_pos = 0;                           // largest position among the rows
   const int4 *blocks = nullptr;              // attention query blocks (device)
   int n_blocks = 0, n_splits = 1, max_block_rows = 0;
+  const CUtensorMap *tm_kv = nullptr;        // TMA view of the single document's pages
+  bool tc5 = false;                          // attention on tcgen05 (set by plan_attention)
 };
 
 bool use_tc_attention(const kvr_model *m) {
@@ -169,25 +171,37 @@ bool use_tc_attention(const kvr_model *m) {
 // document (rows of a document are in ascending position order), at most
 // rows_per_block rows; and a key split count giving about two CTAs per SM.
 kvr_status plan_attention(kvr_model *m, Rows &r, const int32_t *pos, const int32_t *rowdoc) {
+  r.tc5 = false;
   if (!use_tc_attention(m) || r.M <= 0) return KVR_OK;
   const Dims &dm = m->dims;
-  const int qb = attn_tc_rows_per_block(dm.H / dm.G);
+  const int grp = dm.H / dm.G;
+  // one document's rows run on the tcgen05 kernel (query blocks of up to 128
+  // query vectors), several documents' on the mma.sync kernel
+  r.tc5 = m->use_tc5 && !rowdoc && r.tm_kv && attn_tc5_rows_per_block(grp) > 0;
+  const int qb = r.tc5 ? attn_tc5_rows_per_block(grp) : attn_tc_rows_per_block(grp);
   std::vector<int32_t> b;
   int max_chunks = 0, max_rows = 0;
   for (int i = 0; i < r.M;) {
     int doc = rowdoc ? rowdoc[i] : 0;
-    int j = i;
-    while (j < r.M && j - i < qb && (rowdoc ? rowdoc[j] : 0) == doc) ++j;
-    int kmax = pos[j - 1];
-    max_rows = std::max(max_rows, j - i);
-    b.insert(b.end(), {i, j - i, kmax, doc});
-    max_chunks = std::max(max_chunks, kmax / KVR_PAGE + 1);
-    i = j;
+    int e = i;
+    while (e < r.M && (rowdoc ? rowdoc[e] : 0) == doc) ++e;
+    // the document's rows in equal blocks of at most qb rows
+    const int nbd = (e - i + qb - 1) / qb, per = (e - i + nbd - 1) / nbd;
+    for (int j0 = i; j0 < e; j0 += per) {
+      const int j1 = std::min(e, j0 + per);
+      const int kmax = pos[j1 - 1];
+      max_rows = std::max(max_rows, j1 - j0);
+      b.insert(b.end(), {j0, j1 - j0, kmax, doc});
+      max_chunks = std::max(max_chunks, kmax / KVR_PAGE + 1);
+    }
+    i = e;
   }
   int nb = (int)b.size() / 4;
   if (nb > m->max_blocks) return fail(KVR_E_UNSUPPORTED, "too many attention blocks (%d)", nb);
-  int target = m->num_sms;  // one CTA per SM (128 KB of shared memory each)
-  int splits = std::max(1, (target + nb * dm.G - 1) / (nb * dm.G));
+  // about one wave: as many CTAs as fit on the SMs at once
+  const int target = m->num_sms * (r.tc5 ? attn_tc5_ctas_per_sm(dm.dh) : 1);
+  int splits = r.tc5 ? std::max(1, target / (nb * dm.G))  // one wave: no straggler CTAs
+                     : std::max(1, (target + nb * dm.G - 1) / (nb * dm.G));
   splits = std::min(std::min(splits, max_chunks), 64);  // the combine merges <= 64 splits
   while (splits > 1 && attn_tc_ws_floats(splits, nb, dm.G, dm.dh) > m->attn_ws_floats) --splits;
   KVR_TRY(stage_h2d(m, (int32_t *)m->blocks_d, b.data(), b.size()));
@@ -244,7 +258,17 @@ kvr_status layer_rest(kvr_model *m, const Rows &r, int l) {
   {
     int64_t kv_bytes = (int64_t)(r.max_pos + 1) * dm.G * dm.dh * 2 * (int64_t)dm.es();
     Prof pr(m, P_ATTN, kv_bytes);
-    if (use_tc_attention(m)) {
+    if (r.tc5) {
+      const char *e = launch_attention_tc5(m->qb, r.pos, r.blocks, r.n_blocks, r.n_splits, dm, l,
+                                           r.single.pages, r.single.table, *r.tm_kv,
+                                           m->attn_ws_o, m->attn_ws_ml, m->attn, m->dev_flag,
+                                           m->stream);
+      if (!e)
+        e = launch_attention_combine(r.blocks, r.n_blocks, r.n_splits, dm, m->attn_ws_o,
+                                     m->attn_ws_ml, m->attn, m->stream);
+      if (e) return fail(KVR_E_CUDA, "attention: %s", e);
+      KVR_TRY(launch_check(m, r.n_splits > 1 ? 2 : 1));
+    } else if (use_tc_attention(m)) {
       const char *e = launch_attention_tc(m->qb, r.pos, r.blocks, r.n_blocks, r.max_block_rows,
                                           r.n_splits, dm, l, r.views, r.single, m->attn_ws_o,
                                           m->attn_ws_ml, m->attn, m->stream);
@@ -511,6 +535,8 @@ kvr_status kvr_model_create(const kvr_model_config *cfg, const kvr_weights *wts,
     m->use_graphs = !(g && g[0] == '1');
     const char *df = getenv("KVR_DISABLE_DEFERRED_SPLITS");
     m->defer_splits = !(df && df[0] == '1');
+    const char *t5 = getenv("KVR_DISABLE_TC5_ATTENTION");
+    m->use_tc5 = !(t5 && t5[0] == '1');
     const char *pd = getenv("KVR_DISABLE_PDL");
     g_pdl = !(pd && pd[0] == '1');
   }
@@ -796,6 +822,10 @@ kvr_status kvr_prefill(kvr_model *m, const int32_t *tokens, int32_t n, kvr_cache
     kvr_cache_free(c);
     return fail(KVR_E_CUDA, "cache clear");
   }
+  if (dm.dtype == KVR_DTYPE_BF16) {
+    const long long rows = (long long)c->n_pages * dm.L * 2 * dm.G * KVR_PAGE;
+    c->tm_kv_ok = rows < (1ll << 31) && make_tmap_bf16(&c->tm_kv, c->pages, (int)rows, dm.dh, KVR_PAGE);
+  }
   std::vector<int32_t> tab(c->n_pages);
   for (int i = 0; i < c->n_pages; ++i) tab[i] = i;
   kvr_status st = stage_h2d(m, c->table, tab.data(), tab.size());
@@ -803,6 +833,7 @@ kvr_status kvr_prefill(kvr_model *m, const int32_t *tokens, int32_t n, kvr_cache
   Rows r;
   r.tokens = c->tokens_d;
   r.single = c->view();
+  r.tm_kv = c->tm_kv_ok ? &c->tm_kv : nullptr;
   std::vector<int32_t> pos;
   for (int c0 = 0; c0 < n && !st; c0 += dm.max_rows) {
     int M = std::min(dm.max_rows, n - c0);
@@ -866,6 +897,7 @@ kvr_status kvr_repair(kvr_cache *c, const int32_t *new_tokens, int32_t edit_star
     r.pos = m->pos_d;
     r.tokens = c->tokens_d;
     r.single = c->view();
+  r.tm_kv = c->tm_kv_ok ? &c->tm_kv : nullptr;
     r.max_pos = P[M - 1];
     st = plan_attention(m, r, P.data(), nullptr);
     if (!st) st = run_pass_graph(m, c, r);
@@ -988,6 +1020,7 @@ kvr_status kvr_logits(kvr_model *m, const kvr_cache *c, const int32_t *query, in
   r.pos = m->pos_d;
   r.tokens = c->tokens_d;
   r.single = c->view();
+  r.tm_kv = c->tm_kv_ok ? &c->tm_kv : nullptr;
   r.max_pos = c->n + qm - 1;
   KVR_TRY(plan_attention(m, r, P.data(), nullptr));
   KVR_TRY(run_pass(m, r));
@@ -1069,6 +1102,7 @@ kvr_status kvr_select(kvr_model *m, const kvr_cache *c, kvr_policy policy, int32
         r.pos = m->pos_d;
         r.tokens = toks;
         r.single = c->view();
+  r.tm_kv = c->tm_kv_ok ? &c->tm_kv : nullptr;
         r.max_pos = s_end - 1;
         st = plan_attention(m, r, P.data(), nullptr);
         launch_rows_copy(r.single, dm.dtype, r.pos, edit_len, 0, dm.L, save, true, m->stream);
@@ -1108,6 +1142,7 @@ kvr_status kvr_select(kvr_model *m, const kvr_cache *c, kvr_policy policy, int32
       Rows r;
       r.tokens = toks;
       r.single = c->view();
+  r.tm_kv = c->tm_kv_ok ? &c->tm_kv : nullptr;
       if (!st) st = stage_h2d(m, m->pos_d, P.data(), edit_len);
       if (!st) {
         // refresh the span's layer-0 K/V (saved and restored afterwards)
@@ -1234,6 +1269,7 @@ kvr_status kvr_answer_logprob(kvr_model *m, const kvr_cache *c, const int32_t *p
   r.pos = m->pos_d;
   r.tokens = c->tokens_d;
   r.single = c->view();
+  r.tm_kv = c->tm_kv_ok ? &c->tm_kv : nullptr;
   r.max_pos = c->n + rows - 1;
   KVR_TRY(plan_attention(m, r, P.data(), nullptr));
   KVR_TRY(run_pass(m, r));
@@ -1418,6 +1454,7 @@ static cudaError_t trace_attach_all(const TraceBuf &b) {
   cudaError_t e = trace_attach_rows(b);
   if (e == cudaSuccess) e = trace_attach_gemm(b);
   if (e == cudaSuccess) e = trace_attach_attn(b);
+  if (e == cudaSuccess) e = trace_attach_attn5(b);
   return e;
 }
 

@@ -389,7 +389,34 @@ const char *run(const AttnTcParams &p, int max_mq, cudaStream_t s) {
   return e == cudaSuccess ? nullptr : cudaGetErrorString(e);
 }
 
+template <int DH>
+const char *run_combine(const AttnTcParams &p, cudaStream_t s) {
+  const int warps = 2 * p.n_blocks * p.G * MAXQ;
+  launch_pdl(k_attn_combine<DH>, (warps + 7) / 8, 256, 0, s, p);
+  cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? nullptr : cudaGetErrorString(e);
+}
+
 }  // namespace
+
+const char *launch_attention_combine(const int4 *blocks, int n_blocks, int n_splits,
+                                     const Dims &dm, float *ws_o, float2 *ws_ml, void *out,
+                                     cudaStream_t s) {
+  if (n_blocks <= 0 || n_splits <= 1) return nullptr;
+  AttnTcParams p{};
+  p.H = dm.H;
+  p.G = dm.G;
+  p.grp = dm.H / dm.G;
+  p.blocks = blocks;
+  p.n_splits = n_splits;
+  p.ws_o = ws_o;
+  p.ws_ml = ws_ml;
+  p.n_blocks = n_blocks;
+  p.out = (__nv_bfloat16 *)out;
+  if (dm.dh == 128) return run_combine<128>(p, s);
+  if (dm.dh == 64) return run_combine<64>(p, s);
+  return "head_dim not supported";
+}
 
 int attn_tc_rows_per_block(int grp) { return MAXQ / grp; }
 

@@ -1,0 +1,498 @@
+// k_attn_tc5.cu -- scattered-query causal GQA attention of one document's
+// rows on the tcgen05 tensor cores (sm_103a), bf16 cache, head_dim 64 or 128.
+//
+// A CTA owns one query block -- up to 128 query vectors (rows of the pass times
+// the grp query heads of KV head g), the M = 128 rows of the MMA -- and a
+// contiguous range of 64-key chunks (one KV page each).  Per chunk:
+//   S = Q K^T      tcgen05.mma, M 128 x N 64 x K head_dim, into TMEM (two
+//                  S buffers, so S of chunk i+1 is computed while the softmax
+//                  works on chunk i);
+//   softmax        eight warps, two per TMEM lane quarter: one query vector
+//                  per thread pair, each thread half of the chunk's keys and
+//                  half of O's columns, the row maximum exchanged through
+//                  shared memory; S read once from
+//                  TMEM: causal mask key <= position, exponentials in the
+//                  log2 domain (Q is pre-scaled by log2(e)/sqrt(dh)) against
+//                  a reference maximum that is raised -- and the accumulator
+//                  rescaled in TMEM -- only when the running maximum exceeds
+//                  it by more than 8 (so P <= 256); P in bf16 written to one
+//                  of two shared-memory buffers as the next MMA's A operand,
+//                  so the softmax of chunk i overlaps O += P V of chunk i-1;
+//   O += P V       tcgen05.mma, M 128 x N head_dim x K 64, V read MN-major
+//                  straight from the page layout [key][head_dim].
+// K and V tiles arrive by TMA (128-byte swizzle, KV_STAGES stages deep, so a
+// chunk's load is issued long before its MMA); Q by cp.async.
+// With several key splits the CTA writes its unnormalised O and (max, sum)
+// for the combine kernel, else the normalised output.
+//
+// Rows of the pass were written into the cache at this layer before the
+// launch (operator R, Sec. 3); keys are read only after the wait on that
+// kernel, and only L2 prefetches are issued before it.
+//
+// Warp roles (320 threads): warp 0 TMA (one lane), warp 1 TMEM allocation and
+// MMA issue (one lane), warps 2-9 softmax and epilogue.  Every wait is
+// bounded; a wait that runs out sets the device error flag, the roles stop
+// issuing, drain what is in flight, free TMEM and return.
+#include <math.h>
+
+#include "kvr_internal.cuh"
+#include "tc_ptx.cuh"
+
+namespace kvr {
+namespace {
+using namespace ptx;
+
+constexpr int QV = 128;          // query vectors per CTA (UMMA M)
+constexpr int CH = KVR_PAGE;     // keys per chunk
+constexpr int NT5 = 320;         // threads per CTA
+constexpr int WS_MAXQ = 192;     // query slots per (split, block, head) of the split workspace
+constexpr uint32_t TMEM_COLS = 256;  // S buffers at columns 0 and 64, O from column 128
+constexpr int SOFTMAX_THREADS = 256;
+constexpr float RESCALE_LOG2 = 8.f;  // headroom of the reference maximum (P <= 2^8)
+constexpr int KV_STAGES = 4;
+
+struct Attn5Params {
+  const __nv_bfloat16 *q;  // [M][H * dh] post-RoPE, pre-scaled by log2(e)/sqrt(dh)
+  const int32_t *pos;      // [M] ascending (one document)
+  const int4 *blocks;      // (row0, nrows, kmax, doc)
+  const __nv_bfloat16 *pages;  // the cache's page pool
+  const int32_t *table;        // logical page -> physical page
+  int H, G, grp, layer, L;
+  int n_splits, n_blocks;
+  float *ws_o;    // [n_splits][n_blocks][G][WS_MAXQ][dh]
+  float2 *ws_ml;  // [n_splits][n_blocks][G][WS_MAXQ]
+  __nv_bfloat16 *out;  // [M][H * dh]
+  int *dev_flag;
+};
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+
+__device__ __forceinline__ uint32_t pack2(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *(uint32_t *)&v;
+}
+
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// byte offset of 16-byte chunk c of row r in a [rows][128 B] 128-byte-swizzled tile
+__device__ __forceinline__ uint32_t sw_off(int r, int c) {
+  return (uint32_t)((r >> 3) * 1024 + (r & 7) * 128 + ((c ^ (r & 7)) << 4));
+}
+
+template <int DH>
+__global__ void __launch_bounds__(NT5, 1)
+    k_attn_tc5(const __grid_constant__ CUtensorMap tm_kv, const Attn5Params p) {
+  constexpr int HALVES = DH / 64;           // 128-byte column blocks of a row
+  constexpr uint32_t QBYTES = QV * 128 * HALVES;
+  constexpr uint32_t TBYTES = CH * 128 * HALVES;  // one K (or V) tile
+  constexpr uint32_t KVBYTES = 2 * TBYTES;
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t kv_full[KV_STAGES], kv_empty[KV_STAGES], s_full[2], s_free[2],
+      p_full[2], o_done[2], q_full, drain_bar;
+  __shared__ uint32_t tmem_slot;
+  __shared__ int abort_f;
+  __shared__ int spos[QV];
+  __shared__ int sprow[2 * 64];  // pool rows of the CTA's K and V pages (at most 64 chunks)
+  __shared__ float sx[2][2][QV];  // per chunk parity and key half: row maxima
+  __shared__ float ssum[2][QV];   // per key half: sums of exponentials
+
+  TraceScope ts(TK_ATTN);
+  const int split = blockIdx.x, g = blockIdx.y, blk = blockIdx.z;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  // block table, positions and page table are written before the pass
+  const int4 bd = p.blocks[blk];
+  const int row0 = bd.x, nrows = bd.y, kmax = bd.z;
+  const int mq = nrows * p.grp;
+  const int n_chunks = kmax / CH + 1;
+  const int cps = (n_chunks + p.n_splits - 1) / p.n_splits;
+  const int c0 = split * cps, c1 = min(n_chunks, c0 + cps);
+  if (c0 >= c1) {  // empty split: the combine skips it
+    pdl_trigger();
+    return;
+  }
+  const int nch = c1 - c0;
+  const uint32_t base = (su32(smem_raw) + 1023u) & ~1023u;
+  const uint32_t sQ = base, sKV = sQ + QBYTES, sP = sKV + KV_STAGES * KVBYTES;  // P: two tiles
+  volatile int *abort_v = &abort_f;
+  auto page_row = [&](int c, int kv) {  // first row of (chunk c, kv) in the pool's 2D view
+    const long long pg = p.table[c];
+    return (int)((((pg * p.L + p.layer) * 2 + kv) * p.G + g) * CH);
+  };
+  const bool rows_cached = nch <= 64;
+
+  if (tid == 0) {
+    for (int st = 0; st < KV_STAGES; ++st) {
+      mbar_init(&kv_full[st], 1);
+      mbar_init(&kv_empty[st], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&s_full[b], 1);
+      mbar_init(&s_free[b], SOFTMAX_THREADS);
+      mbar_init(&p_full[b], SOFTMAX_THREADS);
+      mbar_init(&o_done[b], 1);
+    }
+    mbar_init(&q_full, SOFTMAX_THREADS);
+    mbar_init(&drain_bar, 1);
+    abort_f = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  for (int v = tid; v < QV; v += NT5) spos[v] = v < mq ? p.pos[row0 + v / p.grp] : -1;
+  // pull this CTA's K and V pages into L2 while the RoPE kernel finishes
+  for (int t = tid; t < 2 * nch; t += NT5) {
+    const int i = t >> 1, kv = t & 1;
+    const int row = page_row(c0 + i, kv);
+    if (rows_cached) sprow[t] = row;
+    const __nv_bfloat16 *pg = p.pages + (size_t)row * DH;
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(pg), "r"(TBYTES) : "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     su32(&tmem_slot)),
+                 "r"(TMEM_COLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tmem_slot;
+  // dependents may launch once this CTA holds its TMEM
+  pdl_trigger();
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA
+    if (lane == 0) {
+      tma_prefetch_desc(&tm_kv);
+      pdl_wait();
+      ts.waited();
+      int issued = 0;
+      for (int i = 0; i < nch && !*abort_v; ++i) {
+        const int b = i % KV_STAGES;
+        if (i >= KV_STAGES &&
+            !mbar_wait(&kv_empty[b], (i / KV_STAGES - 1) & 1, abort_v, p.dev_flag, 64))
+          break;
+        const uint32_t sk = sKV + b * KVBYTES, sv = sk + TBYTES;
+        mbar_expect_tx(&kv_full[b], KVBYTES);
+        const int rk = rows_cached ? sprow[2 * i] : page_row(c0 + i, 0);
+        const int rv = rows_cached ? sprow[2 * i + 1] : page_row(c0 + i, 1);
+        if (i == 0) trace_mark(1);
+#pragma unroll
+        for (int h = 0; h < HALVES; ++h) {
+          tma_load_2d((void *)__cvta_shared_to_generic(sk + h * CH * 128), &tm_kv, &kv_full[b],
+                      h * 64, rk);
+          tma_load_2d((void *)__cvta_shared_to_generic(sv + h * CH * 128), &tm_kv, &kv_full[b],
+                      h * 64, rv);
+        }
+        ++issued;
+      }
+      // copies in flight complete before the CTA may exit
+      for (int i = issued > KV_STAGES ? issued - KV_STAGES : 0; i < issued; ++i)
+        mbar_wait(&kv_full[i % KV_STAGES], (i / KV_STAGES) & 1, abort_v, p.dev_flag, 0, false);
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA
+    if (lane == 0) {
+      const uint32_t id_s = idesc_bf16(QV, CH), id_o = idesc_bf16(QV, DH, 1);
+      bool ok = mbar_wait(&q_full, 0, abort_v, p.dev_flag, 65);
+      auto issue_s = [&](int i) -> bool {
+        const int b = i & 1, st = i % KV_STAGES;
+        if (!mbar_wait(&kv_full[st], (i / KV_STAGES) & 1, abort_v, p.dev_flag, 66)) return false;
+        if (i >= 2 && !mbar_wait(&s_free[b], ((i - 2) >> 1) & 1, abort_v, p.dev_flag, 67))
+          return false;
+        tc_fence_after();
+        const uint32_t sk = sKV + st * KVBYTES;
+#pragma unroll
+        for (int kk = 0; kk < DH / 16; ++kk) {
+          const uint64_t a = sw128_desc(sQ + (kk >> 2) * QV * 128 + (kk & 3) * 32);
+          const uint64_t bb = sw128_desc(sk + (kk >> 2) * CH * 128 + (kk & 3) * 32);
+          mma_bf16(tmem + b * CH, a, bb, id_s, kk > 0 ? 1u : 0u);
+        }
+        mma_commit(&s_full[b]);
+        return true;
+      };
+      if (ok) ok = issue_s(0);
+      for (int i = 0; i < nch && ok; ++i) {
+        if (i + 1 < nch && !(ok = issue_s(i + 1))) break;
+        if (!(ok = mbar_wait(&p_full[i & 1], (i >> 1) & 1, abort_v, p.dev_flag, 68))) break;
+        tc_fence_after();
+        const uint32_t sv = sKV + (i % KV_STAGES) * KVBYTES + TBYTES;
+        const uint32_t sp = sP + (i & 1) * QV * CH * 2;
+#pragma unroll
+        for (int kk = 0; kk < CH / 16; ++kk) {
+          // P: K-major rows of 64 keys.  V: keys are the rows (K), head_dim
+          // runs along them (MN-major) in 64-wide column blocks CH*128 bytes
+          // apart, 8-key groups 1024 bytes apart.
+          const uint64_t a = sw128_desc(sp + kk * 32);
+          const uint64_t bb = sw128_desc_mn(sv + kk * 2048, CH * 128, 1024);
+          mma_bf16(tmem + 2 * CH, a, bb, id_o, (i > 0 || kk > 0) ? 1u : 0u);
+        }
+        mma_commit(&o_done[i & 1]);
+        mma_commit(&kv_empty[i % KV_STAGES]);
+      }
+      // every MMA issued here completes before TMEM is freed
+      mma_commit(&drain_bar);
+      mbar_wait(&drain_bar, 0, abort_v, p.dev_flag, 0, false);
+    }
+  } else {
+    // ------------------------------------------------------------ softmax
+    // Warps w and w + 4 share TMEM lane quarter w % 4: the same 32 query
+    // vectors, keys (and O columns) split in halves.  Their per-chunk maxima
+    // meet at a 64-thread named barrier, which both warps reach on every
+    // iteration -- also after an abort, when they only skip their work -- so
+    // it can never wait on a warp that has left.
+    const int quarter = warp & 3;  // TMEM lanes 32 * quarter .. + 31
+    const int half = (warp - 2) >> 2;
+    const int v = quarter * 32 + lane;
+    const uint32_t tl = tmem + ((uint32_t)(quarter * 32) << 16);
+    const int bar_id = 1 + quarter;
+    auto pair_bar = [&]() { asm volatile("bar.sync %0, 64;" ::"r"(bar_id) : "memory"); };
+    pdl_wait();
+    // this thread's half of the Q row, into the swizzled K-major tile
+    {
+      const bool real = v < mq;
+      const __nv_bfloat16 *src =
+          p.q + ((size_t)(row0 + (real ? v / p.grp : 0)) * p.H + g * p.grp + v % p.grp) * DH;
+#pragma unroll
+      for (int k = 0; k < DH / 16; ++k) {
+        const int ch = half * (DH / 16) + k;
+        const uint32_t dst = sQ + (ch >> 3) * QV * 128 + sw_off(v, ch & 7);
+        if (real)
+          cp_async16(dst, src + ch * 8);
+        else
+          asm volatile("st.shared.v4.u32 [%0], {%1, %1, %1, %1};" ::"r"(dst), "r"(0u)
+                       : "memory");
+      }
+      asm volatile("cp.async.commit_group;" ::: "memory");
+      asm volatile("cp.async.wait_group 0;" ::: "memory");
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      mbar_arrive(&q_full);
+      if (warp == 2 && lane == 0) trace_mark(2);
+    }
+    constexpr int HK = CH / 2;  // keys of this thread per chunk
+    const int pv = spos[v];
+    float m = -INFINITY, l = 0.f;  // reference maximum, this half's sum of exponentials
+    bool dead = false;             // warp-uniform: a wait ran out
+    for (int i = 0; i < nch; ++i) {
+      const int b = i & 1, key0 = (c0 + i) * CH + half * HK;
+      uint32_t sr[HK];
+      float mx = -INFINITY;
+      if (!dead) {
+        dead = !__all_sync(0xffffffffu,
+                           mbar_wait(&s_full[b], (i >> 1) & 1, abort_v, p.dev_flag, 69));
+      }
+      if (!dead) {
+        tc_fence_after();
+        if (i == 0 && warp == 2 && lane == 0) trace_mark(3);
+        tmem_ld32_nowait(tl + b * CH + half * HK, sr);
+        tmem_wait_ld();
+        tc_fence_before();
+        mbar_arrive(&s_free[b]);  // S is in registers: the buffer may be refilled
+        float t[HK];
+#pragma unroll
+        for (int j = 0; j < HK; ++j) t[j] = key0 + j <= pv ? __uint_as_float(sr[j]) : -INFINITY;
+#pragma unroll
+        for (int w = HK / 2; w > 0; w >>= 1)
+#pragma unroll
+          for (int j = 0; j < w; ++j) t[j] = fmaxf(t[j], t[j + w]);
+        mx = t[0];
+        sx[b][half][v] = mx;
+      }
+      pair_bar();
+      if (dead) continue;
+      mx = fmaxf(mx, sx[b][half ^ 1][v]);
+      // O is exactly zero until the first unmasked key: no rescale then
+      if (m == -INFINITY) m = mx;
+      const bool grow = mx > m + RESCALE_LOG2;
+      if (__any_sync(0xffffffffu, grow)) {
+        if (i > 0) {  // O += P V of the previous chunk has landed
+          dead = !__all_sync(0xffffffffu, mbar_wait(&o_done[(i - 1) & 1], ((i - 1) >> 1) & 1,
+                                                    abort_v, p.dev_flag, 70));
+          if (dead) continue;
+          tc_fence_after();
+        }
+        const float alpha = grow ? ex2(m - mx) : 1.f;
+#pragma unroll
+        for (int q = 0; q < DH / 32; ++q) {  // this half's O columns
+          float o[16];
+          tmem_ld16(tl + 2 * CH + half * (DH / 2) + q * 16, o);
+#pragma unroll
+          for (int j = 0; j < 16; ++j) o[j] *= alpha;
+          tmem_st16(tl + 2 * CH + half * (DH / 2) + q * 16, o);
+        }
+        l *= alpha;
+        if (grow) m = mx;
+      }
+      // P buffer b was last read by O += P V of chunk i - 2
+      if (i >= 2) {
+        dead = !__all_sync(0xffffffffu, mbar_wait(&o_done[b], ((i - 2) >> 1) & 1, abort_v,
+                                                  p.dev_flag, 72));
+        if (dead) continue;
+      }
+      const uint32_t prow =
+          sP + b * QV * CH * 2 + (uint32_t)((v >> 3) * 1024 + (v & 7) * 128);
+      float e[HK];
+#pragma unroll
+      for (int j = 0; j < HK; ++j) e[j] = key0 + j <= pv ? ex2(__uint_as_float(sr[j]) - m) : 0.f;
+#pragma unroll
+      for (int q = 0; q < HK / 8; ++q) {
+        const uint32_t d = prow + (((half * (HK / 8) + q) ^ (v & 7)) << 4);
+        asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(d),
+                     "r"(pack2(e[q * 8], e[q * 8 + 1])), "r"(pack2(e[q * 8 + 2], e[q * 8 + 3])),
+                     "r"(pack2(e[q * 8 + 4], e[q * 8 + 5])), "r"(pack2(e[q * 8 + 6], e[q * 8 + 7]))
+                     : "memory");
+      }
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      tc_fence_before();
+      mbar_arrive(&p_full[b]);
+#pragma unroll
+      for (int w = HK / 2; w > 0; w >>= 1)
+#pragma unroll
+        for (int j = 0; j < w; ++j) e[j] += e[j + w];
+      l += e[0];
+      if (warp == 2 && lane == 0) trace_mark(i == 0 ? 4 : 5);
+    }
+    if (!dead)
+      dead = !__all_sync(0xffffffffu, mbar_wait(&o_done[(nch - 1) & 1], ((nch - 1) >> 1) & 1,
+                                                abort_v, p.dev_flag, 71));
+    if (warp == 2 && lane == 0) trace_mark(6);
+    ssum[half][v] = l;
+    pair_bar();
+    const float lt = l + ssum[half ^ 1][v];  // both halves, same reference maximum
+    // O: TMEM -> registers -> shared memory (the K/V stages are free now; rows
+    // of DH floats, 16-byte chunks XOR-swizzled by row so the writes hit
+    // distinct banks) -> global, one coalesced row per warp instruction.
+    // Both named barriers are reached by all 256 softmax threads, live or not.
+    constexpr int RCH = DH / 4;  // 16-byte chunks per staged row
+    const float inv = lt > 0.f ? 1.f / lt : 0.f;
+    const float scale = p.n_splits == 1 ? inv : 1.f;
+    float *stage = (float *)__cvta_shared_to_generic(sKV);
+    if (!dead) {
+      tc_fence_after();
+      const uint32_t to = tl + 2 * CH + half * (DH / 2);
+      uint32_t o[DH / 2];
+      tmem_ld32_nowait(to, o);
+      if (DH / 2 > 32) tmem_ld32_nowait(to + 32, o + 32 * (DH / 64 - 1));
+      tmem_wait_ld();
+      if (warp == 2 && lane == 0) trace_mark(7);
+#pragma unroll
+      for (int k = 0; k < DH / 8; ++k) {  // this half's chunks
+        const int c = half * (DH / 8) + k;
+        *(float4 *)(stage + v * DH + ((c ^ (v & (RCH - 1))) << 2)) =
+            make_float4(__uint_as_float(o[4 * k]) * scale, __uint_as_float(o[4 * k + 1]) * scale,
+                        __uint_as_float(o[4 * k + 2]) * scale, __uint_as_float(o[4 * k + 3]) * scale);
+      }
+      if (half == 0 && p.n_splits > 1 && v < mq) {
+        const size_t bs = ((size_t)split * p.n_blocks + blk) * p.G + g;
+        p.ws_ml[bs * WS_MAXQ + v] = make_float2(m, lt);
+      }
+    }
+    asm volatile("bar.sync 5, 256;" ::: "memory");
+    {
+      const int ws = warp - 2;  // rows ws * 16 .. + 15
+      for (int rr = 0; rr < QV / 8; ++rr) {
+        const int row = ws * (QV / 8) + rr;
+        if (row >= mq || lane >= RCH) continue;
+        const float4 x = *(const float4 *)(stage + row * DH + ((lane ^ (row & (RCH - 1))) << 2));
+        if (p.n_splits == 1) {
+          const int r = row0 + row / p.grp, hh = g * p.grp + row % p.grp;
+          uint2 y;
+          y.x = pack2(x.x, x.y);
+          y.y = pack2(x.z, x.w);
+          *(uint2 *)(p.out + ((size_t)r * p.H + hh) * DH + lane * 4) = y;
+        } else {
+          const size_t bs = ((size_t)split * p.n_blocks + blk) * p.G + g;
+          *(float4 *)(p.ws_o + (bs * WS_MAXQ + row) * DH + lane * 4) = x;
+        }
+      }
+    }
+    if (warp == 2 && lane == 0) trace_mark(0);
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1)
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                 "r"(TMEM_COLS)
+                 : "memory");
+  ts.finish();
+}
+
+template <int DH>
+constexpr size_t smem_bytes() {
+  return 1024 + (size_t)QV * 128 * (DH / 64) + KV_STAGES * 2 * (size_t)CH * 128 * (DH / 64) +
+         2 * (size_t)QV * CH * 2;
+}
+
+template <int DH>
+const char *run(const CUtensorMap &tm, const Attn5Params &p, cudaStream_t s) {
+  constexpr size_t smem = smem_bytes<DH>();
+  static bool set = false;
+  if (!set) {
+    cudaError_t e = cudaFuncSetAttribute(k_attn_tc5<DH>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return cudaGetErrorString(e);
+    set = true;
+  }
+  dim3 grid(p.n_splits, p.G, p.n_blocks);
+  launch_pdl(k_attn_tc5<DH>, grid, NT5, smem, s, tm, p);
+  cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? nullptr : cudaGetErrorString(e);
+}
+
+}  // namespace
+
+int attn_tc5_rows_per_block(int grp) { return grp <= QV ? QV / grp : 0; }
+
+int attn_tc5_ctas_per_sm(int dh) {
+  static int cached[2] = {-1, -1};
+  const int k = dh == 128 ? 1 : 0;
+  if (cached[k] < 0) {
+    int n = 0;
+    size_t smem = dh == 128 ? smem_bytes<128>() : smem_bytes<64>();
+    const void *fn = dh == 128 ? (const void *)k_attn_tc5<128> : (const void *)k_attn_tc5<64>;
+    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
+            cudaSuccess ||
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fn, NT5, smem) != cudaSuccess)
+      n = 1;
+    cached[k] = n < 1 ? 1 : (n > 2 ? 2 : n);  // TMEM holds two CTAs' 256 columns
+  }
+  return cached[k];
+}
+
+const char *launch_attention_tc5(const void *q, const int32_t *pos, const int4 *blocks,
+                                 int n_blocks, int n_splits, const Dims &dm, int layer,
+                                 const void *pages, const int32_t *table, const CUtensorMap &tm_kv,
+                                 float *ws_o, float2 *ws_ml, void *out, int *dev_flag,
+                                 cudaStream_t s) {
+  if (n_blocks <= 0) return nullptr;
+  Attn5Params p{};
+  p.q = (const __nv_bfloat16 *)q;
+  p.pos = pos;
+  p.blocks = blocks;
+  p.pages = (const __nv_bfloat16 *)pages;
+  p.table = table;
+  p.H = dm.H;
+  p.G = dm.G;
+  p.grp = dm.H / dm.G;
+  p.layer = layer;
+  p.L = dm.L;
+  p.n_splits = n_splits;
+  p.n_blocks = n_blocks;
+  p.ws_o = ws_o;
+  p.ws_ml = ws_ml;
+  p.out = (__nv_bfloat16 *)out;
+  p.dev_flag = dev_flag;
+  if (dm.dh == 128) return run<128>(tm_kv, p, s);
+  if (dm.dh == 64) return run<64>(tm_kv, p, s);
+  return "head_dim not supported";
+}
+
+KVR_TRACE_ATTACH(trace_attach_attn5)
+
+}  // namespace kvr

@@ -247,6 +247,7 @@ struct kvr_model {
   kvr::TraceBuf trace{};       // attached device timeline buffer, if any
   kvr::SplitView pending{};    // split tiles of h not yet added (next RMSNorm adds them)
   bool defer_splits = true;    // GEMM split tiles reduced by the consumer
+  bool use_tc5 = true;         // tcgen05 attention for single-document passes
   // pinned staging for host->device argument copies
   int32_t *stage_h = nullptr;
   int32_t *stage_d = nullptr;
@@ -264,6 +265,10 @@ struct kvr_cache {
   int n = 0, cap = 0, n_pages = 0;
   void *pages = nullptr;
   int32_t *table = nullptr;   // device [n_pages]
+  // TMA view of the page pool (bf16): rows of head_dim elements, one row per
+  // (page, layer, k|v, kv head, slot); boxes of 64 rows x 64 elements
+  CUtensorMap tm_kv{};
+  bool tm_kv_ok = false;
   int32_t *tokens_d = nullptr;  // device [cap]
   std::vector<int32_t> tokens_h;
   bool poisoned = false;
@@ -375,6 +380,7 @@ struct TraceScope {
 cudaError_t trace_attach_rows(const TraceBuf &b);
 cudaError_t trace_attach_gemm(const TraceBuf &b);
 cudaError_t trace_attach_attn(const TraceBuf &b);
+cudaError_t trace_attach_attn5(const TraceBuf &b);
 
 // ---- programmatic dependent launch (PDL) ----
 // Kernels of a pass are launched with programmatic stream serialisation: a
@@ -496,6 +502,20 @@ const char *launch_attention_tc(const void *q, const int32_t *pos, const int4 *b
                                 int n_blocks, int max_rows_per_block, int n_splits, const Dims &dm,
                                 int layer, const KVView *views, KVView single, float *ws_o,
                                 float2 *ws_ml, void *out, cudaStream_t s);
+// The split merge alone (after launch_attention_tc5 with n_splits > 1).
+const char *launch_attention_combine(const int4 *blocks, int n_blocks, int n_splits,
+                                     const Dims &dm, float *ws_o, float2 *ws_ml, void *out,
+                                     cudaStream_t s);
+// tcgen05 attention of one document's rows (bf16 cache, head_dim 64 or 128):
+// query blocks of at most attn_tc5_rows_per_block(grp) rows; partials in the
+// same workspace layout as launch_attention_tc.  tm_kv: the cache's TMA view.
+int attn_tc5_rows_per_block(int grp);
+int attn_tc5_ctas_per_sm(int dh);
+const char *launch_attention_tc5(const void *q, const int32_t *pos, const int4 *blocks,
+                                 int n_blocks, int n_splits, const Dims &dm, int layer,
+                                 const void *pages, const int32_t *table, const CUtensorMap &tm_kv,
+                                 float *ws_o, float2 *ws_ml, void *out, int *dev_flag,
+                                 cudaStream_t s);
 
 // ---- kernels: selectors ----
 // bound: device int holding n - 1 (EditLocal@boundary writes the first

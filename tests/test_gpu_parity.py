@@ -481,3 +481,34 @@ def test_model_free_releases_live_caches():
     assert all(c.h is None for c in caches)
     for c in caches:
         c.close()
+
+
+@pytest.mark.parametrize("shape", ["llama8b", "qwen7b"])
+def test_tcgen05_attention_matches_mma_sync_kernel(shape, monkeypatch):
+    # The bf16 path has two attention kernels: tcgen05 for one document's
+    # rows (the default) and mma.sync for batches of documents, forced here
+    # with KVR_DISABLE_TC5_ATTENTION (read when the model is created).  On
+    # the same pass (700 keys: several key splits, a ragged last page; Qwen's
+    # 7 query heads per KV head give blocks of 18 rows) they agree within the
+    # bf16 tolerance, and are different arithmetic: not bit-identical.
+    cfg = synth.preset(shape, n_layers=2)
+    n, s, L = 700, 300, 8
+    doc = synth.document(21, n, cfg["vocab"])
+    new = synth.edit_tokens(22, doc[s:s + L], cfg["vocab"])
+    query = synth.fill_tokens(23, 3, cfg["vocab"], 13)
+    A = np.arange(s + L, s + L + 40)
+    rows = np.arange(n)
+    got = {}
+    for flag in ("0", "1"):
+        monkeypatch.setenv("KVR_DISABLE_TC5_ATTENTION", flag)
+        model = kv.Model(cfg, None, seed=0, max_context=1024, max_rows=512)
+        cache = model.prefill(doc)
+        cache.repair(new, s, A)
+        got[flag] = cache.read(rows) + (model.logits(cache, query),)
+        cache.close()
+        model.close()
+    (k0, v0, lg0), (k1, v1, lg1) = got["0"], got["1"]
+    for l in range(cfg["n_layers"]):
+        assert rel(k0[:, l], k1[:, l]) <= TOL["bf16"] and rel(v0[:, l], v1[:, l]) <= TOL["bf16"], l
+    assert rel(lg0, lg1) <= TOL["bf16"]
+    assert not (np.array_equal(k0, k1) and np.array_equal(v0, v1))
