@@ -264,8 +264,8 @@ kvr_status layer_rest(kvr_model *m, const Rows &r, int l) {
                                            m->attn_ws_o, m->attn_ws_ml, m->attn, m->dev_flag,
                                            m->stream);
       if (!e)
-        e = launch_attention_combine(r.blocks, r.n_blocks, r.n_splits, dm, m->attn_ws_o,
-                                     m->attn_ws_ml, m->attn, m->stream);
+        e = launch_attention_combine(r.blocks, r.n_blocks, r.max_block_rows, r.n_splits, dm,
+                                     m->attn_ws_o, m->attn_ws_ml, m->attn, m->stream);
       if (e) return fail(KVR_E_CUDA, "attention: %s", e);
       KVR_TRY(launch_check(m, r.n_splits > 1 ? 2 : 1));
     } else if (use_tc_attention(m)) {

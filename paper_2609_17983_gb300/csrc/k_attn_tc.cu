@@ -18,6 +18,8 @@
 // elsewhere (operator R, Sec. 3).
 #include <math.h>
 
+#include <algorithm>
+
 #include <type_traits>
 
 #include "kvr_internal.cuh"
@@ -42,6 +44,7 @@ struct AttnTcParams {
   float2 *ws_ml; // [n_splits][n_blocks][MAXQ]
   int n_blocks;
   __nv_bfloat16 *out;  // [M][H*dh]
+  int cq;              // query slots per (block, head) the combine visits: the largest block's
 };
 
 __device__ __forceinline__ uint32_t su32(const void *p) {
@@ -308,9 +311,9 @@ __global__ void __launch_bounds__(256) k_attn_combine(const AttnTcParams p) {
   ts.waited();
   const int gw = (blockIdx.x * 8) + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   const int half = gw & 1, wv = gw >> 1;
-  const int total = p.n_blocks * p.G * MAXQ;
+  const int total = p.n_blocks * p.G * p.cq;
   if (wv >= total) return;
-  const int v = wv % MAXQ, bg = wv / MAXQ;
+  const int v = wv % p.cq, bg = wv / p.cq;
   const int g = bg % p.G, blk = bg / p.G;
   const int4 bd = p.blocks[blk];
   const int mq = bd.y * p.grp;
@@ -382,7 +385,7 @@ const char *run(const AttnTcParams &p, int max_mq, cudaStream_t s) {
   dim3 grid(p.n_splits, p.G, p.n_blocks);
   launch_pdl(k_attn_tc<DH>, grid, warps * 32, smem, s, p);
   if (p.n_splits > 1) {
-    int warps = 2 * p.n_blocks * p.G * MAXQ;
+    int warps = 2 * p.n_blocks * p.G * p.cq;
     launch_pdl(k_attn_combine<DH>, (warps + 7) / 8, 256, 0, s, p);
   }
   cudaError_t e = cudaGetLastError();
@@ -391,7 +394,7 @@ const char *run(const AttnTcParams &p, int max_mq, cudaStream_t s) {
 
 template <int DH>
 const char *run_combine(const AttnTcParams &p, cudaStream_t s) {
-  const int warps = 2 * p.n_blocks * p.G * MAXQ;
+  const int warps = 2 * p.n_blocks * p.G * p.cq;
   launch_pdl(k_attn_combine<DH>, (warps + 7) / 8, 256, 0, s, p);
   cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? nullptr : cudaGetErrorString(e);
@@ -399,11 +402,12 @@ const char *run_combine(const AttnTcParams &p, cudaStream_t s) {
 
 }  // namespace
 
-const char *launch_attention_combine(const int4 *blocks, int n_blocks, int n_splits,
-                                     const Dims &dm, float *ws_o, float2 *ws_ml, void *out,
-                                     cudaStream_t s) {
+const char *launch_attention_combine(const int4 *blocks, int n_blocks, int max_rows_per_block,
+                                     int n_splits, const Dims &dm, float *ws_o, float2 *ws_ml,
+                                     void *out, cudaStream_t s) {
   if (n_blocks <= 0 || n_splits <= 1) return nullptr;
   AttnTcParams p{};
+  p.cq = std::min(MAXQ, max_rows_per_block * (dm.H / dm.G));
   p.H = dm.H;
   p.G = dm.G;
   p.grp = dm.H / dm.G;
@@ -445,6 +449,7 @@ const char *launch_attention_tc(const void *q, const int32_t *pos, const int4 *b
   p.n_blocks = n_blocks;
   p.out = (__nv_bfloat16 *)out;
   const int max_mq = max_rows_per_block * p.grp;
+  p.cq = max_mq;
   if (dm.dh == 128) return run<128>(p, max_mq, s);
   if (dm.dh == 64) return run<64>(p, max_mq, s);
   return "head_dim not supported";
