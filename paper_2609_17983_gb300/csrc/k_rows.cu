@@ -156,11 +156,13 @@ __global__ void __launch_bounds__(NORM_THREADS) k_rmsnorm(float *h, const float 
   }
 }
 
-// grid (M, H + 2G), block dh/2: rotate q and k heads at the row's position;
+// grid (M, ceil((H + 2G) / ROPE_HEADS)), block ROPE_HEADS * dh/2: rotate q and
+// k heads at the row's position;
 // q -> q_out fp32, k and v -> cache (if write_kv).  With a split view the
 // projection is completed from the GEMM's split-tile partials.  Positions,
 // the RoPE table, the page table and the bias are written before the pass,
 // so they are read before the wait on the projection.
+constexpr int ROPE_HEADS = 4;  // heads per CTA
 template <typename T>
 __global__ void k_rope_scatter(const float *qkv, const float2 *rope, const int32_t *pos, int H,
                                int G, int dh, int layer, const KVView *views,
@@ -169,7 +171,10 @@ __global__ void k_rope_scatter(const float *qkv, const float2 *rope, const int32
                                const SplitView sv) {
   TraceScope ts(TK_ROPE);
   pdl_trigger();
-  const int i = blockIdx.x, hh = blockIdx.y, t = threadIdx.x, half = dh >> 1;
+  const int half = dh >> 1;
+  const int i = blockIdx.x, hh = blockIdx.y * ROPE_HEADS + threadIdx.x / half,
+            t = threadIdx.x % half;
+  if (hh >= H + 2 * G) return;
   const int Nqkv = (H + 2 * G) * dh;
   const int n1 = hh * dh + t, n2 = n1 + half;
   const int p = pos[i];
@@ -380,15 +385,16 @@ void launch_rope_scatter(const float *qkv, const float2 *rope, const int32_t *po
                          KVView single, float *q_out, void *qb_out, float qscale, bool write_kv,
                          cudaStream_t s, const SplitView *sv) {
   if (M <= 0) return;
-  dim3 grid(M, dm.H + 2 * dm.G);
+  dim3 grid(M, (dm.H + 2 * dm.G + ROPE_HEADS - 1) / ROPE_HEADS);
+  const int threads = ROPE_HEADS * dm.dh / 2;
   int wk = write_kv ? 1 : 0;
   const SplitView v = sv ? *sv : SplitView{};
   if (dm.dtype == KVR_DTYPE_BF16)
-    launch_pdl(k_rope_scatter<__nv_bfloat16>, grid, dm.dh / 2, 0, s, qkv, rope, pos, dm.H, dm.G,
+    launch_pdl(k_rope_scatter<__nv_bfloat16>, grid, threads, 0, s, qkv, rope, pos, dm.H, dm.G,
                dm.dh, layer, views, rowdoc, single, q_out, (__nv_bfloat16 *)qb_out, qscale, wk,
                v);
   else
-    launch_pdl(k_rope_scatter<float>, grid, dm.dh / 2, 0, s, qkv, rope, pos, dm.H, dm.G, dm.dh,
+    launch_pdl(k_rope_scatter<float>, grid, threads, 0, s, qkv, rope, pos, dm.H, dm.G, dm.dh,
                layer, views, rowdoc, single, q_out, (__nv_bfloat16 *)qb_out, qscale, wk, v);
 }
 
