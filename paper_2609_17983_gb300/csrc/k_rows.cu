@@ -162,7 +162,7 @@ __global__ void __launch_bounds__(NORM_THREADS) k_rmsnorm(float *h, const float 
 // projection is completed from the GEMM's split-tile partials.  Positions,
 // the RoPE table, the page table and the bias are written before the pass,
 // so they are read before the wait on the projection.
-constexpr int ROPE_HEADS = 4;  // heads per CTA
+constexpr int ROPE_HEADS = 8;  // heads per CTA
 template <typename T>
 __global__ void k_rope_scatter(const float *qkv, const float2 *rope, const int32_t *pos, int H,
                                int G, int dh, int layer, const KVView *views,
