@@ -265,7 +265,9 @@ kvr_status layer_rest(kvr_model *m, const Rows &r, int l) {
                                            m->stream);
       if (!e)
         e = launch_attention_combine(r.blocks, r.n_blocks, r.max_block_rows, r.n_splits, dm,
-                                     m->attn_ws_o, m->attn_ws_ml, m->attn, m->stream);
+                                     m->attn_ws_o, m->attn_ws_ml, m->attn, m->stream,
+                                     w.tc_o ? w.wo : nullptr,
+                                     (long long)dm.d * dm.H * dm.dh * (long long)dm.es());
       if (e) return fail(KVR_E_CUDA, "attention: %s", e);
       KVR_TRY(launch_check(m, r.n_splits > 1 ? 2 : 1));
     } else if (use_tc_attention(m)) {

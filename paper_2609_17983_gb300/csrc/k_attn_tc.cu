@@ -45,6 +45,8 @@ struct AttnTcParams {
   int n_blocks;
   __nv_bfloat16 *out;  // [M][H*dh]
   int cq;              // query slots per (block, head) the combine visits: the largest block's
+  const char *pf;      // weights of the next GEMM, warmed into L2 by the combine (HBM is idle)
+  long long pf_bytes;
 };
 
 __device__ __forceinline__ uint32_t su32(const void *p) {
@@ -307,6 +309,19 @@ template <int DH>
 __global__ void __launch_bounds__(256) k_attn_combine(const AttnTcParams p) {
   TraceScope ts(TK_COMBINE);
   pdl_trigger();
+  if (p.pf_bytes > 0) {
+    // this CTA's slice of the next GEMM's weights, in pieces of PF_PIECE bytes
+    constexpr long long PF_PIECE = 32 << 10;
+    const long long slice = (p.pf_bytes / gridDim.x + 15) & ~15ll;
+    const long long b0 = (long long)blockIdx.x * slice;
+    const long long b1 = min(p.pf_bytes, b0 + slice);
+    for (long long o = b0 + (long long)threadIdx.x * PF_PIECE; o < b1; o += 256 * PF_PIECE) {
+      const long long n = min(PF_PIECE, b1 - o) & ~15ll;
+      if (n > 0)
+        asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p.pf + o), "r"((int)n)
+                     : "memory");
+    }
+  }
   pdl_wait();
   ts.waited();
   const int gw = (blockIdx.x * 8) + (threadIdx.x >> 5), lane = threadIdx.x & 31;
@@ -324,7 +339,7 @@ __global__ void __launch_bounds__(256) k_attn_combine(const AttnTcParams p) {
   const size_t stride = (size_t)p.n_blocks * p.G;  // between splits, in (block, head) units
   const size_t base = (size_t)blk * p.G + g;
   constexpr int VPL = DH / 64;  // floats per lane
-  constexpr int NB = 24;        // splits whose partial outputs load in the first round trip
+  constexpr int NB = 12;        // splits whose partial outputs load in the first round trip
   using VecT = typename std::conditional<VPL == 2, float2, float>::type;
   const VecT *src = (const VecT *)(p.ws_o + (base * MAXQ + v) * DH + half * (DH / 2)) + lane;
   const size_t sstride = stride * MAXQ * DH / VPL;  // in vectors
@@ -404,9 +419,12 @@ const char *run_combine(const AttnTcParams &p, cudaStream_t s) {
 
 const char *launch_attention_combine(const int4 *blocks, int n_blocks, int max_rows_per_block,
                                      int n_splits, const Dims &dm, float *ws_o, float2 *ws_ml,
-                                     void *out, cudaStream_t s) {
+                                     void *out, cudaStream_t s, const void *prefetch,
+                                     long long prefetch_bytes) {
   if (n_blocks <= 0 || n_splits <= 1) return nullptr;
   AttnTcParams p{};
+  p.pf = (const char *)prefetch;
+  p.pf_bytes = prefetch && ((uintptr_t)prefetch & 15) == 0 ? prefetch_bytes : 0;
   p.cq = std::min(MAXQ, max_rows_per_block * (dm.H / dm.G));
   p.H = dm.H;
   p.G = dm.G;

@@ -503,9 +503,12 @@ const char *launch_attention_tc(const void *q, const int32_t *pos, const int4 *b
                                 int layer, const KVView *views, KVView single, float *ws_o,
                                 float2 *ws_ml, void *out, cudaStream_t s);
 // The split merge alone (after launch_attention_tc5 with n_splits > 1).
+// prefetch (optional): the next GEMM's weights, pulled into L2 while the
+// combine (bound by L2 latency, not HBM) runs.
 const char *launch_attention_combine(const int4 *blocks, int n_blocks, int max_rows_per_block,
                                      int n_splits, const Dims &dm, float *ws_o, float2 *ws_ml,
-                                     void *out, cudaStream_t s);
+                                     void *out, cudaStream_t s, const void *prefetch = nullptr,
+                                     long long prefetch_bytes = 0);
 // tcgen05 attention of one document's rows (bf16 cache, head_dim 64 or 128):
 // query blocks of at most attn_tc5_rows_per_block(grp) rows; partials in the
 // same workspace layout as launch_attention_tc.  tm_kv: the cache's TMA view.
