@@ -12,10 +12,11 @@
 // tile, 64-wide K block) are linearised feature-tile-major and split into
 // `grid` contiguous, equal ranges, one per CTA (grid <= #SMs), so every SM
 // streams the same number of weight bytes whatever the GEMM shape.  A tile
-// covered by several CTAs is reduced by the last CTA to finish it (atomic
-// arrival counter): each part is written to a per-CTA fp32 slot and the last
-// arriver sums the parts in CTA order, so the result is deterministic.  No CTA
-// ever waits for another.
+// covered by several CTAs is either left to the kernel that next reads Y
+// (deferred mode: each CTA stores its fp32 part and exits), or reduced here
+// by its first CTA, for which it is the last segment: the others store their
+// parts and publish them, the owner waits for them (bounded) and sums all
+// parts in CTA order.  Either way the result is deterministic.
 //
 // Few-row GEMMs whose tiles cannot fill the GPU (e.g. O with 32 tiles) run
 // in cluster split-K mode instead: the P CTAs of a thread-block cluster
@@ -64,7 +65,7 @@ struct TcParams {
   void *out2;  // SwiGLU output (bf16 [M][N/2])
   int ld2;
   float *ws;        // [grid][2][BN][128] fp32 partial tiles
-  int *counters;    // [2][max_tiles]: arrivals, then published parts (self-resetting)
+  int *counters;    // [2][max_tiles]: unused, then published parts per split tile (self-resetting)
   long long max_tiles;
   int *dev_flag;
   int cluster;  // > 1: cluster split-K with this many CTAs per tile
@@ -140,7 +141,6 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       drain_bar;
   __shared__ uint32_t tmem_slot;
   __shared__ int abort_f;
-  __shared__ int last_f;
 
   TraceScope ts(TK_GEMM);
   pdl_trigger();
@@ -366,17 +366,16 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         }
         if (et == 0) trace_mark(3);
       } else {
-        // Reduced by the last CTA to arrive.  Arrival comes first: a CTA that
-        // is not last stores its part and then publishes it; the last one
-        // keeps its own part in TMEM, waits (bounded) until the others are
-        // published, and sums all parts in CTA order.
-        epi_bar();
-        if (et == 0) {
-          last_f = atomicAdd(&p.counters[tl], 1) == parts - 1;
-          trace_mark(4);
-        }
-        epi_bar();
-        if (!last_f) {
+        // Reduced by its first CTA: for it the tile is the last segment, so
+        // the others (for whom it is a first segment, or their whole range)
+        // have usually published their parts long before.  A CTA that is not
+        // the owner stores its part and publishes it; the owner keeps its own
+        // part in TMEM, waits (bounded) until the others are published, and
+        // sums all parts in CTA order.  Every CTA of the grid is resident (the
+        // next kernel cannot launch before all of them have started) and a
+        // publishing CTA waits on nothing, so the wait ends.
+        const bool owner = (int)blockIdx.x == i_first;
+        if (!owner) {
           int slot = range_start(blockIdx.x, p.total, p.grid) >= tile_u0 ? 0 : 1;
           float *w = p.ws + ((size_t)blockIdx.x * 2 + slot) * p.BN * BM;
           for (int c = 0; c < mv; c += 16) {
@@ -393,6 +392,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
             trace_mark(3);
           }
         } else {
+          if (et == 0) trace_mark(4);
           if (et == 0) {
             volatile int *ready = p.counters + p.max_tiles + tl;
             const uint64_t t0w = gtime_ns();
@@ -446,7 +446,6 @@ __global__ void __launch_bounds__(NTHREADS, 1)
               epilogue16(p, t0 + c, n, v, mv - c);
             }
             if (et == 0) {
-              p.counters[tl] = 0;
               p.counters[p.max_tiles + tl] = 0;
               trace_mark(5);
             }
