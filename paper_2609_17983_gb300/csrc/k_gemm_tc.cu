@@ -334,9 +334,6 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       long long tl = a / p.KB;
       long long b = (tl + 1) * p.KB < u1 ? (tl + 1) * p.KB : u1;
       uint32_t buf = seg & 1u, use = seg >> 1;
-      if (!mbar_wait(&accf_bar[buf], use & 1u, abort_v, p.dev_flag, 8)) break;
-      tc_fence_after();
-      if (et == 0) trace_mark(2);
       int ntile = (int)(tl / p.m_tiles), mtile = (int)(tl % p.m_tiles);
       int t0 = mtile * p.BN;
       int mv = min(p.BN, p.M - t0);
@@ -345,6 +342,40 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       int i_first = cta_of(tile_u0, p.total, p.grid);
       int i_last = cta_of(tile_u0 + p.KB - 1, p.total, p.grid);
       int parts = i_last - i_first + 1;
+      // The owner of a split tile waits for the other parts and, with two
+      // parts and at most 48 rows, loads the other one now, while this
+      // tile's MMAs are still running: both L2 round trips leave the tail.
+      const bool own_fix = parts > 1 && !p.defer && (int)blockIdx.x == i_first;
+      const bool pre = own_fix && parts == 2 && mv <= 48;
+      float other[48];
+      if (own_fix) {
+        if (et == 0) {
+          volatile int *ready = p.counters + p.max_tiles + tl;
+          const uint64_t t0w = gtime_ns();
+          for (uint32_t it = 0; *ready < parts - 1; ++it)
+            if ((it & 63) == 63 && (*abort_v || gtime_ns() - t0w > WAIT_NS)) {
+              if (!*abort_v) {
+                *abort_v = 1;
+                atomicOr(p.dev_flag, 32);
+              }
+              break;
+            }
+          trace_mark(4);
+        }
+        epi_bar();
+        if (!*abort_v) {
+          asm volatile("fence.acq_rel.gpu;" ::: "memory");  // acquire the parts
+          if (pre) {
+            const int so = range_start(i_last, p.total, p.grid) >= tile_u0 ? 0 : 1;
+            const float *src = p.ws + ((size_t)i_last * 2 + so) * p.BN * BM + f;
+#pragma unroll
+            for (int j = 0; j < 48; ++j) other[j] = j < mv ? __ldcg(src + (size_t)j * BM) : 0.f;
+          }
+        }
+      }
+      if (!mbar_wait(&accf_bar[buf], use & 1u, abort_v, p.dev_flag, 8)) break;
+      tc_fence_after();
+      if (et == 0) trace_mark(2);
       uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + buf * p.tmem_cols;
       if (parts == 1) {
         for (int c = 0; c < mv; c += 16) {
@@ -392,32 +423,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
             trace_mark(3);
           }
         } else {
-          if (et == 0) trace_mark(4);
-          if (et == 0) {
-            volatile int *ready = p.counters + p.max_tiles + tl;
-            const uint64_t t0w = gtime_ns();
-            for (uint32_t it = 0; *ready < parts - 1; ++it)
-              if ((it & 63) == 63 && (*abort_v || gtime_ns() - t0w > WAIT_NS)) {
-                if (!*abort_v) {
-                  *abort_v = 1;
-                  atomicOr(p.dev_flag, 32);
-                }
-                break;
-              }
-          }
-          epi_bar();
           if (!*abort_v) {
-            asm volatile("fence.acq_rel.gpu;" ::: "memory");  // acquire the parts
-            // two parts and at most 48 rows: the other part in one round trip
-            const bool pre = parts == 2 && mv <= 48;
-            float other[48];
-            if (pre) {
-              const int o = (int)blockIdx.x == i_first ? i_last : i_first;
-              const int so = range_start(o, p.total, p.grid) >= tile_u0 ? 0 : 1;
-              const float *src = p.ws + ((size_t)o * 2 + so) * p.BN * BM + f;
-#pragma unroll
-              for (int j = 0; j < 48; ++j) other[j] = j < mv ? __ldcg(src + (size_t)j * BM) : 0.f;
-            }
 #pragma unroll 1
             for (int c = 0; c < mv; c += 16) {
               float own[16], v[16];
