@@ -70,6 +70,7 @@ struct TcParams {
   int *dev_flag;
   int cluster;  // > 1: cluster split-K with this many CTAs per tile
   int defer;    // 1: split tiles are left as partials for the consumer
+  int stream_w; // 1: each weight tile is read once (one token tile): L2 evict-first
 };
 
 // ------------------------------------------------------------ PTX wrappers
@@ -194,6 +195,13 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       int ntile = (int)(tl0 / p.m_tiles), mtile = (int)(tl0 - (long long)ntile * p.m_tiles);
       int s = 0;
       uint32_t ph = 0, it = 0;
+      const uint64_t wpol = l2_evict_first();
+      auto load_w = [&](uint32_t sa, uint64_t *bar, int x, int y) {
+        if (p.stream_w)
+          tma_load_2d_hint((void *)__cvta_shared_to_generic(sa), &tmW, bar, x, y, wpol);
+        else
+          tma_load_2d((void *)__cvta_shared_to_generic(sa), &tmW, bar, x, y);
+      };
       // The weights never depend on the previous kernel: their tiles for the
       // first stages are requested before waiting for it (PDL), the
       // activation tiles of those stages right after.
@@ -204,8 +212,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         for (long long j = 0; j < npre; ++j) {
           uint32_t sa = base + (uint32_t)j * stage_bytes;
           mbar_expect_tx(&full_bar[j], tx_bytes);
-          tma_load_2d((void *)__cvta_shared_to_generic(sa), &tmW, &full_bar[j], kb2 * BK,
-                      nt2 * BM);
+          load_w(sa, &full_bar[j], kb2 * BK, nt2 * BM);
           if (++kb2 == p.KB) {
             kb2 = 0;
             if (++mt2 == p.m_tiles) {
@@ -238,8 +245,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         if (!mbar_wait(&empty_bar[s], ph ^ 1u, abort_v, p.dev_flag, 1)) break;
         uint32_t sa = base + (uint32_t)s * stage_bytes;
         mbar_expect_tx(&full_bar[s], tx_bytes);
-        tma_load_2d((void *)__cvta_shared_to_generic(sa), &tmW, &full_bar[s], kb * BK,
-                    ntile * BM);
+        load_w(sa, &full_bar[s], kb * BK, ntile * BM);
         tma_load_2d((void *)__cvta_shared_to_generic(sa + A_BYTES), &tmX, &full_bar[s], kb * BK,
                     mtile * p.BN);
         ++it;
@@ -647,6 +653,7 @@ const char *configure(int M, int N, int K, int num_sms, bool defer, TcParams &p,
   smem = 1024 + (size_t)p.stages * stage_bytes;
   p.defer = defer ? 1 : 0;
   p.cluster = p.m_tiles == 1 && !defer ? choose_cluster(M, N, num_sms, smem) : 0;
+  p.stream_w = p.m_tiles == 1;
   if (p.cluster > 1) p.grid = p.n_tiles * p.cluster;
   return nullptr;
 }
