@@ -284,16 +284,19 @@ def main():
     all_w = sum(v["bytes"] for v in gemms.values())
     traffic = (GU_TRAFFIC_BYTES if dom == "gemm_gu" and cfg["n_layers"] == 32
                and gemm_source_sha256() == GU_TRAFFIC_SOURCE_SHA256 else None)
-    # the whole step against the HBM floor: every layer's weights once, the
-    # keys and values of positions 0 .. s_end + K - 1 read once per layer
-    # (the attention's causal range), the K/V of the |S| + K rows written
+    # the whole step against the HBM floor: the weights R needs once -- every
+    # layer's QKV projection; attention output, O and MLP of all layers but
+    # the last, whose outputs feed no K/V -- the keys and values of positions
+    # 0 .. s_end + K - 1 read once per attending layer (the causal range),
+    # the K/V of the |S| + K rows written at every layer
     es = 2
     d, F, L = cfg["d_model"], cfg["ffn"], cfg["n_layers"]
     H, G, dh = cfg["n_heads"], cfg["n_kv_heads"], cfg["head_dim"]
-    layer_w = ((H + 2 * G) * dh * d + d * H * dh + 2 * F * d + d * F) * es
-    kv_read = (EDIT_START + EDIT_LEN + K_BUDGET) * L * 2 * G * dh * es
+    qkv_w = (H + 2 * G) * dh * d * es
+    rest_w = (d * H * dh + 2 * F * d + d * F) * es
+    kv_read = (EDIT_START + EDIT_LEN + K_BUDGET) * (L - 1) * 2 * G * dh * es
     kv_write = M * L * 2 * G * dh * es
-    pass_bytes = L * layer_w + kv_read + kv_write
+    pass_bytes = L * qkv_w + (L - 1) * rest_w + kv_read + kv_write
     pass_gbs = pass_bytes / (ms / 1e3) / 1e9
     all_ms = sum(v["ms"] for v in gemms.values())
 

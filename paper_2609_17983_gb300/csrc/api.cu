@@ -295,13 +295,16 @@ kvr_status layer_rest(kvr_model *m, const Rows &r, int l) {
 }
 
 // Operator R over rows r: every layer, K/V of all rows written before any of
-// them attends at that layer.
-kvr_status run_pass(kvr_model *m, const Rows &r) {
+// them attends at that layer.  kv_only: the pass produces K/V alone (prefill,
+// repair), so the last layer stops after its K/V are written -- K/V of layer l
+// are projections of the layer's input, and the last layer's attention and
+// MLP feed only the final hidden state, which the logits passes need.
+kvr_status run_pass(kvr_model *m, const Rows &r, bool kv_only) {
   if (r.M <= 0) return KVR_OK;
   KVR_TRY(embed(m, r));
   for (int l = 0; l < m->dims.L; ++l) {
     KVR_TRY(layer_qkv(m, r, l, true));
-    KVR_TRY(layer_rest(m, r, l));
+    if (!kv_only || l + 1 < m->dims.L) KVR_TRY(layer_rest(m, r, l));
   }
   return KVR_OK;
 }
@@ -312,7 +315,7 @@ kvr_status run_pass(kvr_model *m, const Rows &r) {
 // so it is captured once per such key and replayed.  Only on a stream that
 // can be captured (not the legacy default stream) and with profiling off.
 kvr_status run_pass_graph(kvr_model *m, kvr_cache *c, const Rows &r) {
-  if (!m->use_graphs || m->prof || m->stream == nullptr) return run_pass(m, r);
+  if (!m->use_graphs || m->prof || m->stream == nullptr) return run_pass(m, r, true);
   for (auto &g : c->graphs)
     if (g.M == r.M && g.nb == r.n_blocks && g.ns == r.n_splits) {
       cudaError_t e = cudaGraphLaunch(g.exec, m->stream);
@@ -323,7 +326,7 @@ kvr_status run_pass_graph(kvr_model *m, kvr_cache *c, const Rows &r) {
   int64_t l0 = m->launches;
   cudaError_t e = cudaStreamBeginCapture(m->stream, cudaStreamCaptureModeThreadLocal);
   if (e != cudaSuccess) return fail(KVR_E_CUDA, "begin capture: %s", cudaGetErrorString(e));
-  kvr_status st = run_pass(m, r);
+  kvr_status st = run_pass(m, r, true);
   cudaGraph_t graph = nullptr;
   e = cudaStreamEndCapture(m->stream, &graph);
   if (st || e != cudaSuccess) {
@@ -847,7 +850,7 @@ kvr_status kvr_prefill(kvr_model *m, const int32_t *tokens, int32_t n, kvr_cache
     r.pos = m->pos_d;
     r.max_pos = c0 + M - 1;
     st = plan_attention(m, r, pos.data(), nullptr);
-    if (!st) st = run_pass(m, r);
+    if (!st) st = run_pass(m, r, true);
   }
   if (st) {
     cudaStreamSynchronize(m->stream);
@@ -993,7 +996,7 @@ kvr_status kvr_repair_batch(kvr_model *m, const kvr_repair_req *reqs, int32_t n_
     r.doc_tokens = (const int32_t *const *)(tab + vb);
     r.max_pos = max_pos;
     st = plan_attention(m, r, P.data(), rowdoc.data());
-    if (!st) st = run_pass(m, r);
+    if (!st) st = run_pass(m, r, true);
   }
   cudaStreamSynchronize(m->stream);
   dev_free(tab);
@@ -1025,7 +1028,7 @@ kvr_status kvr_logits(kvr_model *m, const kvr_cache *c, const int32_t *query, in
   r.tm_kv = c->tm_kv_ok ? &c->tm_kv : nullptr;
   r.max_pos = c->n + qm - 1;
   KVR_TRY(plan_attention(m, r, P.data(), nullptr));
-  KVR_TRY(run_pass(m, r));
+  KVR_TRY(run_pass(m, r, false));
   // final RMSNorm of the last row, lm_head
   {
     Prof pr(m, P_NORM, (int64_t)dm.d * 4);
@@ -1119,7 +1122,8 @@ kvr_status kvr_select(kvr_model *m, const kvr_cache *c, kvr_policy policy, int32
                                       m->stream);
             st = launch_check(m, 2);
           }
-          if (!st) st = layer_rest(m, r, l);
+          // the scores need the queries of every layer; no K/V follow the last
+          if (!st && l + 1 < dm.L) st = layer_rest(m, r, l);
         }
         launch_rows_copy(r.single, dm.dtype, r.pos, edit_len, 0, dm.L, save, false, m->stream);
         if (!st) st = launch_check(m, 1);
@@ -1274,7 +1278,7 @@ kvr_status kvr_answer_logprob(kvr_model *m, const kvr_cache *c, const int32_t *p
   r.tm_kv = c->tm_kv_ok ? &c->tm_kv : nullptr;
   r.max_pos = c->n + rows - 1;
   KVR_TRY(plan_attention(m, r, P.data(), nullptr));
-  KVR_TRY(run_pass(m, r));
+  KVR_TRY(run_pass(m, r, false));
   // rows mp-1 .. mp+ma-2 predict answer[0..ma-1]
   {
     Prof pr(m, P_NORM, (int64_t)ma * dm.d * 4);
