@@ -172,6 +172,24 @@ GU_TRAFFIC_BYTES = 236466176 + 4580608
 GU_TRAFFIC_SOURCE_SHA256 = "b165c07124a41a8ead30ab7391b84980eafa8ccd8f3ab4aa4f3b40a23f914dfb"
 
 
+def max_over_ranks(x: float, device) -> float:
+    """The largest of every rank's x: a replicated job's step ends with its
+    slowest rank.  Identity without an initialised process group."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(x)
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_value(rows_per_rank: int, world: int, seconds: float) -> float:
+    """Whole-job positions/s: the rows every rank repaired per step over the
+    slowest rank's step time."""
+    return world * rows_per_rank / seconds
+
+
 def gemm_source_sha256() -> str:
     import hashlib
     h = hashlib.sha256()
@@ -260,13 +278,9 @@ def main():
             step()
         ev1.record(stream)
         barrier()
-    ms = ev0.elapsed_time(ev1) / args.steps
+    ms = max_over_ranks(ev0.elapsed_time(ev1) / args.steps, "cuda")
     launches = model.launches() - l0
-    if world > 1:
-        t = torch.tensor([ms], device="cuda")
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms = float(t.item())
-    value = world * M / (ms / 1e3)
+    value = job_value(M, world, ms / 1e3)
 
     # per-kernel-class device time over the same steps (CUDA events on the stream)
     kv.kvr_profile_reset(model.h)
@@ -310,7 +324,7 @@ def main():
         cache.repair(new, EDIT_START, A)
         k_rows, v_rows = cache.read(P)
     barrier()
-    e2e_s = (time.perf_counter() - t0) / args.steps
+    e2e_s = max_over_ranks((time.perf_counter() - t0) / args.steps, "cuda")
     h2d = int(new.nbytes + 4 * K_BUDGET + 4 * M)
     d2h = int(k_rows.nbytes + v_rows.nbytes + 4 * K_BUDGET)
 
@@ -342,7 +356,7 @@ def main():
                "repair_ms": ms, "prefill_ms": prefill_ms, "speedup_vs_prefill": prefill_ms / ms,
                "token_layers_per_s": value * cfg["n_layers"],
                "gpu_launches": launches,
-               "e2e": {"value": world * M / e2e_s, "unit": "positions/s",
+               "e2e": {"value": job_value(M, world, e2e_s), "unit": "positions/s",
                        "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
                "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peak,
                             "unit": "GB/s", "frac": achieved / peak, "traffic": traffic,
