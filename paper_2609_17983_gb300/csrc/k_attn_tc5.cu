@@ -7,10 +7,11 @@
 //   S = Q K^T      tcgen05.mma, M 128 x N 64 x K head_dim, into TMEM (two
 //                  S buffers, so S of chunk i+1 is computed while the softmax
 //                  works on chunk i);
-//   softmax        eight warps, two per TMEM lane quarter: one query vector
-//                  per thread pair, each thread half of the chunk's keys and
-//                  half of O's columns, the row maximum exchanged through
-//                  shared memory; S read once from
+//   softmax        sixteen warps, four per TMEM lane quarter: one query
+//                  vector per four threads, each thread a quarter of the
+//                  chunk's keys and of O's columns (four warps per SM
+//                  sub-partition hide each other's latency), the row maximum
+//                  exchanged through shared memory; S read once from
 //                  TMEM: causal mask key <= position, exponentials in the
 //                  log2 domain (Q is pre-scaled by log2(e)/sqrt(dh)) against
 //                  a reference maximum that is raised -- and the accumulator
@@ -29,8 +30,8 @@
 // launch (operator R, Sec. 3); keys are read only after the wait on that
 // kernel, and only L2 prefetches are issued before it.
 //
-// Warp roles (320 threads): warp 0 TMA (one lane), warp 1 TMEM allocation and
-// MMA issue (one lane), warps 2-9 softmax and epilogue.  Every wait is
+// Warp roles (576 threads): warp 0 TMA (one lane), warp 1 TMEM allocation and
+// MMA issue (one lane), warps 2-17 softmax and epilogue.  Every wait is
 // bounded; a wait that runs out sets the device error flag, the roles stop
 // issuing, drain what is in flight, free TMEM and return.
 #include <math.h>
@@ -44,10 +45,11 @@ using namespace ptx;
 
 constexpr int QV = 128;          // query vectors per CTA (UMMA M)
 constexpr int CH = KVR_PAGE;     // keys per chunk
-constexpr int NT5 = 320;         // threads per CTA
+constexpr int SMW = 4;           // softmax warps per TMEM lane quarter
+constexpr int NT5 = 64 + 128 * SMW;  // threads per CTA
 constexpr int WS_MAXQ = 192;     // query slots per (split, block, head) of the split workspace
 constexpr uint32_t TMEM_COLS = 256;  // S buffers at columns 0 and 64, O from column 128
-constexpr int SOFTMAX_THREADS = 256;
+constexpr int SOFTMAX_THREADS = 128 * SMW;
 constexpr float RESCALE_LOG2 = 8.f;  // headroom of the reference maximum (P <= 2^8)
 constexpr int KV_STAGES = 4;
 
@@ -99,8 +101,8 @@ __global__ void __launch_bounds__(NT5, 1)
   __shared__ int abort_f;
   __shared__ int spos[QV];
   __shared__ int sprow[2 * 64];  // pool rows of the CTA's K and V pages (at most 64 chunks)
-  __shared__ float sx[2][2][QV];  // per chunk parity and key half: row maxima
-  __shared__ float ssum[2][QV];   // per key half: sums of exponentials
+  __shared__ float sx[2][SMW][QV];  // per chunk parity and key part: row maxima
+  __shared__ float ssum[SMW][QV];   // per key part: sums of exponentials
 
   TraceScope ts(TK_ATTN);
   const int split = blockIdx.x, g = blockIdx.y, blk = blockIdx.z;
@@ -241,26 +243,28 @@ __global__ void __launch_bounds__(NT5, 1)
     }
   } else {
     // ------------------------------------------------------------ softmax
-    // Warps w and w + 4 share TMEM lane quarter w % 4: the same 32 query
-    // vectors, keys (and O columns) split in halves.  Their per-chunk maxima
-    // meet at a 64-thread named barrier, which both warps reach on every
-    // iteration -- also after an abort, when they only skip their work -- so
-    // it can never wait on a warp that has left.
+    // Warps w, w + 4, ... share TMEM lane quarter w % 4: the same 32 query
+    // vectors, keys (and O columns) split in SMW parts.  Their per-chunk
+    // maxima meet at a named barrier of the quarter's warps, which all of them
+    // reach on every iteration -- also after an abort, when they only skip
+    // their work -- so it can never wait on a warp that has left.
     const int quarter = warp & 3;  // TMEM lanes 32 * quarter .. + 31
-    const int half = (warp - 2) >> 2;
+    const int part = (warp - 2) >> 2;
     const int v = quarter * 32 + lane;
     const uint32_t tl = tmem + ((uint32_t)(quarter * 32) << 16);
     const int bar_id = 1 + quarter;
-    auto pair_bar = [&]() { asm volatile("bar.sync %0, 64;" ::"r"(bar_id) : "memory"); };
+    auto quad_bar = [&]() {
+      asm volatile("bar.sync %0, %1;" ::"r"(bar_id), "n"(32 * SMW) : "memory");
+    };
     pdl_wait();
-    // this thread's half of the Q row, into the swizzled K-major tile
+    // this thread's part of the Q row, into the swizzled K-major tile
     {
       const bool real = v < mq;
       const __nv_bfloat16 *src =
           p.q + ((size_t)(row0 + (real ? v / p.grp : 0)) * p.H + g * p.grp + v % p.grp) * DH;
 #pragma unroll
-      for (int k = 0; k < DH / 16; ++k) {
-        const int ch = half * (DH / 16) + k;
+      for (int k = 0; k < DH / (8 * SMW); ++k) {
+        const int ch = part * (DH / (8 * SMW)) + k;
         const uint32_t dst = sQ + (ch >> 3) * QV * 128 + sw_off(v, ch & 7);
         if (real)
           cp_async16(dst, src + ch * 8);
@@ -274,12 +278,13 @@ __global__ void __launch_bounds__(NT5, 1)
       mbar_arrive(&q_full);
       if (warp == 2 && lane == 0) trace_mark(2);
     }
-    constexpr int HK = CH / 2;  // keys of this thread per chunk
+    constexpr int HK = CH / SMW;  // keys of this thread per chunk
+    constexpr int OC = DH / SMW;  // O columns of this thread
     const int pv = spos[v];
-    float m = -INFINITY, l = 0.f;  // reference maximum, this half's sum of exponentials
+    float m = -INFINITY, l = 0.f;  // reference maximum, this part's sum of exponentials
     bool dead = false;             // warp-uniform: a wait ran out
     for (int i = 0; i < nch; ++i) {
-      const int b = i & 1, key0 = (c0 + i) * CH + half * HK;
+      const int b = i & 1, key0 = (c0 + i) * CH + part * HK;
       uint32_t sr[HK];
       float mx = -INFINITY;
       if (!dead) {
@@ -289,7 +294,10 @@ __global__ void __launch_bounds__(NT5, 1)
       if (!dead) {
         tc_fence_after();
         if (i == 0 && warp == 2 && lane == 0) trace_mark(3);
-        tmem_ld32_nowait(tl + b * CH + half * HK, sr);
+        if constexpr (HK == 32)
+          tmem_ld32_nowait(tl + b * CH + part * HK, sr);
+        else
+          tmem_ld16_nowait(tl + b * CH + part * HK, sr);
         tmem_wait_ld();
         tc_fence_before();
         mbar_arrive(&s_free[b]);  // S is in registers: the buffer may be refilled
@@ -301,11 +309,12 @@ __global__ void __launch_bounds__(NT5, 1)
 #pragma unroll
           for (int j = 0; j < w; ++j) t[j] = fmaxf(t[j], t[j + w]);
         mx = t[0];
-        sx[b][half][v] = mx;
+        sx[b][part][v] = mx;
       }
-      pair_bar();
+      quad_bar();
       if (dead) continue;
-      mx = fmaxf(mx, sx[b][half ^ 1][v]);
+#pragma unroll
+      for (int o = 0; o < SMW; ++o) mx = fmaxf(mx, sx[b][o][v]);
       // O is exactly zero until the first unmasked key: no rescale then
       if (m == -INFINITY) m = mx;
       const bool grow = mx > m + RESCALE_LOG2;
@@ -318,12 +327,12 @@ __global__ void __launch_bounds__(NT5, 1)
         }
         const float alpha = grow ? ex2(m - mx) : 1.f;
 #pragma unroll
-        for (int q = 0; q < DH / 32; ++q) {  // this half's O columns
+        for (int q = 0; q < OC / 16; ++q) {  // this part's O columns
           float o[16];
-          tmem_ld16(tl + 2 * CH + half * (DH / 2) + q * 16, o);
+          tmem_ld16(tl + 2 * CH + part * OC + q * 16, o);
 #pragma unroll
           for (int j = 0; j < 16; ++j) o[j] *= alpha;
-          tmem_st16(tl + 2 * CH + half * (DH / 2) + q * 16, o);
+          tmem_st16(tl + 2 * CH + part * OC + q * 16, o);
         }
         l *= alpha;
         if (grow) m = mx;
@@ -341,7 +350,7 @@ __global__ void __launch_bounds__(NT5, 1)
       for (int j = 0; j < HK; ++j) e[j] = key0 + j <= pv ? ex2(__uint_as_float(sr[j]) - m) : 0.f;
 #pragma unroll
       for (int q = 0; q < HK / 8; ++q) {
-        const uint32_t d = prow + (((half * (HK / 8) + q) ^ (v & 7)) << 4);
+        const uint32_t d = prow + (((part * (HK / 8) + q) ^ (v & 7)) << 4);
         asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(d),
                      "r"(pack2(e[q * 8], e[q * 8 + 1])), "r"(pack2(e[q * 8 + 2], e[q * 8 + 3])),
                      "r"(pack2(e[q * 8 + 4], e[q * 8 + 5])), "r"(pack2(e[q * 8 + 6], e[q * 8 + 7]))
@@ -361,9 +370,11 @@ __global__ void __launch_bounds__(NT5, 1)
       dead = !__all_sync(0xffffffffu, mbar_wait(&o_done[(nch - 1) & 1], ((nch - 1) >> 1) & 1,
                                                 abort_v, p.dev_flag, 71));
     if (warp == 2 && lane == 0) trace_mark(6);
-    ssum[half][v] = l;
-    pair_bar();
-    const float lt = l + ssum[half ^ 1][v];  // both halves, same reference maximum
+    ssum[part][v] = l;
+    quad_bar();
+    float lt = 0.f;  // all parts, same reference maximum, summed in part order
+#pragma unroll
+    for (int o = 0; o < SMW; ++o) lt += ssum[o][v];
     // O: TMEM -> registers -> shared memory (the K/V stages are free now; rows
     // of DH floats, 16-byte chunks XOR-swizzled by row so the writes hit
     // distinct banks) -> global, one coalesced row per warp instruction.
@@ -374,29 +385,36 @@ __global__ void __launch_bounds__(NT5, 1)
     float *stage = (float *)__cvta_shared_to_generic(sKV);
     if (!dead) {
       tc_fence_after();
-      const uint32_t to = tl + 2 * CH + half * (DH / 2);
-      uint32_t o[DH / 2];
-      tmem_ld32_nowait(to, o);
-      if (DH / 2 > 32) tmem_ld32_nowait(to + 32, o + 32 * (DH / 64 - 1));
+      const uint32_t to = tl + 2 * CH + part * OC;
+      uint32_t o[OC];
+      if constexpr (OC == 64) {
+        tmem_ld32_nowait(to, o);
+        tmem_ld32_nowait(to + 32, o + 32);
+      } else if constexpr (OC == 32) {
+        tmem_ld32_nowait(to, o);
+      } else {
+        tmem_ld16_nowait(to, o);
+      }
       tmem_wait_ld();
       if (warp == 2 && lane == 0) trace_mark(7);
 #pragma unroll
-      for (int k = 0; k < DH / 8; ++k) {  // this half's chunks
-        const int c = half * (DH / 8) + k;
+      for (int k = 0; k < OC / 4; ++k) {  // this part's chunks
+        const int c = part * (OC / 4) + k;
         *(float4 *)(stage + v * DH + ((c ^ (v & (RCH - 1))) << 2)) =
             make_float4(__uint_as_float(o[4 * k]) * scale, __uint_as_float(o[4 * k + 1]) * scale,
                         __uint_as_float(o[4 * k + 2]) * scale, __uint_as_float(o[4 * k + 3]) * scale);
       }
-      if (half == 0 && p.n_splits > 1 && v < mq) {
+      if (part == 0 && p.n_splits > 1 && v < mq) {
         const size_t bs = ((size_t)split * p.n_blocks + blk) * p.G + g;
         p.ws_ml[bs * WS_MAXQ + v] = make_float2(m, lt);
       }
     }
-    asm volatile("bar.sync 5, 256;" ::: "memory");
+    asm volatile("bar.sync 5, %0;" ::"n"(SOFTMAX_THREADS) : "memory");
     {
-      const int ws = warp - 2;  // rows ws * 16 .. + 15
-      for (int rr = 0; rr < QV / 8; ++rr) {
-        const int row = ws * (QV / 8) + rr;
+      constexpr int RPW = QV / (4 * SMW);  // rows per softmax warp
+      const int ws = warp - 2;             // rows ws * RPW .. + RPW - 1
+      for (int rr = 0; rr < RPW; ++rr) {
+        const int row = ws * RPW + rr;
         if (row >= mq || lane >= RCH) continue;
         const float4 x = *(const float4 *)(stage + row * DH + ((lane ^ (row & (RCH - 1))) << 2));
         if (p.n_splits == 1) {
