@@ -214,6 +214,18 @@ kvr_status kvr_cache_tokens(const kvr_cache *cache, int32_t *tokens_out);
 kvr_status kvr_cache_read(const kvr_cache *cache, const int32_t *positions, int32_t n_pos,
                           int32_t layer_begin, int32_t layer_end, float *k_out, float *v_out);
 
+/* The same rows in the cache's own element type: bf16 bit patterns (2 bytes
+ * per entry) for a bf16 model, fp32 otherwise -- the repaired K/V exactly as
+ * stored, at half the bytes of kvr_cache_read for bf16.  Same layout; k_out and
+ * v_out are host buffers of n_pos * (layer_end - layer_begin) * n_kv_heads *
+ * head_dim entries each, which the device writes directly when they are
+ * page-locked.  No device allocation during the call (model-owned scratch,
+ * grown when a larger read first needs it).  Synchronous.  Errors as
+ * kvr_cache_read: KVR_E_INVAL for NULL pointers, KVR_E_RANGE for a layer range
+ * or position outside the cache, KVR_E_NOMEM if the scratch cannot grow. */
+kvr_status kvr_cache_read_raw(const kvr_cache *cache, const int32_t *positions, int32_t n_pos,
+                              int32_t layer_begin, int32_t layer_end, void *k_out, void *v_out);
+
 /* Read one weight tensor back in canonical layout and model dtype into host
  * memory of `bytes` bytes.  name: "embed", "lm_head", "final_norm", or per
  * layer "wq","wk","wv","wo","wg","wu","wd","bq","bk","bv","attn_norm",

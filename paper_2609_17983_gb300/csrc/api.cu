@@ -507,6 +507,7 @@ void kvr_model_free(kvr_model *m) {
   dev_free(m->rope);
   dev_free(m->dev_flag);
   dev_free(m->tcw.partials);
+  dev_free(m->read_scratch);
   dev_free(m->tcw.counters);
   dev_free(m->blocks_d);
   dev_free(m->attn_ws_o);
@@ -1309,8 +1310,11 @@ kvr_status kvr_cache_tokens(const kvr_cache *c, int32_t *out) {
   return KVR_OK;
 }
 
-kvr_status kvr_cache_read(const kvr_cache *c, const int32_t *positions, int32_t n_pos,
-                          int32_t l0, int32_t l1, float *k_out, float *v_out) {
+// Rows of positions, layers [l0, l1), gathered on the device into the model's
+// readback scratch (grown, never shrunk) and copied to the host: widened to
+// fp32 (raw false) or as stored (raw true).
+kvr_status cache_read(const kvr_cache *c, const int32_t *positions, int32_t n_pos, int32_t l0,
+                      int32_t l1, void *k_out, void *v_out, bool raw) {
   if (!c || (n_pos > 0 && (!positions || !k_out || !v_out)))
     return fail(KVR_E_INVAL, "NULL argument");
   kvr_model *m = c->model;
@@ -1320,26 +1324,50 @@ kvr_status kvr_cache_read(const kvr_cache *c, const int32_t *positions, int32_t 
     if (positions[i] < 0 || positions[i] >= c->cap) return fail(KVR_E_RANGE, "position");
   if (n_pos == 0 || l0 == l1) return KVR_OK;
   KVR_TRY(use_device(m));
-  size_t elems = (size_t)n_pos * (l1 - l0) * dm.G * dm.dh;
-  int32_t *pd = (int32_t *)dev_alloc((size_t)n_pos * 4);
-  float *kd = (float *)dev_alloc(elems * 4), *vd = (float *)dev_alloc(elems * 4);
-  kvr_status st = KVR_OK;
-  if (!pd || !kd || !vd) st = fail(KVR_E_NOMEM, "readback buffers");
-  if (!st && cudaMemcpyAsync(pd, positions, (size_t)n_pos * 4, cudaMemcpyHostToDevice, m->stream))
+  const size_t elems = (size_t)n_pos * (l1 - l0) * dm.G * dm.dh;
+  const size_t eb = raw ? dm.es() : 4;
+  auto al = [](size_t x) { return (x + 255) / 256 * 256; };
+  const size_t pos_b = al((size_t)n_pos * 4), row_b = al(elems * eb);
+  const size_t need = pos_b + 2 * row_b;
+  if (need > m->read_scratch_bytes) {
+    CUDA_TRY(cudaStreamSynchronize(m->stream));  // the old scratch may still be in use
+    dev_free(m->read_scratch);
+    m->read_scratch = dev_alloc(need);
+    m->read_scratch_bytes = m->read_scratch ? need : 0;
+    if (!m->read_scratch) return fail(KVR_E_NOMEM, "readback scratch: %zu bytes", need);
+  }
+  char *base = (char *)m->read_scratch;
+  int32_t *pd = (int32_t *)base;
+  void *kd = base + pos_b, *vd = base + pos_b + row_b;
+  kvr_status st = (size_t)n_pos <= m->stage_cap ? stage_h2d(m, pd, positions, n_pos) : KVR_OK;
+  if (!st && (size_t)n_pos > m->stage_cap &&
+      cudaMemcpyAsync(pd, positions, (size_t)n_pos * 4, cudaMemcpyHostToDevice, m->stream))
     st = fail(KVR_E_CUDA, "positions upload");
   if (!st) {
-    launch_cache_gather(c->view(), dm.dtype, pd, n_pos, l0, l1, dm.G, dm.dh, kd, vd, m->stream);
+    if (raw)
+      launch_cache_gather_raw(c->view(), dm.dtype, pd, n_pos, l0, l1, dm.G, dm.dh, kd, vd,
+                              m->stream);
+    else
+      launch_cache_gather(c->view(), dm.dtype, pd, n_pos, l0, l1, dm.G, dm.dh, (float *)kd,
+                          (float *)vd, m->stream);
     st = launch_check(m, 1);
   }
-  if (!st && (cudaMemcpyAsync(k_out, kd, elems * 4, cudaMemcpyDeviceToHost, m->stream) ||
-              cudaMemcpyAsync(v_out, vd, elems * 4, cudaMemcpyDeviceToHost, m->stream)))
+  if (!st && (cudaMemcpyAsync(k_out, kd, elems * eb, cudaMemcpyDeviceToHost, m->stream) ||
+              cudaMemcpyAsync(v_out, vd, elems * eb, cudaMemcpyDeviceToHost, m->stream)))
     st = fail(KVR_E_CUDA, "readback");
   if (!st) st = sync_model(m);
   cudaStreamSynchronize(m->stream);
-  dev_free(pd);
-  dev_free(kd);
-  dev_free(vd);
   return st;
+}
+
+kvr_status kvr_cache_read(const kvr_cache *c, const int32_t *positions, int32_t n_pos,
+                          int32_t l0, int32_t l1, float *k_out, float *v_out) {
+  return cache_read(c, positions, n_pos, l0, l1, k_out, v_out, false);
+}
+
+kvr_status kvr_cache_read_raw(const kvr_cache *c, const int32_t *positions, int32_t n_pos,
+                              int32_t l0, int32_t l1, void *k_out, void *v_out) {
+  return cache_read(c, positions, n_pos, l0, l1, k_out, v_out, true);
 }
 
 kvr_status kvr_model_read_tensor(const kvr_model *m, const char *name, int32_t layer, void *out,

@@ -264,6 +264,25 @@ __global__ void k_cache_gather(KVView v, const int32_t *pos, int n_pos, int l0, 
   }
 }
 
+// K/V of the given positions, layers l0 .. l0+nl-1, as stored (T in, T out)
+template <typename T>
+__global__ void k_cache_gather_raw(KVView v, const int32_t *pos, int n_pos, int l0, int nl, int G,
+                                   int dh, T *k_out, T *v_out) {
+  size_t total = (size_t)n_pos * nl * G * dh;
+  const T *c = (const T *)v.pages;
+  for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < total;
+       e += (size_t)gridDim.x * blockDim.x) {
+    int i = (int)(e % dh);
+    size_t r = e / dh;
+    int g = (int)(r % G);
+    r /= G;
+    int l = (int)(r % nl);
+    int p = (int)(r / nl);
+    k_out[e] = c[v.offset(l0 + l, 0, g, pos[p]) + i];
+    v_out[e] = c[v.offset(l0 + l, 1, g, pos[p]) + i];
+  }
+}
+
 // buf layout [n_pos][nl][2][G][dh] in the cache dtype
 template <typename T>
 __global__ void k_rows_copy(KVView v, const int32_t *pos, int n_pos, int l0, int nl, T *buf,
@@ -417,6 +436,18 @@ void launch_cache_gather(KVView v, int dtype, const int32_t *pos, int n_pos, int
   else
     k_cache_gather<float><<<grid_for(n, 256), 256, 0, s>>>(v, pos, n_pos, l0, l1 - l0, G, dh,
                                                             k_out, v_out);
+}
+
+void launch_cache_gather_raw(KVView v, int dtype, const int32_t *pos, int n_pos, int l0, int l1,
+                             int G, int dh, void *k_out, void *v_out, cudaStream_t s) {
+  size_t n = (size_t)n_pos * (l1 - l0) * G * dh;
+  if (n == 0) return;
+  if (dtype == KVR_DTYPE_BF16)
+    k_cache_gather_raw<__nv_bfloat16><<<grid_for(n, 256), 256, 0, s>>>(
+        v, pos, n_pos, l0, l1 - l0, G, dh, (__nv_bfloat16 *)k_out, (__nv_bfloat16 *)v_out);
+  else
+    k_cache_gather_raw<float><<<grid_for(n, 256), 256, 0, s>>>(v, pos, n_pos, l0, l1 - l0, G, dh,
+                                                                (float *)k_out, (float *)v_out);
 }
 
 void launch_transplant(KVView dst, KVView src, int dtype, const int32_t *pos, int n_pos,

@@ -242,6 +242,8 @@ struct kvr_model {
   int32_t *sel_out = nullptr;  // [max_ctx] selected positions
   int32_t *sel_count = nullptr;
   void *save = nullptr;        // stale rows saved by read-only selector passes
+  void *read_scratch = nullptr;  // cache readback: positions, then the gathered K and V
+  size_t read_scratch_bytes = 0;
   size_t save_bytes = 0;
   int *dev_flag = nullptr;     // device error flag (bounded waits)
   kvr::TraceBuf trace{};       // attached device timeline buffer, if any
@@ -446,6 +448,9 @@ void launch_rope_scatter(const float *qkv, const float2 *rope, const int32_t *po
 void launch_swiglu(const float *gu, int M, int F, void *act, int dtype, cudaStream_t s);
 void launch_cache_gather(KVView v, int dtype, const int32_t *pos, int n_pos, int l0, int l1,
                          int G, int dh, float *k_out, float *v_out, cudaStream_t s);
+// The same gather in the cache's element type (no widening).
+void launch_cache_gather_raw(KVView v, int dtype, const int32_t *pos, int n_pos, int l0, int l1,
+                             int G, int dh, void *k_out, void *v_out, cudaStream_t s);
 void launch_rows_copy(KVView v, int dtype, const int32_t *pos, int n_pos, int l0, int l1,
                       void *buf, bool to_buf, cudaStream_t s);
 void launch_transplant(KVView dst, KVView src, int dtype, const int32_t *pos, int n_pos,

@@ -86,6 +86,7 @@ _sigs = {
     "kvr_cache_len": ([_P], _I32),
     "kvr_cache_tokens": ([_P, _P], _I32),
     "kvr_cache_read": ([_P, _P, _I32, _I32, _I32, _P, _P], _I32),
+    "kvr_cache_read_raw": ([_P, _P, _I32, _I32, _I32, _P, _P], _I32),
     "kvr_model_read_tensor": ([_P, ctypes.c_char_p, _I32, _P, ctypes.c_size_t], _I32),
     "kvr_profile_enable": ([_P, _I32], _I32),
     "kvr_profile_reset": ([_P], _I32),
@@ -254,6 +255,22 @@ def kvr_cache_read(cache, positions, layer_begin: int, layer_end: int, n_kv_head
     v = np.zeros(shape, np.float32)
     _check(_lib.kvr_cache_read(cache, _ptr(ps), ps.size, layer_begin, layer_end,
                                k.ctypes.data, v.ctypes.data))
+    return k, v
+
+
+def kvr_cache_read_raw(cache, positions, layer_begin: int, layer_end: int, n_kv_heads: int,
+                       head_dim: int, dtype, k_out=None, v_out=None):
+    """K and V rows as stored (bf16 bit patterns as uint16, or float32); k_out and
+    v_out (optional, e.g. page-locked) receive them in place."""
+    ps = _i32(positions)
+    shape = (ps.size, layer_end - layer_begin, n_kv_heads, head_dim)
+    k = np.empty(shape, dtype) if k_out is None else k_out
+    v = np.empty(shape, dtype) if v_out is None else v_out
+    for a in (k, v):
+        if a.shape != shape or a.dtype != np.dtype(dtype) or not a.flags.c_contiguous:
+            raise ValueError(f"readback buffer must be C-contiguous {np.dtype(dtype)}{shape}")
+    _check(_lib.kvr_cache_read_raw(cache, _ptr(ps), ps.size, layer_begin, layer_end,
+                                   k.ctypes.data, v.ctypes.data))
     return k, v
 
 
@@ -448,3 +465,12 @@ class Cache:
         c = self.model.cfg
         le = c["n_layers"] if layer_end is None else layer_end
         return kvr_cache_read(self.h, positions, layer_begin, le, c["n_kv_heads"], c["head_dim"])
+
+    def read_raw(self, positions, layer_begin: int = 0, layer_end: int | None = None,
+                 k_out=None, v_out=None):
+        """Rows as stored: uint16 bf16 bit patterns for a bf16 model, else float32."""
+        c = self.model.cfg
+        le = c["n_layers"] if layer_end is None else layer_end
+        dt = np.uint16 if c["dtype"] == "bf16" else np.float32
+        return kvr_cache_read_raw(self.h, positions, layer_begin, le, c["n_kv_heads"],
+                                  c["head_dim"], dt, k_out, v_out)

@@ -159,6 +159,32 @@ def test_noop_edit_and_idempotence_gpu(tiny):
     assert np.array_equal(k2, k3) and np.array_equal(v2, v3)
 
 
+@pytest.mark.parametrize("dtype", ["fp32", "bf16"])
+def test_cache_read_raw_is_the_stored_rows(dtype):
+    # kvr_cache_read_raw returns the entries as stored: bf16 bit patterns that
+    # widen (exactly) to kvr_cache_read's floats, or the floats themselves;
+    # twice in a row and into caller buffers (the scratch is reused), and a
+    # larger read after a smaller one (the scratch grows)
+    cfg, W, doc, s, new = tiny_setup(dtype)
+    model = kv.Model(cfg, W, max_context=1024, max_rows=512)
+    cache = model.prefill(doc)
+    for rows in (np.array([3, 200, 201, 511]), np.arange(0, len(doc), 3)):
+        k, v = cache.read(rows)
+        kr, vr = cache.read_raw(rows)
+        k2, v2 = np.empty_like(kr), np.empty_like(vr)
+        cache.read_raw(rows, k_out=k2, v_out=v2)
+        assert np.array_equal(kr, k2) and np.array_equal(vr, v2)
+        if dtype == "bf16":
+            assert kr.dtype == np.uint16
+            kr = (kr.astype(np.uint32) << 16).view(np.float32)
+            vr = (vr.astype(np.uint32) << 16).view(np.float32)
+        assert np.array_equal(kr, k) and np.array_equal(vr, v)
+    with pytest.raises(kv.KvrError):
+        cache.read_raw([len(doc) + 5000])
+    cache.close()
+    model.close()
+
+
 def test_logits_parity_fp32(tiny):
     cfg, W, doc, model = tiny["cfg"], tiny["W"], tiny["doc"], tiny["model"]
     cache = model.prefill(doc)
