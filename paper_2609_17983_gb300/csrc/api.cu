@@ -232,8 +232,11 @@ kvr_status norm(kvr_model *m, const float *g, int M, int row0 = 0) {
 
 // QKV projection, RoPE, and (write_kv) the K/V scatter of layer l.  keep_qkv:
 // m->qkv must hold the complete projection afterwards (else split tiles of
-// the GEMM are completed by the RoPE kernel alone).
-kvr_status layer_qkv(kvr_model *m, const Rows &r, int l, bool write_kv, bool keep_qkv = false) {
+// the GEMM are completed by the RoPE kernel alone).  need_q: the fp32 q
+// (m->q) is read afterwards (attention selector); the tensor-core attention
+// reads only the bf16 q, and the fp32 one is then not written.
+kvr_status layer_qkv(kvr_model *m, const Rows &r, int l, bool write_kv, bool keep_qkv = false,
+                     bool need_q = false) {
   const Dims &dm = m->dims;
   const LayerW &w = m->layers[l];
   KVR_TRY(norm(m, w.attn_norm, r.M));
@@ -242,8 +245,9 @@ kvr_status layer_qkv(kvr_model *m, const Rows &r, int l, bool write_kv, bool kee
                dm.Nqkv(), dm.d, GEMM_EPI_STORE, keep_qkv ? nullptr : &sv));
   {
     Prof pr(m, P_ROPE, (int64_t)r.M * dm.Nqkv() * 4);
-    launch_rope_scatter(m->qkv, m->rope, r.pos, r.M, dm, l, r.views, r.rowdoc, r.single, m->q,
-                        use_tc_attention(m) ? m->qb : nullptr,
+    const bool tc = use_tc_attention(m);
+    launch_rope_scatter(m->qkv, m->rope, r.pos, r.M, dm, l, r.views, r.rowdoc, r.single,
+                        tc && !need_q ? nullptr : m->q, tc ? m->qb : nullptr,
                         (float)(1.4426950408889634 / std::sqrt((double)dm.dh)), write_kv,
                         m->stream, &sv);
     KVR_TRY(launch_check(m, 1));
@@ -1116,7 +1120,7 @@ kvr_status kvr_select(kvr_model *m, const kvr_cache *c, kvr_policy policy, int32
         if (!st) st = launch_check(m, 2);
         if (!st) st = embed(m, r);
         for (int l = 0; l < dm.L && !st; ++l) {
-          st = layer_qkv(m, r, l, true);
+          st = layer_qkv(m, r, l, true, false, true);
           if (!st) {
             Prof pr(m, P_SELECT, 0);
             launch_attn_select_scores(m->q, edit_len, dm, l, r.single, s_end, n, probs, m->scores,

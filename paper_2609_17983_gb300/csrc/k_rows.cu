@@ -86,18 +86,19 @@ __global__ void k_embed_rows(const T *embed, const int32_t *tokens,
   for (int c = threadIdx.x; c < d; c += blockDim.x) h[(size_t)i * d + c] = ld(embed, base + c);
 }
 
-// One block of 1024 threads per row (d <= 8192, d % 4 == 0: NV = 1 float4
-// per thread up to d = 4096, else 2), each load issued before its first use.  Block i
+// One block per row (d <= 8192, d % 4 == 0), each load issued before its
+// first use: 1024 threads with NV = 1 float4 each up to d = 4096 (else 2)
+// for a pass of a few rows, 256 threads with NV = d / 1024 for many.  Block i
 // normalises h row row0 + i into out row i.  With a split view, the row is
 // first completed from the GEMM's split-tile partials (their tile table is
 // built once per block in shared memory) and written back to h.
-constexpr int NORM_THREADS = 1024;
-template <typename T, int NV>
-__global__ void __launch_bounds__(NORM_THREADS) k_rmsnorm(float *h, const float *g, int row0,
-                                                          int d, float eps, T *out,
-                                                          const SplitView sv) {
+constexpr int NORM_THREADS = 1024;   // a few rows: one float4 per thread, one round trip
+constexpr int NORM_THREADS_WIDE = 256;  // many rows: several CTAs per SM, fewer waves
+template <typename T, int NV, int TPB>
+__global__ void __launch_bounds__(TPB) k_rmsnorm(float *h, const float *g, int row0, int d,
+                                                 float eps, T *out, const SplitView sv) {
   __shared__ SplitTile tiles[64];
-  __shared__ float red[NORM_THREADS / 32];
+  __shared__ float red[TPB / 32];
   TraceScope ts(TK_NORM);
   pdl_trigger();
   const int i = blockIdx.x, row = row0 + i;
@@ -110,7 +111,7 @@ __global__ void __launch_bounds__(NORM_THREADS) k_rmsnorm(float *h, const float 
   float4 gw[NV];
 #pragma unroll
   for (int k = 0; k < NV; ++k) {
-    const int q = k * NORM_THREADS + threadIdx.x;
+    const int q = k * TPB + threadIdx.x;
     gw[k] = q < nq ? ((const float4 *)g)[q] : make_float4(0.f, 0.f, 0.f, 0.f);
   }
   pdl_wait();
@@ -121,7 +122,7 @@ __global__ void __launch_bounds__(NORM_THREADS) k_rmsnorm(float *h, const float 
   float ss = 0.f;
 #pragma unroll
   for (int k = 0; k < NV; ++k) {
-    const int q = k * NORM_THREADS + threadIdx.x;
+    const int q = k * TPB + threadIdx.x;
     v[k] = make_float4(0.f, 0.f, 0.f, 0.f);
     if (q < nq) {
       v[k] = x[q];
@@ -140,11 +141,11 @@ __global__ void __launch_bounds__(NORM_THREADS) k_rmsnorm(float *h, const float 
   __syncthreads();
   float tot = 0.f;
 #pragma unroll
-  for (int w = 0; w < NORM_THREADS / 32; ++w) tot += red[w];
+  for (int w = 0; w < TPB / 32; ++w) tot += red[w];
   const float r = 1.0f / sqrtf(tot / (float)d + eps);
 #pragma unroll
   for (int k = 0; k < NV; ++k) {
-    const int q = k * NORM_THREADS + threadIdx.x;
+    const int q = k * TPB + threadIdx.x;
     if (q < nq) {
       const float4 w = gw[k];
       const size_t o = (size_t)i * d + 4 * q;
@@ -158,8 +159,8 @@ __global__ void __launch_bounds__(NORM_THREADS) k_rmsnorm(float *h, const float 
 
 // grid (M, ceil((H + 2G) / ROPE_HEADS)), block ROPE_HEADS * dh/2: rotate q and
 // k heads at the row's position;
-// q -> q_out fp32, k and v -> cache (if write_kv).  With a split view the
-// projection is completed from the GEMM's split-tile partials.  Positions,
+// q -> q_out fp32 (if given) and qb_out, k and v -> cache (if write_kv).  With a
+// split view the projection is completed from the GEMM's split-tile partials.  Positions,
 // the RoPE table, the page table and the bias are written before the pass,
 // so they are read before the wait on the projection.
 constexpr int ROPE_HEADS = 8;  // heads per CTA
@@ -218,9 +219,11 @@ __global__ void k_rope_scatter(const float *qkv, const float2 *rope, const int32
     x2 = r2;
   }
   if (hh < H) {
-    float *qo = q_out + (size_t)i * H * dh + (size_t)hh * dh;
-    qo[t] = x1;
-    qo[t + half] = x2;
+    if (q_out) {
+      float *qo = q_out + (size_t)i * H * dh + (size_t)hh * dh;
+      qo[t] = x1;
+      qo[t + half] = x2;
+    }
     if (qb_out) {
       __nv_bfloat16 *qb = qb_out + (size_t)i * H * dh + (size_t)hh * dh;
       qb[t] = __float2bfloat16_rn(x1 * qscale);
@@ -390,13 +393,35 @@ void launch_rmsnorm(float *h, const float *g, int row0, int M, int d, double eps
                     int out_dtype, cudaStream_t s, const SplitView *sv) {
   if (M <= 0) return;
   const SplitView v = sv ? *sv : SplitView{};
+  // A pass of a few rows is latency-bound: 1024 threads, each with one
+  // float4 in flight.  Hundreds of rows (prefill) run in waves: 256 threads a
+  // row, several rows per SM at once.
+  if (M > 256 && d <= 4 * 8 * NORM_THREADS_WIDE) {
+    constexpr int W = NORM_THREADS_WIDE;
+    const int nv = (d + 4 * W - 1) / (4 * W);
+    if (out_dtype == KVR_DTYPE_BF16) {
+      auto k = nv <= 1 ? k_rmsnorm<__nv_bfloat16, 1, W>
+               : nv <= 2 ? k_rmsnorm<__nv_bfloat16, 2, W>
+               : nv <= 4 ? k_rmsnorm<__nv_bfloat16, 4, W>
+                         : k_rmsnorm<__nv_bfloat16, 8, W>;
+      launch_pdl(k, M, W, 0, s, h, g, row0, d, (float)eps, (__nv_bfloat16 *)out, v);
+    } else {
+      auto k = nv <= 1 ? k_rmsnorm<float, 1, W>
+               : nv <= 2 ? k_rmsnorm<float, 2, W>
+               : nv <= 4 ? k_rmsnorm<float, 4, W>
+                         : k_rmsnorm<float, 8, W>;
+      launch_pdl(k, M, W, 0, s, h, g, row0, d, (float)eps, (float *)out, v);
+    }
+    return;
+  }
   const bool one = d <= 4 * NORM_THREADS;
   if (out_dtype == KVR_DTYPE_BF16)
-    launch_pdl(one ? k_rmsnorm<__nv_bfloat16, 1> : k_rmsnorm<__nv_bfloat16, 2>, M, NORM_THREADS,
-               0, s, h, g, row0, d, (float)eps, (__nv_bfloat16 *)out, v);
+    launch_pdl(one ? k_rmsnorm<__nv_bfloat16, 1, NORM_THREADS>
+                   : k_rmsnorm<__nv_bfloat16, 2, NORM_THREADS>,
+               M, NORM_THREADS, 0, s, h, g, row0, d, (float)eps, (__nv_bfloat16 *)out, v);
   else
-    launch_pdl(one ? k_rmsnorm<float, 1> : k_rmsnorm<float, 2>, M, NORM_THREADS, 0, s, h, g, row0,
-               d, (float)eps, (float *)out, v);
+    launch_pdl(one ? k_rmsnorm<float, 1, NORM_THREADS> : k_rmsnorm<float, 2, NORM_THREADS>, M,
+               NORM_THREADS, 0, s, h, g, row0, d, (float)eps, (float *)out, v);
 }
 
 void launch_rope_scatter(const float *qkv, const float2 *rope, const int32_t *pos, int M,
