@@ -44,6 +44,28 @@ def load_peaks():
         return 6800.0, "fallback"
 
 
+def load_tensor_peak():
+    """Dense bf16 TFLOP/s sustained over seconds (the prefill is a long run)."""
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["bf16_tflops_sustained"]), "measured"
+    except Exception:
+        return 1700.0, "fallback"
+
+
+def prefill_flops(cfg, n: int) -> float:
+    """Dense FLOPs of a prefill of n tokens as the library runs it: every
+    layer's QKV projection; the O projection, MLP and causal attention of all
+    layers but the last (their outputs feed no K/V of the cache)."""
+    d, F, L = cfg["d_model"], cfg["ffn"], cfg["n_layers"]
+    H, G, dh = cfg["n_heads"], cfg["n_kv_heads"], cfg["head_dim"]
+    qkv = 2.0 * n * d * (H + 2 * G) * dh
+    rest = 2.0 * n * (H * dh * d + 2 * F * d + F * d)
+    attn = 4.0 * H * dh * n * (n + 1) / 2  # QK^T and PV over the causal triangle
+    return L * qkv + (L - 1) * (rest + attn)
+
+
 class Clocks:
     """Samples nvidia-smi clocks and throttle reasons while running."""
 
@@ -346,6 +368,8 @@ def main():
         if i:
             pre.append(a.elapsed_time(b))
     prefill_ms = statistics.median(pre)
+    tpeak, tpeak_kind = load_tensor_peak()
+    pf_tflops = prefill_flops(cfg, N_CTX) / (prefill_ms / 1e3) / 1e12
 
     if rank == 0:
         out = {"metric": METRIC, "value": value, "unit": "positions/s", "n_gpus": world,
@@ -358,6 +382,9 @@ def main():
                           "parallelism": "replicas" if world > 1 else "single",
                           "l2": "inputs larger than L2 (14 GB of weights streamed per step)"},
                "repair_ms": ms, "prefill_ms": prefill_ms, "speedup_vs_prefill": prefill_ms / ms,
+               "prefill_roofline": {"bound": "tensor", "flops": prefill_flops(cfg, N_CTX),
+                                    "achieved": pf_tflops, "peak": tpeak, "unit": "TFLOP/s",
+                                    "frac": pf_tflops / tpeak, "peak_kind": tpeak_kind + " sustained"},
                "token_layers_per_s": value * cfg["n_layers"],
                "gpu_launches": launches,
                "e2e": {"value": job_value(M, world, e2e_s), "unit": "positions/s",
