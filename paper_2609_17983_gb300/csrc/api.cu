@@ -742,8 +742,30 @@ kvr_status kvr_model_create(const kvr_model_config *cfg, const kvr_weights *wts,
     m->tcw.counters = (int *)dev_alloc(2 * (size_t)m->tcw.max_tiles * sizeof(int));
     if (!m->tcw.partials || !m->tcw.counters) return bail(fail(KVR_E_NOMEM, "GEMM workspace"));
     cudaMemset(m->tcw.counters, 0, 2 * (size_t)m->tcw.max_tiles * sizeof(int));
-    auto mk = [&](CUtensorMap *tm, const void *w, int N, int K) {
-      return gemm_tc_supported(N, K) && make_tmap_bf16(tm, w, N, K, 128);
+    // each tensor-core weight goes to the GEMM's blocked layout (one 16 KB
+    // block per TMA box), through a scratch buffer of the largest one
+    void *tmp = nullptr;
+    size_t tmp_bytes = 0;
+    bool nomem = false;
+    auto mk = [&](CUtensorMap *tm, void *w, int N, int K) {
+      if (!m->use_tc || nomem || !make_tmap_weight(tm, w, N, K)) return false;
+      const size_t bytes = (size_t)N * K * 2;
+      if (bytes > tmp_bytes) {
+        cudaDeviceSynchronize();
+        dev_free(tmp);
+        tmp = dev_alloc(bytes);
+        tmp_bytes = tmp ? bytes : 0;
+        if (!tmp) {
+          nomem = true;
+          return false;
+        }
+      }
+      if (launch_weight_tile(w, tmp, N, K, false, m->stream) ||
+          cudaMemcpyAsync(w, tmp, bytes, cudaMemcpyDeviceToDevice, m->stream) != cudaSuccess) {
+        nomem = true;  // reported below
+        return false;
+      }
+      return true;
     };
     for (int l = 0; l < dm.L; ++l) {
       LayerW &w = m->layers[l];
@@ -753,6 +775,9 @@ kvr_status kvr_model_create(const kvr_model_config *cfg, const kvr_weights *wts,
       w.tc_d = mk(&w.tm_d, w.wd, dm.d, dm.F);
     }
     m->tc_lm = mk(&m->tm_lm, m->lm_head, dm.V, dm.d);
+    cudaDeviceSynchronize();
+    dev_free(tmp);
+    if (nomem) return bail(fail(KVR_E_NOMEM, "blocked weight layout: scratch or copy failed"));
   }
   if (use_tc_attention(m)) {
     m->max_blocks = dm.max_rows + 256;
@@ -1391,6 +1416,20 @@ kvr_status kvr_model_read_tensor(const kvr_model *m, const char *name, int32_t l
                         cudaMemcpyDeviceToHost));
     return KVR_OK;
   };
+  // a tensor-core weight [N][K] is stored blocked: back to row-major first
+  void *plain = nullptr;
+  auto untiled = [&](const void *src, bool tiled, int N, int K) -> const void * {
+    if (!tiled) return src;
+    plain = dev_alloc((size_t)N * K * es);
+    if (!plain || launch_weight_tile(src, plain, N, K, true, m->stream) ||
+        cudaStreamSynchronize(m->stream) != cudaSuccess)
+      return nullptr;
+    return plain;
+  };
+  struct Freer {
+    void *&p;
+    ~Freer() { dev_free(p); }
+  } freer{plain};
   auto vec_out = [&](const float *src, size_t n) -> kvr_status {
     KVR_TRY(need(n * es));
     std::vector<float> t(n);
@@ -1404,13 +1443,29 @@ kvr_status kvr_model_read_tensor(const kvr_model *m, const char *name, int32_t l
     return KVR_OK;
   };
   if (nm == "embed") return rows_out(m->embed, dm.V, d, 0);
-  if (nm == "lm_head") return rows_out(m->lm_head, dm.V, d, 0);
+  const void *src = nullptr;
+  auto readable = [&](const void *p) -> kvr_status {
+    return p ? KVR_OK : fail(KVR_E_NOMEM, "untiling %s", name);
+  };
+  if (nm == "lm_head") {
+    KVR_TRY(readable(src = untiled(m->lm_head, m->tc_lm, dm.V, (int)d)));
+    return rows_out(src, dm.V, d, 0);
+  }
   if (nm == "final_norm") return vec_out(m->final_norm, d);
-  if (nm == "wq") return rows_out(w->wqkv, HD, d, 0);
-  if (nm == "wk") return rows_out(w->wqkv, GD, d, HD);
-  if (nm == "wv") return rows_out(w->wqkv, GD, d, HD + GD);
-  if (nm == "wo") return rows_out(w->wo, d, HD, 0);
-  if (nm == "wd") return rows_out(w->wd, d, dm.F, 0);
+  if (nm == "wq" || nm == "wk" || nm == "wv") {
+    KVR_TRY(readable(src = untiled(w->wqkv, w->tc_qkv, dm.Nqkv(), (int)d)));
+    if (nm == "wq") return rows_out(src, HD, d, 0);
+    if (nm == "wk") return rows_out(src, GD, d, HD);
+    return rows_out(src, GD, d, HD + GD);
+  }
+  if (nm == "wo") {
+    KVR_TRY(readable(src = untiled(w->wo, w->tc_o, (int)d, (int)HD)));
+    return rows_out(src, d, HD, 0);
+  }
+  if (nm == "wd") {
+    KVR_TRY(readable(src = untiled(w->wd, w->tc_d, (int)d, dm.F)));
+    return rows_out(src, d, dm.F, 0);
+  }
   if (nm == "attn_norm") return vec_out(w->attn_norm, d);
   if (nm == "mlp_norm") return vec_out(w->mlp_norm, d);
   if (nm == "bq" || nm == "bk" || nm == "bv") {
@@ -1420,11 +1475,12 @@ kvr_status kvr_model_read_tensor(const kvr_model *m, const char *name, int32_t l
   }
   if (nm == "wg" || nm == "wu") {
     KVR_TRY(need((size_t)dm.F * d * es));
+    KVR_TRY(readable(src = untiled(w->wgu, w->tc_gu, 2 * dm.F, (int)d)));
     size_t row = d * es;
     for (int b = 0; b < dm.F / GU_BLOCK; ++b) {
       size_t srow = (size_t)b * 2 * GU_BLOCK + (nm == "wu" ? GU_BLOCK : 0);
       CUDA_TRY(cudaMemcpy((char *)out + (size_t)b * GU_BLOCK * row,
-                          (const char *)w->wgu + srow * row, GU_BLOCK * row,
+                          (const char *)src + srow * row, GU_BLOCK * row,
                           cudaMemcpyDeviceToHost));
     }
     return KVR_OK;

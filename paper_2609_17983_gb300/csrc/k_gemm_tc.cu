@@ -212,7 +212,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         for (long long j = 0; j < npre; ++j) {
           uint32_t sa = base + (uint32_t)j * stage_bytes;
           mbar_expect_tx(&full_bar[j], tx_bytes);
-          load_w(sa, &full_bar[j], kb2 * BK, nt2 * BM);
+          load_w(sa, &full_bar[j], 0, (nt2 * p.KB + kb2) * BM);
           if (++kb2 == p.KB) {
             kb2 = 0;
             if (++mt2 == p.m_tiles) {
@@ -245,7 +245,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         if (!mbar_wait(&empty_bar[s], ph ^ 1u, abort_v, p.dev_flag, 1)) break;
         uint32_t sa = base + (uint32_t)s * stage_bytes;
         mbar_expect_tx(&full_bar[s], tx_bytes);
-        load_w(sa, &full_bar[s], kb * BK, ntile * BM);
+        load_w(sa, &full_bar[s], 0, (ntile * p.KB + kb) * BM);
         tma_load_2d((void *)__cvta_shared_to_generic(sa + A_BYTES), &tmX, &full_bar[s], kb * BK,
                     mtile * p.BN);
         ++it;
@@ -535,6 +535,24 @@ EncodeTiledFn encode_fn() {
 
 }  // namespace
 
+// The weight in the blocked layout (make_tmap_weight): 8 bf16 (one uint4) at a
+// time, row-major element (n, k) <-> block (n / 128, k / 64), row n % 128,
+// column k % 64.
+__global__ void k_weight_tile(const uint4 *src, uint4 *dst, int N, int K, int untile) {
+  const int K8 = K / 8, KB = K / BK;
+  const long long total = (long long)N * K8;
+  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
+       e += (long long)gridDim.x * blockDim.x) {
+    const int n = (int)(e / K8), k = (int)(e % K8) * 8;
+    const long long t =
+        (((long long)(n / BM) * KB + k / BK) * BM + n % BM) * (BK / 8) + (k % BK) / 8;
+    if (untile)
+      dst[e] = src[t];
+    else
+      dst[t] = src[e];
+  }
+}
+
 bool make_tmap_bf16(CUtensorMap *map, const void *ptr, int rows, int cols, int box_rows) {
   EncodeTiledFn fn = encode_fn();
   if (!fn || ((uintptr_t)ptr & 15) || (cols * 2) % 16 || box_rows > 256 || box_rows < 1)
@@ -550,6 +568,22 @@ bool make_tmap_bf16(CUtensorMap *map, const void *ptr, int rows, int cols, int b
 }
 
 bool gemm_tc_supported(int N, int K) { return N % BM == 0 && K % BK == 0 && N > 0 && K > 0; }
+
+bool make_tmap_weight(CUtensorMap *map, const void *w, int N, int K) {
+  if (!gemm_tc_supported(N, K)) return false;
+  const long long rows = (long long)N * K / BK;
+  return rows < (1ll << 31) && make_tmap_bf16(map, w, (int)rows, BK, BM);
+}
+
+const char *launch_weight_tile(const void *src, void *dst, int N, int K, bool untile,
+                               cudaStream_t s) {
+  if (!gemm_tc_supported(N, K)) return "weight shape not tiled";
+  const long long n = (long long)N * K / 8;
+  const int grid = (int)std::min<long long>((n + 255) / 256, 65536);
+  k_weight_tile<<<grid, 256, 0, s>>>((const uint4 *)src, (uint4 *)dst, N, K, untile ? 1 : 0);
+  cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? nullptr : cudaGetErrorString(e);
+}
 
 namespace {
 // Cluster split-K width for a few-row GEMM whose n_tiles cannot fill the

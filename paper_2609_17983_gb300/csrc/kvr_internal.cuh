@@ -474,6 +474,15 @@ void launch_gemm_simt(const GemmArgs &g, cudaStream_t s);
 // Tensor-core GEMM (bf16, N % 128 == 0, K % 64 == 0).  Epilogues:
 enum { GEMM_EPI_STORE = 0, GEMM_EPI_ACCUM = 1, GEMM_EPI_SWIGLU = 2 };
 bool make_tmap_bf16(CUtensorMap *map, const void *ptr, int rows, int cols, int box_rows);
+// Weights of the tensor-core GEMM are stored blocked: the 128-row x 64-column
+// tile (feature tile nt, K block kb) of W [N][K] is one contiguous 16 KB
+// block, row-major inside, block nt * K/64 + kb -- so each TMA box the GEMM
+// loads is one run of DRAM.  make_tmap_weight: the tensor map of such a
+// weight (rows of 64 elements); launch_weight_tile: row-major <-> blocked
+// (untile), between distinct buffers of N*K bf16.
+bool make_tmap_weight(CUtensorMap *map, const void *w, int N, int K);
+const char *launch_weight_tile(const void *src, void *dst, int N, int K, bool untile,
+                               cudaStream_t s);
 bool gemm_tc_supported(int N, int K);
 int gemm_tc_bn(int M);
 size_t gemm_tc_ws_bytes(int num_sms);
