@@ -50,6 +50,11 @@ constexpr int BK = 64;              // K per stage: one 128-byte swizzle atom of
 constexpr int UK = 16;              // K per tcgen05.mma kind::f16
 constexpr int NTHREADS = 192;
 constexpr int A_BYTES = BM * BK * 2;  // 16 KB
+// Weight stages requested before the wait on the previous kernel.  All CTAs
+// issue them at once into the same HBM queue; with the full pipeline (8) a CTA
+// that becomes resident late waits behind every other CTA's deep prefetch for
+// its first stage, and its whole range ends late.
+constexpr int PRE_WAIT_STAGES = 4;
 
 struct TcParams {
   int M, N, K;
@@ -206,7 +211,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       // first stages are requested before waiting for it (PDL), the
       // activation tiles of those stages right after.
       {
-        const long long npre = (u1 - u0) < S ? (u1 - u0) : S;
+        const long long npre = std::min<long long>(u1 - u0, std::min(S, PRE_WAIT_STAGES));
         int kb2 = kb, nt2 = ntile;
         int mt2 = mtile;
         for (long long j = 0; j < npre; ++j) {
