@@ -211,7 +211,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       // first stages are requested before waiting for it (PDL), the
       // activation tiles of those stages right after.
       {
-        const long long npre = std::min<long long>(u1 - u0, std::min(S, PRE_WAIT_STAGES));
+        const int pre_stages = S < PRE_WAIT_STAGES ? S : PRE_WAIT_STAGES;
+        const long long npre = (u1 - u0) < pre_stages ? (u1 - u0) : pre_stages;
         int kb2 = kb, nt2 = ntile;
         int mt2 = mtile;
         for (long long j = 0; j < npre; ++j) {
