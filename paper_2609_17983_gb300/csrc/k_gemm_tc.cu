@@ -48,7 +48,12 @@ using namespace ptx;
 constexpr int BM = 128;             // output features per tile (UMMA M)
 constexpr int BK = 64;              // K per stage: one 128-byte swizzle atom of bf16
 constexpr int UK = 16;              // K per tcgen05.mma kind::f16
-constexpr int NTHREADS = 192;
+// Epilogue warp groups: each group's four warps cover the four TMEM lane
+// quarters (all 128 features of a tile); group e takes the 16-row chunks
+// e, e + EPI_GROUPS, ... of a tile, so its chunks run in parallel.
+constexpr int EPI_GROUPS = 2;
+constexpr int EPI_THREADS = 128 * EPI_GROUPS;
+constexpr int NTHREADS = 64 + EPI_THREADS;
 constexpr int A_BYTES = BM * BK * 2;  // 16 KB
 // Weight stages requested before the wait on the previous kernel.  All CTAs
 // issue them at once into the same HBM queue; with the full pipeline (8) a CTA
@@ -80,7 +85,9 @@ struct TcParams {
 
 // ------------------------------------------------------------ PTX wrappers
 
-__device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+__device__ __forceinline__ void epi_bar() {
+  asm volatile("bar.sync 1, %0;" ::"n"(EPI_THREADS) : "memory");
+}
 
 // ------------------------------------------------------------ work split
 
@@ -165,7 +172,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&accf_bar[b], 1);
-      mbar_init(&acce_bar[b], 128);
+      mbar_init(&acce_bar[b], EPI_THREADS);
     }
     mbar_init(&drain_bar, 1);
     abort_f = 0;
@@ -320,7 +327,9 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     pdl_wait();  // outputs, partials and counters may still be in use upstream
     const int q = warp & 3;  // TMEM lane quarter of this warp
     const int f = q * 32 + lane;
-    const int et = threadIdx.x - 64;  // 0..127
+    const int et = threadIdx.x - 64;  // 0 .. EPI_THREADS - 1
+    const int eg = (warp - 2) >> 2;   // epilogue group: chunks 16 eg, 16 (eg + EPI_GROUPS), ...
+    constexpr int CSTEP = 16 * EPI_GROUPS;
     uint32_t seg = 0;
     if (p.cluster > 1) {
       // stage this CTA's partial tile [mv][128] in shared memory (the
@@ -331,7 +340,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         const int mv = min(p.BN, p.M);
         float *sp = (float *)__cvta_shared_to_generic(base);
         uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16);
-        for (int c = 0; c < mv; c += 16) {
+        for (int c = 16 * eg; c < mv; c += CSTEP) {
           float v[16];
           tmem_ld16(taddr + c, v);
 #pragma unroll
@@ -359,7 +368,10 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       // tile's MMAs are still running: both L2 round trips leave the tail.
       const bool own_fix = parts > 1 && !p.defer && (int)blockIdx.x == i_first;
       const bool pre = own_fix && parts == 2 && mv <= 48;
-      float other[48];
+      // this group's chunks of the other part: chunk k of the group at rows
+      // 16 eg + CSTEP k .. + 15
+      constexpr int PRE_CHUNKS = (48 + CSTEP - 1) / CSTEP;
+      float other[16 * PRE_CHUNKS];
       if (own_fix) {
         if (et == 0) {
           volatile int *ready = p.counters + p.max_tiles + tl;
@@ -381,7 +393,12 @@ __global__ void __launch_bounds__(NTHREADS, 1)
             const int so = range_start(i_last, p.total, p.grid) >= tile_u0 ? 0 : 1;
             const float *src = p.ws + ((size_t)i_last * 2 + so) * p.BN * BM + f;
 #pragma unroll
-            for (int j = 0; j < 48; ++j) other[j] = j < mv ? __ldcg(src + (size_t)j * BM) : 0.f;
+            for (int k = 0; k < PRE_CHUNKS; ++k)
+#pragma unroll
+              for (int j = 0; j < 16; ++j) {
+                const int row = 16 * eg + CSTEP * k + j;
+                other[16 * k + j] = row < mv ? __ldcg(src + (size_t)row * BM) : 0.f;
+              }
           }
         }
       }
@@ -390,7 +407,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       if (et == 0) trace_mark(2);
       uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + buf * p.tmem_cols;
       if (parts == 1) {
-        for (int c = 0; c < mv; c += 16) {
+        for (int c = 16 * eg; c < mv; c += CSTEP) {
           float v[16];
           tmem_ld16(taddr + c, v);
           epilogue16(p, t0 + c, n, v, mv - c);
@@ -400,7 +417,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         // the consumer of Y adds this part: store it and go on
         int slot = range_start(blockIdx.x, p.total, p.grid) >= tile_u0 ? 0 : 1;
         float *w = p.ws + ((size_t)blockIdx.x * 2 + slot) * p.BN * BM;
-        for (int c = 0; c < mv; c += 16) {
+        for (int c = 16 * eg; c < mv; c += CSTEP) {
           float v[16];
           tmem_ld16(taddr + c, v);
 #pragma unroll
@@ -421,7 +438,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         if (!owner) {
           int slot = range_start(blockIdx.x, p.total, p.grid) >= tile_u0 ? 0 : 1;
           float *w = p.ws + ((size_t)blockIdx.x * 2 + slot) * p.BN * BM;
-          for (int c = 0; c < mv; c += 16) {
+          for (int c = 16 * eg; c < mv; c += CSTEP) {
             float v[16];
             tmem_ld16(taddr + c, v);
 #pragma unroll
@@ -437,7 +454,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         } else {
           if (!*abort_v) {
 #pragma unroll 1
-            for (int c = 0; c < mv; c += 16) {
+            for (int c = 16 * eg; c < mv; c += CSTEP) {
               float own[16], v[16];
               tmem_ld16(taddr + c, own);
 #pragma unroll
@@ -447,10 +464,11 @@ __global__ void __launch_bounds__(NTHREADS, 1)
 #pragma unroll
                   for (int j = 0; j < 16; ++j) v[j] += own[j];
                 } else if (pre) {
-                  // rows c..c+15 of the preloaded part (c is 0, 16 or 32)
+                  // rows c..c+15 of the preloaded part: this group's chunk 0 or 1
+                  static_assert(PRE_CHUNKS == 2, "preloaded chunks of a group");
+                  const bool first = c == 16 * eg;
 #pragma unroll
-                  for (int j = 0; j < 16; ++j)
-                    v[j] += c == 0 ? other[j] : c == 16 ? other[16 + j] : other[32 + j];
+                  for (int j = 0; j < 16; ++j) v[j] += first ? other[j] : other[16 + j];
                 } else {
                   const int si = range_start(i, p.total, p.grid) >= tile_u0 ? 0 : 1;
                   const float *src = p.ws + (((size_t)i * 2 + si) * p.BN + c) * BM + f;
@@ -492,7 +510,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       const int f = (warp & 3) * 32 + lane;
       const int n = (int)(blockIdx.x / P) * BM + f;
       float *local = (float *)__cvta_shared_to_generic(base);
-      for (int c = r0; c < r1; c += 16) {
+      for (int c = r0 + 16 * ((warp - 2) >> 2); c < r1; c += 16 * EPI_GROUPS) {
         float v[16];
 #pragma unroll
         for (int j = 0; j < 16; ++j) v[j] = 0.f;
