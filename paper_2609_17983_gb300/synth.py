@@ -42,7 +42,7 @@ WEIGHT_STD = 0.02
 # ------------------------------------------------------------------ presets
 
 PRESETS = {
-    # Tiny Llama-style decoder, fp32 (BASELINE config 1).
+    # Tiny Llama-style decoder, fp32 (the small workload the oracle finishes in seconds).
     "tiny": dict(vocab=1024, d_model=256, n_layers=2, n_heads=4, n_kv_heads=2,
                  head_dim=64, ffn=688, rope_theta=10000.0, rms_eps=1e-5,
                  qkv_bias=False, dtype="fp32", delim_id=13),
