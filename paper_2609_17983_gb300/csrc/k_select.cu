@@ -195,7 +195,8 @@ __global__ void __launch_bounds__(TOPK_THREADS)
 
 // Attention selector, one layer: block (span row r, query head hh) writes the
 // softmax over the pool of q_{r,hh} . K_layer[j] / sqrt(dh) into
-// probs[(r*H + hh) * c + (j - s_end)].
+// probs[(r*H + hh) * c + (j - s_end)].  dh * sizeof(T) is 128, 256 or 512
+// bytes (dh 64 or 128), so a key row is 8, 16 or 32 lanes' 16-byte loads.
 template <typename T>
 __global__ void __launch_bounds__(256)
     k_attn_select_probs(const float *q, int H, int G, int dh, int layer, KVView v, int s_end,
@@ -210,20 +211,38 @@ __global__ void __launch_bounds__(256)
   const T *kc = (const T *)v.pages;
   float *pr = probs + (size_t)blockIdx.x * c;
   float mx = -INFINITY;
-  for (int t = threadIdx.x; t < c; t += blockDim.x) {
-    size_t o = v.offset(layer, 0, g, s_end + t);
+  // L lanes read one key row with 16-byte loads (a contiguous row per group
+  // of lanes, so a warp's load is L-way coalesced) and combine their partial
+  // dot products by shuffles: blockDim / L keys per iteration
+  constexpr int EPV = 16 / (int)sizeof(T);  // elements per 16-byte load
+  const int L = dh / EPV;                   // 8, 16 or 32 lanes (dh 64 or 128)
+  const int sub = threadIdx.x % L, kk = threadIdx.x / L, kpi = blockDim.x / L;
+  for (int t0 = 0; t0 < c; t0 += kpi) {
+    const int t = t0 + kk;
     float s = 0.f;
-    for (int i = 0; i < dh; ++i) {
-      float kv;
-      if constexpr (sizeof(T) == 2)
-        kv = __bfloat162float(kc[o + i]);
-      else
-        kv = kc[o + i];
-      s += qs[i] * kv;
+    if (t < c) {
+      const uint4 raw = *(const uint4 *)(kc + v.offset(layer, 0, g, s_end + t) + sub * EPV);
+      const float *qv = qs + sub * EPV;
+      if constexpr (sizeof(T) == 2) {
+        const __nv_bfloat162 *b = (const __nv_bfloat162 *)&raw;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float2 f = __bfloat1622float2(b[e]);
+          s += qv[2 * e] * f.x;
+          s += qv[2 * e + 1] * f.y;
+        }
+      } else {
+        const float *f = (const float *)&raw;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) s += qv[e] * f[e];
+      }
     }
-    s *= scale;
-    pr[t] = s;
-    mx = fmaxf(mx, s);
+    for (int off = L >> 1; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+    if (t < c && sub == 0) {
+      s *= scale;
+      pr[t] = s;
+      mx = fmaxf(mx, s);
+    }
   }
   for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
   if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = mx;
