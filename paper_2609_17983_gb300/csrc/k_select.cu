@@ -200,7 +200,7 @@ __global__ void __launch_bounds__(TOPK_THREADS)
 template <typename T>
 __global__ void __launch_bounds__(256)
     k_attn_select_probs(const float *q, int H, int G, int dh, int layer, KVView v, int s_end,
-                        int n, float *probs, float scale) {
+                        int n, float *probs, float scale, int in_smem) {
   int r = blockIdx.x / H, hh = blockIdx.x % H, g = hh / (H / G);
   int c = n - s_end;
   extern __shared__ float qs[];
@@ -210,6 +210,9 @@ __global__ void __launch_bounds__(256)
   __syncthreads();
   const T *kc = (const T *)v.pages;
   float *pr = probs + (size_t)blockIdx.x * c;
+  // the row's logits: in shared memory after q when they fit (one write of
+  // the probabilities to global at the end), else in place in probs
+  float *buf = in_smem ? qs + dh : pr;
   float mx = -INFINITY;
   // L lanes read one key row with 16-byte loads (a contiguous row per group
   // of lanes, so a warp's load is L-way coalesced) and combine their partial
@@ -217,14 +220,22 @@ __global__ void __launch_bounds__(256)
   constexpr int EPV = 16 / (int)sizeof(T);  // elements per 16-byte load
   const int L = dh / EPV;                   // 8, 16 or 32 lanes (dh 64 or 128)
   const int sub = threadIdx.x % L, kk = threadIdx.x / L, kpi = blockDim.x / L;
-  for (int t0 = 0; t0 < c; t0 += kpi) {
-    const int t = t0 + kk;
-    float s = 0.f;
-    if (t < c) {
-      const uint4 raw = *(const uint4 *)(kc + v.offset(layer, 0, g, s_end + t) + sub * EPV);
-      const float *qv = qs + sub * EPV;
+  const float *qv = qs + sub * EPV;
+  constexpr int U = 8;  // keys per lane group in flight: U loads issued before any use
+  for (int t0 = 0; t0 < c; t0 += kpi * U) {
+    uint4 raw[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int t = t0 + u * kpi + kk;
+      raw[u] = t < c ? *(const uint4 *)(kc + v.offset(layer, 0, g, s_end + t) + sub * EPV)
+                     : make_uint4(0u, 0u, 0u, 0u);
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int t = t0 + u * kpi + kk;
+      float s = 0.f;
       if constexpr (sizeof(T) == 2) {
-        const __nv_bfloat162 *b = (const __nv_bfloat162 *)&raw;
+        const __nv_bfloat162 *b = (const __nv_bfloat162 *)&raw[u];
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
           const float2 f = __bfloat1622float2(b[e]);
@@ -232,16 +243,16 @@ __global__ void __launch_bounds__(256)
           s += qv[2 * e + 1] * f.y;
         }
       } else {
-        const float *f = (const float *)&raw;
+        const float *f = (const float *)&raw[u];
 #pragma unroll
         for (int e = 0; e < 4; ++e) s += qv[e] * f[e];
       }
-    }
-    for (int off = L >> 1; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
-    if (t < c && sub == 0) {
-      s *= scale;
-      pr[t] = s;
-      mx = fmaxf(mx, s);
+      for (int off = L >> 1; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+      if (t < c && sub == 0) {
+        s *= scale;
+        buf[t] = s;
+        mx = fmaxf(mx, s);
+      }
     }
   }
   for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
@@ -257,8 +268,8 @@ __global__ void __launch_bounds__(256)
   __syncthreads();
   float z = 0.f;
   for (int t = threadIdx.x; t < c; t += blockDim.x) {
-    float e = expf(pr[t] - mx);
-    pr[t] = e;
+    float e = expf(buf[t] - mx);
+    buf[t] = e;
     z += e;
   }
   for (int off = 16; off > 0; off >>= 1) z += __shfl_xor_sync(0xffffffffu, z, off);
@@ -271,15 +282,30 @@ __global__ void __launch_bounds__(256)
   }
   __syncthreads();
   float inv = 1.0f / red[0];
-  for (int t = threadIdx.x; t < c; t += blockDim.x) pr[t] *= inv;
+  for (int t = threadIdx.x; t < c; t += blockDim.x) pr[t] = buf[t] * inv;
 }
 
-// score[j] += sum over (row, head) of probs, in a fixed order.
-__global__ void k_attn_select_accum(const float *probs, int RH, int c, int s_end, float *score) {
-  for (int t = blockIdx.x * blockDim.x + threadIdx.x; t < c; t += gridDim.x * blockDim.x) {
-    float s = 0.f;
-    for (int rh = 0; rh < RH; ++rh) s += probs[(size_t)rh * c + t];
-    score[s_end + t] += s;
+// score[j] += sum over (row, head) of probs, in a fixed order: a CTA takes 32
+// keys; its 8 warps sum interleaved slices of the RH rows (coalesced along the
+// keys), then warp 0 adds the 8 slice sums in slice order.
+constexpr int ACC_SLICES = 8;
+__global__ void __launch_bounds__(32 * ACC_SLICES)
+    k_attn_select_accum(const float *probs, int RH, int c, int s_end, float *score) {
+  __shared__ float part[ACC_SLICES][32];
+  const int kk = threadIdx.x & 31, sl = threadIdx.x >> 5;
+  const int t = blockIdx.x * 32 + kk;
+  float s = 0.f;
+  if (t < c) {
+#pragma unroll 8
+    for (int rh = sl; rh < RH; rh += ACC_SLICES) s += probs[(size_t)rh * c + t];
+  }
+  part[sl][kk] = s;
+  __syncthreads();
+  if (sl == 0 && t < c) {
+    float tot = 0.f;
+#pragma unroll
+    for (int i = 0; i < ACC_SLICES; ++i) tot += part[i][kk];
+    score[s_end + t] += tot;
   }
 }
 
@@ -391,14 +417,18 @@ void launch_attn_select_scores(const float *q, int S, const Dims &dm, int layer,
   int c = n - s_end;
   if (c <= 0 || S <= 0) return;
   float scale = (float)(1.0 / sqrt((double)dm.dh));
-  size_t smem = (size_t)dm.dh * sizeof(float);
+  // q, then the row's logits when both fit the default 48 KB of shared memory
+  const size_t with_row = (size_t)(dm.dh + c) * sizeof(float);
+  const int in_smem = with_row <= (48u << 10) ? 1 : 0;
+  const size_t smem = in_smem ? with_row : (size_t)dm.dh * sizeof(float);
   if (dm.dtype == KVR_DTYPE_BF16)
-    k_attn_select_probs<__nv_bfloat16><<<S * dm.H, 256, smem, s>>>(q, dm.H, dm.G, dm.dh, layer,
-                                                                    v, s_end, n, probs_ws, scale);
+    k_attn_select_probs<__nv_bfloat16><<<S * dm.H, 256, smem, s>>>(
+        q, dm.H, dm.G, dm.dh, layer, v, s_end, n, probs_ws, scale, in_smem);
   else
     k_attn_select_probs<float><<<S * dm.H, 256, smem, s>>>(q, dm.H, dm.G, dm.dh, layer, v, s_end,
-                                                            n, probs_ws, scale);
-  k_attn_select_accum<<<grid_for(c, 256), 256, 0, s>>>(probs_ws, S * dm.H, c, s_end, scores);
+                                                            n, probs_ws, scale, in_smem);
+  k_attn_select_accum<<<(c + 31) / 32, 32 * ACC_SLICES, 0, s>>>(probs_ws, S * dm.H, c, s_end,
+                                                                  scores);
 }
 
 void launch_kv_deviation(const float *qkv, const float2 *rope, const int32_t *pos, int M,
