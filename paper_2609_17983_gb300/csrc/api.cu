@@ -363,6 +363,19 @@ kvr_status sync_model(kvr_model *m) {
   return KVR_OK;
 }
 
+// Model-owned scratch that only grows: a call that fits reuses the buffer, so
+// repeated calls make no device allocation (and no cudaFree, which waits for
+// the whole device).
+kvr_status grow_scratch(kvr_model *m, void *&buf, size_t &have, size_t need, const char *what) {
+  if (need <= have) return KVR_OK;
+  CUDA_TRY(cudaStreamSynchronize(m->stream));  // the old buffer may still be in use
+  dev_free(buf);
+  buf = dev_alloc(need);
+  have = buf ? need : 0;
+  if (!buf) return fail(KVR_E_NOMEM, "%s: %zu bytes", what, need);
+  return KVR_OK;
+}
+
 kvr_status use_device(const kvr_model *m) {
   CUDA_TRY(cudaSetDevice(m->device));
   return KVR_OK;
@@ -512,6 +525,7 @@ void kvr_model_free(kvr_model *m) {
   dev_free(m->dev_flag);
   dev_free(m->tcw.partials);
   dev_free(m->read_scratch);
+  dev_free(m->sel_scratch);
   dev_free(m->tcw.counters);
   dev_free(m->blocks_d);
   dev_free(m->attn_ws_o);
@@ -1095,16 +1109,29 @@ kvr_status kvr_select(kvr_model *m, const kvr_cache *c, kvr_policy policy, int32
   int n = c->n, s_end = edit_start + edit_len;
   *count_out = 0;
   if (n - s_end <= 0 || K == 0) return KVR_OK;
-  // the edited context, private to this call
-  int32_t *toks = (int32_t *)dev_alloc((size_t)c->cap * 4);
-  if (!toks) return fail(KVR_E_NOMEM, "token scratch");
+  // scratch: the edited context, then (Attention, CacheBlend) the stale rows
+  // the read-only passes overwrite and the span queries' probabilities
+  auto al = [](size_t x) { return (x + 255) / 256 * 256; };
+  const size_t tok_b = al((size_t)c->cap * 4);
+  size_t save_b = 0, prob_b = 0;
+  if (policy == KVR_POLICY_ATTENTION) {
+    save_b = al((size_t)edit_len * dm.L * 2 * dm.G * dm.dh * dm.es());
+    prob_b = al(attn_select_ws_bytes(edit_len, dm, n - s_end));
+  } else if (policy == KVR_POLICY_CACHEBLEND) {
+    save_b = al((size_t)edit_len * 2 * dm.G * dm.dh * dm.es());
+  }
+  if (edit_len > dm.max_rows) save_b = prob_b = 0;  // refused below
+  KVR_TRY(grow_scratch(m, m->sel_scratch, m->sel_scratch_bytes, tok_b + save_b + prob_b,
+                       "selector scratch"));
+  char *scr = (char *)m->sel_scratch;
+  int32_t *toks = (int32_t *)scr;
   kvr_status st = KVR_OK;
   if (cudaMemcpyAsync(toks, c->tokens_d, (size_t)n * 4, cudaMemcpyDeviceToDevice, m->stream))
     st = fail(KVR_E_CUDA, "token copy");
   if (!st && edit_len) st = stage_h2d(m, toks + edit_start, new_tokens, edit_len);
   int topk_k = K;
   void *save = nullptr;
-  float *probs = nullptr;
+  void *probs = nullptr;  // Attention: the selector workspace
   if (!st && (policy == KVR_POLICY_EDITLOCAL || policy == KVR_POLICY_STRUCTURAL ||
               policy == KVR_POLICY_RANDOM || policy == KVR_POLICY_EDITLOCAL_BOUNDARY)) {
     Prof pr(m, P_SELECT, 0);
@@ -1126,11 +1153,9 @@ kvr_status kvr_select(kvr_model *m, const kvr_cache *c, kvr_policy policy, int32
       // restored), probabilities of the span queries over the stale pool keys
       std::vector<int32_t> P(edit_len);
       for (int i = 0; i < edit_len; ++i) P[i] = edit_start + i;
-      size_t save_bytes = (size_t)edit_len * dm.L * 2 * dm.G * dm.dh * dm.es();
-      save = dev_alloc(save_bytes);
-      probs = (float *)dev_alloc((size_t)edit_len * dm.H * (n - s_end) * 4);
-      if (!save || !probs) st = fail(KVR_E_NOMEM, "selector scratch");
-      if (!st) st = stage_h2d(m, m->pos_d, P.data(), edit_len);
+      save = scr + tok_b;
+      probs = scr + tok_b + save_b;
+      st = stage_h2d(m, m->pos_d, P.data(), edit_len);
       if (!st) {
         Rows r;
         r.M = edit_len;
@@ -1148,8 +1173,8 @@ kvr_status kvr_select(kvr_model *m, const kvr_cache *c, kvr_policy policy, int32
           st = layer_qkv(m, r, l, true, false, true);
           if (!st) {
             Prof pr(m, P_SELECT, 0);
-            launch_attn_select_scores(m->q, edit_len, dm, l, r.single, s_end, n, probs, m->scores,
-                                      m->stream);
+            launch_attn_select_scores(m->q, edit_len, dm, l, r.single, s_end, n, probs, l == 0,
+                                      m->scores, m->stream);
             st = launch_check(m, 2);
           }
           // the scores need the queries of every layer; no K/V follow the last
@@ -1173,8 +1198,7 @@ kvr_status kvr_select(kvr_model *m, const kvr_cache *c, kvr_policy policy, int32
     } else {
       std::vector<int32_t> P(edit_len);
       for (int i = 0; i < edit_len; ++i) P[i] = edit_start + i;
-      save = dev_alloc((size_t)edit_len * 2 * dm.G * dm.dh * dm.es());
-      if (!save) st = fail(KVR_E_NOMEM, "selector scratch");
+      save = scr + tok_b;
       Rows r;
       r.tokens = toks;
       r.single = c->view();
@@ -1244,9 +1268,6 @@ kvr_status kvr_select(kvr_model *m, const kvr_cache *c, kvr_policy policy, int32
     st = fail(KVR_E_CUDA, "select readback");
   if (!st) st = sync_model(m);
   cudaStreamSynchronize(m->stream);
-  dev_free(toks);
-  dev_free(save);
-  dev_free(probs);
   if (!st) *count_out = cnt;
   return st;
 }
@@ -1358,13 +1379,7 @@ kvr_status cache_read(const kvr_cache *c, const int32_t *positions, int32_t n_po
   auto al = [](size_t x) { return (x + 255) / 256 * 256; };
   const size_t pos_b = al((size_t)n_pos * 4), row_b = al(elems * eb);
   const size_t need = pos_b + 2 * row_b;
-  if (need > m->read_scratch_bytes) {
-    CUDA_TRY(cudaStreamSynchronize(m->stream));  // the old scratch may still be in use
-    dev_free(m->read_scratch);
-    m->read_scratch = dev_alloc(need);
-    m->read_scratch_bytes = m->read_scratch ? need : 0;
-    if (!m->read_scratch) return fail(KVR_E_NOMEM, "readback scratch: %zu bytes", need);
-  }
+  KVR_TRY(grow_scratch(m, m->read_scratch, m->read_scratch_bytes, need, "readback scratch"));
   char *base = (char *)m->read_scratch;
   int32_t *pd = (int32_t *)base;
   void *kd = base + pos_b, *vd = base + pos_b + row_b;
@@ -1549,6 +1564,7 @@ static cudaError_t trace_attach_all(const TraceBuf &b) {
   if (e == cudaSuccess) e = trace_attach_gemm(b);
   if (e == cudaSuccess) e = trace_attach_attn(b);
   if (e == cudaSuccess) e = trace_attach_attn5(b);
+  if (e == cudaSuccess) e = trace_attach_select(b);
   return e;
 }
 

@@ -193,111 +193,232 @@ __global__ void __launch_bounds__(TOPK_THREADS)
   if (tid == 0) *count = cnt;
 }
 
-// Attention selector, one layer: block (span row r, query head hh) writes the
-// softmax over the pool of q_{r,hh} . K_layer[j] / sqrt(dh) into
-// probs[(r*H + hh) * c + (j - s_end)].  dh * sizeof(T) is 128, 256 or 512
-// bytes (dh 64 or 128), so a key row is 8, 16 or 32 lanes' 16-byte loads.
-template <typename T>
-__global__ void __launch_bounds__(256)
-    k_attn_select_probs(const float *q, int H, int G, int dh, int layer, KVView v, int s_end,
-                        int n, float *probs, float scale, int in_smem) {
-  int r = blockIdx.x / H, hh = blockIdx.x % H, g = hh / (H / G);
-  int c = n - s_end;
-  extern __shared__ float qs[];
-  __shared__ float red[32];
-  for (int i = threadIdx.x; i < dh; i += blockDim.x)
-    qs[i] = q[(size_t)r * H * dh + (size_t)hh * dh + i];
-  __syncthreads();
-  const T *kc = (const T *)v.pages;
-  float *pr = probs + (size_t)blockIdx.x * c;
-  // the row's logits: in shared memory after q when they fit (one write of
-  // the probabilities to global at the end), else in place in probs
-  float *buf = in_smem ? qs + dh : pr;
-  float mx = -INFINITY;
-  // L lanes read one key row with 16-byte loads (a contiguous row per group
-  // of lanes, so a warp's load is L-way coalesced) and combine their partial
-  // dot products by shuffles: blockDim / L keys per iteration
-  constexpr int EPV = 16 / (int)sizeof(T);  // elements per 16-byte load
-  const int L = dh / EPV;                   // 8, 16 or 32 lanes (dh 64 or 128)
-  const int sub = threadIdx.x % L, kk = threadIdx.x / L, kpi = blockDim.x / L;
-  const float *qv = qs + sub * EPV;
-  constexpr int U = 8;  // keys per lane group in flight: U loads issued before any use
-  for (int t0 = 0; t0 < c; t0 += kpi * U) {
-    uint4 raw[U];
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int t = t0 + u * kpi + kk;
-      raw[u] = t < c ? *(const uint4 *)(kc + v.offset(layer, 0, g, s_end + t) + sub * EPV)
-                     : make_uint4(0u, 0u, 0u, 0u);
-    }
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int t = t0 + u * kpi + kk;
-      float s = 0.f;
-      if constexpr (sizeof(T) == 2) {
-        const __nv_bfloat162 *b = (const __nv_bfloat162 *)&raw[u];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float2 f = __bfloat1622float2(b[e]);
-          s += qv[2 * e] * f.x;
-          s += qv[2 * e + 1] * f.y;
-        }
-      } else {
-        const float *f = (const float *)&raw[u];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) s += qv[e] * f[e];
-      }
-      for (int off = L >> 1; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
-      if (t < c && sub == 0) {
-        s *= scale;
-        buf[t] = s;
-        mx = fmaxf(mx, s);
-      }
-    }
+// Attention selector, one layer, in two kernels over a workspace.  The
+// queries of kv group g are the span rows' heads hh with hh / (H/G) == g;
+// within the group a query is ql = r * (H/G) + (hh mod H/G), globally
+// qg = g * S * (H/G) + ql.  A CTA of k_attn_select_logits takes SEL_KC pool
+// keys and SEL_QT queries of one group: the keys are read once into shared
+// memory and serve every query of the tile (so a group's key rows leave L2
+// once per query tile, not once per query).  It stores the scaled logits,
+// logit[qg * c + (j - s_end)], and per query the chunk's max and sum of
+// exp(logit - max); the last CTA of (group, query tile) to finish folds the
+// chunk statistics into the pool softmax's max and 1 / sum.  Arrival is an
+// atomic count with no waiting: every other CTA just exits.
+constexpr int SEL_KC = 64, SEL_QT = 32, SEL_THREADS = 128;
+constexpr int SEL_KG = SEL_KC / 4;   // key groups of 4 (a thread: 4 queries x 4 keys)
+constexpr int SEL_LTS = SEL_KC + 4;  // logits tile row stride (floats)
+constexpr int SEL_DH_MAX = 128;
+constexpr int SEL_FOLD = 16;         // chunk statistics in flight per thread in the fold
+static_assert(SEL_KG * (SEL_QT / 4) == SEL_THREADS, "one 4x4 micro-tile per thread");
+
+struct SelWs {
+  float *logit;  // [S*H][c]
+  float2 *ml;    // [S*H][n_chunks] chunk (max, sum of exp)
+  float2 *mz;    // [S*H] pool (max, 1 / sum of exp)
+  int *cnt;      // [G][n_qtiles] arrivals
+};
+
+__host__ __device__ inline int sel_chunks(int c) { return (c + SEL_KC - 1) / SEL_KC; }
+
+// (m, z) <- the (max, sum of exp) of the union of two sets, either possibly
+// empty (m = -inf, z = 0).  Symmetric in its operands, bit for bit.
+__device__ __forceinline__ void lse_merge(float &m, float &z, float m2, float z2) {
+  if (m2 == -INFINITY) return;
+  if (m == -INFINITY) {
+    m = m2, z = z2;
+    return;
   }
-  for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = mx;
-  __syncthreads();
-  if (threadIdx.x < 32) {
-    float t = threadIdx.x < (blockDim.x >> 5) ? red[threadIdx.x] : -INFINITY;
-    for (int off = 16; off > 0; off >>= 1) t = fmaxf(t, __shfl_xor_sync(0xffffffffu, t, off));
-    if (threadIdx.x == 0) red[0] = t;
-  }
-  __syncthreads();
-  mx = red[0];
-  __syncthreads();
-  float z = 0.f;
-  for (int t = threadIdx.x; t < c; t += blockDim.x) {
-    float e = expf(buf[t] - mx);
-    buf[t] = e;
-    z += e;
-  }
-  for (int off = 16; off > 0; off >>= 1) z += __shfl_xor_sync(0xffffffffu, z, off);
-  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = z;
-  __syncthreads();
-  if (threadIdx.x < 32) {
-    float t = threadIdx.x < (blockDim.x >> 5) ? red[threadIdx.x] : 0.f;
-    for (int off = 16; off > 0; off >>= 1) t += __shfl_xor_sync(0xffffffffu, t, off);
-    if (threadIdx.x == 0) red[0] = t;
-  }
-  __syncthreads();
-  float inv = 1.0f / red[0];
-  for (int t = threadIdx.x; t < c; t += blockDim.x) pr[t] = buf[t] * inv;
+  const float mm = fmaxf(m, m2);
+  z = z * expf(m - mm) + z2 * expf(m2 - mm);
+  m = mm;
 }
 
-// score[j] += sum over (row, head) of probs, in a fixed order: a CTA takes 32
-// keys; its 8 warps sum interleaved slices of the RH rows (coalesced along the
-// keys), then warp 0 adds the 8 slice sums in slice order.
-constexpr int ACC_SLICES = 8;
-__global__ void __launch_bounds__(32 * ACC_SLICES)
-    k_attn_select_accum(const float *probs, int RH, int c, int s_end, float *score) {
-  __shared__ float part[ACC_SLICES][32];
-  const int kk = threadIdx.x & 31, sl = threadIdx.x >> 5;
-  const int t = blockIdx.x * 32 + kk;
+template <typename T>
+__global__ void __launch_bounds__(SEL_THREADS)
+    k_attn_select_logits(const float *q, int S, int H, int G, int dh, int layer, KVView v,
+                         int s_end, int c, float scale, SelWs ws) {
+  TraceScope ts(TK_SELECT);
+  pdl_trigger();
+  const int chunk = blockIdx.x, g = blockIdx.y, qt = blockIdx.z, nch = gridDim.x;
+  const int hpg = H / G, Nq = S * hpg;
+  const int t0 = chunk * SEL_KC, q0 = qt * SEL_QT;
+  const int nk = min(SEL_KC, c - t0), nq = min(SEL_QT, Nq - q0);
+  // both operands transposed, d-major and in fp32: the thread of micro-tile
+  // (queries 4qg.., keys 4kg..) reads one float4 of each per d
+  extern __shared__ float4 sel_smem[];
+  float *qT = (float *)sel_smem;   // [dh][SEL_QT]
+  float *kT = qT + dh * SEL_QT;    // [dh][SEL_KC]
+  float *lt = kT;                  // [SEL_QT][SEL_LTS] logits, after the keys
+  const int tid = threadIdx.x;
+  // the pool's stale keys: no kernel of the pass writes them, so they are
+  // read before the wait on the predecessor; a thread issues all its loads
+  // (page lookups, then rows) before it uses the first
+  constexpr int EPV = 16 / (int)sizeof(T);  // elements per 16-byte load
+  constexpr int KLD = SEL_KC * (SEL_DH_MAX / EPV) / SEL_THREADS;
+  const T *kc = (const T *)v.pages;
+  const int L = dh / EPV;
+  uint4 kx[KLD];
+#pragma unroll
+  for (int u = 0; u < KLD; ++u) {
+    const int i = tid + u * SEL_THREADS, kk = i % SEL_KC, sub = i / SEL_KC;
+    kx[u] = make_uint4(0u, 0u, 0u, 0u);
+    if (kk < nk && sub < L)
+      kx[u] = *(const uint4 *)(kc + v.offset(layer, 0, g, s_end + t0 + kk) + sub * EPV);
+  }
+#pragma unroll
+  for (int u = 0; u < KLD; ++u) {
+    const int i = tid + u * SEL_THREADS, kk = i % SEL_KC, sub = i / SEL_KC;
+    if (sub < L) {
+      float f[EPV];
+      if constexpr (sizeof(T) == 2) {
+        const __nv_bfloat162 *b = (const __nv_bfloat162 *)&kx[u];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float2 x = __bfloat1622float2(b[e]);
+          f[2 * e] = x.x, f[2 * e + 1] = x.y;
+        }
+      } else {
+        const float *x = (const float *)&kx[u];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) f[e] = x[e];
+      }
+#pragma unroll
+      for (int e = 0; e < EPV; ++e) kT[(sub * EPV + e) * SEL_KC + kk] = f[e];  // lanes: consecutive keys
+    }
+  }
+  pdl_wait();  // the queries come from the RoPE kernel just before
+  ts.waited();
+  constexpr int QLD = SEL_QT * (SEL_DH_MAX / 4) / SEL_THREADS;
+  const int D4 = dh / 4;
+  float4 qx[QLD];
+#pragma unroll
+  for (int u = 0; u < QLD; ++u) {
+    const int i = tid + u * SEL_THREADS, ql = i % SEL_QT, d4 = i / SEL_QT;
+    qx[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (ql < nq && d4 < D4) {
+      const int qq = q0 + ql, r = qq / hpg, hh = g * hpg + qq % hpg;
+      qx[u] = *(const float4 *)(q + ((size_t)r * H + hh) * dh + 4 * d4);
+    }
+  }
+#pragma unroll
+  for (int u = 0; u < QLD; ++u) {
+    const int i = tid + u * SEL_THREADS, ql = i % SEL_QT, d4 = i / SEL_QT;
+    if (d4 < D4) {
+      float *dst = qT + 4 * d4 * SEL_QT + ql;  // lanes: consecutive queries
+      dst[0] = qx[u].x;
+      dst[SEL_QT] = qx[u].y;
+      dst[2 * SEL_QT] = qx[u].z;
+      dst[3 * SEL_QT] = qx[u].w;
+    }
+  }
+  __syncthreads();
+  if (tid == 0) trace_mark(0);  // keys and queries staged
+  const int kg = tid % SEL_KG, qg = tid / SEL_KG;
+  float acc[4][4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
+#pragma unroll 4
+  for (int d = 0; d < dh; ++d) {
+    const float4 a = *(const float4 *)(qT + d * SEL_QT + 4 * qg);
+    const float4 b = *(const float4 *)(kT + d * SEL_KC + 4 * kg);
+    const float av[4] = {a.x, a.y, a.z, a.w}, bv[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+      for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
+  }
+  __syncthreads();  // keys consumed: lt reuses their space
+  if (tid == 0) trace_mark(1);  // logits computed
+  const size_t qg0 = (size_t)g * Nq + q0;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int ql = 4 * qg + i;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int kk = 4 * kg + j;
+      const float l = acc[i][j] * scale;
+      lt[ql * SEL_LTS + kk] = kk < nk ? l : -INFINITY;
+      if (kk < nk && ql < nq) ws.logit[(qg0 + ql) * c + t0 + kk] = l;
+    }
+  }
+  __syncthreads();
+  // chunk statistics: 4 threads per query, keys o, o + 4, ... (the row
+  // stride SEL_LTS = 4 mod 32 puts a warp's 8 queries x 4 lanes on 32 banks)
+  const int ql = tid >> 2, o = tid & 3;
+  {
+    const float *row = lt + ql * SEL_LTS;
+    float mx = -INFINITY;
+#pragma unroll
+    for (int j = 0; j < SEL_KC / 4; ++j) mx = fmaxf(mx, row[o + 4 * j]);
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+    float z = 0.f;  // key 0 is valid: mx is finite
+#pragma unroll
+    for (int j = 0; j < SEL_KC / 4; ++j) z += expf(row[o + 4 * j] - mx);
+    z += __shfl_xor_sync(0xffffffffu, z, 2);
+    z += __shfl_xor_sync(0xffffffffu, z, 1);
+    if (o == 0 && ql < nq) ws.ml[(qg0 + ql) * nch + chunk] = make_float2(mx, z);
+  }
+  __threadfence();
+  __syncthreads();
+  if (tid == 0) trace_mark(2);  // chunk statistics stored
+  int *last = (int *)qT;  // the queries are consumed
+  int *cnt = ws.cnt + (size_t)g * gridDim.z + qt;
+  if (tid == 0) *last = atomicAdd(cnt, 1) == nch - 1;
+  __syncthreads();
+  if (tid == 0) trace_mark(3);  // arrival counted
+  if (!*last) return;
+  if (tid == 0) *cnt = 0;  // ready for the next layer's launch
+  __threadfence();
+  // fold: 4 threads per query, each over chunks o, o + 4, ... (SEL_FOLD
+  // loads in flight), then the quad
+  float mx = -INFINITY, z = 0.f;
+  if (ql < nq) {
+    const float2 *row = ws.ml + (qg0 + ql) * nch;
+    for (int base = o; base < nch; base += 4 * SEL_FOLD) {
+      float2 x[SEL_FOLD];
+#pragma unroll
+      for (int j = 0; j < SEL_FOLD; ++j) {
+        const int ch = base + 4 * j;
+        x[j] = ch < nch ? __ldcg(row + ch) : make_float2(-INFINITY, 0.f);
+      }
+#pragma unroll
+      for (int j = 0; j < SEL_FOLD; ++j) lse_merge(mx, z, x[j].x, x[j].y);
+    }
+  }
+#pragma unroll
+  for (int off = 2; off > 0; off >>= 1) {
+    const float m2 = __shfl_xor_sync(0xffffffffu, mx, off);
+    const float z2 = __shfl_xor_sync(0xffffffffu, z, off);
+    lse_merge(mx, z, m2, z2);
+  }
+  if (o == 0 && ql < nq) ws.mz[qg0 + ql] = make_float2(mx, 1.0f / z);
+  if (tid == 0) trace_mark(4);  // fold done (last CTA of the group)
+}
+
+// score[j] += sum over the S*H queries of exp(logit - max) / sum, in a fixed
+// order: a CTA takes ACC_KEYS keys; its ACC_SLICES thread slices sum
+// interleaved sets of the queries (coalesced along the keys), then one
+// thread per key adds the slice sums in slice order.
+constexpr int ACC_KEYS = 16, ACC_SLICES = 32;
+__global__ void __launch_bounds__(ACC_KEYS * ACC_SLICES)
+    k_attn_select_accum(const float *logit, const float2 *mz, int NQ, int c, int s_end,
+                        float *score) {
+  TraceScope ts(TK_SELECT_ACC);
+  pdl_trigger();
+  __shared__ float part[ACC_SLICES][ACC_KEYS];
+  const int kk = threadIdx.x % ACC_KEYS, sl = threadIdx.x / ACC_KEYS;
+  const int t = blockIdx.x * ACC_KEYS + kk;
+  pdl_wait();  // logits and softmax statistics of the kernel before
   float s = 0.f;
   if (t < c) {
 #pragma unroll 8
-    for (int rh = sl; rh < RH; rh += ACC_SLICES) s += probs[(size_t)rh * c + t];
+    for (int qg = sl; qg < NQ; qg += ACC_SLICES) {
+      const float2 st = mz[qg];
+      s += expf(logit[(size_t)qg * c + t] - st.x) * st.y;
+    }
   }
   part[sl][kk] = s;
   __syncthreads();
@@ -412,23 +533,52 @@ const char *launch_topk(const unsigned long long *keys, int n, int s_end, int K,
   return e == cudaSuccess ? nullptr : cudaGetErrorString(e);
 }
 
+namespace {
+struct SelLayout {
+  size_t logit, ml, mz, cnt, total;  // byte offsets into the workspace
+};
+SelLayout sel_layout(int S, const Dims &dm, int c) {
+  auto al = [](size_t x) { return (x + 255) / 256 * 256; };
+  const size_t NQ = (size_t)S * dm.H, nqt = ((size_t)S * (dm.H / dm.G) + SEL_QT - 1) / SEL_QT;
+  SelLayout o;
+  o.logit = 0;
+  o.ml = o.logit + al(NQ * c * sizeof(float));
+  o.mz = o.ml + al(NQ * sel_chunks(c) * sizeof(float2));
+  o.cnt = o.mz + al(NQ * sizeof(float2));
+  o.total = o.cnt + al((size_t)dm.G * nqt * sizeof(int));
+  return o;
+}
+}  // namespace
+
+size_t attn_select_ws_bytes(int S, const Dims &dm, int n_pool) {
+  return n_pool > 0 && S > 0 ? sel_layout(S, dm, n_pool).total : 0;
+}
+
 void launch_attn_select_scores(const float *q, int S, const Dims &dm, int layer, KVView v,
-                               int s_end, int n, float *probs_ws, float *scores, cudaStream_t s) {
-  int c = n - s_end;
+                               int s_end, int n, void *ws_base, bool first_layer,
+                               float *scores, cudaStream_t s) {
+  const int c = n - s_end;
   if (c <= 0 || S <= 0) return;
-  float scale = (float)(1.0 / sqrt((double)dm.dh));
-  // q, then the row's logits when both fit the default 48 KB of shared memory
-  const size_t with_row = (size_t)(dm.dh + c) * sizeof(float);
-  const int in_smem = with_row <= (48u << 10) ? 1 : 0;
-  const size_t smem = in_smem ? with_row : (size_t)dm.dh * sizeof(float);
-  if (dm.dtype == KVR_DTYPE_BF16)
-    k_attn_select_probs<__nv_bfloat16><<<S * dm.H, 256, smem, s>>>(
-        q, dm.H, dm.G, dm.dh, layer, v, s_end, n, probs_ws, scale, in_smem);
-  else
-    k_attn_select_probs<float><<<S * dm.H, 256, smem, s>>>(q, dm.H, dm.G, dm.dh, layer, v, s_end,
-                                                            n, probs_ws, scale, in_smem);
-  k_attn_select_accum<<<(c + 31) / 32, 32 * ACC_SLICES, 0, s>>>(probs_ws, S * dm.H, c, s_end,
-                                                                  scores);
+  const float scale = (float)(1.0 / sqrt((double)dm.dh));
+  const SelLayout o = sel_layout(S, dm, c);
+  char *b = (char *)ws_base;
+  SelWs ws{(float *)(b + o.logit), (float2 *)(b + o.ml), (float2 *)(b + o.mz), (int *)(b + o.cnt)};
+  const int nqt = (S * (dm.H / dm.G) + SEL_QT - 1) / SEL_QT;
+  // arrival counts start at zero; each launch's last CTAs leave them at zero
+  if (first_layer) cudaMemsetAsync(ws.cnt, 0, (size_t)dm.G * nqt * sizeof(int), s);
+  const dim3 grid(sel_chunks(c), dm.G, nqt);
+  const size_t q_b = (size_t)SEL_QT * dm.dh * sizeof(float);
+  const size_t lt_b = (size_t)SEL_QT * SEL_LTS * sizeof(float);
+  const size_t k_b = (size_t)SEL_KC * dm.dh * sizeof(float);
+  const size_t smem = q_b + (k_b > lt_b ? k_b : lt_b);  // 48 KB at dh 128
+  auto kern = dm.dtype == KVR_DTYPE_BF16 ? k_attn_select_logits<__nv_bfloat16>
+                                         : k_attn_select_logits<float>;
+  // the trace build adds static shared memory: allow the sum above 48 KB
+  cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  launch_pdl(kern, grid, SEL_THREADS, smem, s, q, S, dm.H, dm.G, dm.dh, layer, v, s_end, c, scale,
+             ws);
+  launch_pdl(k_attn_select_accum, (c + ACC_KEYS - 1) / ACC_KEYS, ACC_KEYS * ACC_SLICES, 0, s,
+             (const float *)ws.logit, (const float2 *)ws.mz, S * dm.H, c, s_end, scores);
 }
 
 void launch_kv_deviation(const float *qkv, const float2 *rope, const int32_t *pos, int M,
@@ -439,5 +589,7 @@ void launch_kv_deviation(const float *qkv, const float2 *rope, const int32_t *po
   else
     k_kv_deviation<float><<<M, 256, 0, s>>>(qkv, rope, pos, dm.H, dm.G, dm.dh, v, scores);
 }
+
+KVR_TRACE_ATTACH(trace_attach_select)
 
 }  // namespace kvr

@@ -241,10 +241,10 @@ struct kvr_model {
   unsigned long long *keys = nullptr;  // [max_ctx + reserve] top-K keys
   int32_t *sel_out = nullptr;  // [max_ctx] selected positions
   int32_t *sel_count = nullptr;
-  void *save = nullptr;        // stale rows saved by read-only selector passes
   void *read_scratch = nullptr;  // cache readback: positions, then the gathered K and V
   size_t read_scratch_bytes = 0;
-  size_t save_bytes = 0;
+  void *sel_scratch = nullptr;   // selector: edited tokens, saved stale rows, probabilities
+  size_t sel_scratch_bytes = 0;
   int *dev_flag = nullptr;     // device error flag (bounded waits)
   kvr::TraceBuf trace{};       // attached device timeline buffer, if any
   kvr::SplitView pending{};    // split tiles of h not yet added (next RMSNorm adds them)
@@ -301,7 +301,9 @@ namespace kvr {
 // translation unit, set by its trace_attach_* function).  Even detached, the
 // checks lengthen each kernel's critical path, so tracing is compiled only
 // into the KVR_TRACE build of the library; elsewhere the hooks are empty.
-enum TraceKind : int { TK_EMBED = 1, TK_NORM, TK_GEMM, TK_ROPE, TK_ATTN, TK_COMBINE, TK_OTHER };
+enum TraceKind : int {
+  TK_EMBED = 1, TK_NORM, TK_GEMM, TK_ROPE, TK_ATTN, TK_COMBINE, TK_OTHER, TK_SELECT, TK_SELECT_ACC
+};
 #ifdef KVR_TRACE
 static __constant__ TraceBuf g_trace;
 
@@ -383,6 +385,7 @@ cudaError_t trace_attach_rows(const TraceBuf &b);
 cudaError_t trace_attach_gemm(const TraceBuf &b);
 cudaError_t trace_attach_attn(const TraceBuf &b);
 cudaError_t trace_attach_attn5(const TraceBuf &b);
+cudaError_t trace_attach_select(const TraceBuf &b);
 
 // ---- programmatic dependent launch (PDL) ----
 // Kernels of a pass are launched with programmatic stream serialisation: a
@@ -539,8 +542,14 @@ const char *launch_attention_tc5(const void *q, const int32_t *pos, const int4 *
 // delimiter position at or after s_end into it).
 void launch_scores_simple(int policy, const int32_t *tokens, int n, int s_end, int delim,
                           uint64_t seed, int *bound, unsigned long long *keys, cudaStream_t s);
+// Attention selector, one layer: adds to scores[j], j in [s_end, n), the
+// pool-softmax probabilities of the S span rows' queries (fp32 q, [S][H*dh]).
+// ws_base: attn_select_ws_bytes(S, dm, n - s_end) bytes; first_layer zeroes
+// its arrival counts.
+size_t attn_select_ws_bytes(int S, const Dims &dm, int n_pool);
 void launch_attn_select_scores(const float *q, int S, const Dims &dm, int layer, KVView v,
-                               int s_end, int n, float *probs_ws, float *scores, cudaStream_t s);
+                               int s_end, int n, void *ws_base, bool first_layer,
+                               float *scores, cudaStream_t s);
 void launch_kv_deviation(const float *qkv, const float2 *rope, const int32_t *pos, int M,
                          const Dims &dm, KVView v, float *scores, cudaStream_t s);
 void launch_float_keys(const float *scores, int n, int s_end, unsigned long long *keys,

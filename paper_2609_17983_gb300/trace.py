@@ -6,7 +6,9 @@ time it finished, and eight kernel-specific marks (GEMM, for the CTA's last
 tile: first operand stage landed, all MMAs complete, accumulator taken by the
 epilogue, partial stored, split-tile arrival counted or partials staged across
 the cluster, tile reduced and written, epilogue done, all warps done;
-attention: last key chunk consumed).  `launches` groups the records into kernel launches
+attention: last key chunk consumed; Attention-selector logits: keys and
+queries staged, logits computed, chunk statistics stored, arrival counted,
+fold done).  `launches` groups the records into kernel launches
 (a launch holds each block index once), in issue order; `layer_table`
 averages the launches of a repeating per-layer sequence by position.
 """
@@ -14,7 +16,8 @@ from __future__ import annotations
 
 import numpy as np
 
-KINDS = {1: "embed", 2: "rmsnorm", 3: "gemm", 4: "rope", 5: "attention", 6: "combine"}
+KINDS = {1: "embed", 2: "rmsnorm", 3: "gemm", 4: "rope", 5: "attention", 6: "combine", 7: "other",
+         8: "select", 9: "select_accum"}
 
 
 def launches(rec: np.ndarray) -> list[dict]:
