@@ -946,7 +946,7 @@ kvr_status kvr_repair(kvr_cache *c, const int32_t *new_tokens, int32_t edit_star
     r.pos = m->pos_d;
     r.tokens = c->tokens_d;
     r.single = c->view();
-  r.tm_kv = c->tm_kv_ok ? &c->tm_kv : nullptr;
+    r.tm_kv = c->tm_kv_ok ? &c->tm_kv : nullptr;
     r.max_pos = P[M - 1];
     st = plan_attention(m, r, P.data(), nullptr);
     if (!st) st = run_pass_graph(m, c, r);
@@ -1162,7 +1162,7 @@ kvr_status kvr_select(kvr_model *m, const kvr_cache *c, kvr_policy policy, int32
         r.pos = m->pos_d;
         r.tokens = toks;
         r.single = c->view();
-  r.tm_kv = c->tm_kv_ok ? &c->tm_kv : nullptr;
+        r.tm_kv = c->tm_kv_ok ? &c->tm_kv : nullptr;
         r.max_pos = s_end - 1;
         st = plan_attention(m, r, P.data(), nullptr);
         launch_rows_copy(r.single, dm.dtype, r.pos, edit_len, 0, dm.L, save, true, m->stream);
@@ -1202,7 +1202,7 @@ kvr_status kvr_select(kvr_model *m, const kvr_cache *c, kvr_policy policy, int32
       Rows r;
       r.tokens = toks;
       r.single = c->view();
-  r.tm_kv = c->tm_kv_ok ? &c->tm_kv : nullptr;
+      r.tm_kv = c->tm_kv_ok ? &c->tm_kv : nullptr;
       if (!st) st = stage_h2d(m, m->pos_d, P.data(), edit_len);
       if (!st) {
         // refresh the span's layer-0 K/V (saved and restored afterwards)

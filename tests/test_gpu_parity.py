@@ -245,6 +245,27 @@ def test_select_model_policies_parity(tiny, policy):
     assert np.array_equal(cache.tokens(), doc)
 
 
+@pytest.mark.parametrize("dtype", ["fp32", "bf16"])
+@pytest.mark.parametrize("n,s,L", [(300, 200, 35), (264, 196, 4), (201, 196, 4), (400, 10, 17)])
+def test_attention_selector_chunk_and_tile_edges(dtype, n, s, L):
+    # pools of 65, 64 (one full key chunk of the logits kernel), 1 and 373
+    # keys; spans whose 2L queries per kv group fill 3, 1, 1 and 2 query tiles
+    cfg = synth.preset("tiny", dtype=dtype)
+    W = synth.weights(cfg, 0)
+    doc = synth.document(7, n, cfg["vocab"], cfg["delim_id"])
+    new = synth.edit_tokens(8, doc[s:s + L], cfg["vocab"], cfg["delim_id"])
+    model = kv.Model(cfg, W, max_context=512, max_rows=256)
+    cache = model.prefill(doc)
+    K = min(8, n - s - L)
+    got = model.select(cache, "attention", K, s, new)
+    stale = oracle.prefill(cfg, W, doc)
+    sc, D = oracle.scores(cfg, W, stale, "attention", s, new)
+    ref = oracle.topk(sc, D, K)
+    band = (1e-4 if dtype == "fp32" else 2e-2) * np.abs(sc[D]).max()
+    check_selection(got, ref, sc, band)
+    model.close()
+
+
 # ------------------------------------------------------------------ batch
 
 def test_repair_batch_parity_fp32():
