@@ -233,6 +233,18 @@ __device__ __forceinline__ void lse_merge(float &m, float &z, float m2, float z2
   m = mm;
 }
 
+__device__ __forceinline__ uint32_t bf2_bits(__nv_bfloat162 v) { return *(const uint32_t *)&v; }
+
+// d[0..3] += A (16 x 16, row) . B (16 x 8, col), bf16 operands, fp32 accumulate
+__device__ __forceinline__ void sel_mma_bf16(float *d, uint32_t a0, uint32_t a1, uint32_t a2,
+                                             uint32_t a3, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+      "{%8,%9}, {%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
 template <typename T>
 __global__ void __launch_bounds__(SEL_THREADS)
     k_attn_select_logits(const float *q, int S, int H, int G, int dh, int layer, KVView v,
@@ -243,104 +255,201 @@ __global__ void __launch_bounds__(SEL_THREADS)
   const int hpg = H / G, Nq = S * hpg;
   const int t0 = chunk * SEL_KC, q0 = qt * SEL_QT;
   const int nk = min(SEL_KC, c - t0), nq = min(SEL_QT, Nq - q0);
-  // both operands transposed, d-major and in fp32: the thread of micro-tile
-  // (queries 4qg.., keys 4kg..) reads one float4 of each per d
-  extern __shared__ float4 sel_smem[];
-  float *qT = (float *)sel_smem;   // [dh][SEL_QT]
-  float *kT = qT + dh * SEL_QT;    // [dh][SEL_KC]
-  float *lt = kT;                  // [SEL_QT][SEL_LTS] logits, after the keys
   const int tid = threadIdx.x;
-  // the pool's stale keys: no kernel of the pass writes them, so they are
-  // read before the wait on the predecessor; a thread issues all its loads
-  // (page lookups, then rows) before it uses the first
-  constexpr int EPV = 16 / (int)sizeof(T);  // elements per 16-byte load
-  constexpr int KLD = SEL_KC * (SEL_DH_MAX / EPV) / SEL_THREADS;
-  const T *kc = (const T *)v.pages;
-  const int L = dh / EPV;
-  uint4 kx[KLD];
+  const size_t qg0 = (size_t)g * Nq + q0;
+  extern __shared__ float4 sel_smem[];
+  float *lt;  // [SEL_QT][SEL_LTS] logits, over the keys once they are consumed
+  int *last;  // arrival flag, over the queries once they are consumed
+  if constexpr (sizeof(T) == 2) {
+    // bf16 keys: tensor cores (mma.sync m16n8k16, fp32 accumulate).  Each
+    // query is split into two bf16 parts, q = q_hi + q_lo with q_lo the
+    // rounding remainder, and logit = q_hi . k + q_lo . k: about 16 bits of
+    // q's mantissa, the keys exact.  Rows are d-contiguous with a stride of
+    // dh + 8 elements (4 mod 32 words), so a fragment load's 8 rows x 4
+    // lanes fall on 32 banks.
+    const int RS = dh + 8;
+    __nv_bfloat16 *qh = (__nv_bfloat16 *)sel_smem;  // [SEL_QT][RS]
+    __nv_bfloat16 *qo = qh + SEL_QT * RS;           // [SEL_QT][RS] the remainders
+    __nv_bfloat16 *ks = qo + SEL_QT * RS;           // [SEL_KC][RS]
+    lt = (float *)ks;
+    last = (int *)qh;
+    // the pool's stale keys: no kernel of the pass writes them, so they are
+    // read before the wait on the predecessor; a thread issues all its loads
+    // (page lookups, then rows) before it uses the first
+    constexpr int KLD = SEL_KC * (SEL_DH_MAX / 8) / SEL_THREADS;
+    const __nv_bfloat16 *kc = (const __nv_bfloat16 *)v.pages;
+    const int L = dh / 8;  // 16-byte pieces per key row
+    uint4 kx[KLD];
 #pragma unroll
-  for (int u = 0; u < KLD; ++u) {
-    const int i = tid + u * SEL_THREADS, kk = i % SEL_KC, sub = i / SEL_KC;
-    kx[u] = make_uint4(0u, 0u, 0u, 0u);
-    if (kk < nk && sub < L)
-      kx[u] = *(const uint4 *)(kc + v.offset(layer, 0, g, s_end + t0 + kk) + sub * EPV);
-  }
+    for (int u = 0; u < KLD; ++u) {
+      const int i = tid + u * SEL_THREADS, kk = i / L, sub = i % L;
+      kx[u] = make_uint4(0u, 0u, 0u, 0u);
+      if (kk < nk) kx[u] = *(const uint4 *)(kc + v.offset(layer, 0, g, s_end + t0 + kk) + sub * 8);
+    }
 #pragma unroll
-  for (int u = 0; u < KLD; ++u) {
-    const int i = tid + u * SEL_THREADS, kk = i % SEL_KC, sub = i / SEL_KC;
-    if (sub < L) {
-      float f[EPV];
-      if constexpr (sizeof(T) == 2) {
-        const __nv_bfloat162 *b = (const __nv_bfloat162 *)&kx[u];
+    for (int u = 0; u < KLD; ++u) {
+      const int i = tid + u * SEL_THREADS, kk = i / L, sub = i % L;
+      if (kk < SEL_KC) *(uint4 *)(ks + kk * RS + sub * 8) = kx[u];  // rows of 16-byte multiples
+    }
+    pdl_wait();  // the queries come from the RoPE kernel just before
+    ts.waited();
+    constexpr int QLD = SEL_QT * (SEL_DH_MAX / 4) / SEL_THREADS;
+    const int D4 = dh / 4;
+    float4 qx[QLD];
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float2 x = __bfloat1622float2(b[e]);
-          f[2 * e] = x.x, f[2 * e + 1] = x.y;
-        }
-      } else {
-        const float *x = (const float *)&kx[u];
+    for (int u = 0; u < QLD; ++u) {
+      const int i = tid + u * SEL_THREADS, ql = i / D4, d4 = i % D4;
+      qx[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (ql < nq) {
+        const int qq = q0 + ql, r = qq / hpg, hh = g * hpg + qq % hpg;
+        qx[u] = *(const float4 *)(q + ((size_t)r * H + hh) * dh + 4 * d4);
+      }
+    }
 #pragma unroll
-        for (int e = 0; e < 4; ++e) f[e] = x[e];
+    for (int u = 0; u < QLD; ++u) {
+      const int i = tid + u * SEL_THREADS, ql = i / D4, d4 = i % D4;
+      if (ql < SEL_QT) {
+        const float2 x01 = make_float2(qx[u].x, qx[u].y), x23 = make_float2(qx[u].z, qx[u].w);
+        const __nv_bfloat162 h01 = __float22bfloat162_rn(x01), h23 = __float22bfloat162_rn(x23);
+        const float2 f01 = __bfloat1622float2(h01), f23 = __bfloat1622float2(h23);
+        const __nv_bfloat162 l01 = __floats2bfloat162_rn(x01.x - f01.x, x01.y - f01.y);
+        const __nv_bfloat162 l23 = __floats2bfloat162_rn(x23.x - f23.x, x23.y - f23.y);
+        *(uint2 *)(qh + ql * RS + 4 * d4) = make_uint2(bf2_bits(h01), bf2_bits(h23));
+        *(uint2 *)(qo + ql * RS + 4 * d4) = make_uint2(bf2_bits(l01), bf2_bits(l23));
+      }
+    }
+    __syncthreads();
+    if (tid == 0) trace_mark(0);  // keys and queries staged
+    // warp w: keys 16w .. 16w + 15 (two n-tiles of 8), all SEL_QT queries
+    // (two m-tiles of 16); lane: group gr = lane / 4, pair column gc
+    const int warp = tid >> 5, lane = tid & 31, gr = lane >> 2, gc = (lane & 3) * 2;
+    static_assert(SEL_QT == 32 && SEL_KC == 16 * (SEL_THREADS / 32), "warp tiling");
+    float acc[2][2][4];
+#pragma unroll
+    for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+      for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) acc[mt][nt][e] = 0.f;
+    for (int k0 = 0; k0 < dh; k0 += 16) {
+      uint32_t b[2][2];
+#pragma unroll
+      for (int nt = 0; nt < 2; ++nt) {
+        const __nv_bfloat16 *kr = ks + (16 * warp + 8 * nt + gr) * RS + k0 + gc;
+        b[nt][0] = *(const uint32_t *)kr;
+        b[nt][1] = *(const uint32_t *)(kr + 8);
       }
 #pragma unroll
-      for (int e = 0; e < EPV; ++e) kT[(sub * EPV + e) * SEL_KC + kk] = f[e];  // lanes: consecutive keys
+      for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+        for (int part = 0; part < 2; ++part) {
+          const __nv_bfloat16 *qr = (part ? qo : qh) + (16 * mt + gr) * RS + k0 + gc;
+          const uint32_t a0 = *(const uint32_t *)qr, a1 = *(const uint32_t *)(qr + 8 * RS);
+          const uint32_t a2 = *(const uint32_t *)(qr + 8), a3 = *(const uint32_t *)(qr + 8 * RS + 8);
+#pragma unroll
+          for (int nt = 0; nt < 2; ++nt) sel_mma_bf16(acc[mt][nt], a0, a1, a2, a3, b[nt][0], b[nt][1]);
+        }
     }
-  }
-  pdl_wait();  // the queries come from the RoPE kernel just before
-  ts.waited();
-  constexpr int QLD = SEL_QT * (SEL_DH_MAX / 4) / SEL_THREADS;
-  const int D4 = dh / 4;
-  float4 qx[QLD];
+    __syncthreads();  // keys consumed: lt reuses their space
+    if (tid == 0) trace_mark(1);  // logits computed
 #pragma unroll
-  for (int u = 0; u < QLD; ++u) {
-    const int i = tid + u * SEL_THREADS, ql = i % SEL_QT, d4 = i / SEL_QT;
-    qx[u] = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (ql < nq && d4 < D4) {
-      const int qq = q0 + ql, r = qq / hpg, hh = g * hpg + qq % hpg;
-      qx[u] = *(const float4 *)(q + ((size_t)r * H + hh) * dh + 4 * d4);
+    for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+      for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int ql = 16 * mt + gr + (e >> 1) * 8, kk = 16 * warp + 8 * nt + gc + (e & 1);
+          const float l = acc[mt][nt][e] * scale;
+          lt[ql * SEL_LTS + kk] = kk < nk ? l : -INFINITY;
+          if (kk < nk && ql < nq) ws.logit[(qg0 + ql) * c + t0 + kk] = l;
+        }
+  } else {
+    // fp32 keys: FFMA micro-tiles.  Both operands transposed, d-major: the
+    // thread of micro-tile (queries 4qg.., keys 4kg..) reads one float4 of
+    // each per d
+    float *qT = (float *)sel_smem;   // [dh][SEL_QT]
+    float *kT = qT + dh * SEL_QT;    // [dh][SEL_KC]
+    lt = kT;
+    last = (int *)qT;
+    // the pool's stale keys: no kernel of the pass writes them, so they are
+    // read before the wait on the predecessor; a thread issues all its loads
+    // (page lookups, then rows) before it uses the first
+    constexpr int EPV = 16 / (int)sizeof(T);  // elements per 16-byte load
+    constexpr int KLD = SEL_KC * (SEL_DH_MAX / EPV) / SEL_THREADS;
+    const T *kc = (const T *)v.pages;
+    const int L = dh / EPV;
+    uint4 kx[KLD];
+#pragma unroll
+    for (int u = 0; u < KLD; ++u) {
+      const int i = tid + u * SEL_THREADS, kk = i % SEL_KC, sub = i / SEL_KC;
+      kx[u] = make_uint4(0u, 0u, 0u, 0u);
+      if (kk < nk && sub < L)
+        kx[u] = *(const uint4 *)(kc + v.offset(layer, 0, g, s_end + t0 + kk) + sub * EPV);
     }
-  }
 #pragma unroll
-  for (int u = 0; u < QLD; ++u) {
-    const int i = tid + u * SEL_THREADS, ql = i % SEL_QT, d4 = i / SEL_QT;
-    if (d4 < D4) {
-      float *dst = qT + 4 * d4 * SEL_QT + ql;  // lanes: consecutive queries
-      dst[0] = qx[u].x;
-      dst[SEL_QT] = qx[u].y;
-      dst[2 * SEL_QT] = qx[u].z;
-      dst[3 * SEL_QT] = qx[u].w;
+    for (int u = 0; u < KLD; ++u) {
+      const int i = tid + u * SEL_THREADS, kk = i % SEL_KC, sub = i / SEL_KC;
+      if (sub < L) {
+        const float *f = (const float *)&kx[u];
+#pragma unroll
+        for (int e = 0; e < EPV; ++e) kT[(sub * EPV + e) * SEL_KC + kk] = f[e];  // lanes: consecutive keys
+      }
     }
-  }
-  __syncthreads();
-  if (tid == 0) trace_mark(0);  // keys and queries staged
-  const int kg = tid % SEL_KG, qg = tid / SEL_KG;
-  float acc[4][4];
+    pdl_wait();  // the queries come from the RoPE kernel just before
+    ts.waited();
+    constexpr int QLD = SEL_QT * (SEL_DH_MAX / 4) / SEL_THREADS;
+    const int D4 = dh / 4;
+    float4 qx[QLD];
 #pragma unroll
-  for (int i = 0; i < 4; ++i)
+    for (int u = 0; u < QLD; ++u) {
+      const int i = tid + u * SEL_THREADS, ql = i % SEL_QT, d4 = i / SEL_QT;
+      qx[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (ql < nq && d4 < D4) {
+        const int qq = q0 + ql, r = qq / hpg, hh = g * hpg + qq % hpg;
+        qx[u] = *(const float4 *)(q + ((size_t)r * H + hh) * dh + 4 * d4);
+      }
+    }
 #pragma unroll
-    for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
-#pragma unroll 4
-  for (int d = 0; d < dh; ++d) {
-    const float4 a = *(const float4 *)(qT + d * SEL_QT + 4 * qg);
-    const float4 b = *(const float4 *)(kT + d * SEL_KC + 4 * kg);
-    const float av[4] = {a.x, a.y, a.z, a.w}, bv[4] = {b.x, b.y, b.z, b.w};
+    for (int u = 0; u < QLD; ++u) {
+      const int i = tid + u * SEL_THREADS, ql = i % SEL_QT, d4 = i / SEL_QT;
+      if (d4 < D4) {
+        float *dst = qT + 4 * d4 * SEL_QT + ql;  // lanes: consecutive queries
+        dst[0] = qx[u].x;
+        dst[SEL_QT] = qx[u].y;
+        dst[2 * SEL_QT] = qx[u].z;
+        dst[3 * SEL_QT] = qx[u].w;
+      }
+    }
+    __syncthreads();
+    if (tid == 0) trace_mark(0);  // keys and queries staged
+    const int kg = tid % SEL_KG, qg = tid / SEL_KG;
+    float acc[4][4];
 #pragma unroll
     for (int i = 0; i < 4; ++i)
 #pragma unroll
-      for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
-  }
-  __syncthreads();  // keys consumed: lt reuses their space
-  if (tid == 0) trace_mark(1);  // logits computed
-  const size_t qg0 = (size_t)g * Nq + q0;
+      for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
+#pragma unroll 4
+    for (int d = 0; d < dh; ++d) {
+      const float4 a = *(const float4 *)(qT + d * SEL_QT + 4 * qg);
+      const float4 b = *(const float4 *)(kT + d * SEL_KC + 4 * kg);
+      const float av[4] = {a.x, a.y, a.z, a.w}, bv[4] = {b.x, b.y, b.z, b.w};
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int ql = 4 * qg + i;
+      for (int i = 0; i < 4; ++i)
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const int kk = 4 * kg + j;
-      const float l = acc[i][j] * scale;
-      lt[ql * SEL_LTS + kk] = kk < nk ? l : -INFINITY;
-      if (kk < nk && ql < nq) ws.logit[(qg0 + ql) * c + t0 + kk] = l;
+        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
+    }
+    __syncthreads();  // keys consumed: lt reuses their space
+    if (tid == 0) trace_mark(1);  // logits computed
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int ql = 4 * qg + i;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int kk = 4 * kg + j;
+        const float l = acc[i][j] * scale;
+        lt[ql * SEL_LTS + kk] = kk < nk ? l : -INFINITY;
+        if (kk < nk && ql < nq) ws.logit[(qg0 + ql) * c + t0 + kk] = l;
+      }
     }
   }
   __syncthreads();
@@ -364,7 +473,6 @@ __global__ void __launch_bounds__(SEL_THREADS)
   __threadfence();
   __syncthreads();
   if (tid == 0) trace_mark(2);  // chunk statistics stored
-  int *last = (int *)qT;  // the queries are consumed
   int *cnt = ws.cnt + (size_t)g * gridDim.z + qt;
   if (tid == 0) *last = atomicAdd(cnt, 1) == nch - 1;
   __syncthreads();
@@ -567,13 +675,15 @@ void launch_attn_select_scores(const float *q, int S, const Dims &dm, int layer,
   // arrival counts start at zero; each launch's last CTAs leave them at zero
   if (first_layer) cudaMemsetAsync(ws.cnt, 0, (size_t)dm.G * nqt * sizeof(int), s);
   const dim3 grid(sel_chunks(c), dm.G, nqt);
-  const size_t q_b = (size_t)SEL_QT * dm.dh * sizeof(float);
+  // bf16: q_hi, q_lo and keys as bf16 rows of dh + 8; fp32: q and keys as
+  // fp32 columns of dh.  The logits tile reuses the keys' space.
+  const bool bf16 = dm.dtype == KVR_DTYPE_BF16;
+  const size_t q_b = bf16 ? (size_t)2 * SEL_QT * (dm.dh + 8) * 2 : (size_t)SEL_QT * dm.dh * 4;
+  const size_t k_b = bf16 ? (size_t)SEL_KC * (dm.dh + 8) * 2 : (size_t)SEL_KC * dm.dh * 4;
   const size_t lt_b = (size_t)SEL_QT * SEL_LTS * sizeof(float);
-  const size_t k_b = (size_t)SEL_KC * dm.dh * sizeof(float);
-  const size_t smem = q_b + (k_b > lt_b ? k_b : lt_b);  // 48 KB at dh 128
-  auto kern = dm.dtype == KVR_DTYPE_BF16 ? k_attn_select_logits<__nv_bfloat16>
-                                         : k_attn_select_logits<float>;
-  // the trace build adds static shared memory: allow the sum above 48 KB
+  const size_t smem = q_b + (k_b > lt_b ? k_b : lt_b);  // 34 KB (bf16), 48 KB (fp32) at dh 128
+  auto kern = bf16 ? k_attn_select_logits<__nv_bfloat16> : k_attn_select_logits<float>;
+  // fp32 at dh 128, plus the trace build's static shared memory, passes 48 KB
   cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   launch_pdl(kern, grid, SEL_THREADS, smem, s, q, S, dm.H, dm.G, dm.dh, layer, v, s_end, c, scale,
              ws);
