@@ -177,8 +177,7 @@ def run_reference(args, cfg, rank):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": t * 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic", "impl": "reference",
-            "config": {"workload": f"{WORKLOAD}: n={N_CTX}, edit {EDIT_LEN}@{EDIT_START}, "
-                                   f"editlocal K={K_BUDGET}"},
+            "config": workload_config(cfg, args.gpus),
             "cpu_baseline": {"value": val, "unit": "positions/s", "cores": threads,
                              "kind": "oracle", "sample": sample},
             "e2e": {"value": val, "unit": "positions/s", "h2d_bytes_per_step": 0,
@@ -192,6 +191,15 @@ def run_reference(args, cfg, rank):
 # GEMM kernel's source is the one the capture was taken on.
 GU_TRAFFIC_BYTES = 235293696 + 4597760
 GU_TRAFFIC_SOURCE_SHA256 = "cf8edeeaa92c5a2694529c8c6cb3f63d064c0843eec4aaced7b1a114f5f711de"
+
+
+def workload_config(cfg: dict, world: int) -> dict:
+    """The `config` of both arms' JSON lines: one workload, named the same."""
+    return {"workload": f"{WORKLOAD}: Llama-3-8B shape, n={N_CTX}, "
+                        f"edit {EDIT_LEN}@{EDIT_START}, editlocal K={K_BUDGET}",
+            "rows": EDIT_LEN + K_BUDGET, "layers": cfg["n_layers"],
+            "parallelism": "replicas" if world > 1 else "single",
+            "l2": "inputs larger than L2 (14 GB of weights streamed per step)"}
 
 
 def max_over_ranks(x: float, device) -> float:
@@ -403,11 +411,7 @@ def main():
                "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
                "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
                "dtype": "bf16", "data": "synthetic (seeded random-init weights and tokens)",
-               "config": {"workload": f"{WORKLOAD}: Llama-3-8B shape, n={N_CTX}, "
-                                      f"edit {EDIT_LEN}@{EDIT_START}, editlocal K={K_BUDGET}",
-                          "rows": M, "layers": cfg["n_layers"],
-                          "parallelism": "replicas" if world > 1 else "single",
-                          "l2": "inputs larger than L2 (14 GB of weights streamed per step)"},
+               "config": workload_config(cfg, world),
                "repair_ms": ms, "repair_only_ms": repair_only_ms, "select_ms": sel_ms,
                "prefill_ms": prefill_ms, "speedup_vs_prefill": prefill_ms / ms,
                "prefill_roofline": {"bound": "tensor", "flops": prefill_flops(cfg, N_CTX),
