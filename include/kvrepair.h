@@ -135,7 +135,14 @@ void kvr_cache_free(kvr_cache *cache);
  * cache and leave it bit-identical.  positions_out: host int32[K], receives
  * *count_out ascending positions in [edit_end, n).  *count_out == K except
  * for STRUCTURAL when the pool holds fewer delimiters, and when the pool is
- * smaller than K.  Ties go to the lowest position.  Errors: KVR_E_RANGE. */
+ * smaller than K.  Ties go to the lowest position.  Device scratch (the
+ * edited tokens; for ATTENTION and CACHEBLEND the saved span rows and the
+ * ATTENTION logits) belongs to the model and only grows: a call that fits
+ * allocates nothing.  Errors: KVR_E_RANGE (K < 0, span outside the
+ * context, token id outside the vocabulary, empty span for ATTENTION or
+ * CACHEBLEND), KVR_E_INVAL (NULL argument, cache of another model, unknown
+ * policy), KVR_E_POISONED, KVR_E_UNSUPPORTED (span above max_rows,
+ * CACHEBLEND with fewer than 2 layers), KVR_E_NOMEM (scratch cannot grow). */
 kvr_status kvr_select(kvr_model *model, const kvr_cache *cache, kvr_policy policy, int32_t K,
                       int32_t edit_start, int32_t edit_len, const int32_t *new_tokens,
                       uint64_t seed, int32_t *positions_out, int32_t *count_out);
