@@ -128,14 +128,19 @@ def edit_inputs(cfg):
 
 # ------------------------------------------------------------- CPU oracle
 
-def oracle_sample(cfg, layers: int):
-    """Time the oracle's operator R for the 40 rows of the workload through
-    `layers` layers of the 8B shape (one layer's seeded weights reused for
-    every sampled layer; a seeded synthetic stale cache of the document's
-    length).  Returns (seconds per layer, threads)."""
+# CPU seconds the reference arm's W + K timed samples may take in all, and
+# the GPU arm's one-step oracle sample (cpu_baseline)
+REF_BUDGET_S = 150.0
+CPU_BASELINE_S = 15.0
+
+
+def oracle_setup(cfg, layers: int):
+    """Inputs of one oracle sample: the workload's 40 rows through `layers`
+    layers of the 8B shape (one layer's seeded weights reused for every
+    sampled layer) over a seeded synthetic stale cache of the document's
+    length."""
     import oracle
     from paper_2609_17983_gb300 import synth
-    threads = oracle.set_threads(os.cpu_count() or 1)
     doc, new = edit_inputs(cfg)
     edited = doc.copy()
     edited[EDIT_START:EDIT_START + EDIT_LEN] = new
@@ -153,44 +158,51 @@ def oracle_sample(cfg, layers: int):
     g = synth.tensor(3, 999, cache.k.shape, "fp32")
     cache.k[:] = g
     cache.v[:] = g[::-1]
+    return dict(cfg=ocfg, W=W, cache=cache, toks=toks, P=P, layers=layers)
+
+
+def oracle_time(sample) -> float:
+    """Seconds per layer of the oracle's operator R on one sample (R writes
+    the same rows each time, so a sample can be timed repeatedly)."""
+    import oracle
     t0 = time.perf_counter()
-    oracle.recompute(ocfg, W, cache, toks, P)
-    dt = time.perf_counter() - t0
-    return dt / layers, threads
+    oracle.recompute(sample["cfg"], sample["W"], sample["cache"], sample["toks"], sample["P"])
+    return (time.perf_counter() - t0) / sample["layers"]
 
 
 def run_reference(args, cfg, rank):
+    """The oracle timed on the host cores as the reference arm: W untimed and
+    K timed samples of the workload, each through the same number of layers,
+    chosen (at most --oracle-layers) so the W + K samples fit REF_BUDGET_S
+    by a one-layer probe; every sample is scaled to all layers."""
+    import oracle
     if rank != 0:
         return None
     M = EDIT_LEN + K_BUDGET
+    threads = oracle.set_threads(os.cpu_count() or 1)
+    probe = oracle_setup(cfg, 1)
+    t_layer = oracle_time(probe)
+    runs = args.warmup + args.steps
+    layers = max(1, min(args.oracle_layers, int(REF_BUDGET_S / (runs * t_layer))))
+    sample = probe if layers == 1 else oracle_setup(cfg, layers)
     times = []
-    threads = 1
-    for i in range(args.warmup + args.steps):
-        per_layer, threads = oracle_sample(cfg, args.oracle_layers)
+    for i in range(runs):
+        per_layer = oracle_time(sample)
         if i >= args.warmup:
             times.append(per_layer * cfg["n_layers"])
     t = statistics.median(times)
     val = M / t
-    sample = (f"oracle operator R on the {M} rows through {args.oracle_layers} of "
-              f"{cfg['n_layers']} layers per step, scaled to all layers")
+    desc = (f"oracle operator R on the {M} rows through {layers} of "
+            f"{cfg['n_layers']} layers per step, scaled to all layers")
     return {"metric": METRIC, "value": val, "unit": "positions/s", "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": t * 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic", "impl": "reference",
             "config": workload_config(cfg, args.gpus),
             "cpu_baseline": {"value": val, "unit": "positions/s", "cores": threads,
-                             "kind": "oracle", "sample": sample},
+                             "kind": "oracle", "sample": desc},
             "e2e": {"value": val, "unit": "positions/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
-
-
-# ------------------------------------------------------------- GPU arm
-
-# DRAM bytes (read + write) of one gate/up GEMM launch at this workload's shape
-# (40 x 28672 x 4096), from one ncu capture of that launch; reported only while the
-# GEMM kernel's source is the one the capture was taken on.
-GU_TRAFFIC_BYTES = 235293696 + 4597760
-GU_TRAFFIC_SOURCE_SHA256 = "cf8edeeaa92c5a2694529c8c6cb3f63d064c0843eec4aaced7b1a114f5f711de"
 
 
 def workload_config(cfg: dict, world: int) -> dict:
@@ -238,7 +250,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="kvrepair", choices=["kvrepair", "reference"])
     ap.add_argument("--prefill-steps", type=int, default=3)
-    ap.add_argument("--oracle-layers", type=int, default=4)
+    ap.add_argument("--oracle-layers", type=int, default=4,
+                    help="most layers per oracle sample of the reference arm")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--layers", type=int, default=None,
                     help="decoder layers (default: the model's 32); fewer only for profiling")
@@ -261,12 +274,19 @@ def main():
     # the CPU baseline runs before any GPU work (no forked workers after CUDA init)
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        per_layer, threads = oracle_sample(cfg, args.oracle_layers)
+        import oracle
+        threads = oracle.set_threads(os.cpu_count() or 1)
+        probe = oracle_setup(cfg, 1)
+        t_layer = oracle_time(probe)
+        # one step through as many layers as take about CPU_BASELINE_S
+        layers = max(1, min(cfg["n_layers"], round(CPU_BASELINE_S / t_layer)))
+        per_layer = oracle_time(oracle_setup(cfg, layers)) if layers > 1 else t_layer
         M = EDIT_LEN + K_BUDGET
         cpu = {"value": M / (per_layer * cfg["n_layers"]), "unit": "positions/s",
                "cores": threads, "kind": "oracle",
-               "sample": f"oracle operator R on the {M} rows through {args.oracle_layers} of "
-                         f"{cfg['n_layers']} layers (one step), scaled to all layers"}
+               "sample": f"oracle operator R on the {M} rows through {layers} of "
+                         f"{cfg['n_layers']} layers (one step, about {CPU_BASELINE_S:.0f} s), "
+                         f"scaled to all layers"}
 
     import torch
     local = int(os.environ.get("LOCAL_RANK", "0"))
