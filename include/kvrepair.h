@@ -283,16 +283,20 @@ kvr_status kvr_profile_read(kvr_model *model, int32_t cap, double *ms_out, int64
  * kvr_trace_enable with capacity > 0 returns KVR_E_UNSUPPORTED.  With
  * capacity > 0, a device buffer of `capacity` records is attached and every
  * CTA of the pass kernels (embedding, RMSNorm, GEMM, RoPE/scatter,
- * attention, combine) appends one record of 16 uint64 words:
+ * attention, combine) and of the Attention selector's two kernels appends
+ * one record of 16 uint64 words:
  *   [0] kind (1 embed, 2 rmsnorm, 3 GEMM, 4 RoPE/scatter, 5 attention,
- *       6 combine) | SM id << 8 | linear block index << 16,
+ *       6 combine, 8 selector logits, 9 selector accumulation) | SM id << 8
+ *       | linear block index << 16,
  *   [1] start, [2] return of the wait on the predecessor kernel, [3] end,
  *   [4..11] eight marks, 0 where the kernel sets none.  GEMM, for the CTA's
  *       last tile: first operand stage landed, all MMAs complete,
  *       accumulator taken by the epilogue, partial tile stored, split-tile
  *       arrival counted or partials staged across the cluster, tile reduced
  *       and written, epilogue done, all warps done.  Attention: last key
- *       chunk consumed.
+ *       chunk consumed.  Selector logits: keys and queries staged, logits
+ *       computed, chunk statistics stored, arrival counted, softmax
+ *       statistics folded (the group's last CTA only).
  *   [12..15] zero,
  * times in ns of the device's global timer.  Records past `capacity` are
  * dropped.  capacity == 0 detaches and frees the buffer.  The buffer is
