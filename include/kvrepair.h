@@ -7,7 +7,7 @@
  * its key/value states K(C) are cached.  An edit replaces the half-open span
  * S = [s_start, s_end) with the same number of new tokens, giving C'.  Repair
  * recomputes the positions P = S u A, A a subset of the pool D = [s_end, n),
- * from C' layer by layer against the otherwise-stale cache and writes the
+ * from C' one layer at a time against the otherwise-stale cache and writes the
  * refreshed K/V back in place (operator R, Eq. 1).  A is chosen by one of the
  * five selection policies of Table 1.
  *

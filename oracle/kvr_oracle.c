@@ -8,7 +8,7 @@
  * What it computes (paper: "Contiguity, Not Importance: Budgeted Repair of
  * Stale KV Caches After Document Edits", Sec. 3):
  *   - the repair operator R(K(C), C', P) of Sec. 3 "The repair interface":
- *     positions P are recomputed from the edited context C' layer by layer,
+ *     positions P are recomputed from the edited context C' one layer at a time,
  *     every other cache entry is left as it is;
  *   - full prefill K(C') as the special case P = {0..n-1} on an empty cache
  *     (the endpoint identity, Eq. 1);
@@ -339,8 +339,9 @@ int orc_recompute_token_major(const orc_config *c, const orc_weights *w, float *
   return rc;
 }
 
-/* Stale-query Attention selector score (Table 1, "top-K by stale-cache
- * attention from the query"), with the edit-span rows as the queries.
+/* Stale-query Attention selector score (Table 1: positions ranked by the
+ * attention a query pays them in the stale cache), with the edit-span rows as
+ * the queries.
  * The span rows [s_start, s_end) are run through every layer exactly as in
  * repair (their fresh k, v are written into kc/vc, which the caller passes
  * as a copy).  At layer l, for each span row and query head, logits to the
