@@ -1,11 +1,12 @@
 /*
- * kvrepair.h -- C ABI of libkvrepair: budgeted in-place repair of a stale KV
- * cache after a same-length document edit, on one GB300 GPU (sm_103a).
+ * kvrepair.h -- C ABI of libkvrepair: repairing a stale KV cache in place,
+ * within a budget of positions, after a same-length document edit, on one
+ * GB300 GPU (sm_103a).
  *
  * Method: "Contiguity, Not Importance: Budgeted Repair of Stale KV Caches
  * After Document Edits", Sec. 3.  A context C of n tokens is prefilled and
- * its key/value states K(C) are cached.  An edit replaces the half-open span
- * S = [s_start, s_end) with the same number of new tokens, giving C'.  Repair
+ * its key/value states K(C) are cached.  An edit replaces the tokens of
+ * S = [s_start, s_end) (end excluded) by as many new ones, giving C'.  Repair
  * recomputes the positions P = S u A, A a subset of the pool D = [s_end, n),
  * from C' one layer at a time against the otherwise-stale cache and writes the
  * refreshed K/V back in place (operator R, Eq. 1).  A is chosen by one of the
@@ -56,8 +57,8 @@ typedef enum { KVR_DTYPE_F32 = 0, KVR_DTYPE_BF16 = 1 } kvr_dtype;
 
 /* Selection policies of Table 1.  All pick from the pool D = [s_end, n). */
 typedef enum {
-  KVR_POLICY_EDITLOCAL = 0,  /* the K positions immediately after the span */
-  KVR_POLICY_STRUCTURAL = 1, /* delimiter tokens, nearest to the span first */
+  KVR_POLICY_EDITLOCAL = 0,  /* the first K pool positions, those next to the span */
+  KVR_POLICY_STRUCTURAL = 1, /* delimiter tokens of the pool, closest first */
   KVR_POLICY_ATTENTION = 2,  /* top-K stale-cache attention from the span queries */
   KVR_POLICY_CACHEBLEND = 3, /* top-K layer-1 (0-indexed) K/V deviation */
   KVR_POLICY_RANDOM = 4,     /* uniform K-subset, seeded */
@@ -200,8 +201,8 @@ kvr_status kvr_answer_logprob(kvr_model *model, const kvr_cache *cache, const in
                               int32_t m_prompt, const int32_t *answer, int32_t m_answer,
                               double *mean_logprob_out);
 
-/* Fresh-query logits (Sec. 3: the fresh query is never cached and is
- * recomputed for scoring).  The m query tokens (1 <= m <= 64) take positions
+/* Fresh-query logits (Sec. 3: the query that scores a cache state is
+ * computed anew each time and kept out of the cache).  The m query tokens (1 <= m <= 64) take positions
  * n..n+m-1 and attend to the cache; the document's K/V are not modified.
  * logits_out: host float[vocab], the logits of the last query row. */
 kvr_status kvr_logits(kvr_model *model, const kvr_cache *cache, const int32_t *query, int32_t m,

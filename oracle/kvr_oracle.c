@@ -14,7 +14,8 @@
  *     (the endpoint identity, Eq. 1);
  *   - the two selector forwards of Table 1 that need a model pass
  *     (stale-query Attention and CacheBlend-style KV deviation);
- *   - the fresh-query logits of Sec. 3 ("the fresh query is never cached").
+ *   - the fresh-query logits of Sec. 3 (a query computed anew, kept out of
+ *     the cache).
  * The model is a textbook Llama-style decoder (RMSNorm, rotate-half RoPE at
  * the original position ids, grouped-query causal attention, SwiGLU MLP),
  * which is what the paper's three model families are.
@@ -503,8 +504,8 @@ done:
   return rc;
 }
 
-/* Fresh-query logits (Sec. 3: the fresh query is never cached and is
- * recomputed for scoring).  The m query tokens sit at positions n..n+m-1;
+/* Fresh-query logits (Sec. 3: the query that scores a cache state is
+ * computed anew each time and kept out of the cache).  The m query tokens sit at positions n..n+m-1;
  * their k, v go into the caller's copy of the cache (cap >= n+m) and never
  * into the document's entries.  logits[vocab] = lm_head RMSNorm(h_last). */
 int orc_logits(const orc_config *c, const orc_weights *w, float *kc, float *vc, int cap, int n,
