@@ -205,6 +205,15 @@ def run_reference(args, cfg, rank):
                     "d2h_bytes_per_step": 0}}
 
 
+# ------------------------------------------------------------- GPU arm
+
+# DRAM bytes (read + write) of one gate/up GEMM launch at this workload's shape
+# (40 x 28672 x 4096), from one ncu capture of that launch; reported only while the
+# GEMM kernel's source is the one the capture was taken on.
+GU_TRAFFIC_BYTES = 235293696 + 4597760
+GU_TRAFFIC_SOURCE_SHA256 = "cf8edeeaa92c5a2694529c8c6cb3f63d064c0843eec4aaced7b1a114f5f711de"
+
+
 def workload_config(cfg: dict, world: int) -> dict:
     """The `config` of both arms' JSON lines: one workload, named the same."""
     return {"workload": f"{WORKLOAD}: Llama-3-8B shape, n={N_CTX}, "
