@@ -310,6 +310,14 @@ kvr_status kvr_profile_read(kvr_model *model, int32_t cap, double *ms_out, int64
 kvr_status kvr_trace_enable(kvr_model *model, int32_t capacity);
 kvr_status kvr_trace_read(kvr_model *model, uint64_t *out, int32_t cap, int32_t *n_out);
 
+/* Failure-detection probe (tests): enqueue on the model's stream one thread
+ * that waits for a device word nothing sets, bounded by limit_us (1 ..
+ * 1e6) like every device wait of the library.  When the bound runs out it
+ * sets the model's device flag; the next synchronising call (kvr_synchronize,
+ * kvr_select, the readbacks) returns KVR_E_DEVICE_TIMEOUT and clears the
+ * flag, and the model stays usable.  Errors: KVR_E_INVAL, KVR_E_RANGE. */
+kvr_status kvr_wait_probe(kvr_model *model, int32_t limit_us);
+
 /* Number of library kernels launched so far on this model. */
 int64_t kvr_launch_count(const kvr_model *model);
 

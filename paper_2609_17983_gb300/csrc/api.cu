@@ -469,6 +469,27 @@ bool valid_config(const kvr_model_config *c, std::string &why) {
   return true;
 }
 
+// Failure-detection probe: one thread waits for *word to turn nonzero, which
+// nothing makes it do.  The wait is bounded like every device wait of the
+// library, by %globaltimer (limit_ns) and, should the timer stall, by an
+// iteration cap; when it runs out the thread records `code` in the model's
+// device flag, as a timed-out wait in a pass kernel does, and returns.
+constexpr int WAIT_PROBE_CODE = 1 << 20;
+__global__ void k_wait_probe(const volatile int *word, unsigned long long limit_ns,
+                             unsigned int max_iters, int *dev_flag) {
+  unsigned long long t0;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t0));
+  for (unsigned int it = 0; *word == 0; ++it) {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    if (t - t0 >= limit_ns || it >= max_iters) {
+      atomicOr(dev_flag, WAIT_PROBE_CODE);
+      return;
+    }
+    __nanosleep(256);
+  }
+}
+
 }  // namespace
 
 // ======================================================================== ABI
@@ -818,6 +839,17 @@ kvr_status kvr_synchronize(kvr_model *m) {
   if (!m) return fail(KVR_E_INVAL, "NULL model");
   KVR_TRY(use_device(m));
   return sync_model(m);
+}
+
+kvr_status kvr_wait_probe(kvr_model *m, int32_t limit_us) {
+  if (!m) return fail(KVR_E_INVAL, "NULL model");
+  if (limit_us < 1 || limit_us > 1000000) return fail(KVR_E_RANGE, "limit_us outside [1, 1e6]");
+  KVR_TRY(use_device(m));
+  // word 16 of the zeroed 256-byte flag block: no kernel writes it
+  const unsigned long long limit_ns = (unsigned long long)limit_us * 1000ull;
+  const unsigned int max_iters = (unsigned int)(limit_ns / 64 + 4096);
+  k_wait_probe<<<1, 1, 0, m->stream>>>(m->dev_flag + 16, limit_ns, max_iters, m->dev_flag);
+  return launch_check(m, 1);
 }
 
 int64_t kvr_launch_count(const kvr_model *m) { return m ? m->launches : 0; }

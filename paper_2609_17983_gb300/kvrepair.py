@@ -92,6 +92,7 @@ _sigs = {
     "kvr_profile_reset": ([_P], _I32),
     "kvr_profile_read": ([_P, _I32, _P, _P, _P, _P, _I32, _P], _I32),
     "kvr_launch_count": ([_P], ctypes.c_int64),
+    "kvr_wait_probe": ([_P, _I32], _I32),
     "kvr_trace_enable": ([_P, _I32], _I32),
     "kvr_trace_read": ([_P, _P, _I32, _P], _I32),
     "kvr_linear": ([_P, ctypes.c_char_p, _I32, _P, _I32, _P], _I32),
@@ -389,6 +390,10 @@ class Model:
 
     def synchronize(self):
         kvr_synchronize(self.h)
+
+    def wait_probe(self, limit_us: int):
+        """Enqueue a device wait that runs out after limit_us (see kvr_wait_probe)."""
+        _check(_lib.kvr_wait_probe(self.h, int(limit_us)))
 
     def prefill(self, tokens) -> "Cache":
         return Cache(self, kvr_prefill(self.h, tokens))

@@ -318,6 +318,28 @@ def test_range_errors_leave_cache_unchanged(tiny):
     assert np.array_equal(cache.tokens(), doc)
 
 
+def test_device_wait_timeout_reported_and_model_usable():
+    # failure detection without a fault: a one-thread kernel waits 20 ms for a
+    # device word that nothing sets; its bounded wait runs out and sets the
+    # model's device flag, which the next synchronising call reports once and
+    # clears; the model then repairs as before
+    cfg, W, doc, s, new = tiny_setup("fp32")
+    model = kv.Model(cfg, W, max_context=1024, max_rows=512)
+    cache = model.prefill(doc)
+    model.synchronize()
+    model.wait_probe(20000)
+    with pytest.raises(kv.KvrError) as e:
+        model.synchronize()
+    assert e.value.code == 5  # KVR_E_DEVICE_TIMEOUT
+    model.synchronize()
+    A = model.select(cache, "editlocal", 32, s, new)
+    cache.repair(new, s, A)
+    ref = oracle.repair(cfg, W, oracle.prefill(cfg, W, doc), new, s, A)
+    cmp_rows(cache, ref, oracle.repaired_set(s, len(new), A), TOL["fp32"])
+    cache.close()
+    model.close()
+
+
 # ------------------------------------------------------- bf16 and 8B shapes
 
 def test_tiny_bf16_parity():
