@@ -203,11 +203,12 @@ __global__ void __launch_bounds__(TOPK_THREADS)
 // logit[qg * c + (j - s_end)], and per query the chunk's max and sum of
 // exp(logit - max); the last CTA of (group, query tile) to finish folds the
 // chunk statistics into the pool softmax's max and 1 / sum.  Arrival is an
-// atomic count with no waiting: every other CTA just exits.
+// atomic count with no waiting: every other CTA just exits.  The contraction
+// runs on mma.sync for bf16 caches and on FFMA micro-tiles for fp32 caches.
 constexpr int SEL_KC = 64, SEL_QT = 32, SEL_THREADS = 128;
-constexpr int SEL_KG = SEL_KC / 4;   // key groups of 4 (a thread: 4 queries x 4 keys)
+constexpr int SEL_KG = SEL_KC / 4;   // fp32 path: key groups of 4 (a thread: 4 queries x 4 keys)
 constexpr int SEL_LTS = SEL_KC + 4;  // logits tile row stride (floats)
-constexpr int SEL_DH_MAX = 128;
+constexpr int SEL_DH_MAX = 128;      // head_dim is 64 or 128 (checked at model creation)
 constexpr int SEL_FOLD = 16;         // chunk statistics in flight per thread in the fold
 static_assert(SEL_KG * (SEL_QT / 4) == SEL_THREADS, "one 4x4 micro-tile per thread");
 
