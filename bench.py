@@ -309,6 +309,8 @@ def main():
     # (the legacy default stream cannot be captured)
     stream = torch.cuda.Stream()
     torch.cuda.set_stream(stream)
+    # device memory from PyTorch's caching allocator, work on PyTorch's stream
+    kv.use_torch_allocator()
     model = kv.Model(cfg, None, seed=0, max_context=8192, max_rows=4096)
     model.set_stream(stream.cuda_stream)
     doc, new = edit_inputs(cfg)

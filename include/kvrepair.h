@@ -129,6 +129,21 @@ kvr_status kvr_synchronize(kvr_model *model);
 kvr_status kvr_prefill(kvr_model *model, const int32_t *tokens, int32_t n, kvr_cache **out);
 void kvr_cache_free(kvr_cache *cache);
 
+/* A cache restored from host memory instead of computed: the stored state
+ * K(C) of Sec. 3 for a context C of n tokens, e.g. one saved earlier with
+ * kvr_cache_read_raw over positions 0..n-1 and all layers.  tokens: host
+ * int32[n] (same rules as kvr_prefill); k, v: host arrays
+ * [n][n_layers][n_kv_heads][head_dim] in the cache's element type (bf16 bit
+ * patterns for a bf16 model, fp32 otherwise), only read during the call.
+ * The library does not check that the entries are the prefill of the tokens:
+ * repair and the selectors compute against whatever they hold, except that
+ * the CACHEBLEND policy takes the layer-0 entries of pool positions as the
+ * function of their token and position that every prefill leaves there.
+ * Synchronous.  Errors: KVR_E_INVAL (NULL argument), KVR_E_RANGE (n, token
+ * ids), KVR_E_NOMEM, KVR_E_CUDA. */
+kvr_status kvr_cache_load(kvr_model *model, const int32_t *tokens, int32_t n, const void *k,
+                          const void *v, kvr_cache **out);
+
 /* Select A (Table 1; Sec. 3 "Cost accounting": selector work is outside K).
  * The edit [edit_start, edit_start+edit_len) with host new_tokens[edit_len]
  * is applied to a private copy of the context, not to the cache; the
@@ -201,6 +216,15 @@ kvr_status kvr_answer_logprob(kvr_model *model, const kvr_cache *cache, const in
                               int32_t m_prompt, const int32_t *answer, int32_t m_answer,
                               double *mean_logprob_out);
 
+/* The margin m_x of Eq. 2 for one cache state: the length-averaged
+ * teacher-forced log-probability (kvr_answer_logprob) of the answer a_new
+ * minus that of a_old, both after the same prompt.  MR (Eq. 2) is
+ * (m_repaired - m_stale) / (m_oracle - m_stale) over three cache states.
+ * Errors as kvr_answer_logprob, and KVR_E_INVAL for a NULL margin_out. */
+kvr_status kvr_margin(kvr_model *model, const kvr_cache *cache, const int32_t *prompt,
+                      int32_t m_prompt, const int32_t *a_new, int32_t m_new,
+                      const int32_t *a_old, int32_t m_old, double *margin_out);
+
 /* Fresh-query logits (Sec. 3: the query that scores a cache state is
  * computed anew each time and kept out of the cache).  The m query tokens (1 <= m <= 64) take positions
  * n..n+m-1 and attend to the cache; the document's K/V are not modified.
@@ -258,11 +282,14 @@ kvr_status kvr_linear(kvr_model *model, const char *name, int32_t layer, const v
  * imply, hosts whose allocator belongs to another framework).  x: DEVICE
  * bf16 [M][K], y: DEVICE float [M][N], both owned by the caller; name
  * "wqkv", "wo", "wd" or "lm_head" of a bf16 model on the tensor-core GEMM;
- * 1 <= M <= 64, otherwise KVR_E_UNSUPPORTED.  The GEMM's scratch (partial
- * tiles, arrival counters) is a fixed ~10.5 MB device array that every GPU
- * loading the library holds until exit; the first call on a device looks up
- * its address (make that call before any stream capture).  All calls share
- * the array: calls whose GPU work overlaps race and give wrong results.
+ * 1 <= M <= 64, otherwise KVR_E_UNSUPPORTED; x or y not device memory of the
+ * model's device: KVR_E_INVAL (checked before any launch).  The GEMM's
+ * scratch (partial tiles, arrival counters) is a fixed ~10.5 MB device array
+ * that every GPU loading the library holds until exit; the first call on a
+ * device looks up its address (make that call before any stream capture) and
+ * keeps it for the process: after cudaDeviceReset or a release of the
+ * device's primary context, do not call it on that device again.  All calls
+ * share the array: calls whose GPU work overlaps race and give wrong results.
  * Asynchronous on the model's stream; kvr_synchronize reports device
  * timeouts.  Allocates nothing: no cudaMalloc, cudaFree or allocating
  * library call. */

@@ -873,15 +873,22 @@ void kvr_cache_free(kvr_cache *c) {
 
 int32_t kvr_cache_len(const kvr_cache *c) { return c ? c->n : -1; }
 
-kvr_status kvr_prefill(kvr_model *m, const int32_t *tokens, int32_t n, kvr_cache **out) {
-  if (!m || !tokens || !out) return fail(KVR_E_INVAL, "NULL argument");
-  *out = nullptr;
+// Argument checks shared by the calls that create a cache from host tokens.
+static kvr_status check_context(const kvr_model *m, const int32_t *tokens, int32_t n) {
   const Dims &dm = m->dims;
   if (n < 1 || n > dm.max_ctx) return fail(KVR_E_RANGE, "n=%d outside [1, %d]", n, dm.max_ctx);
   for (int i = 0; i < n; ++i)
     if (tokens[i] < 0 || tokens[i] >= dm.V)
       return fail(KVR_E_RANGE, "token %d at position %d outside [0, %d)", tokens[i], i, dm.V);
-  KVR_TRY(use_device(m));
+  return KVR_OK;
+}
+
+// A new cache of n positions holding `tokens`: zeroed pages (slots never
+// written hold finite values, so a masked key meets probability 0 and never
+// 0 * NaN), the identity block table, the device copy of the tokens and, for
+// bf16, the TMA view of the page pool.  Enqueued on the model's stream.
+static kvr_status new_cache(kvr_model *m, const int32_t *tokens, int32_t n, kvr_cache **out) {
+  const Dims &dm = m->dims;
   kvr_cache *c = new kvr_cache();
   c->model = m;
   m->caches.push_back(c);
@@ -897,8 +904,6 @@ kvr_status kvr_prefill(kvr_model *m, const int32_t *tokens, int32_t n, kvr_cache
     return fail(KVR_E_NOMEM, "cache of %d pages", c->n_pages);
   }
   c->tokens_h.assign(tokens, tokens + n);
-  // zeroed pages: slots never written hold finite values (masked keys meet
-  // probability 0, and 0 * NaN would not vanish)
   if (cudaMemsetAsync(c->pages, 0, (size_t)c->n_pages * page_bytes, m->stream)) {
     kvr_cache_free(c);
     return fail(KVR_E_CUDA, "cache clear");
@@ -911,6 +916,62 @@ kvr_status kvr_prefill(kvr_model *m, const int32_t *tokens, int32_t n, kvr_cache
   for (int i = 0; i < c->n_pages; ++i) tab[i] = i;
   kvr_status st = stage_h2d(m, c->table, tab.data(), tab.size());
   if (!st) st = stage_h2d(m, c->tokens_d, tokens, n);
+  if (st) {
+    cudaStreamSynchronize(m->stream);
+    kvr_cache_free(c);
+    return st;
+  }
+  *out = c;
+  return KVR_OK;
+}
+
+kvr_status kvr_cache_load(kvr_model *m, const int32_t *tokens, int32_t n, const void *k,
+                          const void *v, kvr_cache **out) {
+  if (!m || !tokens || !k || !v || !out) return fail(KVR_E_INVAL, "NULL argument");
+  *out = nullptr;
+  KVR_TRY(check_context(m, tokens, n));
+  KVR_TRY(use_device(m));
+  const Dims &dm = m->dims;
+  kvr_cache *c = nullptr;
+  KVR_TRY(new_cache(m, tokens, n, &c));
+  // positions in chunks of about 32 MB of K (and as much V) through the
+  // model's readback scratch; host rows [n][L][G][dh] are contiguous per chunk
+  const size_t row_b = (size_t)dm.L * dm.G * dm.dh * dm.es();
+  const int chunk = (int)std::max<size_t>(1, std::min<size_t>(n, ((size_t)32 << 20) / row_b));
+  auto al = [](size_t x) { return (x + 255) / 256 * 256; };
+  kvr_status st = grow_scratch(m, m->read_scratch, m->read_scratch_bytes,
+                               2 * al((size_t)chunk * row_b), "cache load scratch");
+  char *kd = (char *)m->read_scratch, *vd = kd + al((size_t)chunk * row_b);
+  for (int p0 = 0; !st && p0 < n; p0 += chunk) {
+    const int cnt = std::min(chunk, n - p0);
+    const size_t b = (size_t)cnt * row_b, off = (size_t)p0 * row_b;
+    if (cudaMemcpyAsync(kd, (const char *)k + off, b, cudaMemcpyHostToDevice, m->stream) ||
+        cudaMemcpyAsync(vd, (const char *)v + off, b, cudaMemcpyHostToDevice, m->stream)) {
+      st = fail(KVR_E_CUDA, "cache load upload");
+      break;
+    }
+    launch_cache_scatter_raw(c->view(), dm.dtype, p0, cnt, kd, vd, m->stream);
+    st = launch_check(m, 1);
+  }
+  if (!st) st = sync_model(m);
+  if (st) {
+    cudaStreamSynchronize(m->stream);
+    kvr_cache_free(c);
+    return st;
+  }
+  *out = c;
+  return KVR_OK;
+}
+
+kvr_status kvr_prefill(kvr_model *m, const int32_t *tokens, int32_t n, kvr_cache **out) {
+  if (!m || !tokens || !out) return fail(KVR_E_INVAL, "NULL argument");
+  *out = nullptr;
+  const Dims &dm = m->dims;
+  KVR_TRY(check_context(m, tokens, n));
+  KVR_TRY(use_device(m));
+  kvr_cache *c = nullptr;
+  KVR_TRY(new_cache(m, tokens, n, &c));
+  kvr_status st = KVR_OK;
   Rows r;
   r.tokens = c->tokens_d;
   r.single = c->view();
@@ -962,14 +1023,17 @@ kvr_status kvr_repair(kvr_cache *c, const int32_t *new_tokens, int32_t edit_star
   if (M > dm.max_rows) return fail(KVR_E_UNSUPPORTED, "|P|=%d above max_rows", M);
   KVR_TRY(use_device(m));
   if (M == 0) return KVR_OK;
-  // a1: apply the edit
-  std::vector<int32_t> P(M);
+  // a1: apply the edit (the old tokens are kept to undo it should the pass
+  // fail before any device work touched the cache)
+  std::vector<int32_t> P(M), old(c->tokens_h.begin() + edit_start,
+                                 c->tokens_h.begin() + edit_start + edit_len);
   for (int i = 0; i < edit_len; ++i) {
     c->tokens_h[edit_start + i] = new_tokens[i];
     P[i] = edit_start + i;
   }
   for (int i = 0; i < n_positions; ++i) P[edit_len + i] = positions[i];
   kvr_status st = KVR_OK;
+  bool launched = false;
   if (edit_len) st = stage_h2d(m, c->tokens_d + edit_start, new_tokens, edit_len);
   if (!st) st = stage_h2d(m, m->pos_d, P.data(), M);
   if (!st) {
@@ -981,9 +1045,17 @@ kvr_status kvr_repair(kvr_cache *c, const int32_t *new_tokens, int32_t edit_star
     r.tm_kv = c->tm_kv_ok ? &c->tm_kv : nullptr;
     r.max_pos = P[M - 1];
     st = plan_attention(m, r, P.data(), nullptr);
-    if (!st) st = run_pass_graph(m, c, r);
+    if (!st) {
+      launched = true;
+      st = run_pass_graph(m, c, r);
+    }
   }
-  if (st == KVR_E_CUDA) c->poisoned = true;
+  if (st && st != KVR_E_CUDA && !launched && edit_len) {
+    // refused before the pass: put the old tokens back, host and device
+    std::copy(old.begin(), old.end(), c->tokens_h.begin() + edit_start);
+    if (stage_h2d(m, c->tokens_d + edit_start, old.data(), edit_len)) c->poisoned = true;
+  }
+  if (st == KVR_E_CUDA || (st && launched)) c->poisoned = true;
   return st;
 }
 
@@ -1383,6 +1455,17 @@ kvr_status kvr_answer_logprob(kvr_model *m, const kvr_cache *c, const int32_t *p
   double acc = 0.0;
   for (int i = 0; i < ma; ++i) acc += h[i];
   *out = acc / ma;
+  return KVR_OK;
+}
+
+kvr_status kvr_margin(kvr_model *m, const kvr_cache *c, const int32_t *prompt, int32_t mp,
+                      const int32_t *a_new, int32_t m_new, const int32_t *a_old, int32_t m_old,
+                      double *margin_out) {
+  if (!margin_out) return fail(KVR_E_INVAL, "NULL argument");
+  double lp_new = 0.0, lp_old = 0.0;
+  KVR_TRY(kvr_answer_logprob(m, c, prompt, mp, a_new, m_new, &lp_new));
+  KVR_TRY(kvr_answer_logprob(m, c, prompt, mp, a_old, m_old, &lp_old));
+  *margin_out = lp_new - lp_old;
   return KVR_OK;
 }
 

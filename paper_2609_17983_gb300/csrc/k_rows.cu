@@ -286,6 +286,26 @@ __global__ void k_cache_gather_raw(KVView v, const int32_t *pos, int n_pos, int 
   }
 }
 
+// The inverse of k_cache_gather_raw for consecutive positions p0 .. p0+n_pos-1
+// and every layer: rows [n_pos][L][G][dh] of k_in / v_in written into the pages.
+template <typename T>
+__global__ void k_cache_scatter_raw(KVView v, int p0, int n_pos, const T *k_in, const T *v_in) {
+  const int L = v.L, G = v.G, dh = v.dh;
+  size_t total = (size_t)n_pos * L * G * dh;
+  T *c = (T *)v.pages;
+  for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < total;
+       e += (size_t)gridDim.x * blockDim.x) {
+    int i = (int)(e % dh);
+    size_t r = e / dh;
+    int g = (int)(r % G);
+    r /= G;
+    int l = (int)(r % L);
+    int p = p0 + (int)(r / L);
+    c[v.offset(l, 0, g, p) + i] = k_in[e];
+    c[v.offset(l, 1, g, p) + i] = v_in[e];
+  }
+}
+
 // buf layout [n_pos][nl][2][G][dh] in the cache dtype
 template <typename T>
 __global__ void k_rows_copy(KVView v, const int32_t *pos, int n_pos, int l0, int nl, T *buf,
@@ -473,6 +493,18 @@ void launch_cache_gather_raw(KVView v, int dtype, const int32_t *pos, int n_pos,
   else
     k_cache_gather_raw<float><<<grid_for(n, 256), 256, 0, s>>>(v, pos, n_pos, l0, l1 - l0, G, dh,
                                                                 (float *)k_out, (float *)v_out);
+}
+
+void launch_cache_scatter_raw(KVView v, int dtype, int p0, int n_pos, const void *k_in,
+                              const void *v_in, cudaStream_t s) {
+  size_t n = (size_t)n_pos * v.L * v.G * v.dh;
+  if (n == 0) return;
+  if (dtype == KVR_DTYPE_BF16)
+    k_cache_scatter_raw<__nv_bfloat16><<<grid_for(n, 256), 256, 0, s>>>(
+        v, p0, n_pos, (const __nv_bfloat16 *)k_in, (const __nv_bfloat16 *)v_in);
+  else
+    k_cache_scatter_raw<float><<<grid_for(n, 256), 256, 0, s>>>(v, p0, n_pos, (const float *)k_in,
+                                                                 (const float *)v_in);
 }
 
 void launch_transplant(KVView dst, KVView src, int dtype, const int32_t *pos, int n_pos,

@@ -454,6 +454,9 @@ void launch_cache_gather(KVView v, int dtype, const int32_t *pos, int n_pos, int
 // The same gather in the cache's element type (no widening).
 void launch_cache_gather_raw(KVView v, int dtype, const int32_t *pos, int n_pos, int l0, int l1,
                              int G, int dh, void *k_out, void *v_out, cudaStream_t s);
+// Rows [n_pos][L][G][dh] (cache dtype) of consecutive positions p0.. into the pages.
+void launch_cache_scatter_raw(KVView v, int dtype, int p0, int n_pos, const void *k_in,
+                              const void *v_in, cudaStream_t s);
 void launch_rows_copy(KVView v, int dtype, const int32_t *pos, int n_pos, int l0, int l1,
                       void *buf, bool to_buf, cudaStream_t s);
 void launch_transplant(KVView dst, KVView src, int dtype, const int32_t *pos, int n_pos,

@@ -16,6 +16,15 @@
 // array is ~10.5 MB of device memory that every GPU which loads the library
 // keeps until the process exits.
 //
+// Pointers: x and y must be device (or managed) memory of the model's device;
+// anything else is refused before the launch (a host address would reach the
+// TMA descriptor and the epilogue stores).
+//
+// Lifetime: the array's device address is looked up once per device and kept
+// until the process exits.  After cudaDeviceReset, or a release of the
+// device's primary context, that address is stale: do not call this entry
+// point on that device again in the same process.
+//
 // Sharing: every call uses the same array and leaves its contents behind.
 // The arrival counters are cleared at the start of each call (stream-ordered
 // memset, no allocation).  Calls whose GPU work overlaps in time (different
@@ -64,6 +73,18 @@ kvr_status scratch_address(int device, void **out) {
   return KVR_OK;
 }
 
+// True if p is device or managed memory that `device` can use as such (the
+// attribute query allocates nothing).
+bool on_device(const void *p, int device) {
+  cudaPointerAttributes a{};
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  if (a.type == cudaMemoryTypeManaged) return true;
+  return a.type == cudaMemoryTypeDevice && a.device == device;
+}
+
 }  // namespace
 
 using namespace kvr;
@@ -105,6 +126,9 @@ extern "C" kvr_status kvr_linear_noalloc(kvr_model *m, const char *name, int32_t
     return na_fail(KVR_E_UNSUPPORTED, "kvr_linear_noalloc: more output tiles than counters");
   if (cudaSetDevice(m->device) != cudaSuccess)
     return na_fail(KVR_E_CUDA, "kvr_linear_noalloc: cudaSetDevice");
+  if (!on_device(x, m->device) || !on_device(y, m->device))
+    return na_fail(KVR_E_INVAL, "kvr_linear_noalloc: x and y must be device memory of the "
+                                "model's device");
   void *scratch = nullptr;
   kvr_status st = scratch_address(m->device, &scratch);
   if (st) return st;

@@ -79,6 +79,7 @@ _sigs = {
     "kvr_synchronize": ([_P], _I32),
     "kvr_prefill": ([_P, _P, _I32, ctypes.POINTER(_P)], _I32),
     "kvr_cache_free": ([_P], None),
+    "kvr_cache_load": ([_P, _P, _I32, _P, _P, ctypes.POINTER(_P)], _I32),
     "kvr_select": ([_P, _P, _I32, _I32, _I32, _I32, _P, ctypes.c_uint64, _P, _P], _I32),
     "kvr_repair": ([_P, _P, _I32, _I32, _P, _I32], _I32),
     "kvr_repair_batch": ([_P, _P, _I32], _I32),
@@ -99,6 +100,7 @@ _sigs = {
     "kvr_linear_noalloc": ([_P, ctypes.c_char_p, _I32, _P, _I32, _P], _I32),
     "kvr_transplant": ([_P, _P, _P, _I32], _I32),
     "kvr_answer_logprob": ([_P, _P, _P, _I32, _P, _I32, _P], _I32),
+    "kvr_margin": ([_P, _P, _P, _I32, _P, _I32, _P, _I32, _P], _I32),
 }
 for _name, (_args, _res) in _sigs.items():
     _f = getattr(_lib, _name)
@@ -189,6 +191,21 @@ def kvr_cache_free(cache):
     _lib.kvr_cache_free(cache)
 
 
+def kvr_cache_load(model, tokens, k, v, dtype) -> ctypes.c_void_p:
+    """k, v: [n][n_layers][n_kv_heads][head_dim] in the cache's element type
+    (uint16 bf16 bit patterns, or float32)."""
+    t = _i32(tokens)
+    k = np.ascontiguousarray(k)
+    v = np.ascontiguousarray(v)
+    for a in (k, v):
+        if a.dtype != np.dtype(dtype) or a.shape[:1] != (t.size,):
+            raise ValueError(f"cache rows must be {np.dtype(dtype)} [{t.size}, L, G, dh]")
+    out = ctypes.c_void_p()
+    _check(_lib.kvr_cache_load(model, _ptr(t), t.size, k.ctypes.data, v.ctypes.data,
+                               ctypes.byref(out)))
+    return out
+
+
 def kvr_select(model, cache, policy: str, K: int, edit_start: int, new_tokens,
                seed: int = 0) -> np.ndarray:
     nt = _i32(new_tokens)
@@ -235,6 +252,14 @@ def kvr_answer_logprob(model, cache, prompt, answer) -> float:
     out = ctypes.c_double(0.0)
     _check(_lib.kvr_answer_logprob(model, cache, _ptr(pr), pr.size, _ptr(an), an.size,
                                    ctypes.byref(out)))
+    return out.value
+
+
+def kvr_margin(model, cache, prompt, a_new, a_old) -> float:
+    pr, an, ao = _i32(prompt), _i32(a_new), _i32(a_old)
+    out = ctypes.c_double(0.0)
+    _check(_lib.kvr_margin(model, cache, _ptr(pr), pr.size, _ptr(an), an.size, _ptr(ao),
+                           ao.size, ctypes.byref(out)))
     return out.value
 
 
@@ -398,6 +423,11 @@ class Model:
     def prefill(self, tokens) -> "Cache":
         return Cache(self, kvr_prefill(self.h, tokens))
 
+    def load_cache(self, tokens, k, v) -> "Cache":
+        """A cache holding the given K/V rows ([n][L][G][dh], cache dtype)."""
+        dt = np.uint16 if self.cfg["dtype"] == "bf16" else np.float32
+        return Cache(self, kvr_cache_load(self.h, tokens, k, v, dt))
+
     def select(self, cache: "Cache", policy: str, K: int, edit_start: int, new_tokens,
                seed: int = 0) -> np.ndarray:
         return kvr_select(self.h, cache.h, policy, K, edit_start, new_tokens, seed)
@@ -409,9 +439,8 @@ class Model:
         return kvr_answer_logprob(self.h, cache.h, prompt, answer)
 
     def margin(self, cache: "Cache", prompt, a_new, a_old) -> float:
-        """m_x of Eq. 2 for this cache state."""
-        return (self.answer_logprob(cache, prompt, a_new)
-                - self.answer_logprob(cache, prompt, a_old))
+        """m_x of Eq. 2 for this cache state (kvr_margin)."""
+        return kvr_margin(self.h, cache.h, prompt, a_new, a_old)
 
     def repair_batch(self, reqs):
         kvr_repair_batch(self.h, [(c.h, e, p) for c, e, p in reqs])

@@ -215,6 +215,28 @@ def weights(cfg: dict, model_seed: int = 0, n_layers: int | None = None,
         layers=[layer_weights(cfg, model_seed, l) for l in range(L)])
 
 
+# ------------------------------------------------------- stale KV caches
+
+# Spread of the synthetic cache entries: a K or V entry of these models is a
+# projection of an RMS-normalised row (unit RMS) by N(0, 0.02^2) weights over
+# d_model = 4096 inputs, whose standard deviation is 0.02 * sqrt(4096) = 1.28.
+KV_STD = 1.28
+TID_CACHE_K, TID_CACHE_V = 1001, 1002
+
+
+def kv_rows(seed: int, n: int, n_layers: int, n_kv_heads: int, head_dim: int, dtype: str,
+            std: float = KV_STD) -> tuple[np.ndarray, np.ndarray]:
+    """A seeded synthetic stale cache: K and V rows [n][n_layers][n_kv_heads][head_dim]
+    with entries approximately N(0, std^2), from the weight generator's counter-based
+    streams (tensor ids TID_CACHE_K / TID_CACHE_V of `seed`); bf16 bit patterns for
+    bf16, else float32.  Used where a test or a timing needs a cached state K(C)
+    of a long context that no CPU prefill could produce: repair is defined over
+    any stale cache."""
+    shape = (n, n_layers, n_kv_heads, head_dim)
+    return (tensor(seed, TID_CACHE_K, shape, dtype, std),
+            tensor(seed, TID_CACHE_V, shape, dtype, std))
+
+
 # --------------------------------------------------------- documents, edits
 
 def _uniform_ints(seed: int, count: int, lo: int, hi: int) -> np.ndarray:

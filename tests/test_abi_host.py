@@ -58,6 +58,8 @@ def test_null_handles_rejected(kv):
     assert lib.kvr_select(None, None, 0, 1, 0, 0, None, 0, None, None) == 1
     assert lib.kvr_logits(None, None, None, 1, None) == 1
     assert lib.kvr_wait_probe(None, 1000) == 1
+    assert lib.kvr_cache_load(None, None, 0, None, None, None) == 1
+    assert lib.kvr_margin(None, None, None, 1, None, 1, None, 1, None) == 1
     assert lib.kvr_synchronize(None) == 1
     assert b"NULL" in lib.kvr_last_error()
     assert lib.kvr_cache_len(None) == -1

@@ -185,6 +185,66 @@ def test_cache_read_raw_is_the_stored_rows(dtype):
     model.close()
 
 
+@pytest.mark.parametrize("dtype", ["fp32", "bf16"])
+def test_cache_load_round_trip(dtype):
+    # a cache saved with kvr_cache_read_raw and restored with kvr_cache_load
+    # holds the same entries and tokens, and repairs bit for bit as the
+    # original does (the same pass over the same state)
+    cfg, W, doc, s, new = tiny_setup(dtype)
+    model = kv.Model(cfg, W, max_context=1024, max_rows=512)
+    orig = model.prefill(doc)
+    rows = np.arange(len(doc))
+    k, v = orig.read_raw(rows)
+    restored = model.load_cache(doc, k, v)
+    k2, v2 = restored.read_raw(rows)
+    assert np.array_equal(k, k2) and np.array_equal(v, v2)
+    assert np.array_equal(restored.tokens(), doc)
+    A = np.arange(s + 4, s + 36)
+    orig.repair(new, s, A)
+    restored.repair(new, s, A)
+    k1, v1 = orig.read_raw(rows)
+    k2, v2 = restored.read_raw(rows)
+    assert np.array_equal(k1, k2) and np.array_equal(v1, v2)
+    bad = doc.copy()
+    bad[7] = cfg["vocab"]
+    with pytest.raises(kv.KvrError) as e:
+        model.load_cache(bad, k, v)
+    assert e.value.code == 2
+    model.close()
+
+
+def test_model_on_torch_caching_allocator():
+    # device memory from PyTorch's caching allocator (kvr_set_allocator through
+    # use_torch_allocator): the model's and cache's allocations appear in
+    # torch.cuda.memory_allocated, the repair matches the oracle as it does
+    # with cudaMalloc, and freeing the model returns every byte
+    import torch
+    cfg, W, doc, s, new = tiny_setup("bf16", qkv_bias=True)
+    weight_bytes = sum(a.nbytes for a in (W["embed"], W["lm_head"], W["final_norm"]))
+    weight_bytes += sum(a.nbytes for ly in W["layers"] for a in ly.values())
+    torch.cuda.synchronize()
+    before = torch.cuda.memory_allocated()
+    kv.use_torch_allocator()
+    model = None
+    try:
+        model = kv.Model(cfg, W, max_context=1024, max_rows=512)
+        assert torch.cuda.memory_allocated() - before >= weight_bytes
+        with_model = torch.cuda.memory_allocated()
+        cache = model.prefill(doc)
+        assert torch.cuda.memory_allocated() > with_model  # the cache's pages
+        A = np.arange(s + 4, s + 36)
+        cache.repair(new, s, A)
+        ref = oracle.repair(cfg, W, oracle.prefill(cfg, W, doc), new, s, A)
+        cmp_rows(cache, ref, oracle.repaired_set(s, 4, A), TOL["bf16"])
+        cache.close()
+    finally:
+        if model is not None:
+            model.close()
+        kv.use_cuda_allocator()
+    torch.cuda.synchronize()
+    assert torch.cuda.memory_allocated() == before
+
+
 def test_logits_parity_fp32(tiny):
     cfg, W, doc, model = tiny["cfg"], tiny["W"], tiny["doc"], tiny["model"]
     cache = model.prefill(doc)
