@@ -128,17 +128,20 @@ def edit_inputs(cfg):
 
 # ------------------------------------------------------------- CPU oracle
 
-# CPU seconds the reference arm's W + K timed samples may take in all, and
-# the GPU arm's one-step oracle sample (cpu_baseline)
+# CPU seconds the reference arm's W + K timed steps may take in all, and the
+# GPU arm's one-step oracle sample (cpu_baseline)
 REF_BUDGET_S = 150.0
-CPU_BASELINE_S = 15.0
+CPU_BASELINE_S = 10.0
+# seed of the synthetic stale cache (the one the full-depth parity test starts from)
+STALE_SEED = 11
 
 
 def oracle_setup(cfg, layers: int):
-    """Inputs of one oracle sample: the workload's 40 rows through `layers`
-    layers of the 8B shape (one layer's seeded weights reused for every
-    sampled layer) over a seeded synthetic stale cache of the document's
-    length."""
+    """Inputs of the oracle's timed step: the workload's 40 rows (the span and
+    its EditLocal window) of the edited document through the model's first
+    `layers` decoder layers, each with its own seeded weights, over the seeded
+    synthetic stale cache of the document's length restricted to those
+    layers."""
     import oracle
     from paper_2609_17983_gb300 import synth
     doc, new = edit_inputs(cfg)
@@ -147,55 +150,66 @@ def oracle_setup(cfg, layers: int):
     P = np.arange(EDIT_START, EDIT_START + EDIT_LEN + K_BUDGET)
     used = np.unique(edited[P])
     remap = {int(t): i for i, t in enumerate(used)}
-    ly = synth.layer_weights(cfg, 0, 0)
     W = dict(embed=synth.rows(0, synth.TID_EMBED, used, cfg["d_model"], cfg["dtype"]),
              final_norm=synth.ones(cfg["d_model"], cfg["dtype"]), lm_head=None,
-             layers=[ly] * layers)
+             layers=[synth.layer_weights(cfg, 0, l) for l in range(layers)])
     ocfg = dict(cfg, n_layers=layers, vocab=len(used))
     toks = np.zeros(N_CTX, np.int32)
     toks[P] = [remap[int(t)] for t in edited[P]]
-    cache = oracle.empty_cache(ocfg, N_CTX)
-    g = synth.tensor(3, 999, cache.k.shape, "fp32")
-    cache.k[:] = g
-    cache.v[:] = g[::-1]
+    k, v = synth.kv_rows(STALE_SEED, N_CTX, cfg["n_layers"], cfg["n_kv_heads"],
+                         cfg["head_dim"], cfg["dtype"])
+    f32 = synth.bf16_bits_to_f32 if cfg["dtype"] == "bf16" else np.asarray
+    cache = oracle.Cache(np.ascontiguousarray(f32(k[:, :layers]).transpose(1, 0, 2, 3)),
+                         np.ascontiguousarray(f32(v[:, :layers]).transpose(1, 0, 2, 3)), toks)
     return dict(cfg=ocfg, W=W, cache=cache, toks=toks, P=P, layers=layers)
 
 
 def oracle_time(sample) -> float:
-    """Seconds per layer of the oracle's operator R on one sample (R writes
-    the same rows each time, so a sample can be timed repeatedly)."""
+    """Seconds of one oracle step: operator R on the sample's rows through its
+    layers (R writes the same rows each time, so a sample can be rerun)."""
     import oracle
     t0 = time.perf_counter()
     oracle.recompute(sample["cfg"], sample["W"], sample["cache"], sample["toks"], sample["P"])
-    return (time.perf_counter() - t0) / sample["layers"]
+    return time.perf_counter() - t0
+
+
+def oracle_value(cfg, layers: int, seconds: float) -> float:
+    """positions/s of an oracle step that took `seconds` for the 40 rows through
+    `layers` of the model's layers (a position is repaired by all of them)."""
+    return (EDIT_LEN + K_BUDGET) * layers / cfg["n_layers"] / seconds
 
 
 def run_reference(args, cfg, rank):
-    """The oracle timed on the host cores as the reference arm: W untimed and
-    K timed samples of the workload, each through the same number of layers,
-    chosen (at most --oracle-layers) so the W + K samples fit REF_BUDGET_S
-    by a one-layer probe; every sample is scaled to all layers."""
+    """The oracle timed on the host cores as the reference arm.  Every step is
+    the same bounded sample of the workload: the 40 rows through the model's
+    first `layers` layers, as many (at most --oracle-layers) as let the W
+    warm-up and K timed steps fit REF_BUDGET_S by a one-layer probe.
+    ms_per_step is the step as it ran; value counts a position once per full
+    depth (positions x layers_per_step / layers_per_position per second)."""
     import oracle
     if rank != 0:
         return None
     M = EDIT_LEN + K_BUDGET
+    L = cfg["n_layers"]
     threads = oracle.set_threads(os.cpu_count() or 1)
     probe = oracle_setup(cfg, 1)
     t_layer = oracle_time(probe)
     runs = args.warmup + args.steps
-    layers = max(1, min(args.oracle_layers, int(REF_BUDGET_S / (runs * t_layer))))
+    cap = args.oracle_layers or L
+    layers = max(1, min(cap, L, int(REF_BUDGET_S / (runs * t_layer))))
     sample = probe if layers == 1 else oracle_setup(cfg, layers)
-    times = []
-    for i in range(runs):
-        per_layer = oracle_time(sample)
-        if i >= args.warmup:
-            times.append(per_layer * cfg["n_layers"])
-    t = statistics.median(times)
-    val = M / t
-    desc = (f"oracle operator R on the {M} rows through {layers} of "
-            f"{cfg['n_layers']} layers per step, scaled to all layers")
+    for _ in range(args.warmup):
+        oracle_time(sample)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle_time(sample)
+    t = (time.perf_counter() - t0) / args.steps
+    val = oracle_value(cfg, layers, t)
+    desc = (f"oracle operator R on the {M} rows through the first {layers} of {L} layers "
+            f"per step (each layer its own seeded weights, seeded synthetic stale cache)")
     return {"metric": METRIC, "value": val, "unit": "positions/s", "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": t * 1e3,
+            "layers_per_step": layers, "layers_per_position": L,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic", "impl": "reference",
             "config": workload_config(cfg, args.gpus),
@@ -252,6 +266,104 @@ def gemm_source_sha256() -> str:
     return h.hexdigest()
 
 
+def time_ms(fn, stream, reps: int = 3, warm: int = 1) -> float:
+    """Median device time (CUDA events on `stream`) of fn over reps calls
+    after warm untimed ones."""
+    import torch
+    t = []
+    for i in range(warm + reps):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        fn()
+        b.record(stream)
+        torch.cuda.synchronize()
+        if i >= warm:
+            t.append(a.elapsed_time(b))
+    return statistics.median(t)
+
+
+def pass_flops(cfg, positions) -> float:
+    """Dense FLOPs of a K/V-only pass over rows at `positions` (as the library
+    runs it: every layer's QKV projection, the O projection, MLP and causal
+    attention over keys 0..p of all layers but the last)."""
+    d, F, L = cfg["d_model"], cfg["ffn"], cfg["n_layers"]
+    H, G, dh = cfg["n_heads"], cfg["n_kv_heads"], cfg["head_dim"]
+    rows = len(positions)
+    qkv = 2.0 * rows * d * (H + 2 * G) * dh
+    rest = 2.0 * rows * (H * dh * d + 3 * F * d)
+    attn = 4.0 * H * dh * float(np.sum(np.asarray(positions, np.float64) + 1))
+    return L * qkv + (L - 1) * (rest + attn)
+
+
+def other_workloads(kv, stream, llama) -> dict:
+    """The other paper-shaped workloads, timed on the device (CUDA events,
+    median of 3 after a warm-up call):
+    - Qwen2.5-7B shape: select and repair for K in 8..128 under EditLocal,
+      Random and Attention (selector time apart from the repair, as the paper
+      reports it);
+    - Mistral-7B shape: the Structural and CacheBlend selectors at K = 32;
+    - 16 Llama-3-8B-shaped documents of 8192 tokens, 4 edits each with an
+      EditLocal window of 32 after every span, in one batched repair call,
+      against the 16 full re-prefills."""
+    from paper_2609_17983_gb300 import synth
+    out = {}
+    tpeak, _ = load_tensor_peak()
+    for name, pols in (("qwen7b", ("editlocal", "random", "attention")),
+                       ("mistral7b", ("structural", "cacheblend"))):
+        cfg = synth.preset(name)
+        w = synth.workload(name)
+        doc, s, new = w["doc"], w["edit_start"], w["new_tokens"]
+        m = kv.Model(cfg, None, seed=0, max_context=8192, max_rows=4096)
+        m.set_stream(stream.cuda_stream)
+        cache = m.prefill(doc)
+        res = {"edit": f"{len(new)}@{s}", "n": len(doc), "layers": cfg["n_layers"]}
+        for pol in pols:
+            res[pol] = {}
+            for K in w["Ks"]:
+                A = m.select(cache, pol, K, s, new, 0)
+                sel = time_ms(lambda: m.select(cache, pol, K, s, new, 0), stream)
+                rep = time_ms(lambda: cache.repair(new, s, A), stream)
+                rows = len(new) + len(A)
+                res[pol][str(K)] = {"select_ms": sel, "repair_ms": rep, "rows": rows,
+                                    "positions_per_s": rows / (rep / 1e3)}
+        cache.close()
+        m.close()
+        out[name] = res
+    # batched repair: 16 x 8192, 64 edits (span U[2, 16], window of 32 each)
+    cfg = synth.preset(WORKLOAD)
+    docs, reqs, P_all = [], [], []
+    for d in range(16):
+        doc = synth.document(100 + d, 8192, cfg["vocab"], cfg["delim_id"])
+        edits, A, P = [], [], set()
+        for (st, ln) in synth.batch_edits(200 + d, 8192, 4, (2, 16), K_BUDGET):
+            new = synth.edit_tokens(300 + d * 7 + st, doc[st:st + ln], cfg["vocab"])
+            edits.append((st, new))
+            A += list(range(st + ln, st + ln + K_BUDGET))
+            P |= set(range(st, st + ln + K_BUDGET))
+        docs.append(doc)
+        reqs.append((edits, np.array(sorted(set(A)))))
+        P_all += sorted(P)
+    caches = [llama.prefill(doc) for doc in docs]
+    batch = [(c, e, A) for c, (e, A) in zip(caches, reqs)]
+    b_ms = time_ms(lambda: llama.repair_batch(batch), stream)
+    for c in caches:
+        c.close()
+    edited = []
+    for doc, (edits, _) in zip(docs, reqs):
+        t = doc.copy()
+        for st, new in edits:
+            t[st:st + len(new)] = new
+        edited.append(t)
+    p_ms = time_ms(lambda: [llama.prefill(t).close() for t in edited], stream, reps=1)
+    fl = pass_flops(cfg, P_all)
+    out["batch_16x8192"] = {"docs": 16, "n": 8192, "edits": 64, "rows": len(P_all),
+                            "repair_ms": b_ms, "positions_per_s": len(P_all) / (b_ms / 1e3),
+                            "prefill_16_ms": p_ms, "speedup_vs_prefill": p_ms / b_ms,
+                            "flops": fl, "tflops": fl / (b_ms / 1e3) / 1e12,
+                            "frac_of_bf16_sustained": fl / (b_ms / 1e3) / 1e12 / tpeak}
+    return out
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -259,9 +371,11 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="kvrepair", choices=["kvrepair", "reference"])
     ap.add_argument("--prefill-steps", type=int, default=3)
-    ap.add_argument("--oracle-layers", type=int, default=4,
-                    help="most layers per oracle sample of the reference arm")
+    ap.add_argument("--oracle-layers", type=int, default=None,
+                    help="most layers per oracle step of the reference arm")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-other-workloads", action="store_true",
+                    help="skip the Qwen/Mistral/batched workloads (profiling runs)")
     ap.add_argument("--layers", type=int, default=None,
                     help="decoder layers (default: the model's 32); fewer only for profiling")
     args = ap.parse_args()
@@ -285,17 +399,17 @@ def main():
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         import oracle
         threads = oracle.set_threads(os.cpu_count() or 1)
-        probe = oracle_setup(cfg, 1)
-        t_layer = oracle_time(probe)
-        # one step through as many layers as take about CPU_BASELINE_S
+        t_layer = oracle_time(oracle_setup(cfg, 1))
+        # one step through as many of the model's first layers as take about
+        # CPU_BASELINE_S
         layers = max(1, min(cfg["n_layers"], round(CPU_BASELINE_S / t_layer)))
-        per_layer = oracle_time(oracle_setup(cfg, layers)) if layers > 1 else t_layer
+        t = oracle_time(oracle_setup(cfg, layers)) if layers > 1 else t_layer
         M = EDIT_LEN + K_BUDGET
-        cpu = {"value": M / (per_layer * cfg["n_layers"]), "unit": "positions/s",
-               "cores": threads, "kind": "oracle",
-               "sample": f"oracle operator R on the {M} rows through {layers} of "
-                         f"{cfg['n_layers']} layers (one step, about {CPU_BASELINE_S:.0f} s), "
-                         f"scaled to all layers"}
+        cpu = {"value": oracle_value(cfg, layers, t), "unit": "positions/s",
+               "cores": threads, "kind": "oracle", "step_s": t, "layers_per_step": layers,
+               "sample": f"oracle operator R on the {M} rows through the first {layers} of "
+                         f"{cfg['n_layers']} layers (one step; each layer its own seeded "
+                         f"weights, seeded synthetic stale cache)"}
 
     import torch
     local = int(os.environ.get("LOCAL_RANK", "0"))
@@ -436,6 +550,9 @@ def main():
     prefill_ms = statistics.median(pre)
     tpeak, tpeak_kind = load_tensor_peak()
     pf_tflops = prefill_flops(cfg, N_CTX) / (prefill_ms / 1e3) / 1e12
+    others = None
+    if not args.no_other_workloads and cfg["n_layers"] == 32:
+        others = other_workloads(kv, stream, model)
 
     if rank == 0:
         out = {"metric": METRIC, "value": value, "unit": "positions/s", "n_gpus": world,
@@ -462,6 +579,7 @@ def main():
                "kernel_ms_per_step": {k: v["ms"] / args.steps for k, v in prof.items()
                                       if v["launches"]},
                "clocks": clk.summary(),
+               "other_workloads": others,
                "cpu_baseline": cpu}
         print(json.dumps(out), flush=True)
     cache.close()

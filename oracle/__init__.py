@@ -21,6 +21,10 @@ Pin status (what each function is checked against, in tests/test_oracle_*.py):
                           complex-number RoPE), Eq. 1 endpoint identity,
                           no-op edit, token-major brute force, upstream
                           invariance, split-call and idempotence.
+  bf16 path            -- the same textbook decoder with the bf16 path's
+                          rounding points (torch's own bf16 conversions, an
+                          attention written out over all heads), to 1e-9;
+                          the Eq. 1 identities hold bit-exact on it too.
   logits               -- the same textbook decoder run over C' + query.
   editlocal/structural -- closed forms and hand-written golden cases.
   editlocal_boundary   -- hand-written golden case.
@@ -81,6 +85,7 @@ class _Config(ctypes.Structure):
                 ("n_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
                 ("ffn", ctypes.c_int32), ("qkv_bias", ctypes.c_int32),
                 ("wdtype", ctypes.c_int32), ("cdtype", ctypes.c_int32),
+                ("operands", ctypes.c_int32),
                 ("rope_theta", ctypes.c_double), ("rms_eps", ctypes.c_double)]
 
 
@@ -131,11 +136,23 @@ def _wdtype(cfg) -> int:
     return 1 if cfg["dtype"] == "bf16" else 0
 
 
+# Operand precision of the matrix products (kvr_oracle.c, orc_config.operands):
+# "fp64" keeps them in double; "bf16" rounds every operand of a matrix product
+# to bf16, as the bf16 path does; "bf16_dense" only those of the weight
+# products; "bf16_f32sums" is the bf16 path with the weight products' results
+# and the residual stream rounded to fp32 (a null control: how far last-bit
+# changes of the sums carry through the layers).  A config's "operands" key
+# selects it; by default a bf16 model is computed on the bf16 path and an
+# fp32 model in double.
+OPERANDS = {"fp64": 0, "bf16_dense": 1, "bf16": 3, "bf16_f32sums": 7}
+
+
 def _cfg_struct(cfg) -> _Config:
     bf = _wdtype(cfg)
     return _Config(cfg["vocab"], cfg["d_model"], cfg["n_layers"], cfg["n_heads"],
                    cfg["n_kv_heads"], cfg["head_dim"], cfg["ffn"],
                    1 if cfg.get("qkv_bias") else 0, bf, bf,
+                   OPERANDS[cfg.get("operands", "bf16" if bf else "fp64")],
                    float(cfg["rope_theta"]), float(cfg["rms_eps"]))
 
 

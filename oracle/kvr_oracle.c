@@ -23,7 +23,10 @@
  * Arithmetic: IEEE double everywhere.  Weights arrive as fp32 or as bf16 bit
  * patterns and are widened exactly.  Cache entries are stored in the cache's
  * dtype (fp32 or bf16, round-to-nearest-even) because the cache is a stored
- * data structure of that dtype; everything else stays in double.  Build with
+ * data structure of that dtype; everything else stays in double -- except, on
+ * the bf16 path (orc_config.operands), the operands of the matrix products,
+ * which that path holds in bf16: they are rounded where they enter a product
+ * and every sum stays in double.  Build with
  * -ffp-contract=off so that a*b+c is never fused: each output element is one
  * sequential sum in a fixed order, independent of which other rows are in the
  * batch and of the thread count.  That is what makes the bit-exact invariants
@@ -45,6 +48,20 @@ typedef struct {
   int32_t qkv_bias; /* 1: the q/k/v projections carry a bias (Qwen-style) */
   int32_t wdtype;   /* storage of every weight: 0 = fp32, 1 = bf16 bit patterns */
   int32_t cdtype;   /* storage of cache entries: 0 = fp32, 1 = bf16 */
+  /* Operands of the matrix products (the bf16 path of Sec. 4 takes them in
+   * bf16 and accumulates wider): 0 = kept in double; bit 0 = the rows that
+   * enter a weight product (normalised rows into the QKV and gate/up
+   * projections and the lm_head, the attention output into O, the SwiGLU
+   * activation into down) are rounded to bf16; bit 1 = so are the two
+   * attention products' operands: the post-RoPE query, and the weights of V,
+   * 2^(x_j - E) with x_j = log2(e) s_j the scores in base 2 and E an integer
+   * at or above their maximum (any integer gives the same bf16 mantissas;
+   * O = sum_j bf16(2^(x_j - E)) v_j / sum_j 2^(x_j - E)).  Accumulation and
+   * everything else stay in double -- unless bit 2 is set: then every weight
+   * product's result and the residual stream are rounded to fp32 as well (the
+   * bf16 path with fp32 sums; a null control, which measures how far a last-
+   * bit change of the sums carries through the layers). */
+  int32_t operands;
   double rope_theta, rms_eps;
 } orc_config;
 
@@ -59,6 +76,8 @@ typedef struct {
 } orc_weights;
 
 enum { ORC_OK = 0, ORC_EINVAL = 1, ORC_ENOMEM = 2 };
+
+static const double LOG2E = 1.44269504088896340736; /* log2(e) */
 
 /* ---------------------------------------------------------------- helpers */
 
@@ -86,6 +105,15 @@ static float to_cache(double x, int cdtype) {
   return f;
 }
 
+/* An operand of a matrix product as the bf16 path holds it: rounded to bf16
+ * (through fp32, as to_cache) when `on`, else unchanged. */
+static double operand(double x, int on) { return on ? (double)to_cache(x, 1) : x; }
+
+static void round_operands(double *x, size_t n, int on) {
+  if (on)
+    for (size_t i = 0; i < n; ++i) x[i] = operand(x[i], 1);
+}
+
 /* RMSNorm: y_i = x_i / sqrt(mean(x^2) + eps) * g_i. */
 static void rmsnorm(const double *x, const void *g, int gbf16, int d, double eps, double *y) {
   double ss = 0.0;
@@ -93,6 +121,12 @@ static void rmsnorm(const double *x, const void *g, int gbf16, int d, double eps
   double r = 1.0 / sqrt(ss / (double)d + eps);
   for (int i = 0; i < d; ++i) y[i] = x[i] * r * wval(g, (size_t)i, gbf16);
 }
+
+/* Set by the entry points from orc_config.operands bit 2: round the results
+ * of the weight products and the residual stream to fp32. */
+static int g_f32_sums = 0;
+
+static double sum_round(double x) { return g_f32_sums ? (double)(float)x : x; }
 
 /* y[r][o] = sum_k W[o][k] * x[r][k] (+ b[o]) for m rows. */
 static void linear_rows(const double *x, int m, int in, const void *W, const void *b, int bf16,
@@ -104,7 +138,7 @@ static void linear_rows(const double *x, int m, int in, const void *W, const voi
       double acc = 0.0;
       for (int k = 0; k < in; ++k) acc += wval(W, (size_t)o * in + k, bf16) * xr[k];
       if (b) acc += wval(b, (size_t)o, bf16);
-      y[(size_t)r * out + o] = acc;
+      y[(size_t)r * out + o] = sum_round(acc);
     }
   }
 }
@@ -138,6 +172,7 @@ static void stage_qkv(const orc_config *c, const orc_weights *w, int l, const do
   int d = c->d_model, dh = c->head_dim, H = c->n_heads, G = c->n_kv_heads, bf = c->wdtype;
   for (int r = 0; r < m; ++r)
     rmsnorm(h + (size_t)r * d, w->attn_norm[l], bf, d, c->rms_eps, scratch + (size_t)r * d);
+  round_operands(scratch, (size_t)m * d, c->operands & 1);
   linear_rows(scratch, m, d, w->wq[l], c->qkv_bias ? w->bq[l] : NULL, bf, H * dh, q);
   linear_rows(scratch, m, d, w->wk[l], c->qkv_bias ? w->bk[l] : NULL, bf, G * dh, k);
   linear_rows(scratch, m, d, w->wv[l], c->qkv_bias ? w->bv[l] : NULL, bf, G * dh, v);
@@ -166,6 +201,7 @@ static void stage_write_kv(const orc_config *c, int l, float *kc, float *vc, int
 static void attend_row(const orc_config *c, int l, const float *kc, const float *vc, int cap,
                        const double *q, int64_t p, double *o, double *sbuf) {
   int H = c->n_heads, G = c->n_kv_heads, dh = c->head_dim, grp = H / G;
+  const int rnd = c->operands & 2;
   double scale = 1.0 / sqrt((double)dh);
   for (int hh = 0; hh < H; ++hh) {
     int g = hh / grp;
@@ -174,14 +210,25 @@ static void attend_row(const orc_config *c, int l, const float *kc, const float 
     for (int64_t j = 0; j <= p; ++j) {
       const float *kj = kc + cache_index(c, cap, l, j, g);
       double s = 0.0;
-      for (int i = 0; i < dh; ++i) s += qh[i] * (double)kj[i];
+      for (int i = 0; i < dh; ++i) s += operand(qh[i], rnd) * (double)kj[i];
       sbuf[j] = s * scale;
       if (sbuf[j] > mx) mx = sbuf[j];
     }
     double z = 0.0;
-    for (int64_t j = 0; j <= p; ++j) {
-      sbuf[j] = exp(sbuf[j] - mx);
-      z += sbuf[j];
+    if (rnd) {
+      /* base-2 scores against the integer E = ceil(max): the weights of V
+       * are rounded, their sum is not */
+      const double E = ceil(mx * LOG2E);
+      for (int64_t j = 0; j <= p; ++j) {
+        sbuf[j] = exp2(sbuf[j] * LOG2E - E);
+        z += sbuf[j];
+        sbuf[j] = operand(sbuf[j], 1);
+      }
+    } else {
+      for (int64_t j = 0; j <= p; ++j) {
+        sbuf[j] = exp(sbuf[j] - mx);
+        z += sbuf[j];
+      }
     }
     double *oh = o + (size_t)hh * dh;
     for (int i = 0; i < dh; ++i) {
@@ -228,8 +275,9 @@ static int stage_attn_mlp(const orc_config *c, const orc_weights *w, int l, cons
     return ORC_ENOMEM;
   }
   /* h += o Wo */
+  round_operands(o, (size_t)m * H * dh, c->operands & 1);
   linear_rows(o, m, H * dh, w->wo[l], NULL, bf, d, t);
-  for (size_t i = 0; i < (size_t)m * d; ++i) h[i] += t[i];
+  for (size_t i = 0; i < (size_t)m * d; ++i) h[i] = sum_round(h[i] + t[i]);
   /* h += Wd (silu(Wg b) * (Wu b)) */
   double *bb = malloc(sizeof(double) * (size_t)m * d);
   double *gg = malloc(sizeof(double) * (size_t)m * F);
@@ -244,11 +292,13 @@ static int stage_attn_mlp(const orc_config *c, const orc_weights *w, int l, cons
   }
   for (int r = 0; r < m; ++r)
     rmsnorm(h + (size_t)r * d, w->mlp_norm[l], bf, d, c->rms_eps, bb + (size_t)r * d);
+  round_operands(bb, (size_t)m * d, c->operands & 1);
   linear_rows(bb, m, d, w->wg[l], NULL, bf, F, gg);
   linear_rows(bb, m, d, w->wu[l], NULL, bf, F, uu);
   for (size_t i = 0; i < (size_t)m * F; ++i) gg[i] = silu(gg[i]) * uu[i];
+  round_operands(gg, (size_t)m * F, c->operands & 1);
   linear_rows(gg, m, F, w->wd[l], NULL, bf, d, t);
-  for (size_t i = 0; i < (size_t)m * d; ++i) h[i] += t[i];
+  for (size_t i = 0; i < (size_t)m * d; ++i) h[i] = sum_round(h[i] + t[i]);
   free(bb);
   free(gg);
   free(uu);
@@ -297,6 +347,7 @@ int orc_set_threads(int n) {
  * receives the rows' final residual stream [m][d_model]. */
 int orc_recompute(const orc_config *c, const orc_weights *w, float *kc, float *vc, int cap,
                   const int32_t *tokens, const int64_t *pos, int m, double *h_out) {
+  g_f32_sums = (c->operands & 4) != 0;
   if (m <= 0) return ORC_OK;
   int rc = check_rows(c, cap, tokens, pos, m);
   if (rc) return rc;
@@ -351,6 +402,7 @@ int orc_recompute_token_major(const orc_config *c, const orc_weights *w, float *
  * score has n entries; entries outside D are set to 0. */
 int orc_score_attention(const orc_config *c, const orc_weights *w, float *kc, float *vc, int cap,
                         int n, const int32_t *tokens, int s_start, int s_end, double *score) {
+  g_f32_sums = (c->operands & 4) != 0;
   int m = s_end - s_start;
   if (m <= 0 || s_start < 0 || s_end > n || n > cap) return ORC_EINVAL;
   int d = c->d_model, H = c->n_heads, G = c->n_kv_heads, dh = c->head_dim, grp = H / G;
@@ -417,6 +469,7 @@ done:
  * over all kv heads and dims.  Entries outside D are 0.  Needs >= 2 layers. */
 int orc_score_cacheblend(const orc_config *c, const orc_weights *w, float *kc, float *vc, int cap,
                          int n, const int32_t *tokens, int s_start, int s_end, double *score) {
+  g_f32_sums = (c->operands & 4) != 0;
   int ms = s_end - s_start, md = n - s_end;
   if (ms <= 0 || s_start < 0 || s_end > n || n > cap || c->n_layers < 2) return ORC_EINVAL;
   int d = c->d_model, H = c->n_heads, G = c->n_kv_heads, dh = c->head_dim;
@@ -481,6 +534,7 @@ done:
  * lm_head RMSNorm(h_row).  Used for teacher-forced answer scoring (Eq. 2). */
 int orc_logits_all(const orc_config *c, const orc_weights *w, float *kc, float *vc, int cap,
                    int n, const int32_t *tokens, int m, double *logits) {
+  g_f32_sums = (c->operands & 4) != 0;
   if (m <= 0 || n < 0 || n + m > cap) return ORC_EINVAL;
   int d = c->d_model;
   int64_t *pos = malloc(sizeof(int64_t) * (size_t)m);
@@ -496,6 +550,7 @@ int orc_logits_all(const orc_config *c, const orc_weights *w, float *kc, float *
   if (rc) goto done;
   for (int r = 0; r < m; ++r)
     rmsnorm(h + (size_t)r * d, w->final_norm, c->wdtype, d, c->rms_eps, a + (size_t)r * d);
+  round_operands(a, (size_t)m * d, c->operands & 1);
   linear_rows(a, m, d, w->lm_head, NULL, c->wdtype, c->vocab, logits);
 done:
   free(pos);
@@ -510,6 +565,7 @@ done:
  * into the document's entries.  logits[vocab] = lm_head RMSNorm(h_last). */
 int orc_logits(const orc_config *c, const orc_weights *w, float *kc, float *vc, int cap, int n,
                const int32_t *tokens /* [n+m], query at n.. */, int m, double *logits) {
+  g_f32_sums = (c->operands & 4) != 0;
   if (m <= 0 || n < 0 || n + m > cap) return ORC_EINVAL;
   int d = c->d_model;
   int64_t *pos = malloc(sizeof(int64_t) * (size_t)m);
@@ -524,6 +580,7 @@ int orc_logits(const orc_config *c, const orc_weights *w, float *kc, float *vc, 
   rc = orc_recompute(c, w, kc, vc, cap, tokens, pos, m, h);
   if (rc) goto done;
   rmsnorm(h + (size_t)(m - 1) * d, w->final_norm, c->wdtype, d, c->rms_eps, a);
+  round_operands(a, (size_t)d, c->operands & 1);
   linear_rows(a, 1, d, w->lm_head, NULL, c->wdtype, c->vocab, logits);
 done:
   free(pos);

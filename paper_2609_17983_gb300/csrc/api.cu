@@ -160,6 +160,7 @@ struct Rows {
   const int4 *blocks = nullptr;              // attention query blocks (device)
   int n_blocks = 0, n_splits = 1, max_block_rows = 0;
   const CUtensorMap *tm_kv = nullptr;        // TMA view of the single document's pages
+  const CUtensorMap *tmaps = nullptr;        // device [docs]: TMA views of a batch's pages
   bool tc5 = false;                          // attention on tcgen05 (set by plan_attention)
 };
 
@@ -175,9 +176,10 @@ kvr_status plan_attention(kvr_model *m, Rows &r, const int32_t *pos, const int32
   if (!use_tc_attention(m) || r.M <= 0) return KVR_OK;
   const Dims &dm = m->dims;
   const int grp = dm.H / dm.G;
-  // one document's rows run on the tcgen05 kernel (query blocks of up to 128
-  // query vectors), several documents' on the mma.sync kernel
-  r.tc5 = m->use_tc5 && !rowdoc && r.tm_kv && attn_tc5_rows_per_block(grp) > 0;
+  // the tcgen05 kernel (query blocks of up to 128 query vectors) when every
+  // document has a TMA view of its pages, else the mma.sync kernel
+  r.tc5 = m->use_tc5 && (rowdoc ? r.tmaps != nullptr : r.tm_kv != nullptr) &&
+          attn_tc5_rows_per_block(grp) > 0;
   const int qb = r.tc5 ? attn_tc5_rows_per_block(grp) : attn_tc_rows_per_block(grp);
   std::vector<int32_t> b;
   int max_chunks = 0, max_rows = 0;
@@ -247,8 +249,7 @@ kvr_status layer_qkv(kvr_model *m, const Rows &r, int l, bool write_kv, bool kee
     Prof pr(m, P_ROPE, (int64_t)r.M * dm.Nqkv() * 4);
     const bool tc = use_tc_attention(m);
     launch_rope_scatter(m->qkv, m->rope, r.pos, r.M, dm, l, r.views, r.rowdoc, r.single,
-                        tc && !need_q ? nullptr : m->q, tc ? m->qb : nullptr,
-                        (float)(1.4426950408889634 / std::sqrt((double)dm.dh)), write_kv,
+                        tc && !need_q ? nullptr : m->q, tc ? m->qb : nullptr, 1.0f, write_kv,
                         m->stream, &sv);
     KVR_TRY(launch_check(m, 1));
   }
@@ -263,10 +264,11 @@ kvr_status layer_rest(kvr_model *m, const Rows &r, int l) {
     int64_t kv_bytes = (int64_t)(r.max_pos + 1) * dm.G * dm.dh * 2 * (int64_t)dm.es();
     Prof pr(m, P_ATTN, kv_bytes);
     if (r.tc5) {
-      const char *e = launch_attention_tc5(m->qb, r.pos, r.blocks, r.n_blocks, r.n_splits, dm, l,
-                                           r.single.pages, r.single.table, *r.tm_kv,
-                                           m->attn_ws_o, m->attn_ws_ml, m->attn, m->dev_flag,
-                                           m->stream);
+      static const CUtensorMap unused{};  // a batch's views come from r.tmaps
+      const char *e = launch_attention_tc5(
+          m->qb, r.pos, r.blocks, r.n_blocks, r.n_splits, dm, l, r.single.pages, r.single.table,
+          r.tm_kv ? *r.tm_kv : unused, m->attn_ws_o, m->attn_ws_ml, m->attn, m->dev_flag,
+          m->stream, r.tmaps ? r.views : nullptr, r.tmaps);
       if (!e)
         e = launch_attention_combine(r.blocks, r.n_blocks, r.max_block_rows, r.n_splits, dm,
                                      m->attn_ws_o, m->attn_ws_ml, m->attn, m->stream,
@@ -547,6 +549,7 @@ void kvr_model_free(kvr_model *m) {
   dev_free(m->tcw.partials);
   dev_free(m->read_scratch);
   dev_free(m->sel_scratch);
+  dev_free(m->batch_scratch);
   dev_free(m->tcw.counters);
   dev_free(m->blocks_d);
   dev_free(m->attn_ws_o);
@@ -760,7 +763,9 @@ kvr_status kvr_model_create(const kvr_model_config *cfg, const kvr_weights *wts,
     m->dev_flag = (int *)dev_alloc(256);
     if (!m->dev_flag) return bail(fail(KVR_E_NOMEM, "flag"));
     cudaMemset(m->dev_flag, 0, 256);
-    m->stage_cap = std::max<size_t>(R * 4, P) + 4096;
+    // positions and tokens of a pass, plus the tables of a 256-document batch
+    m->stage_cap = std::max<size_t>(R * 4, P) + 4096 +
+                   256 * (sizeof(CUtensorMap) + sizeof(KVView) + sizeof(void *)) / 4;
     if (cudaMallocHost(&m->stage_h, m->stage_cap * sizeof(int32_t)) != cudaSuccess)
       return bail(fail(KVR_E_NOMEM, "pinned staging"));
     cudaEventCreateWithFlags(&m->stage_ev, cudaEventDisableTiming);
@@ -1116,20 +1121,26 @@ kvr_status kvr_repair_batch(kvr_model *m, const kvr_repair_req *reqs, int32_t n_
       tk += L;
     }
   }
-  // device tables: views and token pointers of the documents
-  std::vector<KVView> views(n_reqs);
-  std::vector<const int32_t *> toks(n_reqs);
+  // device tables, in the model's batch scratch (grown, never shrunk; reused
+  // in stream order): the documents' TMA views of their pages (when every
+  // cache has one), their cache views and token pointers
+  bool all_tm = true;
+  for (int r = 0; r < n_reqs; ++r) all_tm = all_tm && reqs[r].cache->tm_kv_ok;
+  const size_t mb = all_tm ? (size_t)n_reqs * sizeof(CUtensorMap) : 0;
+  const size_t vb = n_reqs * sizeof(KVView), tb = n_reqs * sizeof(void *);
+  std::vector<int32_t> host((mb + vb + tb + 3) / 4);
+  char *hb = (char *)host.data();
   for (int r = 0; r < n_reqs; ++r) {
-    views[r] = reqs[r].cache->view();
-    toks[r] = reqs[r].cache->tokens_d;
+    if (all_tm) memcpy(hb + r * sizeof(CUtensorMap), &reqs[r].cache->tm_kv, sizeof(CUtensorMap));
+    const KVView v = reqs[r].cache->view();
+    memcpy(hb + mb + r * sizeof(KVView), &v, sizeof(KVView));
+    const int32_t *t = reqs[r].cache->tokens_d;
+    memcpy(hb + mb + vb + r * sizeof(void *), &t, sizeof(void *));
   }
-  size_t vb = n_reqs * sizeof(KVView), tb = n_reqs * sizeof(void *);
-  char *tab = (char *)dev_alloc(vb + tb + 64);
-  if (!tab) return fail(KVR_E_NOMEM, "batch tables");
-  kvr_status st = KVR_OK;
-  if (cudaMemcpyAsync(tab, views.data(), vb, cudaMemcpyHostToDevice, m->stream) ||
-      cudaMemcpyAsync(tab + vb, toks.data(), tb, cudaMemcpyHostToDevice, m->stream))
-    st = fail(KVR_E_CUDA, "batch table upload");
+  KVR_TRY(grow_scratch(m, m->batch_scratch, m->batch_scratch_bytes, host.size() * 4,
+                       "batch tables"));
+  char *tab = (char *)m->batch_scratch;
+  kvr_status st = stage_h2d(m, (int32_t *)tab, host.data(), host.size());
   if (!st) st = stage_h2d(m, m->pos_d, P.data(), M);
   if (!st) {
     // rowdoc goes through a second staging round
@@ -1140,14 +1151,13 @@ kvr_status kvr_repair_batch(kvr_model *m, const kvr_repair_req *reqs, int32_t n_
     r.M = M;
     r.pos = m->pos_d;
     r.rowdoc = m->rowdoc_d;
-    r.views = (const KVView *)tab;
-    r.doc_tokens = (const int32_t *const *)(tab + vb);
+    r.views = (const KVView *)(tab + mb);
+    r.doc_tokens = (const int32_t *const *)(tab + mb + vb);
+    r.tmaps = all_tm ? (const CUtensorMap *)tab : nullptr;
     r.max_pos = max_pos;
     st = plan_attention(m, r, P.data(), rowdoc.data());
     if (!st) st = run_pass(m, r, true);
   }
-  cudaStreamSynchronize(m->stream);
-  dev_free(tab);
   if (st == KVR_E_CUDA)
     for (int r = 0; r < n_reqs; ++r) reqs[r].cache->poisoned = true;
   return st;

@@ -19,6 +19,7 @@
 #include <math.h>
 
 #include <algorithm>
+#include <cmath>
 
 #include <type_traits>
 
@@ -32,7 +33,8 @@ constexpr int MAXW = 12;         // warps per CTA, 16 query vectors each
 constexpr int MAXQ = MAXW * 16;  // query vectors per CTA
 
 struct AttnTcParams {
-  const __nv_bfloat16 *q;  // [M][H*dh] post-RoPE, pre-scaled by log2(e)/sqrt(dh)
+  const __nv_bfloat16 *q;  // [M][H*dh] post-RoPE
+  float qk_scale;          // log2(e) / sqrt(dh): scores into the log2 domain
   int H, G, grp;
   const int32_t *pos;
   const int4 *blocks;  // (row0, nrows, kmax, doc)
@@ -200,11 +202,15 @@ __global__ void __launch_bounds__(MAXW * 32, 1) k_attn_tc(const AttnTcParams p) 
         }
       }
       // causal mask on original positions, online softmax (log2 domain)
+      // against integer reference maxima, so that bf16(P) is a power of two
+      // times the rounding of 2^(x - E) for any integer E
       const int kbase = c * CHUNK + 2 * (lane & 3);
       float mx0 = -INFINITY, mx1 = -INFINITY;
 #pragma unroll
       for (int nt = 0; nt < 8; ++nt) {
         int j = kbase + 8 * nt;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) s[nt][k] *= p.qk_scale;
         if (j > p0) s[nt][0] = -INFINITY;
         if (j + 1 > p0) s[nt][1] = -INFINITY;
         if (j > p1) s[nt][2] = -INFINITY;
@@ -216,7 +222,7 @@ __global__ void __launch_bounds__(MAXW * 32, 1) k_attn_tc(const AttnTcParams p) 
       mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
       mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
       mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
-      const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
+      const float mn0 = fmaxf(m0, ceilf(mx0)), mn1 = fmaxf(m1, ceilf(mx1));
       const float b0s = mn0 == -INFINITY ? 0.f : mn0, b1s = mn1 == -INFINITY ? 0.f : mn1;
       const float cr0 = exp2f(m0 - b0s), cr1 = exp2f(m1 - b1s);
       m0 = mn0;
@@ -453,6 +459,7 @@ const char *launch_attention_tc(const void *q, const int32_t *pos, const int4 *b
   if (n_blocks <= 0) return nullptr;
   AttnTcParams p{};
   p.q = (const __nv_bfloat16 *)q;
+  p.qk_scale = (float)(1.4426950408889634 / std::sqrt((double)dm.dh));
   p.H = dm.H;
   p.G = dm.G;
   p.grp = dm.H / dm.G;

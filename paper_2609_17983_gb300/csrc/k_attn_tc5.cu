@@ -2,8 +2,9 @@
 // rows on the tcgen05 tensor cores (sm_103a), bf16 cache, head_dim 64 or 128.
 //
 // A CTA owns one query block -- up to 128 query vectors (rows of the pass times
-// the grp query heads of KV head g), the M = 128 rows of the MMA -- and a
-// contiguous range of 64-key chunks (one KV page each).  Per chunk:
+// the grp query heads of KV head g, all of one document), the M = 128 rows of
+// the MMA -- and a contiguous range of 64-key chunks (one KV page each).  A
+// pass over several documents gives each its own page table and TMA view.  Per chunk:
 //   S = Q K^T      tcgen05.mma, M 128 x N 64 x K head_dim, into TMEM (two
 //                  S buffers, so S of chunk i+1 is computed while the softmax
 //                  works on chunk i);
@@ -12,11 +13,14 @@
 //                  chunk's keys and of O's columns (four warps per SM
 //                  sub-partition hide each other's latency), the row maximum
 //                  exchanged through shared memory; S read once from
-//                  TMEM: causal mask key <= position, exponentials in the
-//                  log2 domain (Q is pre-scaled by log2(e)/sqrt(dh)) against
-//                  a reference maximum that is raised -- and the accumulator
-//                  rescaled in TMEM -- only when the running maximum exceeds
-//                  it by more than 8 (so P <= 256); P in bf16 written to one
+//                  TMEM: causal mask key <= position, scores scaled by
+//                  log2(e)/sqrt(dh) into the log2 domain, exponentials
+//                  against an integer reference maximum that is raised -- and
+//                  the accumulator rescaled in TMEM by a power of two -- only
+//                  when the running maximum exceeds it by more than 8 (so
+//                  P <= 256); with an integer reference, bf16(P) is a power
+//                  of two times the rounding of 2^(x - E) for any integer E,
+//                  whichever chunk set it; P in bf16 written to one
 //                  of two shared-memory buffers as the next MMA's A operand,
 //                  so the softmax of chunk i overlaps O += P V of chunk i-1;
 //   O += P V       tcgen05.mma, M 128 x N head_dim x K 64, V read MN-major
@@ -54,11 +58,16 @@ constexpr float RESCALE_LOG2 = 8.f;  // headroom of the reference maximum (P <= 
 constexpr int KV_STAGES = 4;
 
 struct Attn5Params {
-  const __nv_bfloat16 *q;  // [M][H * dh] post-RoPE, pre-scaled by log2(e)/sqrt(dh)
+  const __nv_bfloat16 *q;  // [M][H * dh] post-RoPE
+  float qk_scale;          // log2(e) / sqrt(dh): scores into the log2 domain
   const int32_t *pos;      // [M] ascending (one document)
   const int4 *blocks;      // (row0, nrows, kmax, doc)
-  const __nv_bfloat16 *pages;  // the cache's page pool
-  const int32_t *table;        // logical page -> physical page
+  const __nv_bfloat16 *pages;  // the cache's page pool (one document)
+  const int32_t *table;        // logical page -> physical page (one document)
+  // several documents: their views and the TMA views of their page pools
+  // (device memory, 64-byte aligned), indexed by the block's document
+  const KVView *views;
+  const CUtensorMap *tmaps;
   int H, G, grp, layer, L;
   int n_splits, n_blocks;
   float *ws_o;    // [n_splits][n_blocks][G][WS_MAXQ][dh]
@@ -111,6 +120,11 @@ __global__ void __launch_bounds__(NT5, 1)
   const int4 bd = p.blocks[blk];
   const int row0 = bd.x, nrows = bd.y, kmax = bd.z;
   const int mq = nrows * p.grp;
+  // the block's document: its page table, page pool and TMA view
+  const int32_t *table = p.views ? p.views[bd.w].table : p.table;
+  const __nv_bfloat16 *pages =
+      p.views ? (const __nv_bfloat16 *)p.views[bd.w].pages : p.pages;
+  const CUtensorMap *tmap = p.tmaps ? p.tmaps + bd.w : &tm_kv;
   const int n_chunks = kmax / CH + 1;
   const int cps = (n_chunks + p.n_splits - 1) / p.n_splits;
   const int c0 = split * cps, c1 = min(n_chunks, c0 + cps);
@@ -123,7 +137,7 @@ __global__ void __launch_bounds__(NT5, 1)
   const uint32_t sQ = base, sKV = sQ + QBYTES, sP = sKV + KV_STAGES * KVBYTES;  // P: two tiles
   volatile int *abort_v = &abort_f;
   auto page_row = [&](int c, int kv) {  // first row of (chunk c, kv) in the pool's 2D view
-    const long long pg = p.table[c];
+    const long long pg = table[c];
     return (int)((((pg * p.L + p.layer) * 2 + kv) * p.G + g) * CH);
   };
   const bool rows_cached = nch <= 64;
@@ -155,7 +169,7 @@ __global__ void __launch_bounds__(NT5, 1)
     const int i = t >> 1, kv = t & 1;
     const int row = page_row(c0 + i, kv);
     if (rows_cached) sprow[t] = row;
-    const __nv_bfloat16 *pg = p.pages + (size_t)row * DH;
+    const __nv_bfloat16 *pg = pages + (size_t)row * DH;
     if (nch <= PREFETCH_MAX_CHUNKS)
       asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(pg), "r"(TBYTES)
                    : "memory");
@@ -177,7 +191,11 @@ __global__ void __launch_bounds__(NT5, 1)
   if (warp == 0) {
     // ------------------------------------------------------------ TMA
     if (lane == 0) {
-      tma_prefetch_desc(&tm_kv);
+      // a tensor map in global memory is read through the tensor-map proxy
+      if (p.tmaps)
+        asm volatile("fence.proxy.tensormap::generic.acquire.gpu [%0], 128;" ::"l"(tmap)
+                     : "memory");
+      tma_prefetch_desc(tmap);
       pdl_wait();
       ts.waited();
       int issued = 0;
@@ -193,9 +211,9 @@ __global__ void __launch_bounds__(NT5, 1)
         if (i == 0) trace_mark(1);
 #pragma unroll
         for (int h = 0; h < HALVES; ++h) {
-          tma_load_2d((void *)__cvta_shared_to_generic(sk + h * CH * 128), &tm_kv, &kv_full[b],
+          tma_load_2d((void *)__cvta_shared_to_generic(sk + h * CH * 128), tmap, &kv_full[b],
                       h * 64, rk);
-          tma_load_2d((void *)__cvta_shared_to_generic(sv + h * CH * 128), &tm_kv, &kv_full[b],
+          tma_load_2d((void *)__cvta_shared_to_generic(sv + h * CH * 128), tmap, &kv_full[b],
                       h * 64, rv);
         }
         ++issued;
@@ -310,7 +328,11 @@ __global__ void __launch_bounds__(NT5, 1)
         mbar_arrive(&s_free[b]);  // S is in registers: the buffer may be refilled
         float t[HK];
 #pragma unroll
-        for (int j = 0; j < HK; ++j) t[j] = key0 + j <= pv ? __uint_as_float(sr[j]) : -INFINITY;
+        for (int j = 0; j < HK; ++j) {
+          const float x = __uint_as_float(sr[j]) * p.qk_scale;
+          sr[j] = __float_as_uint(x);
+          t[j] = key0 + j <= pv ? x : -INFINITY;
+        }
 #pragma unroll
         for (int w = HK / 2; w > 0; w >>= 1)
 #pragma unroll
@@ -322,8 +344,9 @@ __global__ void __launch_bounds__(NT5, 1)
       if (dead) continue;
 #pragma unroll
       for (int o = 0; o < SMW; ++o) mx = fmaxf(mx, sx[b][o][v]);
-      // O is exactly zero until the first unmasked key: no rescale then
-      if (m == -INFINITY) m = mx;
+      // O is exactly zero until the first unmasked key: no rescale then.
+      // The reference is an integer (see the header).
+      if (m == -INFINITY) m = ceilf(mx);
       const bool grow = mx > m + RESCALE_LOG2;
       if (__any_sync(0xffffffffu, grow)) {
         if (i > 0) {  // O += P V of the previous chunk has landed
@@ -332,7 +355,8 @@ __global__ void __launch_bounds__(NT5, 1)
           if (dead) continue;
           tc_fence_after();
         }
-        const float alpha = grow ? ex2(m - mx) : 1.f;
+        const float mn = ceilf(mx);
+        const float alpha = grow ? ex2(m - mn) : 1.f;
 #pragma unroll
         for (int q = 0; q < OC / 16; ++q) {  // this part's O columns
           float o[16];
@@ -342,7 +366,7 @@ __global__ void __launch_bounds__(NT5, 1)
           tmem_st16(tl + 2 * CH + part * OC + q * 16, o);
         }
         l *= alpha;
-        if (grow) m = mx;
+        if (grow) m = mn;
       }
       // P buffer b was last read by O += P V of chunk i - 2
       if (i >= 2) {
@@ -494,10 +518,15 @@ const char *launch_attention_tc5(const void *q, const int32_t *pos, const int4 *
                                  int n_blocks, int n_splits, const Dims &dm, int layer,
                                  const void *pages, const int32_t *table, const CUtensorMap &tm_kv,
                                  float *ws_o, float2 *ws_ml, void *out, int *dev_flag,
-                                 cudaStream_t s) {
+                                 cudaStream_t s, const KVView *views,
+                                 const CUtensorMap *tmaps) {
   if (n_blocks <= 0) return nullptr;
+  if ((views == nullptr) != (tmaps == nullptr)) return "document views without tensor maps";
   Attn5Params p{};
+  p.views = views;
+  p.tmaps = tmaps;
   p.q = (const __nv_bfloat16 *)q;
+  p.qk_scale = (float)(1.4426950408889634 / std::sqrt((double)dm.dh));
   p.pos = pos;
   p.blocks = blocks;
   p.pages = (const __nv_bfloat16 *)pages;

@@ -73,14 +73,16 @@ struct TraceBuf {
   unsigned int cap = 0;
 };
 
-// silu(g) * u for the bf16 tensor-core GEMM's fused epilogue: the logistic
-// function through tanh, sigma(g) = (1 + tanh(g / 2)) / 2, on the hardware
-// tanh approximation (one special-function op per element; its relative
-// error, below 1e-3, is far under the bf16 rounding of the result).
+// silu(g) * u for the bf16 tensor-core GEMM's fused epilogue: g sigma(g) with
+// sigma(g) = 1 / (1 + 2^(-g log2 e)) from the hardware base-2 exponential and
+// reciprocal (relative error about 1e-7, so the bf16 rounding of the result is
+// that of the exact product up to rare ties; the hardware tanh, one op fewer,
+// is off by up to 1e-3, half a bf16 step).  Large |g| saturate to g or -0.
 __device__ __forceinline__ float swiglu_bf16path(float g, float u) {
-  float t;
-  asm("tanh.approx.f32 %0, %1;" : "=f"(t) : "f"(0.5f * g));
-  return 0.5f * g * (1.0f + t) * u;
+  float e, r;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(e) : "f"(-1.4426950408889634f * g));
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(1.0f + e));
+  return g * r * u;
 }
 
 // ---- split-K tiles reduced by the consumer ----
@@ -235,7 +237,7 @@ struct kvr_model {
   int32_t *pos_d = nullptr;  // [R] positions of the rows of a pass
   int32_t *rowdoc_d = nullptr;  // [R] batch: document of each row
   float *h = nullptr, *qkv = nullptr, *q = nullptr, *gu = nullptr, *logits = nullptr;
-  void *qb = nullptr;  // bf16 scaled q for the tensor-core attention
+  void *qb = nullptr;  // bf16 post-RoPE q for the tensor-core attention
   void *a = nullptr, *attn = nullptr, *act = nullptr;
   float *scores = nullptr;     // [max_ctx + reserve] selector scores
   unsigned long long *keys = nullptr;  // [max_ctx + reserve] top-K keys
@@ -245,6 +247,8 @@ struct kvr_model {
   size_t read_scratch_bytes = 0;
   void *sel_scratch = nullptr;   // selector: edited tokens, saved stale rows, probabilities
   size_t sel_scratch_bytes = 0;
+  void *batch_scratch = nullptr; // batched repair: documents' TMA views, cache views, tokens
+  size_t batch_scratch_bytes = 0;
   int *dev_flag = nullptr;     // device error flag (bounded waits)
   kvr::TraceBuf trace{};       // attached device timeline buffer, if any
   kvr::SplitView pending{};    // split tiles of h not yet added (next RMSNorm adds them)
@@ -517,7 +521,7 @@ void launch_attention_simt(const float *q, const int32_t *pos, int M, const Dims
 // chunks (ws_o/ws_ml hold the partials when n_splits > 1).
 int attn_tc_rows_per_block(int grp);
 size_t attn_tc_ws_floats(int n_splits, int n_blocks, int G, int dh);
-// q: bf16 [M][H*dh], rotated and scaled by log2(e)/sqrt(dh).
+// q: bf16 [M][H*dh], rotated (the kernels scale the scores by log2(e)/sqrt(dh)).
 const char *launch_attention_tc(const void *q, const int32_t *pos, const int4 *blocks,
                                 int n_blocks, int max_rows_per_block, int n_splits, const Dims &dm,
                                 int layer, const KVView *views, KVView single, float *ws_o,
@@ -529,16 +533,19 @@ const char *launch_attention_combine(const int4 *blocks, int n_blocks, int max_r
                                      int n_splits, const Dims &dm, float *ws_o, float2 *ws_ml,
                                      void *out, cudaStream_t s, const void *prefetch = nullptr,
                                      long long prefetch_bytes = 0);
-// tcgen05 attention of one document's rows (bf16 cache, head_dim 64 or 128):
-// query blocks of at most attn_tc5_rows_per_block(grp) rows; partials in the
-// same workspace layout as launch_attention_tc.  tm_kv: the cache's TMA view.
+// tcgen05 attention (bf16 cache, head_dim 64 or 128): query blocks of at most
+// attn_tc5_rows_per_block(grp) rows of one document each; partials in the
+// same workspace layout as launch_attention_tc.  One document: pages, table
+// and tm_kv (its TMA view).  Several: views and tmaps, device arrays indexed
+// by a block's document (blocks[].w), tmaps 64-byte aligned.
 int attn_tc5_rows_per_block(int grp);
 int attn_tc5_ctas_per_sm(int dh);
 const char *launch_attention_tc5(const void *q, const int32_t *pos, const int4 *blocks,
                                  int n_blocks, int n_splits, const Dims &dm, int layer,
                                  const void *pages, const int32_t *table, const CUtensorMap &tm_kv,
                                  float *ws_o, float2 *ws_ml, void *out, int *dev_flag,
-                                 cudaStream_t s);
+                                 cudaStream_t s, const KVView *views = nullptr,
+                                 const CUtensorMap *tmaps = nullptr);
 
 // ---- kernels: selectors ----
 // bound: device int holding n - 1 (EditLocal@boundary writes the first

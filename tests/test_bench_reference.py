@@ -24,9 +24,11 @@ def test_reference_arm_line():
     assert d["config"] == bench.workload_config(synth.preset(bench.WORKLOAD), 1)
     assert d["steps"] == 1 and d["warmup"] == 3 and d["n_gpus"] == 1
     assert d["higher_is_better"] is True and d["vs_baseline"] is None
-    assert d["value"] > 0 and abs(d["value"] * d["ms_per_step"] / 1e3 - 40) < 1e-6
+    # a step is the 40 rows through the first layers_per_step of 32 layers, as it ran
+    assert d["layers_per_step"] == 1 and d["layers_per_position"] == 32
+    assert d["value"] > 0 and abs(d["value"] * d["ms_per_step"] / 1e3 - 40 / 32) < 1e-9
     cb = d["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["value"] == d["value"] and cb["cores"] >= 1
-    assert "1 of 32 layers" in cb["sample"]
+    assert "first 1 of 32 layers" in cb["sample"]
     assert d["e2e"] == {"value": d["value"], "unit": "positions/s", "h2d_bytes_per_step": 0,
                         "d2h_bytes_per_step": 0}

@@ -9,8 +9,15 @@ same bits reach the GPU (``kvr_cache_load``) and the oracle.  Nothing the
 oracle receives comes from the CUDA path: weights and tokens are seeded,
 positions are the oracle's own selections.
 
-Tolerances are those of the other parity tests: max|gpu - ref| / max|ref| <=
-2e-2 per layer, for K and V over the repaired rows, and for the logits.
+The oracle runs the bf16 path (every operand of a matrix product in bf16,
+sums in double).  Tolerance: max|gpu - ref| / max|ref| <= 2e-2 per layer, for
+K and V over the repaired rows, and for the logits -- or, where more, twice
+the oracle's own null control at that depth: the same bf16 path with its
+sums and residual rounded to fp32 (the arithmetic the bf16 path specifies),
+compared with the double-sum run.  On these random-init models a last-bit
+change of the sums grows with depth to about 2% of the largest entry by
+layer 31, so at depth that measured spread, not 2e-2, is what any
+implementation of the path can promise; near the input the 2e-2 bound holds.
 Selections must match the oracle's top-K except where the oracle scores of
 swapped positions lie within 2e-2 * max|score| of the K-th score.
 """
@@ -92,14 +99,25 @@ def oracle_cache(k, v, tokens, layers=None):
     return oracle.Cache(kf, vf, np.asarray(tokens, np.int32).copy())
 
 
-def compare_rows(gk, gv, ref, P):
+def null_cfg(cfg):
+    """The oracle's null control of the bf16 path: sums rounded to fp32."""
+    return dict(cfg, operands="bf16_f32sums")
+
+
+def compare_rows(gk, gv, ref, null, P, name):
     """GPU rows [m][L][G][dh] (fp32) against the oracle cache at positions P,
-    per layer, K and V separately; returns the worst relative error."""
-    worst = 0.0
+    per layer, K and V separately, each within max(TOL, 2 x the null
+    control's distance from the oracle at that layer); prints the table and
+    returns the worst error relative to its bound."""
+    worst, lines = 0.0, []
     for l in range(gk.shape[1]):
         ek, ev = rel(gk[:, l], ref.k[l, P]), rel(gv[:, l], ref.v[l, P])
-        worst = max(worst, ek, ev)
-        assert ek <= TOL and ev <= TOL, (l, ek, ev)
+        nk, nv = rel(null.k[l, P], ref.k[l, P]), rel(null.v[l, P], ref.v[l, P])
+        tk, tv = max(TOL, 2 * nk), max(TOL, 2 * nv)
+        worst = max(worst, ek / tk, ev / tv)
+        lines.append(f"{l}:{max(ek, ev):.4f}/{max(nk, nv):.4f}")
+        assert ek <= tk and ev <= tv, (name, l, ek, ev, nk, nv)
+    print(f"{name} per layer gpu/null: " + " ".join(lines))
     return worst
 
 
@@ -144,10 +162,13 @@ def test_llama8b_full_depth_repair_logits_and_margin():
     W = host_weights(cfg, np.concatenate([edited[P], query, prompt, a_new, a_old]),
                      lm_head=True)
     ref = oracle.repair(cfg, W, oracle_cache(k, v, doc), new, s, A)
+    null = oracle.repair(null_cfg(cfg), W, oracle_cache(k, v, doc), new, s, A)
     del k, v
-    worst = compare_rows(gk, gv, ref, P)
+    worst = compare_rows(gk, gv, ref, null, P, "llama8b")
     rlog = oracle.logits(cfg, W, ref, query)
-    assert rel(glog, rlog) <= TOL, rel(glog, rlog)
+    nlog = oracle.logits(null_cfg(cfg), W, null, query)
+    tlog = max(TOL, 2 * rel(nlog, rlog))
+    assert rel(glog, rlog) <= tlog, (rel(glog, rlog), rel(nlog, rlog))
     # answer log-probabilities: lp = logit(target) - logsumexp(logits), so an
     # error of at most e in every logit moves lp by at most 2e; e is the logits
     # tolerance times the largest logit of the answer rows
@@ -155,15 +176,16 @@ def test_llama8b_full_depth_repair_logits_and_margin():
     for name, a in (("new", a_new), ("old", a_old)):
         feed = np.concatenate([prompt, a[:-1]])
         rows = oracle.logits_all(cfg, W, ref, feed)[len(prompt) - 1:]
-        bound[name] = 2 * TOL * float(np.abs(rows).max())
+        bound[name] = 2 * tlog * float(np.abs(rows).max())
     r_new = oracle.answer_logprob(cfg, W, ref, prompt, a_new)
     r_old = oracle.answer_logprob(cfg, W, ref, prompt, a_old)
     assert abs(g_new - r_new) <= bound["new"], (g_new, r_new, bound)
     assert abs(g_old - r_old) <= bound["old"], (g_old, r_old, bound)
     assert abs(g_margin - (g_new - g_old)) <= 1e-12 * max(1.0, abs(g_margin))
     assert abs(g_margin - (r_new - r_old)) <= bound["new"] + bound["old"]
-    print(f"llama8b full depth: worst K/V rel err {worst:.2e}, logits {rel(glog, rlog):.2e}, "
-          f"margin gpu {g_margin:.4f} oracle {r_new - r_old:.4f}")
+    print(f"llama8b full depth: worst K/V error {worst:.2f} of its bound, logits "
+          f"{rel(glog, rlog):.2e} (null control {rel(nlog, rlog):.2e}), margin gpu "
+          f"{g_margin:.4f} oracle {r_new - r_old:.4f} bound {bound['new'] + bound['old']:.3f}")
 
 
 def test_qwen7b_full_depth_attention_selector_and_repair():
@@ -198,9 +220,10 @@ def test_qwen7b_full_depth_attention_selector_and_repair():
     cache.close()
     m.close()
     ref = oracle.repair(cfg, W, oracle_cache(k, v, doc), new, s, A)
-    worst = compare_rows(gk, gv, ref, P)
+    null = oracle.repair(null_cfg(cfg), W, oracle_cache(k, v, doc), new, s, A)
+    worst = compare_rows(gk, gv, ref, null, P, "qwen7b")
     print(f"qwen7b full depth: attention selections within the tie band for K in {w['Ks']}, "
-          f"worst K/V rel err {worst:.2e}")
+          f"worst K/V error {worst:.2f} of its bound")
 
 
 def test_mistral7b_full_size_cacheblend_selector():

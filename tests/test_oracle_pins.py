@@ -92,6 +92,35 @@ def test_prefill_matches_textbook_decoder(bias):
     np.testing.assert_allclose(h, hr, rtol=0, atol=1e-6 * np.abs(hr).max())
 
 
+@pytest.mark.parametrize("bias", [False, True])
+def test_bf16_path_matches_textbook_decoder(bias):
+    # The oracle's bf16 path (a bf16 model's default: every operand of a matrix
+    # product rounded to bf16, the cache in bf16, sums in double) against the
+    # textbook decoder with the same rounding points, made by torch's own
+    # conversions, its library products and an attention written out over all
+    # heads at once.  The values before each rounding agree to double
+    # precision, so every rounding lands the same way: agreement to 1e-9.
+    cfg, W, doc, s, new = small_workload(dtype="bf16", qkv_bias=bias)
+    query = synth.fill_tokens(98, 5, cfg["vocab"], cfg["delim_id"])
+    ref = textbook.forward(cfg, W, np.concatenate([doc, query]), operands="bf16")
+    got = oracle.prefill(cfg, W, doc)
+    n = len(doc)
+    for l in range(cfg["n_layers"]):
+        k = textbook.bf16(ref["layers"][l]["k"][:n]).numpy()
+        v = textbook.bf16(ref["layers"][l]["v"][:n]).numpy()
+        np.testing.assert_allclose(got.k[l], k, rtol=0, atol=1e-9 * np.abs(k).max())
+        np.testing.assert_allclose(got.v[l], v, rtol=0, atol=1e-9 * np.abs(v).max())
+    lg = oracle.logits(cfg, W, got, query)
+    rl = ref["logits"][-1].numpy()
+    np.testing.assert_allclose(lg, rl, rtol=0, atol=1e-9 * np.abs(rl).max())
+    # and it is a different computation from the double one: at layer 0 the
+    # rounded operands move K by at most a few bf16 steps
+    exact = oracle.prefill(dict(cfg, operands="fp64"), W, doc)
+    d0 = np.abs(exact.k[0].astype(np.float64) - got.k[0]).max()
+    assert 0 < d0 <= 2.0 ** -6 * np.abs(exact.k[0]).max()
+    assert not np.array_equal(exact.k[-1], got.k[-1])
+
+
 def test_logits_match_textbook_decoder():
     cfg, W, doc, s, new = small_workload()
     query = synth.fill_tokens(99, 5, cfg["vocab"], cfg["delim_id"])
