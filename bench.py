@@ -224,8 +224,8 @@ def run_reference(args, cfg, rank):
 # DRAM bytes (read + write) of one gate/up GEMM launch at this workload's shape
 # (40 x 28672 x 4096), from one ncu capture of that launch; reported only while the
 # GEMM kernel's source is the one the capture was taken on.
-GU_TRAFFIC_BYTES = 235293696 + 4597760
-GU_TRAFFIC_SOURCE_SHA256 = "cf8edeeaa92c5a2694529c8c6cb3f63d064c0843eec4aaced7b1a114f5f711de"
+GU_TRAFFIC_BYTES = 235282432 + 2532608
+GU_TRAFFIC_SOURCE_SHA256 = "ecbcbd0008452f3092e11bb7a240b0914a64dff6ea6883cbceb89c547ce0c6eb"
 
 
 def workload_config(cfg: dict, world: int) -> dict:

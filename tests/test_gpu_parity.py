@@ -357,6 +357,41 @@ def test_repair_batch_parity_fp32():
     model.close()
 
 
+@pytest.mark.parametrize("n_docs", [3, 20])
+def test_repair_batch_parity_bf16(n_docs):
+    # several documents in one pass on the tcgen05 attention (each block's
+    # document has its own page table and TMA view), against the oracle's
+    # per-document repair; 20 documents of about 40 rows each give many query
+    # blocks and no key splits, 3 documents give key splits and the combine
+    cfg = synth.preset("tiny", dtype="bf16", qkv_bias=True)
+    W = synth.weights(cfg, 0)
+    model = kv.Model(cfg, W, max_context=1024, max_rows=1024)
+    docs = [synth.document(50 + i, 300 + 23 * i, cfg["vocab"]) for i in range(n_docs)]
+    caches = [model.prefill(d) for d in docs]
+    reqs, refs = [], []
+    for i, (d, c) in enumerate(zip(docs, caches)):
+        s0 = 40 + 7 * i
+        edits = [(s0, synth.edit_tokens(60 + i, d[s0:s0 + 3], cfg["vocab"])),
+                 (s0 + 120, synth.edit_tokens(80 + i, d[s0 + 120:s0 + 122], cfg["vocab"]))]
+        A = np.concatenate([np.arange(s0 + 3, s0 + 19), np.arange(s0 + 122, s0 + 140)])
+        reqs.append((c, edits, A))
+        toks = d.copy()
+        P = list(A)
+        for st, nt in edits:
+            toks[st:st + len(nt)] = nt
+            P += list(range(st, st + len(nt)))
+        P = np.array(sorted(P))
+        ref = oracle.prefill(cfg, W, d)
+        ref.tokens = toks
+        oracle.recompute(cfg, W, ref, toks, P)
+        refs.append((ref, P))
+    model.repair_batch(reqs)
+    for c, (ref, P) in zip(caches, refs):
+        cmp_rows(c, ref, P, TOL["bf16"])
+        assert np.array_equal(c.tokens(), ref.tokens)
+    model.close()
+
+
 # ------------------------------------------------------------ error paths
 
 def test_range_errors_leave_cache_unchanged(tiny):
