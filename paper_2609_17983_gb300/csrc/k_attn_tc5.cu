@@ -114,7 +114,9 @@ __global__ void __launch_bounds__(NT5, 1)
   __shared__ float ssum[SMW][QV];   // per key part: sums of exponentials
 
   TraceScope ts(TK_ATTN);
-  const int split = blockIdx.x, g = blockIdx.y, blk = blockIdx.z;
+  // blocks in descending order: a document's later blocks see more keys, so
+  // the longest CTAs launch first and the last wave holds the shortest
+  const int split = blockIdx.x, g = blockIdx.y, blk = gridDim.z - 1 - blockIdx.z;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   // block table, positions and page table are written before the pass
   const int4 bd = p.blocks[blk];
