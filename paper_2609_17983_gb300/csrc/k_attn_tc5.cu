@@ -20,13 +20,17 @@
 //                  when the running maximum exceeds it by more than 8 (so
 //                  P <= 256); with an integer reference, bf16(P) is a power
 //                  of two times the rounding of 2^(x - E) for any integer E,
-//                  whichever chunk set it; P in bf16 written to one
-//                  of two shared-memory buffers as the next MMA's A operand,
-//                  so the softmax of chunk i overlaps O += P V of chunk i-1;
+//                  whichever chunk set it; P in bf16 written with
+//                  tcgen05.st to one of two tensor-memory buffers as the next
+//                  MMA's A operand, so the softmax of chunk i overlaps
+//                  O += P V of chunk i-1;
 //   O += P V       tcgen05.mma, M 128 x N head_dim x K 64, V read MN-major
 //                  straight from the page layout [key][head_dim].
-// K and V tiles arrive by TMA (128-byte swizzle, KV_STAGES stages deep, so a
-// chunk's load is issued long before its MMA); Q by cp.async.
+// Both MMAs take A (Q, then P) from tensor memory and only B (K, then V) from
+// shared memory, so a chunk's shared-memory traffic is its K and V tiles, each
+// written once by TMA and read once by an MMA.  K and V tiles arrive by TMA
+// (128-byte swizzle, KV_STAGES stages deep, so a chunk's load is issued long
+// before its MMA); the softmax warps write Q into tensor memory once.
 // With several key splits the CTA writes its unnormalised O and (max, sum)
 // for the combine kernel, else the normalised output.
 //
@@ -52,7 +56,14 @@ constexpr int CH = KVR_PAGE;     // keys per chunk
 constexpr int SMW = 4;           // softmax warps per TMEM lane quarter
 constexpr int NT5 = 64 + 128 * SMW;  // threads per CTA
 constexpr int WS_MAXQ = 192;     // query slots per (split, block, head) of the split workspace
-constexpr uint32_t TMEM_COLS = 256;  // S buffers at columns 0 and 64, O from column 128
+// Tensor-memory columns: S buffers at 0 and 64, O (head_dim columns) at 128,
+// Q (head_dim / 2 columns of bf16 pairs) at T_Q, P buffers (32 columns each) at T_P.
+constexpr uint32_t TMEM_COLS = 512;
+constexpr uint32_t T_Q = 256, T_P = 320;
+// Holding all of TMEM cannot stall on another grid: the other kernel that
+// allocates TMEM (the GEMM) cannot share an SM with this one (their register
+// files together exceed the SM's), and dependents launch only after every CTA
+// here holds its columns.
 constexpr int SOFTMAX_THREADS = 128 * SMW;
 constexpr float RESCALE_LOG2 = 8.f;  // headroom of the reference maximum (P <= 2^8)
 constexpr int KV_STAGES = 4;
@@ -76,8 +87,28 @@ struct Attn5Params {
   int *dev_flag;
 };
 
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+// A from tensor memory: row m of A in TMEM lane m, two bf16 of K per 32-bit
+// column (K-major), a_tmem the column of its first K element; B a shared-memory
+// descriptor.
+__device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b,
+                                            uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// 8 consecutive 32-bit TMEM columns of the warp's 32 lanes, one lane per
+// thread, without the wait (tmem_wait_st before the data is consumed).
+__device__ __forceinline__ void tmem_st8_nowait(uint32_t taddr, const uint32_t *r) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7])
+      : "memory");
+}
+__device__ __forceinline__ void tmem_wait_st() {
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 
 __device__ __forceinline__ uint32_t pack2(float lo, float hi) {
@@ -91,16 +122,10 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
-// byte offset of 16-byte chunk c of row r in a [rows][128 B] 128-byte-swizzled tile
-__device__ __forceinline__ uint32_t sw_off(int r, int c) {
-  return (uint32_t)((r >> 3) * 1024 + (r & 7) * 128 + ((c ^ (r & 7)) << 4));
-}
-
 template <int DH>
 __global__ void __launch_bounds__(NT5, 1)
     k_attn_tc5(const __grid_constant__ CUtensorMap tm_kv, const Attn5Params p) {
   constexpr int HALVES = DH / 64;           // 128-byte column blocks of a row
-  constexpr uint32_t QBYTES = QV * 128 * HALVES;
   constexpr uint32_t TBYTES = CH * 128 * HALVES;  // one K (or V) tile
   constexpr uint32_t KVBYTES = 2 * TBYTES;
   extern __shared__ uint8_t smem_raw[];
@@ -136,7 +161,7 @@ __global__ void __launch_bounds__(NT5, 1)
   }
   const int nch = c1 - c0;
   const uint32_t base = (su32(smem_raw) + 1023u) & ~1023u;
-  const uint32_t sQ = base, sKV = sQ + QBYTES, sP = sKV + KV_STAGES * KVBYTES;  // P: two tiles
+  const uint32_t sKV = base;
   volatile int *abort_v = &abort_f;
   auto page_row = [&](int c, int kv) {  // first row of (chunk c, kv) in the pool's 2D view
     const long long pg = table[c];
@@ -237,10 +262,9 @@ __global__ void __launch_bounds__(NT5, 1)
         tc_fence_after();
         const uint32_t sk = sKV + st * KVBYTES;
 #pragma unroll
-        for (int kk = 0; kk < DH / 16; ++kk) {
-          const uint64_t a = sw128_desc(sQ + (kk >> 2) * QV * 128 + (kk & 3) * 32);
+        for (int kk = 0; kk < DH / 16; ++kk) {  // 16 elements of head_dim: 8 columns of Q
           const uint64_t bb = sw128_desc(sk + (kk >> 2) * CH * 128 + (kk & 3) * 32);
-          mma_bf16(tmem + b * CH, a, bb, id_s, kk > 0 ? 1u : 0u);
+          mma_bf16_ts(tmem + b * CH, tmem + T_Q + kk * 8, bb, id_s, kk > 0 ? 1u : 0u);
         }
         mma_commit(&s_full[b]);
         return true;
@@ -251,15 +275,14 @@ __global__ void __launch_bounds__(NT5, 1)
         if (!(ok = mbar_wait(&p_full[i & 1], (i >> 1) & 1, abort_v, p.dev_flag, 68))) break;
         tc_fence_after();
         const uint32_t sv = sKV + (i % KV_STAGES) * KVBYTES + TBYTES;
-        const uint32_t sp = sP + (i & 1) * QV * CH * 2;
+        const uint32_t tp = tmem + T_P + (i & 1) * (CH / 2);
 #pragma unroll
         for (int kk = 0; kk < CH / 16; ++kk) {
-          // P: K-major rows of 64 keys.  V: keys are the rows (K), head_dim
-          // runs along them (MN-major) in 64-wide column blocks CH*128 bytes
-          // apart, 8-key groups 1024 bytes apart.
-          const uint64_t a = sw128_desc(sp + kk * 32);
+          // P: a TMEM lane per query vector, 16 keys in 8 columns.  V: keys
+          // are the rows (K), head_dim runs along them (MN-major) in 64-wide
+          // column blocks CH*128 bytes apart, 8-key groups 1024 bytes apart.
           const uint64_t bb = sw128_desc_mn(sv + kk * 2048, CH * 128, 1024);
-          mma_bf16(tmem + 2 * CH, a, bb, id_o, (i > 0 || kk > 0) ? 1u : 0u);
+          mma_bf16_ts(tmem + 2 * CH, tp + kk * 8, bb, id_o, (i > 0 || kk > 0) ? 1u : 0u);
         }
         mma_commit(&o_done[i & 1]);
         mma_commit(&kv_empty[i % KV_STAGES]);
@@ -284,24 +307,27 @@ __global__ void __launch_bounds__(NT5, 1)
       asm volatile("bar.sync %0, %1;" ::"r"(bar_id), "n"(32 * SMW) : "memory");
     };
     pdl_wait();
-    // this thread's part of the Q row, into the swizzled K-major tile
+    // this thread's part of the Q row (DH / SMW elements, zero past the
+    // block's query vectors) into the TMEM lane of query vector v
     {
+      constexpr int QW = DH / (2 * SMW);  // 32-bit words (columns) of this part
       const bool real = v < mq;
-      const __nv_bfloat16 *src =
-          p.q + ((size_t)(row0 + (real ? v / p.grp : 0)) * p.H + g * p.grp + v % p.grp) * DH;
+      const uint4 *src = (const uint4 *)(p.q + ((size_t)(row0 + (real ? v / p.grp : 0)) * p.H +
+                                                g * p.grp + v % p.grp) * DH) +
+                         part * (QW / 4);
+      uint32_t w[QW];
 #pragma unroll
-      for (int k = 0; k < DH / (8 * SMW); ++k) {
-        const int ch = part * (DH / (8 * SMW)) + k;
-        const uint32_t dst = sQ + (ch >> 3) * QV * 128 + sw_off(v, ch & 7);
-        if (real)
-          cp_async16(dst, src + ch * 8);
-        else
-          asm volatile("st.shared.v4.u32 [%0], {%1, %1, %1, %1};" ::"r"(dst), "r"(0u)
-                       : "memory");
+      for (int k = 0; k < QW / 4; ++k) {
+        const uint4 x = real ? src[k] : make_uint4(0u, 0u, 0u, 0u);
+        w[4 * k] = x.x;
+        w[4 * k + 1] = x.y;
+        w[4 * k + 2] = x.z;
+        w[4 * k + 3] = x.w;
       }
-      asm volatile("cp.async.commit_group;" ::: "memory");
-      asm volatile("cp.async.wait_group 0;" ::: "memory");
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+#pragma unroll
+      for (int k = 0; k < QW / 8; ++k) tmem_st8_nowait(tl + T_Q + part * QW + k * 8, w + 8 * k);
+      tmem_wait_st();
+      tc_fence_before();
       mbar_arrive(&q_full);
       if (warp == 2 && lane == 0) trace_mark(2);
     }
@@ -376,20 +402,18 @@ __global__ void __launch_bounds__(NT5, 1)
                                                   p.dev_flag, 72));
         if (dead) continue;
       }
-      const uint32_t prow =
-          sP + b * QV * CH * 2 + (uint32_t)((v >> 3) * 1024 + (v & 7) * 128);
       float e[HK];
 #pragma unroll
       for (int j = 0; j < HK; ++j) e[j] = key0 + j <= pv ? ex2(__uint_as_float(sr[j]) - m) : 0.f;
+      {  // P in bf16 pairs: this part's HK keys are HK / 2 columns of buffer b
+        uint32_t w[HK / 2];
 #pragma unroll
-      for (int q = 0; q < HK / 8; ++q) {
-        const uint32_t d = prow + (((part * (HK / 8) + q) ^ (v & 7)) << 4);
-        asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(d),
-                     "r"(pack2(e[q * 8], e[q * 8 + 1])), "r"(pack2(e[q * 8 + 2], e[q * 8 + 3])),
-                     "r"(pack2(e[q * 8 + 4], e[q * 8 + 5])), "r"(pack2(e[q * 8 + 6], e[q * 8 + 7]))
-                     : "memory");
+        for (int j = 0; j < HK / 2; ++j) w[j] = pack2(e[2 * j], e[2 * j + 1]);
+#pragma unroll
+        for (int q = 0; q < HK / 16; ++q)
+          tmem_st8_nowait(tl + T_P + b * (CH / 2) + part * (HK / 2) + q * 8, w + 8 * q);
       }
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      tmem_wait_st();
       tc_fence_before();
       mbar_arrive(&p_full[b]);
 #pragma unroll
@@ -476,8 +500,7 @@ __global__ void __launch_bounds__(NT5, 1)
 
 template <int DH>
 constexpr size_t smem_bytes() {
-  return 1024 + (size_t)QV * 128 * (DH / 64) + KV_STAGES * 2 * (size_t)CH * 128 * (DH / 64) +
-         2 * (size_t)QV * CH * 2;
+  return 1024 + KV_STAGES * 2 * (size_t)CH * 128 * (DH / 64);
 }
 
 template <int DH>
@@ -500,21 +523,8 @@ const char *run(const CUtensorMap &tm, const Attn5Params &p, cudaStream_t s) {
 
 int attn_tc5_rows_per_block(int grp) { return grp <= QV ? QV / grp : 0; }
 
-int attn_tc5_ctas_per_sm(int dh) {
-  static int cached[2] = {-1, -1};
-  const int k = dh == 128 ? 1 : 0;
-  if (cached[k] < 0) {
-    int n = 0;
-    size_t smem = dh == 128 ? smem_bytes<128>() : smem_bytes<64>();
-    const void *fn = dh == 128 ? (const void *)k_attn_tc5<128> : (const void *)k_attn_tc5<64>;
-    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
-            cudaSuccess ||
-        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fn, NT5, smem) != cudaSuccess)
-      n = 1;
-    cached[k] = n < 1 ? 1 : (n > 2 ? 2 : n);  // TMEM holds two CTAs' 256 columns
-  }
-  return cached[k];
-}
+// A CTA allocates all 512 tensor-memory columns of its SM.
+int attn_tc5_ctas_per_sm(int) { return 1; }
 
 const char *launch_attention_tc5(const void *q, const int32_t *pos, const int4 *blocks,
                                  int n_blocks, int n_splits, const Dims &dm, int layer,
