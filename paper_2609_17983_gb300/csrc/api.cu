@@ -104,14 +104,22 @@ void prof_collect(kvr_model *m) {
 // ------------------------------------------------------------ staging
 
 // Copy host int32 data to device through the model's pinned staging buffer.
+// Copies take consecutive 128-byte-aligned slots, so a call does not wait for
+// the copies queued before it; when the next slot would not fit, the buffer
+// starts over after every queued copy has completed.
 kvr_status stage_h2d(kvr_model *m, int32_t *dst_dev, const int32_t *src, size_t count) {
   if (count == 0) return KVR_OK;
   if (count > m->stage_cap) return fail(KVR_E_UNSUPPORTED, "staging overflow (%zu)", count);
-  CUDA_TRY(cudaEventSynchronize(m->stage_ev));
-  memcpy(m->stage_h, src, count * sizeof(int32_t));
-  CUDA_TRY(cudaMemcpyAsync(dst_dev, m->stage_h, count * sizeof(int32_t), cudaMemcpyHostToDevice,
+  if (m->stage_off + count > m->stage_cap) {
+    CUDA_TRY(cudaEventSynchronize(m->stage_ev));
+    m->stage_off = 0;
+  }
+  int32_t *h = m->stage_h + m->stage_off;
+  memcpy(h, src, count * sizeof(int32_t));
+  CUDA_TRY(cudaMemcpyAsync(dst_dev, h, count * sizeof(int32_t), cudaMemcpyHostToDevice,
                            m->stream));
   CUDA_TRY(cudaEventRecord(m->stage_ev, m->stream));
+  m->stage_off += (count + 31) / 32 * 32;
   return KVR_OK;
 }
 
@@ -555,6 +563,7 @@ void kvr_model_free(kvr_model *m) {
   dev_free(m->attn_ws_o);
   dev_free(m->attn_ws_ml);
   if (m->stage_h) cudaFreeHost(m->stage_h);
+  if (m->rb_h) cudaFreeHost(m->rb_h);
   if (m->stage_ev) cudaEventDestroy(m->stage_ev);
   delete m;
 }
@@ -770,6 +779,8 @@ kvr_status kvr_model_create(const kvr_model_config *cfg, const kvr_weights *wts,
       return bail(fail(KVR_E_NOMEM, "pinned staging"));
     cudaEventCreateWithFlags(&m->stage_ev, cudaEventDisableTiming);
     cudaEventRecord(m->stage_ev, 0);
+    if (cudaMallocHost(&m->rb_h, ((size_t)P + 8) * sizeof(int32_t)) != cudaSuccess)
+      return bail(fail(KVR_E_NOMEM, "pinned readback"));
   }
   // ---- tensor-core GEMM: workspace and weight TMA descriptors
   if (dm.dtype == KVR_DTYPE_BF16) {
@@ -1371,16 +1382,27 @@ kvr_status kvr_select(kvr_model *m, const kvr_cache *c, kvr_policy policy, int32
     const char *e = launch_topk(m->keys, n, s_end, topk_k, m->sel_out, m->sel_count, m->stream);
     st = e ? fail(KVR_E_CUDA, "top-K over %d candidates: %s", n - s_end, e) : launch_check(m, 1);
   }
+  // one readback: the count, the device error flag and up to K positions
   int32_t cnt = 0;
-  if (!st && (cudaMemcpyAsync(&cnt, m->sel_count, 4, cudaMemcpyDeviceToHost, m->stream) ||
-              cudaStreamSynchronize(m->stream)))
-    st = fail(KVR_E_CUDA, "select readback");
-  if (!st && cnt > 0 &&
-      (cudaMemcpyAsync(positions_out, m->sel_out, (size_t)cnt * 4, cudaMemcpyDeviceToHost,
-                       m->stream) ||
-       cudaStreamSynchronize(m->stream)))
-    st = fail(KVR_E_CUDA, "select readback");
-  if (!st) st = sync_model(m);
+  if (!st) {
+    const int kmax = std::min(K, n - s_end);
+    int32_t *rb = m->rb_h;
+    cudaError_t e = cudaMemcpyAsync(rb, m->sel_count, 4, cudaMemcpyDeviceToHost, m->stream);
+    if (e == cudaSuccess)
+      e = cudaMemcpyAsync(rb + 1, m->dev_flag, 4, cudaMemcpyDeviceToHost, m->stream);
+    if (e == cudaSuccess && kmax > 0)
+      e = cudaMemcpyAsync(rb + 2, m->sel_out, (size_t)kmax * 4, cudaMemcpyDeviceToHost,
+                          m->stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(m->stream);
+    if (e != cudaSuccess) {
+      st = fail(KVR_E_CUDA, "select readback: %s", cudaGetErrorString(e));
+    } else if (rb[1]) {
+      st = sync_model(m);  // reports the bounded wait that ran out and clears the flag
+    } else {
+      cnt = std::min(rb[0], kmax);
+      std::copy(rb + 2, rb + 2 + cnt, positions_out);
+    }
+  }
   cudaStreamSynchronize(m->stream);
   if (!st) *count_out = cnt;
   return st;

@@ -258,7 +258,9 @@ struct kvr_model {
   int32_t *stage_h = nullptr;
   int32_t *stage_d = nullptr;
   size_t stage_cap = 0;
-  cudaEvent_t stage_ev = nullptr;
+  size_t stage_off = 0;           // next free slot (copies take consecutive slots)
+  cudaEvent_t stage_ev = nullptr;  // recorded after the last staged copy
+  int32_t *rb_h = nullptr;         // pinned readback: selector count, flag, positions
   // profiling
   bool prof = false;
   std::vector<kvr::ProfClass> prof_classes;
