@@ -1255,18 +1255,26 @@ kvr_status kvr_select(kvr_model *m, const kvr_cache *c, kvr_policy policy, int32
     st = fail(KVR_E_CUDA, "token copy");
   if (!st && edit_len) st = stage_h2d(m, toks + edit_start, new_tokens, edit_len);
   int topk_k = K;
+  SimpleKeys gen;  // simple policies: keys made inside the top-K kernel
   void *save = nullptr;
   void *probs = nullptr;  // Attention: the selector workspace
   if (!st && (policy == KVR_POLICY_EDITLOCAL || policy == KVR_POLICY_STRUCTURAL ||
               policy == KVR_POLICY_RANDOM || policy == KVR_POLICY_EDITLOCAL_BOUNDARY)) {
-    Prof pr(m, P_SELECT, 0);
     int *bound = (int *)(m->sel_count + 1);
-    int init = n - 1;
-    if (policy == KVR_POLICY_EDITLOCAL_BOUNDARY) st = stage_h2d(m, bound, &init, 1);
-    if (!st) {
-      launch_scores_simple(policy, toks, n, s_end, dm.delim, seed, bound, m->keys, m->stream);
-      st = launch_check(m, policy == KVR_POLICY_EDITLOCAL_BOUNDARY ? 2 : 1);
+    if (policy == KVR_POLICY_EDITLOCAL_BOUNDARY) {
+      Prof pr(m, P_SELECT, 0);
+      int init = n - 1;
+      st = stage_h2d(m, bound, &init, 1);
+      if (!st) {
+        launch_first_delim(toks, n, s_end, dm.delim, bound, m->stream);
+        st = launch_check(m, 1);
+      }
     }
+    gen.policy = (int)policy;
+    gen.tokens = toks;
+    gen.delim = dm.delim;
+    gen.seed = seed;
+    gen.bound = bound;
     if (policy == KVR_POLICY_STRUCTURAL || policy == KVR_POLICY_EDITLOCAL_BOUNDARY) topk_k = -K;
   } else if (!st && policy == KVR_POLICY_ATTENTION) {
     if (edit_len == 0) {
@@ -1379,7 +1387,9 @@ kvr_status kvr_select(kvr_model *m, const kvr_cache *c, kvr_policy policy, int32
   }
   if (!st) {
     Prof pr(m, P_SELECT, 0);
-    const char *e = launch_topk(m->keys, n, s_end, topk_k, m->sel_out, m->sel_count, m->stream);
+    // sel_out: [count][device flag][positions ...], read back in one copy
+    const char *e = launch_topk(m->keys, n, s_end, topk_k, m->sel_out + 2, m->sel_out,
+                                m->stream, gen, m->dev_flag, m->sel_out + 1);
     st = e ? fail(KVR_E_CUDA, "top-K over %d candidates: %s", n - s_end, e) : launch_check(m, 1);
   }
   // one readback: the count, the device error flag and up to K positions
@@ -1387,12 +1397,8 @@ kvr_status kvr_select(kvr_model *m, const kvr_cache *c, kvr_policy policy, int32
   if (!st) {
     const int kmax = std::min(K, n - s_end);
     int32_t *rb = m->rb_h;
-    cudaError_t e = cudaMemcpyAsync(rb, m->sel_count, 4, cudaMemcpyDeviceToHost, m->stream);
-    if (e == cudaSuccess)
-      e = cudaMemcpyAsync(rb + 1, m->dev_flag, 4, cudaMemcpyDeviceToHost, m->stream);
-    if (e == cudaSuccess && kmax > 0)
-      e = cudaMemcpyAsync(rb + 2, m->sel_out, (size_t)kmax * 4, cudaMemcpyDeviceToHost,
-                          m->stream);
+    cudaError_t e = cudaMemcpyAsync(rb, m->sel_out, (size_t)(kmax + 2) * 4,
+                                    cudaMemcpyDeviceToHost, m->stream);
     if (e == cudaSuccess) e = cudaStreamSynchronize(m->stream);
     if (e != cudaSuccess) {
       st = fail(KVR_E_CUDA, "select readback: %s", cudaGetErrorString(e));

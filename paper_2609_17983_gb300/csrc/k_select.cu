@@ -34,23 +34,20 @@ __global__ void k_first_delim(const int32_t *tokens, int n, int s_end, int delim
     if (tokens[j] == delim) atomicMin(bound, j);
 }
 
-__global__ void k_scores_simple(int policy, const int32_t *tokens, int n, int s_end, int delim,
-                                uint64_t seed, const int *bound, unsigned long long *keys) {
-  int c = n - s_end;
-  for (int t = blockIdx.x * blockDim.x + threadIdx.x; t < c; t += gridDim.x * blockDim.x) {
-    int j = s_end + t;
-    unsigned long long k;
-    if (policy == KVR_POLICY_RANDOM) {
-      // first SplitMix64 output of state seed ^ (j * gamma)
-      k = mix64((seed ^ ((uint64_t)j * GAMMA)) + GAMMA);
-    } else {
-      // nearest to the span first
-      k = 0x100000000ull - (unsigned long long)t;
-      if (policy == KVR_POLICY_STRUCTURAL && tokens[j] != delim) k = 0;
-      if (policy == KVR_POLICY_EDITLOCAL_BOUNDARY && j > *bound) k = 0;
-    }
-    keys[t] = k;
+// Key of pool entry t (position s_end + t) under a simple policy; bnd: the
+// EditLocal@boundary boundary.
+__device__ __forceinline__ unsigned long long simple_key(const SimpleKeys &g, int s_end, int t,
+                                                        int bnd) {
+  const int j = s_end + t;
+  if (g.policy == KVR_POLICY_RANDOM) {
+    // first SplitMix64 output of state seed ^ (j * gamma)
+    return mix64((g.seed ^ ((uint64_t)j * GAMMA)) + GAMMA);
   }
+  // nearest to the span first
+  unsigned long long k = 0x100000000ull - (unsigned long long)t;
+  if (g.policy == KVR_POLICY_STRUCTURAL && g.tokens[j] != g.delim) k = 0;
+  if (g.policy == KVR_POLICY_EDITLOCAL_BOUNDARY && j > bnd) k = 0;
+  return k;
 }
 
 __global__ void k_float_keys(const float *scores, int n, int s_end, unsigned long long *keys) {
@@ -62,7 +59,9 @@ __global__ void k_float_keys(const float *scores, int n, int s_end, unsigned lon
 // Top-K of c (key, index) pairs, one CTA of TOPK_THREADS: key descending, ties to
 // the lowest index, the chosen indices written ascending.  Instead of a sort,
 // the K-th key T is found by an MSB-first radix select (8 bits per pass, a
-// shared-memory histogram of the keys that still match the prefix); then
+// shared-memory histogram of the keys that still match the prefix), starting
+// at the highest 8-bit digit in which the keys differ (the AND and OR of all
+// keys give the digits they share, which the passes would only confirm); then
 // every key above T is taken, and of the keys equal to T the lowest-indexed
 // ones until K are taken.  Thread i owns the contiguous keys [i*E, (i+1)*E),
 // so a block-wide scan of per-thread counts writes the output in index order.
@@ -94,40 +93,64 @@ __device__ __forceinline__ int block_excl_scan(int x, int *tmp) {
 
 __global__ void __launch_bounds__(TOPK_THREADS)
     k_topk(const unsigned long long *keys, int c, int s_end, int K, int nonzero_only,
-           int32_t *out, int32_t *count) {
+           int32_t *out, int32_t *count, const SimpleKeys gen, const int *flag_in,
+           int32_t *flag_out) {
   extern __shared__ unsigned long long sk[];  // c keys
   __shared__ int hist[256];
   __shared__ int scan_tmp[TOPK_THREADS / 32];
   __shared__ int s_elig, s_bin, s_above;
+  __shared__ unsigned long long s_and, s_or;
   const int tid = threadIdx.x;
   const int E = (c + TOPK_THREADS - 1) / TOPK_THREADS;
   const int t0 = min(c, tid * E), t1 = min(c, t0 + E);
-  if (tid == 0) s_elig = 0;
+  if (tid == 0) {
+    s_elig = 0;
+    s_and = ~0ull;
+    s_or = 0ull;
+  }
   __syncthreads();
+  const int bnd = gen.policy == KVR_POLICY_EDITLOCAL_BOUNDARY ? *gen.bound : 0;
   int local = 0;
+  unsigned long long kand = ~0ull, kor = 0ull;
   for (int t = tid; t < c; t += TOPK_THREADS) {
-    const unsigned long long k = keys[t];
+    const unsigned long long k = gen.policy >= 0 ? simple_key(gen, s_end, t, bnd) : keys[t];
     sk[t] = k;
+    kand &= k;
+    kor |= k;
     local += (!nonzero_only || k != 0ull) ? 1 : 0;
   }
-  local += __shfl_xor_sync(0xffffffffu, local, 16);
-  local += __shfl_xor_sync(0xffffffffu, local, 8);
-  local += __shfl_xor_sync(0xffffffffu, local, 4);
-  local += __shfl_xor_sync(0xffffffffu, local, 2);
-  local += __shfl_xor_sync(0xffffffffu, local, 1);
-  if ((tid & 31) == 0) atomicAdd(&s_elig, local);
+  for (int o = 16; o > 0; o >>= 1) {
+    local += __shfl_xor_sync(0xffffffffu, local, o);
+    kand &= __shfl_xor_sync(0xffffffffu, kand, o);
+    kor |= __shfl_xor_sync(0xffffffffu, kor, o);
+  }
+  if ((tid & 31) == 0) {
+    atomicAdd(&s_elig, local);
+    atomicAnd(&s_and, kand);
+    atomicOr(&s_or, kor);
+  }
   __syncthreads();
   const int cnt = min(K, s_elig);
   // radix select: prefix/mask of T, need = how many keys equal to the prefix
-  // (so far) are still to be taken
-  unsigned long long pref = 0ull, mask = 0ull;
+  // (so far) are still to be taken.  The digits above dtop are the same in
+  // every key: they start the prefix.
+  const unsigned long long differ = s_or ^ s_and;
+  const int dtop = differ ? (63 - __clzll((long long)differ)) / 8 * 8 : -8;
+  unsigned long long mask = dtop >= 56 ? 0ull : ~0ull << (dtop + 8);
+  unsigned long long pref = s_and & mask;
   int need = cnt;
-  for (int d = 56; d >= 0 && need > 0; d -= 8) {
+  for (int d = dtop; d >= 0 && need > 0; d -= 8) {
     for (int i = tid; i < 256; i += TOPK_THREADS) hist[i] = 0;
     __syncthreads();
-    for (int t = t0; t < t1; ++t) {
-      const unsigned long long k = sk[t];
-      if ((k & mask) == pref) atomicAdd(&hist[(int)(k >> d) & 255], 1);
+    // lanes whose keys fall in the same bin add their count once: keys near
+    // the span (EditLocal) share their upper digits, and one shared-memory
+    // address taking every key serialises the pass
+    for (int e = 0; e < E; ++e) {
+      const int t = t0 + e;
+      const unsigned long long k = t < t1 ? sk[t] : 0ull;
+      const int bin = t < t1 && (k & mask) == pref ? (int)(k >> d) & 255 : -1;
+      const unsigned peers = __match_any_sync(0xffffffffu, bin);
+      if (bin >= 0 && (tid & 31) == __ffs(peers) - 1) atomicAdd(&hist[bin], __popc(peers));
     }
     __syncthreads();
     if (tid < 32) {
@@ -190,7 +213,10 @@ __global__ void __launch_bounds__(TOPK_THREADS)
       }
       if (take) out[pos++] = s_end + t;
     }
-  if (tid == 0) *count = cnt;
+  if (tid == 0) {
+    *count = cnt;
+    if (flag_in) *flag_out = *flag_in;
+  }
 }
 
 // Attention selector, one layer, in two kernels over a workspace.  The
@@ -605,14 +631,11 @@ int grid_for(int n, int block) {
 
 }  // namespace
 
-void launch_scores_simple(int policy, const int32_t *tokens, int n, int s_end, int delim,
-                          uint64_t seed, int *bound, unsigned long long *keys, cudaStream_t s) {
+void launch_first_delim(const int32_t *tokens, int n, int s_end, int delim, int *bound,
+                        cudaStream_t s) {
   int c = n - s_end;
   if (c <= 0) return;
-  if (policy == KVR_POLICY_EDITLOCAL_BOUNDARY)
-    k_first_delim<<<grid_for(c, 256), 256, 0, s>>>(tokens, n, s_end, delim, bound);
-  k_scores_simple<<<grid_for(c, 256), 256, 0, s>>>(policy, tokens, n, s_end, delim, seed, bound,
-                                                   keys);
+  k_first_delim<<<grid_for(c, 256), 256, 0, s>>>(tokens, n, s_end, delim, bound);
 }
 
 void launch_float_keys(const float *scores, int n, int s_end, unsigned long long *keys,
@@ -626,7 +649,8 @@ void launch_float_keys(const float *scores, int n, int s_end, unsigned long long
 // encoded in the sign of K: K < 0 means "only nonzero keys are eligible".
 // Returns nullptr on success, else what failed.
 const char *launch_topk(const unsigned long long *keys, int n, int s_end, int K, int32_t *out,
-                        int32_t *count, cudaStream_t s) {
+                        int32_t *count, cudaStream_t s, const SimpleKeys &gen,
+                        const int *flag_in, int32_t *flag_out) {
   int c = n - s_end;
   int nonzero_only = K < 0 ? 1 : 0;
   if (K < 0) K = -K;
@@ -637,7 +661,8 @@ const char *launch_topk(const unsigned long long *keys, int n, int s_end, int K,
                                          (int)smem);
     if (e != cudaSuccess) return cudaGetErrorString(e);
   }
-  k_topk<<<1, TOPK_THREADS, smem, s>>>(keys, c, s_end, K, nonzero_only, out, count);
+  k_topk<<<1, TOPK_THREADS, smem, s>>>(keys, c, s_end, K, nonzero_only, out, count, gen,
+                                       flag_in, flag_out);
   cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? nullptr : cudaGetErrorString(e);
 }

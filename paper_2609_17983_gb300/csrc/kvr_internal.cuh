@@ -550,10 +550,20 @@ const char *launch_attention_tc5(const void *q, const int32_t *pos, const int4 *
                                  const CUtensorMap *tmaps = nullptr);
 
 // ---- kernels: selectors ----
-// bound: device int holding n - 1 (EditLocal@boundary writes the first
-// delimiter position at or after s_end into it).
-void launch_scores_simple(int policy, const int32_t *tokens, int n, int s_end, int delim,
-                          uint64_t seed, int *bound, unsigned long long *keys, cudaStream_t s);
+// The keys of a simple policy (EditLocal, Structural, Random,
+// EditLocal@boundary), generated inside the top-K kernel instead of read from
+// a keys array.
+struct SimpleKeys {
+  int policy = -1;                  // < 0: the top-K reads the keys array
+  const int32_t *tokens = nullptr;  // the edited context (device)
+  int delim = 0;
+  uint64_t seed = 0;
+  const int *bound = nullptr;       // EditLocal@boundary: launch_first_delim's result
+};
+// EditLocal@boundary: the first delimiter position at or after s_end into
+// *bound, which must hold n - 1 on entry.
+void launch_first_delim(const int32_t *tokens, int n, int s_end, int delim, int *bound,
+                        cudaStream_t s);
 // Attention selector, one layer: adds to scores[j], j in [s_end, n), the
 // pool-softmax probabilities of the S span rows' queries (fp32 q, [S][H*dh]).
 // ws_base: attn_select_ws_bytes(S, dm, n - s_end) bytes; first_layer zeroes
@@ -566,7 +576,10 @@ void launch_kv_deviation(const float *qkv, const float2 *rope, const int32_t *po
                          const Dims &dm, KVView v, float *scores, cudaStream_t s);
 void launch_float_keys(const float *scores, int n, int s_end, unsigned long long *keys,
                        cudaStream_t s);
+// flag_in (optional): the device error flag, copied to *flag_out once every
+// kernel queued before has run, so that one readback returns both.
 const char *launch_topk(const unsigned long long *keys, int n, int s_end, int K, int32_t *out,
-                        int32_t *count, cudaStream_t s);
+                        int32_t *count, cudaStream_t s, const SimpleKeys &gen = SimpleKeys{},
+                        const int *flag_in = nullptr, int32_t *flag_out = nullptr);
 
 }  // namespace kvr
