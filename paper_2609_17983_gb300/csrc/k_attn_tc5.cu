@@ -253,6 +253,13 @@ __global__ void __launch_bounds__(NT5, 1)
     // ------------------------------------------------------------ MMA
     if (lane == 0) {
       const uint32_t id_s = idesc_bf16(QV, CH), id_o = idesc_bf16(QV, DH, 1);
+      // This one thread's issue path bounds the chunk rate (it shares its SM
+      // sub-partition with four softmax warps), so the shared-memory
+      // descriptors are built once: a stage, a 64-wide column block or a
+      // 16-key slice only moves the start address, the descriptor's low field
+      // (address / 16; the operands lie below 256 KB, so the field never
+      // carries).
+      const uint64_t dk0 = sw128_desc(sKV), dv0 = sw128_desc_mn(sKV + TBYTES, CH * 128, 1024);
       bool ok = mbar_wait(&q_full, 0, abort_v, p.dev_flag, 65);
       auto issue_s = [&](int i) -> bool {
         const int b = i & 1, st = i % KV_STAGES;
@@ -260,29 +267,38 @@ __global__ void __launch_bounds__(NT5, 1)
         if (i >= 2 && !mbar_wait(&s_free[b], ((i - 2) >> 1) & 1, abort_v, p.dev_flag, 67))
           return false;
         tc_fence_after();
-        const uint32_t sk = sKV + st * KVBYTES;
+        const uint64_t dk = dk0 + (uint64_t)((st * KVBYTES) >> 4);
+        const uint32_t ts = tmem + b * CH;
 #pragma unroll
-        for (int kk = 0; kk < DH / 16; ++kk) {  // 16 elements of head_dim: 8 columns of Q
-          const uint64_t bb = sw128_desc(sk + (kk >> 2) * CH * 128 + (kk & 3) * 32);
-          mma_bf16_ts(tmem + b * CH, tmem + T_Q + kk * 8, bb, id_s, kk > 0 ? 1u : 0u);
-        }
+        for (int kk = 0; kk < DH / 16; ++kk)  // 16 elements of head_dim: 8 columns of Q
+          mma_bf16_ts(ts, tmem + T_Q + kk * 8,
+                      dk + (uint64_t)(((kk >> 2) * CH * 128 + (kk & 3) * 32) >> 4), id_s,
+                      kk > 0 ? 1u : 0u);
         mma_commit(&s_full[b]);
         return true;
       };
+      // S of chunk i + 2 is issued as soon as the softmax has taken S of chunk
+      // i out of its buffer (early in chunk i), ahead of O += P V of chunk i,
+      // which waits for the end of that softmax: so S is ready before the
+      // softmax reaches it, and the chunk rate is the softmax's own.  Issued
+      // after P V of chunk i instead, it came about 1 us after that P.
       if (ok) ok = issue_s(0);
+      if (ok && nch > 1) ok = issue_s(1);
       for (int i = 0; i < nch && ok; ++i) {
-        if (i + 1 < nch && !(ok = issue_s(i + 1))) break;
+        if (i + 2 < nch && !(ok = issue_s(i + 2))) break;
         if (!(ok = mbar_wait(&p_full[i & 1], (i >> 1) & 1, abort_v, p.dev_flag, 68))) break;
         tc_fence_after();
-        const uint32_t sv = sKV + (i % KV_STAGES) * KVBYTES + TBYTES;
-        const uint32_t tp = tmem + T_P + (i & 1) * (CH / 2);
+        const uint64_t dv = dv0 + (uint64_t)(((i % KV_STAGES) * KVBYTES) >> 4);
+        const uint32_t tp = tmem + T_P + (i & 1) * (CH / 2), to = tmem + 2 * CH;
+        const uint32_t acc0 = i > 0 ? 1u : 0u;
 #pragma unroll
         for (int kk = 0; kk < CH / 16; ++kk) {
           // P: a TMEM lane per query vector, 16 keys in 8 columns.  V: keys
           // are the rows (K), head_dim runs along them (MN-major) in 64-wide
-          // column blocks CH*128 bytes apart, 8-key groups 1024 bytes apart.
-          const uint64_t bb = sw128_desc_mn(sv + kk * 2048, CH * 128, 1024);
-          mma_bf16_ts(tmem + 2 * CH, tp + kk * 8, bb, id_o, (i > 0 || kk > 0) ? 1u : 0u);
+          // column blocks CH*128 bytes apart, 8-key groups 1024 bytes apart;
+          // 16 keys are 2048 bytes.
+          mma_bf16_ts(to, tp + kk * 8, dv + (uint64_t)((kk * 2048) >> 4), id_o,
+                      kk > 0 ? 1u : acc0);
         }
         mma_commit(&o_done[i & 1]);
         mma_commit(&kv_empty[i % KV_STAGES]);
