@@ -63,11 +63,11 @@ kvr_status launch_check(kvr_model *m, int kernels) {
 
 enum ProfId {
   P_EMBED, P_NORM, P_GEMM_QKV, P_ROPE, P_ATTN, P_GEMM_O, P_GEMM_GU, P_SWIGLU, P_GEMM_DOWN,
-  P_LMHEAD, P_SELECT, P_NCLASS
+  P_LMHEAD, P_SELECT, P_GEMM_CHAIN, P_NCLASS
 };
 const char *kProfNames[P_NCLASS] = {"embed",  "rmsnorm",  "gemm_qkv",  "rope_scatter",
                                     "attention", "gemm_o", "gemm_gu",   "swiglu",
-                                    "gemm_down", "lm_head", "select"};
+                                    "gemm_down", "lm_head", "select",    "gemm_chain"};
 
 struct Prof {
   kvr_model *m;
@@ -245,6 +245,20 @@ kvr_status norm(kvr_model *m, const float *g, int M, int row0 = 0) {
 // the GEMM are completed by the RoPE kernel alone).  need_q: the fp32 q
 // (m->q) is read afterwards (attention selector); the tensor-core attention
 // reads only the bf16 q, and the fp32 one is then not written.
+// RoPE of layer l's projection in m->qkv (completed from sv, the QKV GEMM's
+// deferred split tiles), q to m->qb (and m->q when need_q or no tensor-core
+// attention), and (write_kv) the K/V rows into the cache.
+kvr_status rope(kvr_model *m, const Rows &r, int l, bool write_kv, bool need_q,
+                const SplitView &sv) {
+  const Dims &dm = m->dims;
+  Prof pr(m, P_ROPE, (int64_t)r.M * dm.Nqkv() * 4);
+  const bool tc = use_tc_attention(m);
+  launch_rope_scatter(m->qkv, m->rope, r.pos, r.M, dm, l, r.views, r.rowdoc, r.single,
+                      tc && !need_q ? nullptr : m->q, tc ? m->qb : nullptr, 1.0f, write_kv,
+                      m->stream, &sv);
+  return launch_check(m, 1);
+}
+
 kvr_status layer_qkv(kvr_model *m, const Rows &r, int l, bool write_kv, bool keep_qkv = false,
                      bool need_q = false) {
   const Dims &dm = m->dims;
@@ -253,19 +267,11 @@ kvr_status layer_qkv(kvr_model *m, const Rows &r, int l, bool write_kv, bool kee
   SplitView sv;
   KVR_TRY(gemm(m, P_GEMM_QKV, m->a, w.wqkv, w.tc_qkv ? &w.tm_qkv : nullptr, w.bqkv, m->qkv, r.M,
                dm.Nqkv(), dm.d, GEMM_EPI_STORE, keep_qkv ? nullptr : &sv));
-  {
-    Prof pr(m, P_ROPE, (int64_t)r.M * dm.Nqkv() * 4);
-    const bool tc = use_tc_attention(m);
-    launch_rope_scatter(m->qkv, m->rope, r.pos, r.M, dm, l, r.views, r.rowdoc, r.single,
-                        tc && !need_q ? nullptr : m->q, tc ? m->qb : nullptr, 1.0f, write_kv,
-                        m->stream, &sv);
-    KVR_TRY(launch_check(m, 1));
-  }
-  return KVR_OK;
+  return rope(m, r, l, write_kv, need_q, sv);
 }
 
-// Attention, O projection, MLP of layer l (after layer_qkv).
-kvr_status layer_rest(kvr_model *m, const Rows &r, int l) {
+// Attention of layer l (after its RoPE and K/V write) into m->attn.
+kvr_status attention(kvr_model *m, const Rows &r, int l) {
   const Dims &dm = m->dims;
   const LayerW &w = m->layers[l];
   {
@@ -296,6 +302,14 @@ kvr_status layer_rest(kvr_model *m, const Rows &r, int l) {
       KVR_TRY(launch_check(m, 1));
     }
   }
+  return KVR_OK;
+}
+
+// Attention, O projection, MLP of layer l (after layer_qkv).
+kvr_status layer_rest(kvr_model *m, const Rows &r, int l) {
+  const Dims &dm = m->dims;
+  const LayerW &w = m->layers[l];
+  KVR_TRY(attention(m, r, l));
   KVR_TRY(gemm(m, P_GEMM_O, m->attn, w.wo, w.tc_o ? &w.tm_o : nullptr, nullptr, m->h, r.M, dm.d,
                dm.H * dm.dh, GEMM_EPI_ACCUM, &m->pending));
   KVR_TRY(norm(m, w.mlp_norm, r.M));
@@ -313,8 +327,96 @@ kvr_status layer_rest(kvr_model *m, const Rows &r, int l) {
 // repair), so the last layer stops after its K/V are written -- K/V of layer l
 // are projections of the layer's input, and the last layer's attention and
 // MLP feed only the final hidden state, which the logits passes need.
+// Whether the pass's GEMMs and norms can run as chains (launch_gemm_chain):
+// every projection on the tensor cores, rows no more than the SMs, the
+// residual width within the chain norm's reach.
+bool chain_ok(const kvr_model *m, const Rows &r) {
+  const Dims &dm = m->dims;
+  if (!m->use_chain || !m->chain_bar || !m->use_tc || !m->defer_splits ||
+      dm.dtype != KVR_DTYPE_BF16 || r.M <= 0 || r.M > m->num_sms || dm.d > 4096 || dm.d % 4)
+    return false;
+  for (int l = 0; l < dm.L; ++l) {
+    const LayerW &w = m->layers[l];
+    if (!w.tc_qkv || !w.tc_o || !w.tc_gu || !w.tc_d) return false;
+  }
+  return true;
+}
+
+// The pass with the projections and norms in chains, one launch per layer
+// boundary: [norm, QKV] of layer 0, then after each layer's attention
+// [O, norm, gate/up, down] and the next layer's [norm, QKV].  RoPE and the
+// attention stay kernels of their own.
+kvr_status run_pass_chain(kvr_model *m, const Rows &r, bool kv_only) {
+  const Dims &dm = m->dims;
+  const size_t words = gemm_chain_bar_words();
+  if (cudaMemsetAsync(m->chain_bar, 0, (size_t)(dm.L + 1) * words * sizeof(unsigned),
+                      m->stream) != cudaSuccess)
+    return fail(KVR_E_CUDA, "chain counters");
+  KVR_TRY(embed(m, r));
+  auto norm_step = [&](const float *gain) {
+    ChainStep st;
+    st.norm = true;
+    st.h = m->h;
+    st.gain = gain;
+    st.eps = (float)dm.eps;
+    st.d = dm.d;
+    st.out = m->a;
+    return st;
+  };
+  auto gemm_step = [&](const void *X, const void *W, const CUtensorMap *tm, const float *bias,
+                       float *Y, int N, int K, int epi, bool defer) {
+    ChainStep st;
+    st.g = GemmArgs{X, W, bias, Y, r.M, N, K, K, N, dm.dtype, epi == GEMM_EPI_ACCUM};
+    st.tmW = tm;
+    st.epi = epi;
+    st.out2 = epi == GEMM_EPI_SWIGLU ? m->act : nullptr;
+    st.ld2 = N / 2;
+    st.defer = defer;
+    return st;
+  };
+  auto qkv_step = [&](int l) {
+    const LayerW &w = m->layers[l];
+    return gemm_step(m->a, w.wqkv, &w.tm_qkv, w.bqkv, m->qkv, dm.Nqkv(), dm.d, GEMM_EPI_STORE,
+                     true);
+  };
+  int ci = 0;
+  auto run = [&](const std::vector<ChainStep> &st, SplitView *last) -> kvr_status {
+    int64_t bytes = 0;
+    for (const ChainStep &x : st)
+      if (!x.norm) bytes += (int64_t)x.g.N * x.g.K * dm.es();
+    Prof pr(m, P_GEMM_CHAIN, bytes);
+    const char *e = launch_gemm_chain(st.data(), (int)st.size(), m->tcw,
+                                      m->chain_bar + (size_t)ci * words, m->stream, last);
+    ++ci;
+    if (e) return fail(KVR_E_CUDA, "GEMM chain (%d steps): %s", (int)st.size(), e);
+    return launch_check(m, 1);
+  };
+  SplitView sv;
+  KVR_TRY(run({norm_step(m->layers[0].attn_norm), qkv_step(0)}, &sv));
+  for (int l = 0; l < dm.L; ++l) {
+    const LayerW &w = m->layers[l];
+    KVR_TRY(rope(m, r, l, true, false, sv));
+    if (kv_only && l + 1 == dm.L) break;
+    KVR_TRY(attention(m, r, l));
+    std::vector<ChainStep> st = {
+        gemm_step(m->attn, w.wo, &w.tm_o, nullptr, m->h, dm.d, dm.H * dm.dh, GEMM_EPI_ACCUM, true),
+        norm_step(w.mlp_norm),
+        gemm_step(m->a, w.wgu, &w.tm_gu, nullptr, nullptr, 2 * dm.F, dm.d, GEMM_EPI_SWIGLU, false),
+        gemm_step(m->act, w.wd, &w.tm_d, nullptr, m->h, dm.d, dm.F, GEMM_EPI_ACCUM, true)};
+    if (l + 1 < dm.L) {
+      st.push_back(norm_step(m->layers[l + 1].attn_norm));
+      st.push_back(qkv_step(l + 1));
+      KVR_TRY(run(st, &sv));
+    } else {
+      KVR_TRY(run(st, &m->pending));  // the final norm adds the down projection's split tiles
+    }
+  }
+  return KVR_OK;
+}
+
 kvr_status run_pass(kvr_model *m, const Rows &r, bool kv_only) {
   if (r.M <= 0) return KVR_OK;
+  if (chain_ok(m, r)) return run_pass_chain(m, r, kv_only);
   KVR_TRY(embed(m, r));
   for (int l = 0; l < m->dims.L; ++l) {
     KVR_TRY(layer_qkv(m, r, l, true));
@@ -554,6 +656,7 @@ void kvr_model_free(kvr_model *m) {
   dev_free(m->ws_block);
   dev_free(m->rope);
   dev_free(m->dev_flag);
+  dev_free(m->chain_bar);
   dev_free(m->tcw.partials);
   dev_free(m->read_scratch);
   dev_free(m->sel_scratch);
@@ -596,6 +699,9 @@ kvr_status kvr_model_create(const kvr_model_config *cfg, const kvr_weights *wts,
     m->use_tc5 = !(t5 && t5[0] == '1');
     const char *pd = getenv("KVR_DISABLE_PDL");
     g_pdl = !(pd && pd[0] == '1');
+    // GEMM chains are opt-in: they measured slower than separate launches
+    const char *ch = getenv("KVR_ENABLE_CHAIN");
+    m->use_chain = ch && ch[0] == '1';
   }
   cudaDeviceGetAttribute(&m->num_sms, cudaDevAttrMultiProcessorCount, m->device);
   m->prof_classes.resize(P_NCLASS);
@@ -772,6 +878,10 @@ kvr_status kvr_model_create(const kvr_model_config *cfg, const kvr_weights *wts,
     m->dev_flag = (int *)dev_alloc(256);
     if (!m->dev_flag) return bail(fail(KVR_E_NOMEM, "flag"));
     cudaMemset(m->dev_flag, 0, 256);
+    // hand-off counters of a pass's GEMM chains (one set per chain)
+    m->chain_bar =
+        (unsigned *)dev_alloc((size_t)(dm.L + 1) * gemm_chain_bar_words() * sizeof(unsigned));
+    if (!m->chain_bar) return bail(fail(KVR_E_NOMEM, "chain counters"));
     // positions and tokens of a pass, plus the tables of a 256-document batch
     m->stage_cap = std::max<size_t>(R * 4, P) + 4096 +
                    256 * (sizeof(CUtensorMap) + sizeof(KVView) + sizeof(void *)) / 4;

@@ -109,8 +109,8 @@ __device__ __forceinline__ void unit_range(long long i, long long total, int gri
 // feature n of W.  All lanes of the warp call it together (SwiGLU exchanges
 // lanes); every load is issued before any dependent use, so the chunk costs
 // one L2 round trip, not sixteen.
-__device__ __forceinline__ void epilogue16(const TcParams &p, int t0, int n, const float *v,
-                                           int cnt) {
+template <class P>
+__device__ __forceinline__ void epilogue16(const P &p, int t0, int n, const float *v, int cnt) {
   if (p.epi == GEMM_EPI_SWIGLU) {
     // rows 32b..32b+15 of W are gate, 32b+16..32b+31 up, of features
     // 16b..16b+15; lane = n % 32.  Lanes r and r ^ 16 swap their values, so
@@ -144,6 +144,204 @@ __device__ __forceinline__ void epilogue16(const TcParams &p, int t0, int n, con
 #pragma unroll
   for (int j = 0; j < 16; ++j)
     if (j < cnt) y[(size_t)j * p.ldy] = v[j] + b;
+}
+
+// The MMAs of units [u0, u1) of one GEMM: one TMEM accumulator per
+// (feature tile, token tile) segment, double-buffered (seg counts segments);
+// stage s / phase ph continue from the caller.  False if a wait ran out.
+template <class P>
+__device__ __forceinline__ bool mma_range(const P &p, long long u0, long long u1, int &s,
+                                          uint32_t &ph, uint32_t &seg, int S, uint32_t base,
+                                          uint32_t stage_bytes, uint32_t tmem_base,
+                                          uint32_t idesc, uint64_t *full_bar, uint64_t *empty_bar,
+                                          uint64_t *accf_bar, uint64_t *acce_bar,
+                                          volatile int *abort_v) {
+  bool ok = true;
+  for (long long a = u0; a < u1 && ok;) {
+    long long tl = a / p.KB;
+    long long b = (tl + 1) * p.KB < u1 ? (tl + 1) * p.KB : u1;
+    uint32_t buf = seg & 1u, use = seg >> 1;
+    if (!mbar_wait(&acce_bar[buf], (use & 1u) ^ 1u, abort_v, p.dev_flag, 2)) break;
+    tc_fence_after();
+    uint32_t d = tmem_base + buf * p.tmem_cols;
+    for (long long u = a; u < b; ++u) {
+      if (!mbar_wait(&full_bar[s], ph, abort_v, p.dev_flag, 4)) {
+        ok = false;
+        break;
+      }
+      if (u == u0) trace_mark(0);
+      tc_fence_after();
+      uint32_t sa = base + (uint32_t)s * stage_bytes;
+      uint64_t da = sw128_desc(sa), db = sw128_desc(sa + A_BYTES);
+#pragma unroll
+      for (int k = 0; k < BK / UK; ++k)
+        mma_bf16(d, da + (uint64_t)(k * UK * 2 / 16), db + (uint64_t)(k * UK * 2 / 16), idesc,
+                 (u > a || k > 0) ? 1u : 0u);
+      mma_commit(&empty_bar[s]);
+      if (++s == S) {
+        s = 0;
+        ph ^= 1u;
+      }
+    }
+    if (ok) mma_commit(&accf_bar[buf]);
+    ++seg;
+    a = b;
+  }
+  return ok;
+}
+
+// The epilogue of units [u0, u1) of one GEMM (stream-K, one CTA's range):
+// per segment, the accumulator from TMEM into Y (whole tiles), into the
+// split-tile workspace (deferred mode), or, for a split tile's first CTA,
+// summed with the other parts (bounded wait for them) in CTA order.
+template <class P>
+__device__ __forceinline__ void epi_range(const P &p, long long u0, long long u1, uint32_t &seg,
+                                          uint32_t tmem_base, uint64_t *accf_bar,
+                                          uint64_t *acce_bar, volatile int *abort_v, int q,
+                                          int f, int et, int eg) {
+  constexpr int CSTEP = 16 * EPI_GROUPS;
+  for (long long a = u0; a < u1;) {
+    long long tl = a / p.KB;
+    long long b = (tl + 1) * p.KB < u1 ? (tl + 1) * p.KB : u1;
+    uint32_t buf = seg & 1u, use = seg >> 1;
+    int ntile = (int)(tl / p.m_tiles), mtile = (int)(tl % p.m_tiles);
+    int t0 = mtile * p.BN;
+    int mv = min(p.BN, p.M - t0);
+    int n = ntile * BM + f;
+    long long tile_u0 = tl * p.KB;
+    int i_first = cta_of(tile_u0, p.total, p.grid);
+    int i_last = cta_of(tile_u0 + p.KB - 1, p.total, p.grid);
+    int parts = i_last - i_first + 1;
+    // The owner of a split tile waits for the other parts and, with two
+    // parts and at most 48 rows, loads the other one now, while this
+    // tile's MMAs are still running: both L2 round trips leave the tail.
+    const bool own_fix = parts > 1 && !p.defer && (int)blockIdx.x == i_first;
+    const bool pre = own_fix && parts == 2 && mv <= 48;
+    // this group's chunks of the other part: chunk k of the group at rows
+    // 16 eg + CSTEP k .. + 15
+    constexpr int PRE_CHUNKS = (48 + CSTEP - 1) / CSTEP;
+    float other[16 * PRE_CHUNKS];
+    if (own_fix) {
+      if (et == 0) {
+        volatile int *ready = p.counters + p.max_tiles + tl;
+        const uint64_t t0w = gtime_ns();
+        for (uint32_t it = 0; *ready < parts - 1; ++it)
+          if ((it & 63) == 63 && (*abort_v || gtime_ns() - t0w > WAIT_NS)) {
+            if (!*abort_v) {
+              *abort_v = 1;
+              atomicOr(p.dev_flag, 32);
+            }
+            break;
+          }
+        trace_mark(4);
+      }
+      epi_bar();
+      if (!*abort_v) {
+        asm volatile("fence.acq_rel.gpu;" ::: "memory");  // acquire the parts
+        if (pre) {
+          const int so = range_start(i_last, p.total, p.grid) >= tile_u0 ? 0 : 1;
+          const float *src = p.ws + ((size_t)i_last * 2 + so) * p.BN * BM + f;
+#pragma unroll
+          for (int k = 0; k < PRE_CHUNKS; ++k)
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+              const int row = 16 * eg + CSTEP * k + j;
+              other[16 * k + j] = row < mv ? __ldcg(src + (size_t)row * BM) : 0.f;
+            }
+        }
+      }
+    }
+    if (!mbar_wait(&accf_bar[buf], use & 1u, abort_v, p.dev_flag, 8)) break;
+    tc_fence_after();
+    if (et == 0) trace_mark(2);
+    uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + buf * p.tmem_cols;
+    if (parts == 1) {
+      for (int c = 16 * eg; c < mv; c += CSTEP) {
+        float v[16];
+        tmem_ld16(taddr + c, v);
+        epilogue16(p, t0 + c, n, v, mv - c);
+      }
+      if (et == 0) trace_mark(5);
+    } else if (p.defer) {
+      // the consumer of Y adds this part: store it and go on
+      int slot = range_start(blockIdx.x, p.total, p.grid) >= tile_u0 ? 0 : 1;
+      float *w = p.ws + ((size_t)blockIdx.x * 2 + slot) * p.BN * BM;
+      for (int c = 16 * eg; c < mv; c += CSTEP) {
+        float v[16];
+        tmem_ld16(taddr + c, v);
+#pragma unroll
+        for (int j = 0; j < 16; ++j)
+          if (c + j < mv) w[(size_t)(c + j) * BM + f] = v[j];
+      }
+      if (et == 0) trace_mark(3);
+    } else {
+      // Reduced by its first CTA: for it the tile is the last segment, so
+      // the others (for whom it is a first segment, or their whole range)
+      // have usually published their parts long before.  A CTA that is not
+      // the owner stores its part and publishes it; the owner keeps its own
+      // part in TMEM, waits (bounded) until the others are published, and
+      // sums all parts in CTA order.  Every CTA of the grid is resident (the
+      // next kernel cannot launch before all of them have started) and a
+      // publishing CTA waits on nothing, so the wait ends.
+      const bool owner = (int)blockIdx.x == i_first;
+      if (!owner) {
+        int slot = range_start(blockIdx.x, p.total, p.grid) >= tile_u0 ? 0 : 1;
+        float *w = p.ws + ((size_t)blockIdx.x * 2 + slot) * p.BN * BM;
+        for (int c = 16 * eg; c < mv; c += CSTEP) {
+          float v[16];
+          tmem_ld16(taddr + c, v);
+#pragma unroll
+          for (int j = 0; j < 16; ++j)
+            if (c + j < mv) w[(size_t)(c + j) * BM + f] = v[j];
+        }
+        asm volatile("fence.acq_rel.gpu;" ::: "memory");  // release the part
+        epi_bar();
+        if (et == 0) {
+          atomicAdd(&p.counters[p.max_tiles + tl], 1);
+          trace_mark(3);
+        }
+      } else {
+        if (!*abort_v) {
+#pragma unroll 1
+          for (int c = 16 * eg; c < mv; c += CSTEP) {
+            float own[16], v[16];
+            tmem_ld16(taddr + c, own);
+#pragma unroll
+            for (int j = 0; j < 16; ++j) v[j] = 0.f;
+            for (int i = i_first; i <= i_last; ++i) {
+              if (i == (int)blockIdx.x) {
+#pragma unroll
+                for (int j = 0; j < 16; ++j) v[j] += own[j];
+              } else if (pre) {
+                // rows c..c+15 of the preloaded part: this group's chunk 0 or 1
+                static_assert(PRE_CHUNKS == 2, "preloaded chunks of a group");
+                const bool first = c == 16 * eg;
+#pragma unroll
+                for (int j = 0; j < 16; ++j) v[j] += first ? other[j] : other[16 + j];
+              } else {
+                const int si = range_start(i, p.total, p.grid) >= tile_u0 ? 0 : 1;
+                const float *src = p.ws + (((size_t)i * 2 + si) * p.BN + c) * BM + f;
+                float x[16];
+#pragma unroll
+                for (int j = 0; j < 16; ++j) x[j] = c + j < mv ? __ldcg(src + (size_t)j * BM) : 0.f;
+#pragma unroll
+                for (int j = 0; j < 16; ++j) v[j] += x[j];
+              }
+            }
+            epilogue16(p, t0 + c, n, v, mv - c);
+          }
+          if (et == 0) {
+            p.counters[p.max_tiles + tl] = 0;
+            trace_mark(5);
+          }
+        }
+      }
+    }
+    tc_fence_before();
+    mbar_arrive(&acce_bar[buf]);
+    ++seg;
+    a = b;
+  }
 }
 
 __global__ void __launch_bounds__(NTHREADS, 1)
@@ -286,37 +484,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       const uint32_t idesc = idesc_bf16(BM, p.BN);
       uint32_t seg = 0, ph = 0;
       int s = 0;
-      bool ok = true;
-      for (long long a = u0; a < u1 && ok;) {
-        long long tl = a / p.KB;
-        long long b = (tl + 1) * p.KB < u1 ? (tl + 1) * p.KB : u1;
-        uint32_t buf = seg & 1u, use = seg >> 1;
-        if (!mbar_wait(&acce_bar[buf], (use & 1u) ^ 1u, abort_v, p.dev_flag, 2)) break;
-        tc_fence_after();
-        uint32_t d = tmem_base + buf * p.tmem_cols;
-        for (long long u = a; u < b; ++u) {
-          if (!mbar_wait(&full_bar[s], ph, abort_v, p.dev_flag, 4)) {
-            ok = false;
-            break;
-          }
-          if (u == u0) trace_mark(0);
-          tc_fence_after();
-          uint32_t sa = base + (uint32_t)s * stage_bytes;
-          uint64_t da = sw128_desc(sa), db = sw128_desc(sa + A_BYTES);
-#pragma unroll
-          for (int k = 0; k < BK / UK; ++k)
-            mma_bf16(d, da + (uint64_t)(k * UK * 2 / 16), db + (uint64_t)(k * UK * 2 / 16), idesc,
-                     (u > a || k > 0) ? 1u : 0u);
-          mma_commit(&empty_bar[s]);
-          if (++s == S) {
-            s = 0;
-            ph ^= 1u;
-          }
-        }
-        if (ok) mma_commit(&accf_bar[buf]);
-        ++seg;
-        a = b;
-      }
+      mma_range(p, u0, u1, s, ph, seg, S, base, stage_bytes, tmem_base, idesc, full_bar,
+                empty_bar, accf_bar, acce_bar, abort_v);
       // all MMAs issued by this thread complete before TMEM is freed
       mma_commit(&drain_bar);
       mbar_wait(&drain_bar, 0, abort_v, p.dev_flag, 0, false);
@@ -351,148 +520,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       }
       tc_fence_before();
     }
-    for (long long a = u0; a < u1 && p.cluster <= 1;) {
-      long long tl = a / p.KB;
-      long long b = (tl + 1) * p.KB < u1 ? (tl + 1) * p.KB : u1;
-      uint32_t buf = seg & 1u, use = seg >> 1;
-      int ntile = (int)(tl / p.m_tiles), mtile = (int)(tl % p.m_tiles);
-      int t0 = mtile * p.BN;
-      int mv = min(p.BN, p.M - t0);
-      int n = ntile * BM + f;
-      long long tile_u0 = tl * p.KB;
-      int i_first = cta_of(tile_u0, p.total, p.grid);
-      int i_last = cta_of(tile_u0 + p.KB - 1, p.total, p.grid);
-      int parts = i_last - i_first + 1;
-      // The owner of a split tile waits for the other parts and, with two
-      // parts and at most 48 rows, loads the other one now, while this
-      // tile's MMAs are still running: both L2 round trips leave the tail.
-      const bool own_fix = parts > 1 && !p.defer && (int)blockIdx.x == i_first;
-      const bool pre = own_fix && parts == 2 && mv <= 48;
-      // this group's chunks of the other part: chunk k of the group at rows
-      // 16 eg + CSTEP k .. + 15
-      constexpr int PRE_CHUNKS = (48 + CSTEP - 1) / CSTEP;
-      float other[16 * PRE_CHUNKS];
-      if (own_fix) {
-        if (et == 0) {
-          volatile int *ready = p.counters + p.max_tiles + tl;
-          const uint64_t t0w = gtime_ns();
-          for (uint32_t it = 0; *ready < parts - 1; ++it)
-            if ((it & 63) == 63 && (*abort_v || gtime_ns() - t0w > WAIT_NS)) {
-              if (!*abort_v) {
-                *abort_v = 1;
-                atomicOr(p.dev_flag, 32);
-              }
-              break;
-            }
-          trace_mark(4);
-        }
-        epi_bar();
-        if (!*abort_v) {
-          asm volatile("fence.acq_rel.gpu;" ::: "memory");  // acquire the parts
-          if (pre) {
-            const int so = range_start(i_last, p.total, p.grid) >= tile_u0 ? 0 : 1;
-            const float *src = p.ws + ((size_t)i_last * 2 + so) * p.BN * BM + f;
-#pragma unroll
-            for (int k = 0; k < PRE_CHUNKS; ++k)
-#pragma unroll
-              for (int j = 0; j < 16; ++j) {
-                const int row = 16 * eg + CSTEP * k + j;
-                other[16 * k + j] = row < mv ? __ldcg(src + (size_t)row * BM) : 0.f;
-              }
-          }
-        }
-      }
-      if (!mbar_wait(&accf_bar[buf], use & 1u, abort_v, p.dev_flag, 8)) break;
-      tc_fence_after();
-      if (et == 0) trace_mark(2);
-      uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + buf * p.tmem_cols;
-      if (parts == 1) {
-        for (int c = 16 * eg; c < mv; c += CSTEP) {
-          float v[16];
-          tmem_ld16(taddr + c, v);
-          epilogue16(p, t0 + c, n, v, mv - c);
-        }
-        if (et == 0) trace_mark(5);
-      } else if (p.defer) {
-        // the consumer of Y adds this part: store it and go on
-        int slot = range_start(blockIdx.x, p.total, p.grid) >= tile_u0 ? 0 : 1;
-        float *w = p.ws + ((size_t)blockIdx.x * 2 + slot) * p.BN * BM;
-        for (int c = 16 * eg; c < mv; c += CSTEP) {
-          float v[16];
-          tmem_ld16(taddr + c, v);
-#pragma unroll
-          for (int j = 0; j < 16; ++j)
-            if (c + j < mv) w[(size_t)(c + j) * BM + f] = v[j];
-        }
-        if (et == 0) trace_mark(3);
-      } else {
-        // Reduced by its first CTA: for it the tile is the last segment, so
-        // the others (for whom it is a first segment, or their whole range)
-        // have usually published their parts long before.  A CTA that is not
-        // the owner stores its part and publishes it; the owner keeps its own
-        // part in TMEM, waits (bounded) until the others are published, and
-        // sums all parts in CTA order.  Every CTA of the grid is resident (the
-        // next kernel cannot launch before all of them have started) and a
-        // publishing CTA waits on nothing, so the wait ends.
-        const bool owner = (int)blockIdx.x == i_first;
-        if (!owner) {
-          int slot = range_start(blockIdx.x, p.total, p.grid) >= tile_u0 ? 0 : 1;
-          float *w = p.ws + ((size_t)blockIdx.x * 2 + slot) * p.BN * BM;
-          for (int c = 16 * eg; c < mv; c += CSTEP) {
-            float v[16];
-            tmem_ld16(taddr + c, v);
-#pragma unroll
-            for (int j = 0; j < 16; ++j)
-              if (c + j < mv) w[(size_t)(c + j) * BM + f] = v[j];
-          }
-          asm volatile("fence.acq_rel.gpu;" ::: "memory");  // release the part
-          epi_bar();
-          if (et == 0) {
-            atomicAdd(&p.counters[p.max_tiles + tl], 1);
-            trace_mark(3);
-          }
-        } else {
-          if (!*abort_v) {
-#pragma unroll 1
-            for (int c = 16 * eg; c < mv; c += CSTEP) {
-              float own[16], v[16];
-              tmem_ld16(taddr + c, own);
-#pragma unroll
-              for (int j = 0; j < 16; ++j) v[j] = 0.f;
-              for (int i = i_first; i <= i_last; ++i) {
-                if (i == (int)blockIdx.x) {
-#pragma unroll
-                  for (int j = 0; j < 16; ++j) v[j] += own[j];
-                } else if (pre) {
-                  // rows c..c+15 of the preloaded part: this group's chunk 0 or 1
-                  static_assert(PRE_CHUNKS == 2, "preloaded chunks of a group");
-                  const bool first = c == 16 * eg;
-#pragma unroll
-                  for (int j = 0; j < 16; ++j) v[j] += first ? other[j] : other[16 + j];
-                } else {
-                  const int si = range_start(i, p.total, p.grid) >= tile_u0 ? 0 : 1;
-                  const float *src = p.ws + (((size_t)i * 2 + si) * p.BN + c) * BM + f;
-                  float x[16];
-#pragma unroll
-                  for (int j = 0; j < 16; ++j) x[j] = c + j < mv ? __ldcg(src + (size_t)j * BM) : 0.f;
-#pragma unroll
-                  for (int j = 0; j < 16; ++j) v[j] += x[j];
-                }
-              }
-              epilogue16(p, t0 + c, n, v, mv - c);
-            }
-            if (et == 0) {
-              p.counters[p.max_tiles + tl] = 0;
-              trace_mark(5);
-            }
-          }
-        }
-      }
-      tc_fence_before();
-      mbar_arrive(&acce_bar[buf]);
-      ++seg;
-      a = b;
-    }
+    if (p.cluster <= 1)
+      epi_range(p, u0, u1, seg, tmem_base, accf_bar, acce_bar, abort_v, q, f, et, eg);
     if (et == 0) trace_mark(6);
   }
   tc_fence_before();
@@ -555,6 +584,373 @@ EncodeTiledFn encode_fn() {
       fn = (EncodeTiledFn)f;
   }
   return fn;
+}
+
+
+// ------------------------------------------------------------ chained GEMMs
+//
+// A chain runs several GEMMs of one row set, with RMSNorms between them, in one
+// persistent launch: the repair pass's O projection, RMSNorm, gate/up, down,
+// the next layer's RMSNorm and QKV projection.  Every CTA keeps its pipeline,
+// its TMEM and its role loops across the steps, and the steps meet at
+// counters in device memory instead of kernel boundaries: the weight stream of
+// the next GEMM starts while the last tiles of the previous one drain and
+// while the norm runs (its weights do not depend on them), and no CTA leaves
+// or is scheduled between steps.
+//
+// Step hand-offs (counters 128 bytes apart, zeroed before the pass):
+//   after a GEMM, every CTA's epilogue, once its stores are done, adds one
+//   behind a gpu-scope fence;
+//   a norm (its row per CTA, CTAs 0 .. M-1) waits for all of them, completes
+//   the GEMM's deferred split tiles into the residual, writes its row and adds
+//   one;
+//   a GEMM's TMA thread issues the first stages' weight tiles, waits for the
+//   step before (the norm's M rows, or every CTA of the GEMM before) and only
+//   then loads activations (after a generic-to-async proxy fence); its
+//   epilogue waits for the same count before it writes outputs or split-tile
+//   parts (the norm reads the previous GEMM's parts from the same workspace).
+// All CTAs are resident at once (one per SM, grid = SM count, and the next
+// kernel launches only after each has started), so every wait ends; each is
+// bounded all the same.
+constexpr int CHAIN_MAX = 6;         // steps per chain
+constexpr int CHAIN_GEMMS = 4;       // GEMM steps per chain
+constexpr int CHAIN_NORMS = 2;       // norm steps per chain
+constexpr int CHAIN_BAR_STRIDE = 32;  // counters 128 bytes apart
+constexpr int CHAIN_NORM_NV = 4;     // float4s per epilogue thread: d <= 4096
+
+struct ChainNorm {
+  float *h;            // [M][d] residual; split tiles of the GEMM before are added in place
+  const float *g;      // [d] gains
+  float eps;
+  int d;               // multiple of 4, at most 4 * EPI_THREADS * CHAIN_NORM_NV
+  __nv_bfloat16 *out;  // [M][d]
+  SplitView sv;        // deferred split tiles of the GEMM before (ws null: none)
+};
+
+// Indexed by step.  The kernel takes it as a grid constant, so a step's fields
+// are read in place from the parameter space (as an ordinary parameter,
+// indexed by a run-time step, it was copied to local memory).
+struct ChainParams {
+  int n_steps, M;
+  int is_norm[CHAIN_MAX];
+  TcParams g[CHAIN_MAX];     // GEMM steps
+  ChainNorm nrm[CHAIN_MAX];  // norm steps
+  unsigned *bar;             // [CHAIN_MAX][CHAIN_BAR_STRIDE], zero at launch
+  int *dev_flag;
+};
+
+struct ChainMaps {
+  CUtensorMap w[CHAIN_MAX], x[CHAIN_MAX];  // GEMM steps
+};
+
+// Arrivals step k must see before it goes on: a norm's rows, or every CTA
+// of a GEMM.
+__device__ __forceinline__ unsigned chain_target(const ChainParams &c, int k) {
+  return c.is_norm[k] ? (unsigned)c.M : (unsigned)c.g[k].grid;
+}
+
+// Bounded wait (2 s) until *ctr >= target: relaxed gpu-scope loads while it
+// polls, then one acquire fence.
+__device__ __forceinline__ bool chain_wait(const unsigned *ctr, unsigned target,
+                                           volatile int *abort_f, int *dev_flag, int code) {
+  unsigned v;
+  asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(ctr) : "memory");
+  if (v >= target) {
+    asm volatile("fence.acq_rel.gpu;" ::: "memory");
+    return true;
+  }
+  const uint64_t t0 = gtime_ns();
+  for (uint32_t it = 0;; ++it) {
+    asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(ctr) : "memory");
+    if (v >= target) {
+      asm volatile("fence.acq_rel.gpu;" ::: "memory");
+      return true;
+    }
+    if ((it & 63) == 63) {
+      if (*abort_f) return false;
+      if (gtime_ns() - t0 > WAIT_NS) {
+        *abort_f = 1;
+        atomicOr(dev_flag, code);
+        return false;
+      }
+    }
+  }
+}
+
+__device__ __forceinline__ uint32_t chain_pack(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *(uint32_t *)&v;
+}
+
+// RMSNorm of residual row `row` by the CTA's EPI_THREADS epilogue threads
+// (et = 0 .. EPI_THREADS - 1): the row, completed from the split view (and
+// written back), normalised into out in bf16.  red: EPI_THREADS / 32 floats.
+// The row's float4s are completed two at a time (each with up to
+// SPLIT_MAX_PARTS part loads in flight): all four at once held too many
+// registers for the kernel's budget.
+__device__ __forceinline__ void chain_norm(const ChainNorm nm, int row, int et, float *red) {
+  const int nq = nm.d >> 2;
+  float4 *x = (float4 *)(nm.h + (size_t)row * nm.d);
+  float4 v[CHAIN_NORM_NV];
+  float ss = 0.f;
+#pragma unroll 1
+  for (int k0 = 0; k0 < CHAIN_NORM_NV; k0 += 2) {
+#pragma unroll
+    for (int k = k0; k < k0 + 2; ++k) {
+      const int q = k * EPI_THREADS + et;
+      float4 y = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (q < nq) {
+        y = x[q];
+        if (nm.sv.ws) {
+          const SplitTile st =
+              split_tile(nm.sv, (long long)(q >> 5) * nm.sv.m_tiles + row / nm.sv.BN);
+          if (st.i0 != st.i1) {
+            y = split_value4(nm.sv, st, y, row, 4 * q);
+            x[q] = y;
+          }
+        }
+      }
+      ss += y.x * y.x + y.y * y.y + y.z * y.z + y.w * y.w;
+      v[k] = y;
+    }
+  }
+  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+  if ((et & 31) == 0) red[et >> 5] = ss;
+  epi_bar();
+  float tot = 0.f;
+#pragma unroll
+  for (int w = 0; w < EPI_THREADS / 32; ++w) tot += red[w];
+  const float r = 1.0f / sqrtf(tot / (float)nm.d + nm.eps);
+#pragma unroll
+  for (int k = 0; k < CHAIN_NORM_NV; ++k) {
+    const int q = k * EPI_THREADS + et;
+    if (q < nq) {
+      const float4 w = ((const float4 *)nm.g)[q];
+      __nv_bfloat16 *o = nm.out + (size_t)row * nm.d + 4 * q;
+      *(uint2 *)o = make_uint2(chain_pack(v[k].x * r * w.x, v[k].y * r * w.y),
+                               chain_pack(v[k].z * r * w.z, v[k].w * r * w.w));
+    }
+  }
+}
+
+__global__ void __launch_bounds__(NTHREADS, 1)
+    k_gemm_chain(const __grid_constant__ ChainMaps maps, const __grid_constant__ ChainParams c) {
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t full_bar[8], empty_bar[8], accf_bar[2], acce_bar[2],
+      drain_bar;
+  __shared__ uint32_t tmem_slot;
+  __shared__ int abort_f;
+  __shared__ float red[EPI_THREADS / 32];
+
+  TraceScope ts(TK_GEMM);
+  pdl_trigger();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // every GEMM of a chain has the chain's rows: the same token tile, stage
+  // layout, pipeline depth and accumulator width
+  const TcParams &g0 = c.g[c.is_norm[0] ? 1 : 0];
+  const int S = g0.stages;
+  const uint32_t base = (su32(smem_raw) + 1023u) & ~1023u;
+  const uint32_t stage_bytes = A_BYTES + (uint32_t)g0.BN * 128u;
+  const uint32_t tx_bytes = A_BYTES + (uint32_t)g0.brows * 128u;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(&full_bar[s], 1);
+      mbar_init(&empty_bar[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&accf_bar[b], 1);
+      mbar_init(&acce_bar[b], EPI_THREADS);
+    }
+    mbar_init(&drain_bar, 1);
+    abort_f = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 0) {
+    if (lane < c.n_steps && !c.is_norm[lane]) {
+      tma_prefetch_desc(&maps.w[lane]);
+      tma_prefetch_desc(&maps.x[lane]);
+    }
+    __syncwarp();
+    uint32_t ncols = 2 * g0.tmem_cols;
+    asm volatile(
+        "tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+            su32(&tmem_slot)),
+        "r"(ncols)
+        : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = tmem_slot;
+  volatile int *abort_v = &abort_f;
+
+  if (warp == 0) {
+    // ---------------------------------------------------------------- TMA
+    if (lane == 0) {
+      int s = 0;
+      uint32_t ph = 0, it = 0;
+      const uint64_t wpol = l2_evict_first();
+#pragma unroll 1
+      for (int k = 0; k < CHAIN_MAX; ++k) {
+        if (k >= c.n_steps || *abort_v) break;
+        if (c.is_norm[k]) continue;
+        const TcParams &p = c.g[k];
+        const CUtensorMap *tW = &maps.w[k], *tX = &maps.x[k];
+        long long u0, u1;
+        unit_range(blockIdx.x, p.total, p.grid, p.KB, 0, u0, u1);
+        long long tl0 = u0 / p.KB;
+        int kb = (int)(u0 - tl0 * p.KB);
+        int ntile = (int)(tl0 / p.m_tiles), mtile = (int)(tl0 - (long long)ntile * p.m_tiles);
+        auto advance = [&]() {
+          ++it;
+          if (++s == S) {
+            s = 0;
+            ph ^= 1u;
+          }
+          if (++kb == p.KB) {
+            kb = 0;
+            if (++mtile == p.m_tiles) {
+              mtile = 0;
+              ++ntile;
+            }
+          }
+        };
+        auto load_w = [&](uint32_t sa) {
+          const int y = (ntile * p.KB + kb) * BM;
+          if (p.stream_w)
+            tma_load_2d_hint((void *)__cvta_shared_to_generic(sa), tW, &full_bar[s], 0, y, wpol);
+          else
+            tma_load_2d((void *)__cvta_shared_to_generic(sa), tW, &full_bar[s], 0, y);
+        };
+        // the first stages' weights before the step's input is ready
+        const long long npre = (u1 - u0) < S ? (u1 - u0) : S;
+        int pre_s[8], pre_kb[8], pre_mt[8];
+        long long u = u0;
+        for (; u < u0 + npre; ++u) {
+          if (!mbar_wait(&empty_bar[s], ph ^ 1u, abort_v, c.dev_flag, 1)) break;
+          const uint32_t sa = base + (uint32_t)s * stage_bytes;
+          mbar_expect_tx(&full_bar[s], tx_bytes);
+          load_w(sa);
+          pre_s[u - u0] = s;
+          pre_kb[u - u0] = kb;
+          pre_mt[u - u0] = mtile;
+          advance();
+        }
+        const int npre_done = (int)(u - u0);
+        bool ready = true;
+        if (k == 0) {
+          pdl_wait();
+        } else {
+          ready = chain_wait(c.bar + (size_t)(k - 1) * CHAIN_BAR_STRIDE, chain_target(c, k - 1),
+                             abort_v, c.dev_flag, 80 + k);
+          // the input was written by generic stores; TMA reads it
+          asm volatile("fence.proxy.async.global;" ::: "memory");
+        }
+        if (k == 0) ts.waited();
+        // the activations of the stages begun (read even after a wait ran
+        // out, so that every stage's transaction completes)
+        for (int j = 0; j < npre_done; ++j) {
+          const uint32_t sa = base + (uint32_t)pre_s[j] * stage_bytes;
+          tma_load_2d((void *)__cvta_shared_to_generic(sa + A_BYTES), tX, &full_bar[pre_s[j]],
+                      pre_kb[j] * BK, pre_mt[j] * p.BN);
+        }
+        if (!ready || npre_done < npre) break;
+        for (; u < u1; ++u) {
+          if (!mbar_wait(&empty_bar[s], ph ^ 1u, abort_v, c.dev_flag, 1)) break;
+          const uint32_t sa = base + (uint32_t)s * stage_bytes;
+          mbar_expect_tx(&full_bar[s], tx_bytes);
+          load_w(sa);
+          tma_load_2d((void *)__cvta_shared_to_generic(sa + A_BYTES), tX, &full_bar[s], kb * BK,
+                      mtile * p.BN);
+          advance();
+        }
+      }
+      // copies in flight complete before the CTA may exit
+      for (uint32_t j = it > (uint32_t)S ? it - S : 0; j < it; ++j)
+        mbar_wait(&full_bar[j % S], (j / S) & 1u, abort_v, c.dev_flag, 0, false);
+    }
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- MMA
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16(BM, g0.BN);
+      uint32_t seg = 0, ph = 0;
+      int s = 0;
+#pragma unroll 1
+      for (int k = 0; k < CHAIN_MAX; ++k) {
+        if (k >= c.n_steps) break;
+        if (c.is_norm[k]) continue;
+        const TcParams &p = c.g[k];
+        long long u0, u1;
+        unit_range(blockIdx.x, p.total, p.grid, p.KB, 0, u0, u1);
+        if (!mma_range(p, u0, u1, s, ph, seg, S, base, stage_bytes, tmem_base, idesc, full_bar,
+                       empty_bar, accf_bar, acce_bar, abort_v))
+          break;
+      }
+      // all MMAs issued by this thread complete before TMEM is freed
+      mma_commit(&drain_bar);
+      mbar_wait(&drain_bar, 0, abort_v, c.dev_flag, 0, false);
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int q = warp & 3;  // TMEM lane quarter of this warp
+    const int f = q * 32 + lane;
+    const int et = threadIdx.x - 64;  // 0 .. EPI_THREADS - 1
+    const int eg = (warp - 2) >> 2;   // epilogue group
+    uint32_t seg = 0;
+#pragma unroll 1
+    for (int k = 0; k < CHAIN_MAX; ++k) {
+      if (k >= c.n_steps) break;
+      unsigned *arrive = c.bar + (size_t)k * CHAIN_BAR_STRIDE;
+      if (!c.is_norm[k]) {
+        // the step before is done before outputs or parts are written:
+        // the norm before reads the workspace this GEMM's parts go to
+        if (k == 0) {
+          pdl_wait();
+        } else {
+          if (et == 0)
+            chain_wait(c.bar + (size_t)(k - 1) * CHAIN_BAR_STRIDE, chain_target(c, k - 1),
+                       abort_v, c.dev_flag, 90 + k);
+          epi_bar();
+        }
+        const TcParams &p = c.g[k];
+        long long u0, u1;
+        unit_range(blockIdx.x, p.total, p.grid, p.KB, 0, u0, u1);
+        epi_range(p, u0, u1, seg, tmem_base, accf_bar, acce_bar, abort_v, q, f, et, eg);
+        epi_bar();  // every store of the step is issued by now
+        if (et == 0) {
+          __threadfence();
+          atomicAdd(arrive, 1u);
+        }
+      } else if ((int)blockIdx.x < c.M) {
+        if (k == 0) {
+          pdl_wait();
+        } else {
+          if (et == 0)
+            chain_wait(c.bar + (size_t)(k - 1) * CHAIN_BAR_STRIDE, chain_target(c, k - 1),
+                       abort_v, c.dev_flag, 90 + k);
+          epi_bar();
+        }
+        chain_norm(c.nrm[k], blockIdx.x, et, red);
+        epi_bar();
+        if (et == 0) {
+          __threadfence();
+          atomicAdd(arrive, 1u);
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 0) {
+    uint32_t ncols = 2 * g0.tmem_cols;
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
+                 "r"(ncols)
+                 : "memory");
+  }
+  ts.finish();
 }
 
 }  // namespace
@@ -788,6 +1184,118 @@ const char *launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, v
     }
   }
   return e == cudaSuccess ? nullptr : cudaGetErrorString(e);
+}
+
+size_t gemm_chain_bar_words() { return (size_t)CHAIN_MAX * CHAIN_BAR_STRIDE; }
+
+const char *launch_gemm_chain(const ChainStep *st, int n, const TcWorkspace &ws, unsigned *bar,
+                              cudaStream_t s, SplitView *last_defer) {
+  if (last_defer) *last_defer = SplitView{};
+  if (n < 1 || n > CHAIN_MAX) return "chain length outside [1, 6]";
+  ChainParams c{};
+  ChainMaps maps{};
+  c.n_steps = n;
+  c.bar = bar;
+  c.dev_flag = ws.dev_flag;
+  int ng = 0, nn = 0, M = -1, first = -1;
+  size_t smem = 0;
+  SplitView prev{};  // deferred split tiles of the GEMM just before
+  for (int k = 0; k < n; ++k) {
+    c.is_norm[k] = st[k].norm ? 1 : 0;
+    if (st[k].norm) {
+      if (nn == CHAIN_NORMS) return "more than two norms in a chain";
+      if (k + 1 < n && st[k + 1].norm) return "two norms in a row";
+      ChainNorm &nm = c.nrm[k];
+      nm.h = st[k].h;
+      nm.g = st[k].gain;
+      nm.eps = st[k].eps;
+      nm.d = st[k].d;
+      nm.out = (__nv_bfloat16 *)st[k].out;
+      nm.sv = prev;
+      if (nm.d % 4 || nm.d > 4 * EPI_THREADS * CHAIN_NORM_NV) return "norm width";
+      if (((uintptr_t)nm.h | (uintptr_t)nm.g | (uintptr_t)nm.out) & 15) return "norm alignment";
+      prev = SplitView{};
+      ++nn;
+      continue;
+    }
+    if (ng == CHAIN_GEMMS) return "more than four GEMMs in a chain";
+    const GemmArgs &g = st[k].g;
+    if (M < 0) M = g.M;
+    if (g.M != M || g.M <= 0) return "chain GEMMs of different row counts";
+    if (first < 0) first = k;
+    TcParams &p = c.g[k];
+    const bool dfr = st[k].defer && st[k].epi != GEMM_EPI_SWIGLU;
+    size_t sm = 0;
+    if (const char *e = configure(g.M, g.N, g.K, ws.num_sms, dfr, p, sm)) return e;
+    p.cluster = 0;  // stream-K over the whole grid
+    p.grid = (int)(p.total < ws.num_sms ? p.total : ws.num_sms);
+    if (p.grid != ws.num_sms) return "chain GEMM with fewer units than SMs";
+    if (dfr) {
+      const long long per = p.total / p.grid;
+      if (per < 1 || (p.KB + per - 1) / per + 1 > SPLIT_MAX_PARTS) return "chain GEMM split too fine";
+    }
+    if ((long long)p.n_tiles * p.m_tiles > ws.max_tiles) return "more tiles than counters";
+    if (first != k && (p.stages != c.g[first].stages || p.BN != c.g[first].BN))
+      return "chain GEMMs of different tilings";
+    p.Y = g.Y;
+    p.ldy = g.ldy;
+    p.bias = g.bias;
+    p.epi = st[k].epi;
+    p.out2 = st[k].out2;
+    p.ld2 = st[k].ld2;
+    p.ws = ws.partials;
+    p.counters = ws.counters;
+    p.max_tiles = ws.max_tiles;
+    p.dev_flag = ws.dev_flag;
+    maps.w[k] = *st[k].tmW;
+    if (!make_tmap_bf16(&maps.x[k], g.X, g.M, g.K, p.brows))
+      return "activation TMA descriptor rejected";
+    smem = sm > smem ? sm : smem;
+    prev = SplitView{};
+    if (dfr) {
+      bool split = false;
+      for (int i = 0; i < p.grid && !split; ++i) split = range_start(i, p.total, p.grid) % p.KB != 0;
+      if (split) {
+        prev.ws = ws.partials;
+        prev.bias = p.epi == GEMM_EPI_STORE ? g.bias : nullptr;
+        prev.total = p.total;
+        prev.grid = p.grid;
+        prev.KB = p.KB;
+        prev.BN = p.BN;
+        prev.m_tiles = p.m_tiles;
+        prev.accum = p.epi == GEMM_EPI_ACCUM ? 1 : 0;
+        prev.small = (p.total + 1) * (long long)p.grid < (1ll << 31) ? 1 : 0;
+      }
+    }
+    p.defer = dfr ? 1 : 0;
+    ++ng;
+  }
+  if (ng == 0) return "chain without a GEMM";
+  if (st[0].norm && (n < 2 || st[1].norm)) return "a chain's first norm feeds no GEMM";
+  if (nn > 0 && M > ws.num_sms) return "chain norm rows above the SM count";
+  c.M = M;
+  static int set_smem = -1;
+  if (set_smem < (int)smem) {
+    cudaError_t e = cudaFuncSetAttribute(k_gemm_chain, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return cudaGetErrorString(e);
+    set_smem = (int)smem;
+  }
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(ws.num_sms);
+  cfg.blockDim = dim3(NTHREADS);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = g_pdl ? 1 : 0;
+  cudaLaunchKernelEx(&cfg, k_gemm_chain, maps, c);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cudaGetErrorString(e);
+  if (last_defer) *last_defer = prev;
+  return nullptr;
 }
 
 KVR_TRACE_ATTACH(trace_attach_gemm)

@@ -254,6 +254,8 @@ struct kvr_model {
   kvr::SplitView pending{};    // split tiles of h not yet added (next RMSNorm adds them)
   bool defer_splits = true;    // GEMM split tiles reduced by the consumer
   bool use_tc5 = true;         // tcgen05 attention for single-document passes
+  bool use_chain = false;      // a pass's projections and norms as GEMM chains (opt-in)
+  unsigned *chain_bar = nullptr;  // hand-off counters of a pass's chains, zeroed per pass
   // pinned staging for host->device argument copies
   int32_t *stage_h = nullptr;
   int32_t *stage_d = nullptr;
@@ -505,6 +507,31 @@ size_t gemm_tc_ws_bytes(int num_sms);
 // (ws stays null when no tile was split, or when a tile would span more
 // than SPLIT_MAX_PARTS CTAs: then the GEMM reduces them itself).  Not for
 // the SwiGLU epilogue, which needs complete sums.
+// One step of a GEMM chain (launch_gemm_chain): a tensor-core GEMM with
+// launch_gemm_tc's arguments, or an RMSNorm of the chain's rows (h completed
+// in place from the previous GEMM's deferred split tiles, out in bf16).
+struct ChainStep {
+  bool norm = false;
+  GemmArgs g{};
+  const CUtensorMap *tmW = nullptr;
+  int epi = 0;
+  void *out2 = nullptr;
+  int ld2 = 0;
+  bool defer = false;  // split tiles left to the next step (a norm) or kernel
+  float *h = nullptr;
+  const float *gain = nullptr;
+  float eps = 0.f;
+  int d = 0;
+  void *out = nullptr;
+};
+// Up to 6 steps (at most 4 GEMMs, 2 norms) in one persistent launch of
+// num_sms CTAs; every GEMM has the same rows M (<= num_sms when a norm is
+// present) and at least num_sms stream-K units.  bar: gemm_chain_bar_words()
+// zeroed device words for this launch.  last_defer: the last GEMM's deferred
+// split tiles (ws null when it has none).  nullptr on success.
+size_t gemm_chain_bar_words();
+const char *launch_gemm_chain(const ChainStep *steps, int n, const TcWorkspace &ws, unsigned *bar,
+                              cudaStream_t s, SplitView *last_defer);
 const char *launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, void *out2,
                            int ld2, const TcWorkspace &ws, cudaStream_t s,
                            SplitView *defer = nullptr);

@@ -471,8 +471,13 @@ def compact_inputs(cfg, seed, docs, vocab_sample):
     return ocfg, W, [np.array([remap[int(t)] for t in d], np.int32) for d in docs]
 
 
-@pytest.mark.parametrize("shape", ["llama8b", "qwen7b"])
-def test_8b_shape_two_layer_parity(shape):
+@pytest.mark.parametrize("shape,chain", [("llama8b", False), ("qwen7b", False),
+                                         ("llama8b", True), ("qwen7b", True)])
+def test_8b_shape_two_layer_parity(shape, chain, monkeypatch):
+    # chain: the repair and logits passes' projections and norms as GEMM chains
+    # (one persistent launch per layer boundary, KVR_ENABLE_CHAIN)
+    if chain:
+        monkeypatch.setenv("KVR_ENABLE_CHAIN", "1")
     cfg = synth.preset(shape, n_layers=2)
     n, s, L, K = 200, 90, 6, 32
     doc = synth.document(1, n, cfg["vocab"])
@@ -483,7 +488,12 @@ def test_8b_shape_two_layer_parity(shape):
     model = kv.Model(cfg, None, seed=0, max_context=512, max_rows=256)
     cache = model.prefill(doc)
     A = np.arange(s + L, s + L + K)
+    l0 = model.launches()
     cache.repair(new, s, A)
+    # separate launches: embed, 9 kernels of layer 0 (with the split
+    # merge), norm/QKV/RoPE of layer 1; chained: embed, [norm, QKV],
+    # RoPE, attention, merge, [O, norm, gate/up, down, norm, QKV], RoPE
+    assert (model.launches() - l0 <= 7) == chain
     lg = model.logits(cache, query)
     ocfg, W, (odoc, onew, oq) = compact_inputs(cfg, 0, [doc, new, query], vs)
     ref = oracle.repair(ocfg, W, oracle.prefill(ocfg, W, odoc), onew, s, A)
