@@ -224,8 +224,8 @@ def run_reference(args, cfg, rank):
 # DRAM bytes (read + write) of one gate/up GEMM launch at this workload's shape
 # (40 x 28672 x 4096), from one ncu capture of that launch; reported only while the
 # GEMM kernel's source is the one the capture was taken on.
-GU_TRAFFIC_BYTES = 235282432 + 2532608
-GU_TRAFFIC_SOURCE_SHA256 = "ecbcbd0008452f3092e11bb7a240b0914a64dff6ea6883cbceb89c547ce0c6eb"
+GU_TRAFFIC_BYTES = 235282688 + 2533632
+GU_TRAFFIC_SOURCE_SHA256 = "ffd8f455c1db58864f815e38aac09aacd1cc5ddb1219730457d745c7b0bbfb17"
 
 
 def workload_config(cfg: dict, world: int) -> dict:

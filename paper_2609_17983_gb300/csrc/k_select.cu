@@ -101,6 +101,20 @@ __global__ void __launch_bounds__(TOPK_THREADS)
   __shared__ int s_elig, s_bin, s_above;
   __shared__ unsigned long long s_and, s_or;
   const int tid = threadIdx.x;
+  if (gen.policy == KVR_POLICY_EDITLOCAL ||
+      (gen.policy == KVR_POLICY_EDITLOCAL_BOUNDARY && nonzero_only)) {
+    // EditLocal's keys fall strictly with t, all nonzero (@boundary: nonzero
+    // up to the boundary, zero after it, and only nonzero keys eligible): the
+    // K largest are the first K candidates, already in index order.
+    const int avail = gen.policy == KVR_POLICY_EDITLOCAL ? c : min(c, *gen.bound - s_end + 1);
+    const int cnt = min(K, max(avail, 0));
+    for (int t = tid; t < cnt; t += TOPK_THREADS) out[t] = s_end + t;
+    if (tid == 0) {
+      *count = cnt;
+      if (flag_in) *flag_out = *flag_in;
+    }
+    return;
+  }
   const int E = (c + TOPK_THREADS - 1) / TOPK_THREADS;
   const int t0 = min(c, tid * E), t1 = min(c, t0 + E);
   if (tid == 0) {
