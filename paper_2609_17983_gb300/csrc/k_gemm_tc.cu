@@ -81,6 +81,11 @@ struct TcParams {
   int cluster;  // > 1: cluster split-K with this many CTAs per tile
   int defer;    // 1: split tiles are left as partials for the consumer
   int stream_w; // 1: each weight tile is read once (one token tile): L2 evict-first
+  // grouped data-parallel mode (dp_groups > 0, many rows): grid = dp_groups x
+  // m_tiles CTAs; CTA i owns whole tiles -- token tile i % m_tiles of feature
+  // tiles (i / m_tiles) * dp_tpc ... + dp_tpc - 1 -- so the m_tiles CTAs of a
+  // group walk the same weight tiles in step and read each from DRAM once.
+  int dp_groups, dp_tpc;
 };
 
 // ------------------------------------------------------------ PTX wrappers
@@ -205,12 +210,16 @@ __device__ __forceinline__ void epi_range(const P &p, long long u0, long long u1
     long long b = (tl + 1) * p.KB < u1 ? (tl + 1) * p.KB : u1;
     uint32_t buf = seg & 1u, use = seg >> 1;
     int ntile = (int)(tl / p.m_tiles), mtile = (int)(tl % p.m_tiles);
+    if (p.dp_groups) {  // a CTA-local tile of the grouped data-parallel mode
+      ntile = (int)(blockIdx.x / p.m_tiles) * p.dp_tpc + (int)tl;
+      mtile = (int)(blockIdx.x % p.m_tiles);
+    }
     int t0 = mtile * p.BN;
     int mv = min(p.BN, p.M - t0);
     int n = ntile * BM + f;
     long long tile_u0 = tl * p.KB;
-    int i_first = cta_of(tile_u0, p.total, p.grid);
-    int i_last = cta_of(tile_u0 + p.KB - 1, p.total, p.grid);
+    int i_first = p.dp_groups ? (int)blockIdx.x : cta_of(tile_u0, p.total, p.grid);
+    int i_last = p.dp_groups ? (int)blockIdx.x : cta_of(tile_u0 + p.KB - 1, p.total, p.grid);
     int parts = i_last - i_first + 1;
     // The owner of a split tile waits for the other parts and, with two
     // parts and at most 48 rows, loads the other one now, while this
@@ -361,7 +370,12 @@ __global__ void __launch_bounds__(NTHREADS, 1)
   const uint32_t stage_bytes = A_BYTES + (uint32_t)p.BN * 128u;
   const uint32_t tx_bytes = A_BYTES + (uint32_t)p.brows * 128u;
   long long u0, u1;
-  unit_range(blockIdx.x, p.total, p.grid, p.KB, p.cluster, u0, u1);
+  if (p.dp_groups) {  // CTA-local units: dp_tpc whole tiles
+    u0 = 0;
+    u1 = (long long)p.dp_tpc * p.KB;
+  } else {
+    unit_range(blockIdx.x, p.total, p.grid, p.KB, p.cluster, u0, u1);
+  }
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
@@ -403,6 +417,11 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       long long tl0 = u0 / p.KB;
       int kb = (int)(u0 - tl0 * p.KB);
       int ntile = (int)(tl0 / p.m_tiles), mtile = (int)(tl0 - (long long)ntile * p.m_tiles);
+      if (p.dp_groups) {
+        ntile = (int)(blockIdx.x / p.m_tiles) * p.dp_tpc;
+        mtile = (int)(blockIdx.x % p.m_tiles);
+      }
+      const int mstep = p.dp_groups ? 0 : 1;  // the data-parallel walk keeps its token tile
       int s = 0;
       uint32_t ph = 0, it = 0;
       const uint64_t wpol = l2_evict_first();
@@ -426,8 +445,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           load_w(sa, &full_bar[j], 0, (nt2 * p.KB + kb2) * BM);
           if (++kb2 == p.KB) {
             kb2 = 0;
-            if (++mt2 == p.m_tiles) {
-              mt2 = 0;
+            if ((mt2 += mstep) == p.m_tiles || !mstep) {
+              mt2 = mstep ? 0 : mt2;
               ++nt2;
             }
           }
@@ -445,8 +464,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           }
           if (++kb == p.KB) {
             kb = 0;
-            if (++mtile == p.m_tiles) {
-              mtile = 0;
+            if ((mtile += mstep) == p.m_tiles || !mstep) {
+              mtile = mstep ? 0 : mtile;
               ++ntile;
             }
           }
@@ -466,13 +485,12 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         }
         if (++kb == p.KB) {
           kb = 0;
-          if (++mtile == p.m_tiles) {
-            mtile = 0;
+          if ((mtile += mstep) == p.m_tiles || !mstep) {
+            mtile = mstep ? 0 : mtile;
             ++ntile;
           }
         }
       }
-      // warm L2 with the start of this CTA's share of the next GEMM's weights
       // copies in flight complete before the CTA may exit
       uint32_t n_issued = it;
       for (uint32_t j = n_issued > (uint32_t)S ? n_issued - S : 0; j < n_issued; ++j)
@@ -1109,6 +1127,52 @@ const char *configure(int M, int N, int K, int num_sms, bool defer, TcParams &p,
   p.cluster = p.m_tiles == 1 && !defer ? choose_cluster(M, N, num_sms, smem) : 0;
   p.stream_w = p.m_tiles == 1;
   if (p.cluster > 1) p.grid = p.n_tiles * p.cluster;
+  p.dp_groups = p.dp_tpc = 0;
+  // Many rows (a prefill chunk): the grouped data-parallel mode when some
+  // token tile width and group count fill at least 90% of the SMs' slots with
+  // useful rows.  Stream-K there walks all token tiles of a feature tile per
+  // CTA, so the 152 CTAs' weights (about 1 MB each) overflow L2 and every
+  // weight tile came from DRAM once per token tile.
+  static const bool dp_off = [] {
+    const char *e = getenv("KVR_DISABLE_DP_GEMM");
+    return e && e[0] == '1';
+  }();
+  if (!dp_off && M >= 512) {
+    double best = 0.0;
+    int bbn = 0, bmt = 0, bg = 0;
+    for (int bn = 256; bn >= 128; bn -= 16) {
+      const int mt = (M + bn - 1) / bn;
+      for (int g = 1; g <= p.n_tiles && g * mt <= num_sms; ++g) {
+        if (p.n_tiles % g) continue;
+        const double eff = (double)M / ((double)mt * bn) * (double)(g * mt) / num_sms;
+        if (eff > best + 1e-9) {
+          best = eff;
+          bbn = bn;
+          bmt = mt;
+          bg = g;
+        }
+      }
+    }
+    const uint32_t sb = A_BYTES + (uint32_t)bbn * 128u;
+    const int st = bbn ? smem_budget / (int)sb : 0;
+    if (best >= 0.9 && st >= 2) {
+      p.BN = bbn;
+      p.m_tiles = bmt;
+      p.brows = bbn < M ? bbn : M;
+      p.total = (long long)p.n_tiles * p.m_tiles * p.KB;
+      p.grid = bg * bmt;
+      p.dp_groups = bg;
+      p.dp_tpc = p.n_tiles / bg;
+      p.stages = st > 8 ? 8 : st;
+      uint32_t c2 = 32;
+      while (c2 < (uint32_t)p.BN) c2 <<= 1;
+      p.tmem_cols = c2;
+      smem = 1024 + (size_t)p.stages * sb;
+      p.defer = 0;  // whole tiles: nothing is split
+      p.cluster = 0;
+      p.stream_w = 0;
+    }
+  }
   return nullptr;
 }
 
@@ -1122,6 +1186,7 @@ const char *launch_gemm_tc(const GemmArgs &g, const CUtensorMap &tmW, int epi, v
   TcParams p{};
   size_t smem = 0;
   if (const char *e = configure(g.M, g.N, g.K, ws.num_sms, dfr, p, smem)) return e;
+  if (p.dp_groups) dfr = false;  // whole tiles per CTA: no split tiles to leave
   if (dfr) {
     // CTAs per tile: at most ceil(KB / (units per CTA)) + 1
     long long per = p.total / p.grid;
@@ -1227,6 +1292,7 @@ const char *launch_gemm_chain(const ChainStep *st, int n, const TcWorkspace &ws,
     const bool dfr = st[k].defer && st[k].epi != GEMM_EPI_SWIGLU;
     size_t sm = 0;
     if (const char *e = configure(g.M, g.N, g.K, ws.num_sms, dfr, p, sm)) return e;
+    if (p.dp_groups) return "chain GEMM with many rows (data-parallel tiling)";
     p.cluster = 0;  // stream-K over the whole grid
     p.grid = (int)(p.total < ws.num_sms ? p.total : ws.num_sms);
     if (p.grid != ws.num_sms) return "chain GEMM with fewer units than SMs";

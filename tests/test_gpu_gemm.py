@@ -61,3 +61,29 @@ def test_lm_head_matches_fp64_matmul(model):
     lm = model.read_tensor("lm_head")
     got = kv.kvr_linear(model.h, "lm_head", 0, x, lm.shape[0])
     assert rel(got, f64(x) @ f64(lm).T) <= 1e-3
+
+
+@pytest.mark.parametrize("M", [512, 4096])
+def test_many_row_projections_match_fp64_matmul(M):
+    # a prefill chunk's row counts: the grouped data-parallel tiling (whole
+    # tiles per CTA, token tiles of up to 256 rows with a ragged last one);
+    # the fp64 reference on a sample of rows from every token tile
+    cfg = synth.preset("llama8b", n_layers=1)
+    m = kv.Model(cfg, None, seed=0, max_context=512, max_rows=4096)
+    d, F = cfg["d_model"], cfg["ffn"]
+    rows = np.unique(np.concatenate([np.arange(0, M, 61), np.arange(M - 8, M)]))
+    x = synth.tensor(300 + M, 5, (M, d), "bf16", std=1.0)
+    xf = f64(x[rows])
+    for name, w in (("wqkv", np.concatenate([m.read_tensor(n, 0) for n in ("wq", "wk", "wv")])),
+                    ("wo", m.read_tensor("wo", 0))):
+        got = kv.kvr_linear(m.h, name, 0, x, w.shape[0])
+        assert rel(got[rows], xf @ f64(w).T) <= 1e-3, name
+    xd = synth.tensor(400 + M, 5, (M, F), "bf16", std=1.0)
+    wd = m.read_tensor("wd", 0)
+    got = kv.kvr_linear(m.h, "wd", 0, xd, d)
+    assert rel(got[rows], f64(xd[rows]) @ f64(wd).T) <= 1e-3
+    g = xf @ f64(m.read_tensor("wg", 0)).T
+    u = xf @ f64(m.read_tensor("wu", 0)).T
+    got = kv.kvr_linear(m.h, "wgu", 0, x, F)
+    assert rel(got[rows], g / (1.0 + np.exp(-g)) * u) <= 1e-2  # output rounded to bf16
+    m.close()
