@@ -224,8 +224,8 @@ def run_reference(args, cfg, rank):
 # DRAM bytes (read + write) of one gate/up GEMM launch at this workload's shape
 # (40 x 28672 x 4096), from one ncu capture of that launch; reported only while the
 # GEMM kernel's source is the one the capture was taken on.
-GU_TRAFFIC_BYTES = 235282688 + 2533632
-GU_TRAFFIC_SOURCE_SHA256 = "ffd8f455c1db58864f815e38aac09aacd1cc5ddb1219730457d745c7b0bbfb17"
+GU_TRAFFIC_BYTES = 235280384 + 2372864
+GU_TRAFFIC_SOURCE_SHA256 = "8c50084a4dde7e11d5b7e916f8acb26422331cd7d45204691d56920573cc9aa6"
 
 
 def workload_config(cfg: dict, world: int) -> dict:
