@@ -165,75 +165,82 @@ __global__ void __launch_bounds__(TPB) k_rmsnorm(float *h, const float *g, int r
 // so they are read before the wait on the projection.
 constexpr int ROPE_HEADS = 8;  // heads per CTA
 template <typename T>
-__global__ void k_rope_scatter(const float *qkv, const float2 *rope, const int32_t *pos, int H,
-                               int G, int dh, int layer, const KVView *views,
+__global__ void k_rope_scatter(const float *qkv, const float2 *rope, const int32_t *pos, int M,
+                               int rpb, int H, int G, int dh, int layer, const KVView *views,
                                const int32_t *rowdoc, KVView single, float *q_out,
                                __nv_bfloat16 *qb_out, float qscale, int write_kv,
                                const SplitView sv) {
   TraceScope ts(TK_ROPE);
   pdl_trigger();
   const int half = dh >> 1;
-  const int i = blockIdx.x, hh = blockIdx.y * ROPE_HEADS + threadIdx.x / half,
-            t = threadIdx.x % half;
+  const int hh = blockIdx.y * ROPE_HEADS + threadIdx.x / half, t = threadIdx.x % half;
   if (hh >= H + 2 * G) return;
   const int Nqkv = (H + 2 * G) * dh;
   const int n1 = hh * dh + t, n2 = n1 + half;
-  const int p = pos[i];
-  float2 cs = make_float2(1.f, 0.f);
-  if (hh < H + G) cs = rope[(size_t)p * half + t];
-  T *c = nullptr;
-  size_t o = 0;
-  if (hh >= H && write_kv) {
-    const KVView v = views ? views[rowdoc[i]] : single;
-    const int kv = hh < H + G ? 0 : 1;
-    c = (T *)v.pages;
-    o = v.offset(layer, kv, hh - H - kv * G, p);
-  }
-  // dh divides 128: both halves of the head lie in one feature tile
-  SplitTile stl{0, 0, 0};
-  float b1 = 0.f, b2 = 0.f;
-  if (sv.ws) {
-    stl = split_tile(sv, (long long)((hh * dh) >> 7) * sv.m_tiles + i / sv.BN);
-    if (sv.bias) {
-      b1 = sv.bias[n1];
-      b2 = sv.bias[n2];
+  // rows r0 .. r1-1 (one for a pass of a few rows; several for a prefill
+  // chunk, where one row per CTA spent its time starting CTAs); the first
+  // row's position, table entries and split tile are read before the wait
+  const int r0 = blockIdx.x * rpb, r1 = min(M, r0 + rpb);
+  for (int i = r0; i < r1; ++i) {
+    const int p = pos[i];
+    float2 cs = make_float2(1.f, 0.f);
+    if (hh < H + G) cs = rope[(size_t)p * half + t];
+    T *c = nullptr;
+    size_t o = 0;
+    if (hh >= H && write_kv) {
+      const KVView v = views ? views[rowdoc[i]] : single;
+      const int kv = hh < H + G ? 0 : 1;
+      c = (T *)v.pages;
+      o = v.offset(layer, kv, hh - H - kv * G, p);
     }
-  }
-  const bool split = sv.ws && stl.i0 != stl.i1;
-  pdl_wait();
-  ts.waited();
-  float x1, x2;
-  if (split) {
-    const size_t off = (size_t)(i - (i / sv.BN) * sv.BN) * 128;
-    x1 = b1 + split_sum(sv, stl, off + (n1 & 127));
-    x2 = b2 + split_sum(sv, stl, off + (n2 & 127));
-  } else {
-    const float *x = qkv + (size_t)i * Nqkv;
-    x1 = x[n1];
-    x2 = x[n2];
-  }
-  if (hh < H + G) {
-    const float r1 = x1 * cs.x - x2 * cs.y;
-    const float r2 = x2 * cs.x + x1 * cs.y;
-    x1 = r1;
-    x2 = r2;
-  }
-  if (hh < H) {
-    if (q_out) {
-      float *qo = q_out + (size_t)i * H * dh + (size_t)hh * dh;
-      qo[t] = x1;
-      qo[t + half] = x2;
+    // dh divides 128: both halves of the head lie in one feature tile
+    SplitTile stl{0, 0, 0};
+    float b1 = 0.f, b2 = 0.f;
+    if (sv.ws) {
+      stl = split_tile(sv, (long long)((hh * dh) >> 7) * sv.m_tiles + i / sv.BN);
+      if (sv.bias) {
+        b1 = sv.bias[n1];
+        b2 = sv.bias[n2];
+      }
     }
-    if (qb_out) {
-      __nv_bfloat16 *qb = qb_out + (size_t)i * H * dh + (size_t)hh * dh;
-      qb[t] = __float2bfloat16_rn(x1 * qscale);
-      qb[t + half] = __float2bfloat16_rn(x2 * qscale);
+    const bool split = sv.ws && stl.i0 != stl.i1;
+    if (i == r0) {
+      pdl_wait();
+      ts.waited();
     }
-    return;
+    float x1, x2;
+    if (split) {
+      const size_t off = (size_t)(i - (i / sv.BN) * sv.BN) * 128;
+      x1 = b1 + split_sum(sv, stl, off + (n1 & 127));
+      x2 = b2 + split_sum(sv, stl, off + (n2 & 127));
+    } else {
+      const float *x = qkv + (size_t)i * Nqkv;
+      x1 = x[n1];
+      x2 = x[n2];
+    }
+    if (hh < H + G) {
+      const float r1r = x1 * cs.x - x2 * cs.y;
+      const float r2r = x2 * cs.x + x1 * cs.y;
+      x1 = r1r;
+      x2 = r2r;
+    }
+    if (hh < H) {
+      if (q_out) {
+        float *qo = q_out + (size_t)i * H * dh + (size_t)hh * dh;
+        qo[t] = x1;
+        qo[t + half] = x2;
+      }
+      if (qb_out) {
+        __nv_bfloat16 *qb = qb_out + (size_t)i * H * dh + (size_t)hh * dh;
+        qb[t] = __float2bfloat16_rn(x1 * qscale);
+        qb[t + half] = __float2bfloat16_rn(x2 * qscale);
+      }
+      continue;
+    }
+    if (!c) continue;
+    st(c, o + t, x1);
+    st(c, o + t + half, x2);
   }
-  if (!c) return;
-  st(c, o + t, x1);
-  st(c, o + t + half, x2);
 }
 
 template <typename T>
@@ -449,17 +456,19 @@ void launch_rope_scatter(const float *qkv, const float2 *rope, const int32_t *po
                          KVView single, float *q_out, void *qb_out, float qscale, bool write_kv,
                          cudaStream_t s, const SplitView *sv) {
   if (M <= 0) return;
-  dim3 grid(M, (dm.H + 2 * dm.G + ROPE_HEADS - 1) / ROPE_HEADS);
+  const int rpb = M >= 1024 ? 8 : 1;  // rows per CTA
+  dim3 grid((M + rpb - 1) / rpb, (dm.H + 2 * dm.G + ROPE_HEADS - 1) / ROPE_HEADS);
   const int threads = ROPE_HEADS * dm.dh / 2;
   int wk = write_kv ? 1 : 0;
   const SplitView v = sv ? *sv : SplitView{};
   if (dm.dtype == KVR_DTYPE_BF16)
-    launch_pdl(k_rope_scatter<__nv_bfloat16>, grid, threads, 0, s, qkv, rope, pos, dm.H, dm.G,
+    launch_pdl(k_rope_scatter<__nv_bfloat16>, grid, threads, 0, s, qkv, rope, pos, M, rpb, dm.H,
+               dm.G, dm.dh, layer, views, rowdoc, single, q_out, (__nv_bfloat16 *)qb_out, qscale,
+               wk, v);
+  else
+    launch_pdl(k_rope_scatter<float>, grid, threads, 0, s, qkv, rope, pos, M, rpb, dm.H, dm.G,
                dm.dh, layer, views, rowdoc, single, q_out, (__nv_bfloat16 *)qb_out, qscale, wk,
                v);
-  else
-    launch_pdl(k_rope_scatter<float>, grid, threads, 0, s, qkv, rope, pos, dm.H, dm.G, dm.dh,
-               layer, views, rowdoc, single, q_out, (__nv_bfloat16 *)qb_out, qscale, wk, v);
 }
 
 void launch_swiglu(const float *gu, int M, int F, void *act, int dtype, cudaStream_t s) {
