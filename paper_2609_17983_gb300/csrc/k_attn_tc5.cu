@@ -356,6 +356,9 @@ __global__ void __launch_bounds__(NT5, 1)
       const int b = i & 1, key0 = (c0 + i) * CH + part * HK;
       uint32_t sr[HK];
       float mx = -INFINITY;
+      // every key of this part is causal for every query vector of the warp:
+      // the chunk needs no mask (all but the diagonal chunk of a block)
+      const bool unmasked = __all_sync(0xffffffffu, key0 + HK - 1 <= pv);
       if (!dead) {
         dead = !__all_sync(0xffffffffu,
                            mbar_wait(&s_full[b], (i >> 1) & 1, abort_v, p.dev_flag, 69));
@@ -371,11 +374,20 @@ __global__ void __launch_bounds__(NT5, 1)
         tc_fence_before();
         mbar_arrive(&s_free[b]);  // S is in registers: the buffer may be refilled
         float t[HK];
+        if (unmasked) {
 #pragma unroll
-        for (int j = 0; j < HK; ++j) {
-          const float x = __uint_as_float(sr[j]) * p.qk_scale;
-          sr[j] = __float_as_uint(x);
-          t[j] = key0 + j <= pv ? x : -INFINITY;
+          for (int j = 0; j < HK; ++j) {
+            const float x = __uint_as_float(sr[j]) * p.qk_scale;
+            sr[j] = __float_as_uint(x);
+            t[j] = x;
+          }
+        } else {
+#pragma unroll
+          for (int j = 0; j < HK; ++j) {
+            const float x = __uint_as_float(sr[j]) * p.qk_scale;
+            sr[j] = __float_as_uint(x);
+            t[j] = key0 + j <= pv ? x : -INFINITY;
+          }
         }
 #pragma unroll
         for (int w = HK / 2; w > 0; w >>= 1)
@@ -419,8 +431,13 @@ __global__ void __launch_bounds__(NT5, 1)
         if (dead) continue;
       }
       float e[HK];
+      if (unmasked) {
 #pragma unroll
-      for (int j = 0; j < HK; ++j) e[j] = key0 + j <= pv ? ex2(__uint_as_float(sr[j]) - m) : 0.f;
+        for (int j = 0; j < HK; ++j) e[j] = ex2(__uint_as_float(sr[j]) - m);
+      } else {
+#pragma unroll
+        for (int j = 0; j < HK; ++j) e[j] = key0 + j <= pv ? ex2(__uint_as_float(sr[j]) - m) : 0.f;
+      }
       {  // P in bf16 pairs: this part's HK keys are HK / 2 columns of buffer b
         uint32_t w[HK / 2];
 #pragma unroll
