@@ -503,6 +503,22 @@ def test_8b_shape_two_layer_parity(shape, chain, monkeypatch):
     model.close()
 
 
+def test_8b_shape_prefill_many_rows_parity():
+    # a prefill chunk of 600 rows: enough for the GEMMs' grouped data-parallel
+    # tiling (whole tiles per CTA, a ragged last token tile) where it fills
+    # the SMs (the QKV projection here), stream-K elsewhere; every row's K/V
+    # at both layers against the oracle's prefill
+    cfg = synth.preset("llama8b", n_layers=2)
+    n = 600
+    doc = synth.document(4, n, cfg["vocab"])
+    model = kv.Model(cfg, None, seed=0, max_context=1024, max_rows=1024)
+    cache = model.prefill(doc)
+    ocfg, W, (odoc,) = compact_inputs(cfg, 0, [doc], np.array([0], np.int32))
+    ref = oracle.prefill(ocfg, W, odoc)
+    cmp_rows(cache, ref, np.arange(n), TOL["bf16"])
+    model.close()
+
+
 @pytest.mark.parametrize("n", [5000, 8192])
 def test_select_long_context_exact(n):
     # the top-K at the largest pools (up to max_context candidates)
