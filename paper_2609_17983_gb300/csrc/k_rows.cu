@@ -94,12 +94,11 @@ __global__ void k_embed_rows(const T *embed, const int32_t *tokens,
 // built once per block in shared memory) and written back to h.
 constexpr int NORM_THREADS = 1024;   // a few rows: one float4 per thread, one round trip
 constexpr int NORM_THREADS_WIDE = 256;  // many rows: several CTAs per SM, fewer waves
-// (The wide variant asks for four CTAs per SM: at 86 registers only two fit,
-// and a prefill chunk's rows then ran at about half the copy bandwidth.)
+// The wide variant asks for four CTAs per SM: at 86 registers only two fit
+// (prefill norms 3.2 against 2.9 ms).
 template <typename T, int NV, int TPB>
 __global__ void __launch_bounds__(TPB, TPB == NORM_THREADS_WIDE && NV <= 4 ? 4 : 1)
-    k_rmsnorm(float *h, const float *g, int row0, int d,
-                                                 float eps, T *out, const SplitView sv) {
+    k_rmsnorm(float *h, const float *g, int row0, int d, float eps, T *out, const SplitView sv) {
   __shared__ SplitTile tiles[64];
   __shared__ float red[TPB / 32];
   TraceScope ts(TK_NORM);
