@@ -490,9 +490,8 @@ def main():
     all_ms = sum(v["ms"] for v in gemms.values())
 
     # e2e through the public API: host inputs in, the repaired rows' K/V out as
-    # stored (bf16) into page-locked host buffers allocated once
-    P = np.concatenate([np.arange(EDIT_START, EDIT_START + EDIT_LEN),
-                        np.arange(EDIT_START + EDIT_LEN, EDIT_START + EDIT_LEN + K_BUDGET)])
+    # stored (bf16) into page-locked host buffers allocated once; the rows of
+    # each layer group are copied out while the pass computes the next ones
     shape = (M, cfg["n_layers"], cfg["n_kv_heads"], cfg["head_dim"])
     k_rows = torch.empty(shape, dtype=torch.int16, pin_memory=True).numpy().view(np.uint16)
     v_rows = torch.empty(shape, dtype=torch.int16, pin_memory=True).numpy().view(np.uint16)
@@ -500,8 +499,7 @@ def main():
     t0 = time.perf_counter()
     for _ in range(args.steps):
         A = model.select(cache, "editlocal", K_BUDGET, EDIT_START, new)
-        cache.repair(new, EDIT_START, A)
-        cache.read_raw(P, k_out=k_rows, v_out=v_rows)
+        cache.repair_read(new, EDIT_START, A, k_out=k_rows, v_out=v_rows)
     barrier()
     e2e_s = max_over_ranks((time.perf_counter() - t0) / args.steps, "cuda")
     h2d = int(new.nbytes + 4 * K_BUDGET + 4 * M)

@@ -174,6 +174,21 @@ kvr_status kvr_select(kvr_model *model, const kvr_cache *cache, kvr_policy polic
 kvr_status kvr_repair(kvr_cache *cache, const int32_t *new_tokens, int32_t edit_start,
                       int32_t edit_len, const int32_t *positions, int32_t n_positions);
 
+/* kvr_repair, returning the recomputed entries (Sec. 3, Eq. 1: the rows of P
+ * of the repaired cache) in host memory: k_out, v_out receive
+ * [|P|][n_layers][n_kv_heads][head_dim] in the cache's element type (bf16 bit
+ * patterns for a bf16 model, fp32 otherwise), rows in P's ascending order
+ * (the span, then positions) -- what kvr_cache_read_raw returns for P after
+ * kvr_repair.  The rows of each group of layers are copied while the pass
+ * computes the later layers; with page-locked k_out/v_out the copies overlap
+ * the pass, pageable memory is accepted.  Synchronous: returns once the rows
+ * are in host memory, reporting device-side timeouts like kvr_synchronize.
+ * A row buffer on the device belongs to the model and only grows.  Errors as
+ * kvr_repair; KVR_E_INVAL for NULL k_out or v_out with |P| > 0. */
+kvr_status kvr_repair_read(kvr_cache *cache, const int32_t *new_tokens, int32_t edit_start,
+                           int32_t edit_len, const int32_t *positions, int32_t n_positions,
+                           void *k_out, void *v_out);
+
 /* One repair request of a batch: a cache, its edits and the union of the
  * selected positions.  Edits must not overlap; positions must not fall in
  * any edit span. */

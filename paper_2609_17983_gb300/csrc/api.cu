@@ -170,6 +170,10 @@ struct Rows {
   const CUtensorMap *tm_kv = nullptr;        // TMA view of the single document's pages
   const CUtensorMap *tmaps = nullptr;        // device [docs]: TMA views of a batch's pages
   bool tc5 = false;                          // attention on tcgen05 (set by plan_attention)
+  // kvr_repair_read: RoPE also writes the rows' K/V to rows_out (K then V,
+  // [M][L][G][dh]); after every rd_every layers an event marks them ready
+  void *rows_out = nullptr;
+  int rd_every = 0;
 };
 
 bool use_tc_attention(const kvr_model *m) {
@@ -255,7 +259,7 @@ kvr_status rope(kvr_model *m, const Rows &r, int l, bool write_kv, bool need_q,
   const bool tc = use_tc_attention(m);
   launch_rope_scatter(m->qkv, m->rope, r.pos, r.M, dm, l, r.views, r.rowdoc, r.single,
                       tc && !need_q ? nullptr : m->q, tc ? m->qb : nullptr, 1.0f, write_kv,
-                      m->stream, &sv);
+                      m->stream, &sv, write_kv ? r.rows_out : nullptr);
   return launch_check(m, 1);
 }
 
@@ -332,7 +336,7 @@ kvr_status layer_rest(kvr_model *m, const Rows &r, int l) {
 // residual width within the chain norm's reach.
 bool chain_ok(const kvr_model *m, const Rows &r) {
   const Dims &dm = m->dims;
-  if (!m->use_chain || !m->chain_bar || !m->use_tc || !m->defer_splits ||
+  if (!m->use_chain || !m->chain_bar || !m->use_tc || !m->defer_splits || r.rows_out ||
       dm.dtype != KVR_DTYPE_BF16 || r.M <= 0 || r.M > m->num_sms || dm.d > 4096 || dm.d % 4)
     return false;
   for (int l = 0; l < dm.L; ++l) {
@@ -414,13 +418,41 @@ kvr_status run_pass_chain(kvr_model *m, const Rows &r, bool kv_only) {
   return KVR_OK;
 }
 
+// With rows_out: after layer l's RoPE, at the end of each group of rd_every
+// layers, the event the group's host copies wait on.  Inside a capture the
+// event is recorded on a side branch (rd_cap), so that the pass's kernels
+// keep their programmatic edges; the branch rejoins at the end of the pass.
+kvr_status rows_ready(kvr_model *m, const Rows &r, int l, bool capturing) {
+  const int L = m->dims.L;
+  if (!r.rows_out || ((l + 1) % r.rd_every && l + 1 < L)) return KVR_OK;
+  const int g = l / r.rd_every;
+  cudaError_t e;
+  if (capturing) {
+    e = cudaEventRecord(m->rd_fork[g], m->stream);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(m->rd_cap, m->rd_fork[g], 0);
+    if (e == cudaSuccess)
+      e = cudaEventRecordWithFlags(m->rd_ev[g], m->rd_cap, cudaEventRecordExternal);
+  } else {
+    e = cudaEventRecord(m->rd_ev[g], m->stream);
+  }
+  return e == cudaSuccess ? KVR_OK : fail(KVR_E_CUDA, "readback event: %s", cudaGetErrorString(e));
+}
+
 kvr_status run_pass(kvr_model *m, const Rows &r, bool kv_only) {
   if (r.M <= 0) return KVR_OK;
   if (chain_ok(m, r)) return run_pass_chain(m, r, kv_only);
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  if (r.rows_out) CUDA_TRY(cudaStreamIsCapturing(m->stream, &cs));
+  const bool capturing = cs == cudaStreamCaptureStatusActive;
   KVR_TRY(embed(m, r));
   for (int l = 0; l < m->dims.L; ++l) {
     KVR_TRY(layer_qkv(m, r, l, true));
+    KVR_TRY(rows_ready(m, r, l, capturing));
     if (!kv_only || l + 1 < m->dims.L) KVR_TRY(layer_rest(m, r, l));
+  }
+  if (capturing) {
+    CUDA_TRY(cudaEventRecord(m->rd_join, m->rd_cap));
+    CUDA_TRY(cudaStreamWaitEvent(m->stream, m->rd_join, 0));
   }
   return KVR_OK;
 }
@@ -433,7 +465,7 @@ kvr_status run_pass(kvr_model *m, const Rows &r, bool kv_only) {
 kvr_status run_pass_graph(kvr_model *m, kvr_cache *c, const Rows &r) {
   if (!m->use_graphs || m->prof || m->stream == nullptr) return run_pass(m, r, true);
   for (auto &g : c->graphs)
-    if (g.M == r.M && g.nb == r.n_blocks && g.ns == r.n_splits) {
+    if (g.M == r.M && g.nb == r.n_blocks && g.ns == r.n_splits && g.rows_out == r.rows_out) {
       cudaError_t e = cudaGraphLaunch(g.exec, m->stream);
       if (e != cudaSuccess) return fail(KVR_E_CUDA, "graph launch: %s", cudaGetErrorString(e));
       m->launches += g.kernels;
@@ -454,18 +486,19 @@ kvr_status run_pass_graph(kvr_model *m, kvr_cache *c, const Rows &r) {
   e = cudaGraphInstantiate(&exec, graph, 0);
   cudaGraphDestroy(graph);
   if (e != cudaSuccess) return fail(KVR_E_CUDA, "graph instantiate: %s", cudaGetErrorString(e));
-  c->graphs.push_back({r.M, r.n_blocks, r.n_splits, m->launches - l0, exec});
+  c->graphs.push_back({r.M, r.n_blocks, r.n_splits, r.rows_out, m->launches - l0, exec});
   e = cudaGraphLaunch(exec, m->stream);
   if (e != cudaSuccess) return fail(KVR_E_CUDA, "graph launch: %s", cudaGetErrorString(e));
   return KVR_OK;
 }
 
 kvr_status sync_model(kvr_model *m) {
-  cudaError_t e = cudaStreamSynchronize(m->stream);
+  // the flag's copy joins the stream's work: one round trip to the host
+  cudaError_t e = cudaMemcpyAsync(m->flag_h, m->dev_flag, sizeof(int), cudaMemcpyDeviceToHost,
+                                  m->stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(m->stream);
   if (e != cudaSuccess) return fail(KVR_E_CUDA, "device error: %s", cudaGetErrorString(e));
-  int flag = 0;
-  e = cudaMemcpy(&flag, m->dev_flag, sizeof(int), cudaMemcpyDeviceToHost);
-  if (e != cudaSuccess) return fail(KVR_E_CUDA, "device error: %s", cudaGetErrorString(e));
+  const int flag = *m->flag_h;
   if (flag) {
     cudaMemset(m->dev_flag, 0, sizeof(int));
     if (m->tcw.counters)
@@ -659,6 +692,14 @@ void kvr_model_free(kvr_model *m) {
   dev_free(m->chain_bar);
   dev_free(m->tcw.partials);
   dev_free(m->read_scratch);
+  dev_free(m->rows_scratch);
+  for (int g = 0; g < KVR_RD_GROUPS; ++g) {
+    if (m->rd_ev[g]) cudaEventDestroy(m->rd_ev[g]);
+    if (m->rd_fork[g]) cudaEventDestroy(m->rd_fork[g]);
+  }
+  if (m->rd_join) cudaEventDestroy(m->rd_join);
+  if (m->rd_stream) cudaStreamDestroy(m->rd_stream);
+  if (m->rd_cap) cudaStreamDestroy(m->rd_cap);
   dev_free(m->sel_scratch);
   dev_free(m->batch_scratch);
   dev_free(m->tcw.counters);
@@ -667,6 +708,7 @@ void kvr_model_free(kvr_model *m) {
   dev_free(m->attn_ws_ml);
   if (m->stage_h) cudaFreeHost(m->stage_h);
   if (m->rb_h) cudaFreeHost(m->rb_h);
+  if (m->flag_h) cudaFreeHost(m->flag_h);
   if (m->stage_ev) cudaEventDestroy(m->stage_ev);
   delete m;
 }
@@ -889,7 +931,15 @@ kvr_status kvr_model_create(const kvr_model_config *cfg, const kvr_weights *wts,
       return bail(fail(KVR_E_NOMEM, "pinned staging"));
     cudaEventCreateWithFlags(&m->stage_ev, cudaEventDisableTiming);
     cudaEventRecord(m->stage_ev, 0);
-    if (cudaMallocHost(&m->rb_h, ((size_t)P + 8) * sizeof(int32_t)) != cudaSuccess)
+    bool rd_ok = cudaStreamCreateWithFlags(&m->rd_stream, cudaStreamNonBlocking) == cudaSuccess &&
+                 cudaStreamCreateWithFlags(&m->rd_cap, cudaStreamNonBlocking) == cudaSuccess &&
+                 cudaEventCreateWithFlags(&m->rd_join, cudaEventDisableTiming) == cudaSuccess;
+    for (int g = 0; g < KVR_RD_GROUPS && rd_ok; ++g)
+      rd_ok = cudaEventCreateWithFlags(&m->rd_ev[g], cudaEventDisableTiming) == cudaSuccess &&
+              cudaEventCreateWithFlags(&m->rd_fork[g], cudaEventDisableTiming) == cudaSuccess;
+    if (!rd_ok) return bail(fail(KVR_E_CUDA, "readback streams and events"));
+    if (cudaMallocHost(&m->rb_h, ((size_t)P + 8) * sizeof(int32_t)) != cudaSuccess ||
+        cudaMallocHost(&m->flag_h, sizeof(int32_t)) != cudaSuccess)
       return bail(fail(KVR_E_NOMEM, "pinned readback"));
   }
   // ---- tensor-core GEMM: workspace and weight TMA descriptors
@@ -1124,8 +1174,12 @@ kvr_status kvr_prefill(kvr_model *m, const int32_t *tokens, int32_t n, kvr_cache
   return KVR_OK;
 }
 
-kvr_status kvr_repair(kvr_cache *c, const int32_t *new_tokens, int32_t edit_start,
-                      int32_t edit_len, const int32_t *positions, int32_t n_positions) {
+namespace {
+// kvr_repair, and with k_out/v_out (kvr_repair_read) the copy of the rows'
+// K/V to the host overlapping the pass.
+kvr_status repair_impl(kvr_cache *c, const int32_t *new_tokens, int32_t edit_start,
+                       int32_t edit_len, const int32_t *positions, int32_t n_positions,
+                       void *k_out, void *v_out) {
   if (!c) return fail(KVR_E_INVAL, "NULL cache");
   if (c->poisoned) return fail(KVR_E_POISONED, "cache poisoned by an earlier CUDA error");
   kvr_model *m = c->model;
@@ -1171,9 +1225,33 @@ kvr_status kvr_repair(kvr_cache *c, const int32_t *new_tokens, int32_t edit_star
     r.tm_kv = c->tm_kv_ok ? &c->tm_kv : nullptr;
     r.max_pos = P[M - 1];
     st = plan_attention(m, r, P.data(), nullptr);
+    const size_t row_b = (size_t)dm.L * dm.G * dm.dh * dm.es();  // one row, all layers
+    if (!st && k_out) {
+      st = grow_scratch(m, m->rows_scratch, m->rows_scratch_bytes, 2 * M * row_b, "row buffer");
+      r.rows_out = m->rows_scratch;
+      r.rd_every = (dm.L + KVR_RD_GROUPS - 1) / KVR_RD_GROUPS;
+    }
     if (!st) {
       launched = true;
       st = run_pass_graph(m, c, r);
+    }
+    if (!st && k_out) {
+      // group g's rows leave as soon as the pass has written them
+      const char *kd = (const char *)r.rows_out, *vd = kd + M * row_b;
+      const size_t lb = row_b / dm.L;
+      for (int g = 0, l0 = 0; l0 < dm.L && !st; ++g, l0 += r.rd_every) {
+        const size_t w = (size_t)(std::min(dm.L, l0 + r.rd_every) - l0) * lb;
+        if (cudaStreamWaitEvent(m->rd_stream, m->rd_ev[g], 0) != cudaSuccess ||
+            cudaMemcpy2DAsync((char *)k_out + l0 * lb, row_b, kd + l0 * lb, row_b, w, M,
+                              cudaMemcpyDeviceToHost, m->rd_stream) != cudaSuccess ||
+            cudaMemcpy2DAsync((char *)v_out + l0 * lb, row_b, vd + l0 * lb, row_b, w, M,
+                              cudaMemcpyDeviceToHost, m->rd_stream) != cudaSuccess)
+          st = fail(KVR_E_CUDA, "row readback");
+      }
+      const kvr_status s2 = sync_model(m);
+      if (!st) st = s2;
+      if (cudaStreamSynchronize(m->rd_stream) != cudaSuccess && !st)
+        st = fail(KVR_E_CUDA, "row readback");
     }
   }
   if (st && st != KVR_E_CUDA && !launched && edit_len) {
@@ -1183,6 +1261,21 @@ kvr_status kvr_repair(kvr_cache *c, const int32_t *new_tokens, int32_t edit_star
   }
   if (st == KVR_E_CUDA || (st && launched)) c->poisoned = true;
   return st;
+}
+}  // namespace
+
+kvr_status kvr_repair(kvr_cache *c, const int32_t *new_tokens, int32_t edit_start,
+                      int32_t edit_len, const int32_t *positions, int32_t n_positions) {
+  return repair_impl(c, new_tokens, edit_start, edit_len, positions, n_positions, nullptr,
+                     nullptr);
+}
+
+kvr_status kvr_repair_read(kvr_cache *c, const int32_t *new_tokens, int32_t edit_start,
+                           int32_t edit_len, const int32_t *positions, int32_t n_positions,
+                           void *k_out, void *v_out) {
+  if (edit_len + n_positions > 0 && (!k_out || !v_out))
+    return fail(KVR_E_INVAL, "NULL k_out or v_out");
+  return repair_impl(c, new_tokens, edit_start, edit_len, positions, n_positions, k_out, v_out);
 }
 
 kvr_status kvr_repair_batch(kvr_model *m, const kvr_repair_req *reqs, int32_t n_reqs) {

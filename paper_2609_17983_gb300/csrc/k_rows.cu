@@ -171,7 +171,7 @@ __global__ void k_rope_scatter(const float *qkv, const float2 *rope, const int32
                                int rpb, int H, int G, int dh, int layer, const KVView *views,
                                const int32_t *rowdoc, KVView single, float *q_out,
                                __nv_bfloat16 *qb_out, float qscale, int write_kv,
-                               const SplitView sv) {
+                               const SplitView sv, T *rows_out, int L) {
   TraceScope ts(TK_ROPE);
   pdl_trigger();
   const int half = dh >> 1;
@@ -188,12 +188,14 @@ __global__ void k_rope_scatter(const float *qkv, const float2 *rope, const int32
     float2 cs = make_float2(1.f, 0.f);
     if (hh < H + G) cs = rope[(size_t)p * half + t];
     T *c = nullptr;
-    size_t o = 0;
+    size_t o = 0, ro = 0;
     if (hh >= H && write_kv) {
       const KVView v = views ? views[rowdoc[i]] : single;
       const int kv = hh < H + G ? 0 : 1;
       c = (T *)v.pages;
       o = v.offset(layer, kv, hh - H - kv * G, p);
+      // rows_out: K then V, each [M][L][G][dh]
+      ro = ((((size_t)kv * M + i) * L + layer) * G + (hh - H - kv * G)) * dh;
     }
     // dh divides 128: both halves of the head lie in one feature tile
     SplitTile stl{0, 0, 0};
@@ -242,6 +244,10 @@ __global__ void k_rope_scatter(const float *qkv, const float2 *rope, const int32
     if (!c) continue;
     st(c, o + t, x1);
     st(c, o + t + half, x2);
+    if (rows_out) {
+      st(rows_out, ro + t, x1);
+      st(rows_out, ro + t + half, x2);
+    }
   }
 }
 
@@ -276,22 +282,23 @@ __global__ void k_cache_gather(KVView v, const int32_t *pos, int n_pos, int l0, 
   }
 }
 
-// K/V of the given positions, layers l0 .. l0+nl-1, as stored (T in, T out)
-template <typename T>
+// K/V of the given positions, layers l0 .. l0+nl-1, as stored: 16-byte
+// pieces of the cache rows (a row is head_dim elements, a multiple of 16
+// bytes), vr pieces a row, output [n_pos][nl][G][row].
 __global__ void k_cache_gather_raw(KVView v, const int32_t *pos, int n_pos, int l0, int nl, int G,
-                                   int dh, T *k_out, T *v_out) {
-  size_t total = (size_t)n_pos * nl * G * dh;
-  const T *c = (const T *)v.pages;
-  for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < total;
-       e += (size_t)gridDim.x * blockDim.x) {
-    int i = (int)(e % dh);
-    size_t r = e / dh;
-    int g = (int)(r % G);
+                                   int vr, int es, uint4 *k_out, uint4 *v_out) {
+  const unsigned total = (unsigned)n_pos * nl * G * vr;
+  const uint4 *c = (const uint4 *)v.pages;
+  for (unsigned e = blockIdx.x * blockDim.x + threadIdx.x; e < total;
+       e += gridDim.x * blockDim.x) {
+    const unsigned i = e % vr;
+    unsigned r = e / vr;
+    const int g = (int)(r % G);
     r /= G;
-    int l = (int)(r % nl);
-    int p = (int)(r / nl);
-    k_out[e] = c[v.offset(l0 + l, 0, g, pos[p]) + i];
-    v_out[e] = c[v.offset(l0 + l, 1, g, pos[p]) + i];
+    const int l = (int)(r % nl);
+    const int p = pos[r / nl];
+    k_out[e] = c[v.offset(l0 + l, 0, g, p) * es / 16 + i];
+    v_out[e] = c[v.offset(l0 + l, 1, g, p) * es / 16 + i];
   }
 }
 
@@ -456,7 +463,7 @@ void launch_rmsnorm(float *h, const float *g, int row0, int M, int d, double eps
 void launch_rope_scatter(const float *qkv, const float2 *rope, const int32_t *pos, int M,
                          const Dims &dm, int layer, const KVView *views, const int32_t *rowdoc,
                          KVView single, float *q_out, void *qb_out, float qscale, bool write_kv,
-                         cudaStream_t s, const SplitView *sv) {
+                         cudaStream_t s, const SplitView *sv, void *rows_out) {
   if (M <= 0) return;
   const int rpb = M >= 1024 ? 8 : 1;  // rows per CTA
   dim3 grid((M + rpb - 1) / rpb, (dm.H + 2 * dm.G + ROPE_HEADS - 1) / ROPE_HEADS);
@@ -466,11 +473,11 @@ void launch_rope_scatter(const float *qkv, const float2 *rope, const int32_t *po
   if (dm.dtype == KVR_DTYPE_BF16)
     launch_pdl(k_rope_scatter<__nv_bfloat16>, grid, threads, 0, s, qkv, rope, pos, M, rpb, dm.H,
                dm.G, dm.dh, layer, views, rowdoc, single, q_out, (__nv_bfloat16 *)qb_out, qscale,
-               wk, v);
+               wk, v, (__nv_bfloat16 *)rows_out, dm.L);
   else
     launch_pdl(k_rope_scatter<float>, grid, threads, 0, s, qkv, rope, pos, M, rpb, dm.H, dm.G,
                dm.dh, layer, views, rowdoc, single, q_out, (__nv_bfloat16 *)qb_out, qscale, wk,
-               v);
+               v, (float *)rows_out, dm.L);
 }
 
 void launch_swiglu(const float *gu, int M, int F, void *act, int dtype, cudaStream_t s) {
@@ -496,14 +503,17 @@ void launch_cache_gather(KVView v, int dtype, const int32_t *pos, int n_pos, int
 
 void launch_cache_gather_raw(KVView v, int dtype, const int32_t *pos, int n_pos, int l0, int l1,
                              int G, int dh, void *k_out, void *v_out, cudaStream_t s) {
-  size_t n = (size_t)n_pos * (l1 - l0) * G * dh;
-  if (n == 0) return;
-  if (dtype == KVR_DTYPE_BF16)
-    k_cache_gather_raw<__nv_bfloat16><<<grid_for(n, 256), 256, 0, s>>>(
-        v, pos, n_pos, l0, l1 - l0, G, dh, (__nv_bfloat16 *)k_out, (__nv_bfloat16 *)v_out);
-  else
-    k_cache_gather_raw<float><<<grid_for(n, 256), 256, 0, s>>>(v, pos, n_pos, l0, l1 - l0, G, dh,
-                                                                (float *)k_out, (float *)v_out);
+  const int es = dtype == KVR_DTYPE_BF16 ? 2 : 4, vr = dh * es / 16;
+  const size_t per_pos = (size_t)(l1 - l0) * G * vr;
+  if (per_pos == 0) return;
+  // launches of fewer than 2^31 pieces (the kernel indexes in 32 bits)
+  const int chunk = (int)std::min<size_t>((size_t)n_pos, ((size_t)1 << 31) / per_pos);
+  for (int p0 = 0; p0 < n_pos; p0 += chunk) {
+    const int np = std::min(chunk, n_pos - p0);
+    k_cache_gather_raw<<<grid_for(np * per_pos, 256), 256, 0, s>>>(
+        v, pos + p0, np, l0, l1 - l0, G, vr, es, (uint4 *)k_out + p0 * per_pos,
+        (uint4 *)v_out + p0 * per_pos);
+  }
 }
 
 void launch_cache_scatter_raw(KVView v, int dtype, int p0, int n_pos, const void *k_in,

@@ -32,6 +32,7 @@
 namespace kvr {
 
 constexpr int KVR_PAGE = 64;          // positions per KV page
+constexpr int KVR_RD_GROUPS = 8;      // layer groups of kvr_repair_read's overlapped copies
 constexpr int KVR_QUERY_RESERVE = 64; // positions past n reserved for fresh queries
 constexpr int GU_BLOCK = 16;          // gate/up interleave block (rows)
 
@@ -245,6 +246,14 @@ struct kvr_model {
   int32_t *sel_count = nullptr;
   void *read_scratch = nullptr;  // cache readback: positions, then the gathered K and V
   size_t read_scratch_bytes = 0;
+  // kvr_repair_read: the pass's K/V rows as RoPE writes them, copied to the
+  // host group by group (on rd_stream, after the graph's rd_ev[g]) while the
+  // pass goes on; rd_cap carries the events' side branch inside a capture
+  void *rows_scratch = nullptr;
+  size_t rows_scratch_bytes = 0;
+  cudaStream_t rd_stream = nullptr, rd_cap = nullptr;
+  cudaEvent_t rd_ev[kvr::KVR_RD_GROUPS] = {}, rd_fork[kvr::KVR_RD_GROUPS] = {};
+  cudaEvent_t rd_join = nullptr;
   void *sel_scratch = nullptr;   // selector: edited tokens, saved stale rows, probabilities
   size_t sel_scratch_bytes = 0;
   void *batch_scratch = nullptr; // batched repair: documents' TMA views, cache views, tokens
@@ -263,6 +272,7 @@ struct kvr_model {
   size_t stage_off = 0;           // next free slot (copies take consecutive slots)
   cudaEvent_t stage_ev = nullptr;  // recorded after the last staged copy
   int32_t *rb_h = nullptr;         // pinned readback: selector count, flag, positions
+  int32_t *flag_h = nullptr;       // pinned readback of the device error flag
   // profiling
   bool prof = false;
   std::vector<kvr::ProfClass> prof_classes;
@@ -284,6 +294,7 @@ struct kvr_cache {
   bool poisoned = false;
   struct Graph {
     int M, nb, ns;
+    const void *rows_out;  // kvr_repair_read's row buffer, or null
     int64_t kernels;
     cudaGraphExec_t exec;
   };
@@ -451,11 +462,13 @@ void launch_embed_rows(const void *embed, int dtype, const int32_t *tokens,
 // view (rows indexed from h's base), the completed rows are written back to h.
 void launch_rmsnorm(float *h, const float *g, int row0, int M, int d, double eps, void *out,
                     int out_dtype, cudaStream_t s, const SplitView *sv = nullptr);
-// q_out: fp32 rotated q; qb_out (optional): bf16 rotated q times qscale.
+// q_out: fp32 rotated q; qb_out (optional): bf16 rotated q times qscale;
+// rows_out (optional, with write_kv): the K/V rows as written into the cache,
+// K then V, each [M][L][G][dh] in the cache dtype.
 void launch_rope_scatter(const float *qkv, const float2 *rope, const int32_t *pos, int M,
                          const Dims &dm, int layer, const KVView *views, const int32_t *rowdoc,
                          KVView single, float *q_out, void *qb_out, float qscale, bool write_kv,
-                         cudaStream_t s, const SplitView *sv = nullptr);
+                         cudaStream_t s, const SplitView *sv = nullptr, void *rows_out = nullptr);
 void launch_swiglu(const float *gu, int M, int F, void *act, int dtype, cudaStream_t s);
 void launch_cache_gather(KVView v, int dtype, const int32_t *pos, int n_pos, int l0, int l1,
                          int G, int dh, float *k_out, float *v_out, cudaStream_t s);

@@ -12,6 +12,7 @@ no fallback.
 """
 from __future__ import annotations
 
+import atexit
 import ctypes
 import os
 import weakref
@@ -82,6 +83,7 @@ _sigs = {
     "kvr_cache_load": ([_P, _P, _I32, _P, _P, ctypes.POINTER(_P)], _I32),
     "kvr_select": ([_P, _P, _I32, _I32, _I32, _I32, _P, ctypes.c_uint64, _P, _P], _I32),
     "kvr_repair": ([_P, _P, _I32, _I32, _P, _I32], _I32),
+    "kvr_repair_read": ([_P, _P, _I32, _I32, _P, _I32, _P, _P], _I32),
     "kvr_repair_batch": ([_P, _P, _I32], _I32),
     "kvr_logits": ([_P, _P, _P, _I32, _P], _I32),
     "kvr_cache_len": ([_P], _I32),
@@ -219,6 +221,23 @@ def kvr_select(model, cache, policy: str, K: int, edit_start: int, new_tokens,
 def kvr_repair(cache, new_tokens, edit_start: int, positions):
     nt, ps = _i32(new_tokens), _i32(positions)
     _check(_lib.kvr_repair(cache, _ptr(nt), edit_start, nt.size, _ptr(ps), ps.size))
+
+
+def kvr_repair_read(cache, new_tokens, edit_start: int, positions, n_layers: int,
+                    n_kv_heads: int, head_dim: int, dtype, k_out=None, v_out=None):
+    """kvr_repair, returning the K and V rows of P (the span, then positions)
+    as stored; k_out and v_out (optional, page-locked for the copies to
+    overlap the pass) receive them in place."""
+    nt, ps = _i32(new_tokens), _i32(positions)
+    shape = (nt.size + ps.size, n_layers, n_kv_heads, head_dim)
+    k = np.empty(shape, dtype) if k_out is None else k_out
+    v = np.empty(shape, dtype) if v_out is None else v_out
+    for a in (k, v):
+        if a.shape != shape or a.dtype != np.dtype(dtype) or not a.flags.c_contiguous:
+            raise ValueError(f"readback buffer must be C-contiguous {np.dtype(dtype)}{shape}")
+    _check(_lib.kvr_repair_read(cache, _ptr(nt), edit_start, nt.size, _ptr(ps), ps.size,
+                                k.ctypes.data, v.ctypes.data))
+    return k, v
 
 
 def kvr_repair_batch(model, reqs):
@@ -364,6 +383,18 @@ def kvr_launch_count(model) -> int:
 _ALLOC = ctypes.CFUNCTYPE(ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p)
 _FREE = ctypes.CFUNCTYPE(None, ctypes.c_void_p, ctypes.c_void_p)
 _hooks = []
+_live_models = weakref.WeakSet()
+
+
+def _close_all():
+    """Free every model still open (and with it its caches) while the
+    allocator that gave them their device memory is still alive: at
+    interpreter exit, finalisers otherwise run in no defined order."""
+    for m in list(_live_models):
+        m.close()
+
+
+atexit.register(_close_all)
 
 
 def use_torch_allocator():
@@ -379,11 +410,17 @@ def use_torch_allocator():
 
     def free(ptr, ctx):
         if ptr:
-            torch.cuda.caching_allocator_delete(ptr)
+            try:
+                torch.cuda.caching_allocator_delete(ptr)
+            except Exception:  # an exception cannot cross into the library
+                pass
 
     a, f = _ALLOC(alloc), _FREE(free)
     _hooks[:] = [a, f]
     _check(_lib.kvr_set_allocator(ctypes.cast(a, _P), ctypes.cast(f, _P), None))
+    # run before PyTorch's own exit handlers (registered at its import, earlier)
+    atexit.unregister(_close_all)
+    atexit.register(_close_all)
 
 
 def use_cuda_allocator():
@@ -399,6 +436,7 @@ class Model:
         self.cfg = dict(cfg)
         self._caches = weakref.WeakSet()
         self.h = kvr_model_create(cfg, weights, seed, max_context, max_rows)
+        _live_models.add(self)
 
     def close(self):
         if getattr(self, "h", None):
@@ -476,7 +514,9 @@ class Cache:
 
     def close(self):
         if getattr(self, "h", None):
-            kvr_cache_free(self.h)
+            # a freed model has freed its caches with it
+            if getattr(self.model, "h", None):
+                kvr_cache_free(self.h)
             self.h = None
 
     def __del__(self):
@@ -499,6 +539,13 @@ class Cache:
         c = self.model.cfg
         le = c["n_layers"] if layer_end is None else layer_end
         return kvr_cache_read(self.h, positions, layer_begin, le, c["n_kv_heads"], c["head_dim"])
+
+    def repair_read(self, new_tokens, edit_start: int, positions, k_out=None, v_out=None):
+        """repair, returning the K/V rows of P as stored (as read_raw over P)."""
+        c = self.model.cfg
+        dt = np.uint16 if c["dtype"] == "bf16" else np.float32
+        return kvr_repair_read(self.h, new_tokens, edit_start, positions, c["n_layers"],
+                               c["n_kv_heads"], c["head_dim"], dt, k_out, v_out)
 
     def read_raw(self, positions, layer_begin: int = 0, layer_end: int | None = None,
                  k_out=None, v_out=None):

@@ -5,6 +5,7 @@ import ctypes
 import os
 import re
 
+import numpy as np
 import pytest
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
@@ -54,6 +55,10 @@ def test_invalid_config_rejected_on_host(kv):
 def test_null_handles_rejected(kv):
     lib = kv._lib
     assert lib.kvr_repair(None, None, 0, 0, None, 0) == 1
+    assert lib.kvr_repair_read(None, None, 0, 0, None, 0, None, None) == 1
+    one = np.array([5], np.int32)
+    assert lib.kvr_repair_read(None, None, 0, 0, one.ctypes.data, 1, None, None) == 1
+    assert b"k_out" in lib.kvr_last_error()
     assert lib.kvr_prefill(None, None, 0, None) == 1
     assert lib.kvr_select(None, None, 0, 1, 0, 0, None, 0, None, None) == 1
     assert lib.kvr_logits(None, None, None, 1, None) == 1

@@ -6,6 +6,8 @@ logits.  Selected position sets must be identical except where the oracle's
 scores of the swapped positions lie within a tie band of the K-th score
 (exact ties for editlocal/structural/random).
 """
+import os
+
 import numpy as np
 import pytest
 
@@ -243,6 +245,53 @@ def test_model_on_torch_caching_allocator():
         kv.use_cuda_allocator()
     torch.cuda.synchronize()
     assert torch.cuda.memory_allocated() == before
+
+
+def test_unclosed_model_exits_cleanly():
+    # A program that leaves its model and cache open as module globals, on
+    # PyTorch's caching allocator, next to closures over them and PyTorch
+    # tensors of its own, exits with status 0 and no error from the free hook.
+    # (Without the binding's exit handler this program died with SIGSEGV at
+    # interpreter exit: the handles were freed after PyTorch's teardown.)
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    prog = """
+import numpy as np, torch
+from paper_2609_17983_gb300 import kvrepair as kv, synth
+cfg = synth.preset("tiny", dtype="bf16", n_layers=4)
+stream = torch.cuda.Stream(); torch.cuda.set_stream(stream)
+kv.use_torch_allocator()
+model = kv.Model(cfg, None, seed=0, max_context=8192, max_rows=512)
+model.set_stream(stream.cuda_stream)
+doc = synth.document(1, 5000, cfg["vocab"], cfg["delim_id"])
+new = synth.edit_tokens(2, doc[2500:2508], cfg["vocab"], cfg["delim_id"])
+cache = model.prefill(doc); model.synchronize()
+P = np.arange(2500, 2540)
+shape = (40, cfg["n_layers"], cfg["n_kv_heads"], cfg["head_dim"])
+k_rows = torch.empty(shape, dtype=torch.int16, pin_memory=True).numpy().view(np.uint16)
+v_rows = torch.empty(shape, dtype=torch.int16, pin_memory=True).numpy().view(np.uint16)
+A = model.select(cache, "editlocal", 32, 2500, new)
+def dev(fn, n=3):
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(n): fn()
+    e1.record(stream); torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / n
+sel = lambda: model.select(cache, "editlocal", 32, 2500, new)
+rep = lambda: cache.repair(new, 2500, A)
+rd = lambda: cache.read_raw(P, k_out=k_rows, v_out=v_rows)
+res = {"select": dev(sel), "repair": dev(rep), "read": dev(rd)}
+dsrc = torch.empty(k_rows.nbytes * 2, dtype=torch.uint8, device="cuda")
+hdst = torch.empty(k_rows.nbytes * 2, dtype=torch.uint8, pin_memory=True)
+res["d2h"] = dev(lambda: hdst.copy_(dsrc, non_blocking=True))
+print("done", sorted(res))
+"""
+    r = subprocess.run([sys.executable, "-c", prog], cwd=root, capture_output=True, text=True,
+                       timeout=300)
+    assert r.returncode == 0, r.stderr[-2000:]
+    assert "done" in r.stdout
+    assert "Exception ignored" not in r.stderr and "invalid device pointer" not in r.stderr
 
 
 def test_logits_parity_fp32(tiny):
@@ -565,6 +614,45 @@ def test_graph_replay_matches_eager():
         assert np.array_equal(k1, k2) and np.array_equal(v1, v2)
     eager.close()
     graph.close()
+
+
+@pytest.mark.parametrize("shape,layers", [("llama8b", 11), ("tiny", 3)])
+@pytest.mark.parametrize("graphs", [True, False])
+def test_repair_read_returns_the_repaired_rows(shape, layers, graphs):
+    # kvr_repair_read leaves the cache as kvr_repair does and returns exactly
+    # what kvr_cache_read_raw returns for P afterwards: on the capturing call
+    # and on replays (the copies wait on events the graph records on a side
+    # branch, layer groups with a ragged last one), and after eager launches
+    # (no stream of its own: no graph); into page-locked and pageable buffers
+    import torch
+    cfg = synth.preset(shape, n_layers=layers)
+    n, s, L = 600, 300, 8
+    doc = synth.document(1, n, cfg["vocab"])
+    new = synth.edit_tokens(2, doc[s:s + L], cfg["vocab"])
+    model = kv.Model(cfg, None, seed=0, max_context=1024, max_rows=256)
+    if graphs:
+        st = torch.cuda.Stream()
+        model.set_stream(st.cuda_stream)
+    ca, cb = model.prefill(doc), model.prefill(doc)
+    model.synchronize()
+    dt = np.uint16 if cfg["dtype"] == "bf16" else np.float32
+    shape_rows = (L + 32, layers, cfg["n_kv_heads"], cfg["head_dim"])
+    tdt = torch.int16 if dt == np.uint16 else torch.float32
+    pinned = [torch.empty(shape_rows, dtype=tdt, pin_memory=True).numpy().view(dt)
+              for _ in range(2)]
+    everything = np.arange(n)
+    for i, A in enumerate((np.arange(s + L, s + L + 32), np.arange(s + L + 5, s + L + 37),
+                           np.arange(s + L + 40, s + L + 72))):
+        P = np.concatenate([np.arange(s, s + L), A])
+        ca.repair(new, s, A)
+        want = ca.read_raw(P)
+        out = dict(k_out=pinned[0], v_out=pinned[1]) if i < 2 else {}
+        got = cb.repair_read(new, s, A, **out)
+        assert np.array_equal(got[0], want[0]) and np.array_equal(got[1], want[1])
+        ka, va = ca.read_raw(everything)
+        kb, vb = cb.read_raw(everything)
+        assert np.array_equal(ka, kb) and np.array_equal(va, vb)
+    model.close()
 
 
 @pytest.mark.parametrize("shape,policy", [("qwen7b", "attention"), ("mistral7b", "cacheblend"),
