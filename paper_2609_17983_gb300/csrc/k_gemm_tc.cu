@@ -82,11 +82,18 @@ struct TcParams {
   int defer;    // 1: split tiles are left as partials for the consumer
   int stream_w; // 1: each weight tile is read once (one token tile): L2 evict-first
   // grouped data-parallel mode (dp_groups > 0, many rows): grid = dp_groups x
-  // m_tiles CTAs; CTA i owns whole tiles -- token tile i % m_tiles of feature
-  // tiles (i / m_tiles) * dp_tpc ... + dp_tpc - 1 -- so the m_tiles CTAs of a
-  // group walk the same weight tiles in step and read each from DRAM once.
-  int dp_groups, dp_tpc;
+  // m_tiles CTAs; CTA i owns whole tiles -- token tile i % m_tiles of the
+  // feature tiles dp_first(j) .. dp_first(j + 1) - 1 of group j = i / m_tiles
+  // -- so the m_tiles CTAs of a group walk the same weight tiles in step and
+  // read each from DRAM once.
+  int dp_groups;
 };
+
+// First feature tile of data-parallel group j: groups take n_tiles / groups
+// tiles, rounded down or up.
+__device__ __forceinline__ int dp_first(const TcParams &p, int j) {
+  return (int)((long long)j * p.n_tiles / p.dp_groups);
+}
 
 // ------------------------------------------------------------ PTX wrappers
 
@@ -211,7 +218,7 @@ __device__ __forceinline__ void epi_range(const P &p, long long u0, long long u1
     uint32_t buf = seg & 1u, use = seg >> 1;
     int ntile = (int)(tl / p.m_tiles), mtile = (int)(tl % p.m_tiles);
     if (p.dp_groups) {  // a CTA-local tile of the grouped data-parallel mode
-      ntile = (int)(blockIdx.x / p.m_tiles) * p.dp_tpc + (int)tl;
+      ntile = dp_first(p, (int)(blockIdx.x / p.m_tiles)) + (int)tl;
       mtile = (int)(blockIdx.x % p.m_tiles);
     }
     int t0 = mtile * p.BN;
@@ -370,9 +377,10 @@ __global__ void __launch_bounds__(NTHREADS, 1)
   const uint32_t stage_bytes = A_BYTES + (uint32_t)p.BN * 128u;
   const uint32_t tx_bytes = A_BYTES + (uint32_t)p.brows * 128u;
   long long u0, u1;
-  if (p.dp_groups) {  // CTA-local units: dp_tpc whole tiles
+  if (p.dp_groups) {  // CTA-local units: the group's whole tiles
+    const int j = (int)(blockIdx.x / p.m_tiles);
     u0 = 0;
-    u1 = (long long)p.dp_tpc * p.KB;
+    u1 = (long long)(dp_first(p, j + 1) - dp_first(p, j)) * p.KB;
   } else {
     unit_range(blockIdx.x, p.total, p.grid, p.KB, p.cluster, u0, u1);
   }
@@ -418,7 +426,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       int kb = (int)(u0 - tl0 * p.KB);
       int ntile = (int)(tl0 / p.m_tiles), mtile = (int)(tl0 - (long long)ntile * p.m_tiles);
       if (p.dp_groups) {
-        ntile = (int)(blockIdx.x / p.m_tiles) * p.dp_tpc;
+        ntile = dp_first(p, (int)(blockIdx.x / p.m_tiles));
         mtile = (int)(blockIdx.x % p.m_tiles);
       }
       const int mstep = p.dp_groups ? 0 : 1;  // the data-parallel walk keeps its token tile
@@ -1127,12 +1135,14 @@ const char *configure(int M, int N, int K, int num_sms, bool defer, TcParams &p,
   p.cluster = p.m_tiles == 1 && !defer ? choose_cluster(M, N, num_sms, smem) : 0;
   p.stream_w = p.m_tiles == 1;
   if (p.cluster > 1) p.grid = p.n_tiles * p.cluster;
-  p.dp_groups = p.dp_tpc = 0;
+  p.dp_groups = 0;
   // Many rows (a prefill chunk): the grouped data-parallel mode when some
   // token tile width and group count fill at least 90% of the SMs' slots with
-  // useful rows.  Stream-K there walks all token tiles of a feature tile per
-  // CTA, so the 152 CTAs' weights (about 1 MB each) overflow L2 and every
-  // weight tile came from DRAM once per token tile.
+  // useful work: rows over padded rows, CTAs over SMs, and a group's tiles
+  // over the largest group's (groups need not divide the feature tiles).
+  // Stream-K there walks all token tiles of a feature tile per CTA, so the
+  // 152 CTAs' weights (about 1 MB each) overflow L2 and every weight tile
+  // came from DRAM once per token tile.
   static const bool dp_off = [] {
     const char *e = getenv("KVR_DISABLE_DP_GEMM");
     return e && e[0] == '1';
@@ -1143,8 +1153,9 @@ const char *configure(int M, int N, int K, int num_sms, bool defer, TcParams &p,
     for (int bn = 256; bn >= 128; bn -= 16) {
       const int mt = (M + bn - 1) / bn;
       for (int g = 1; g <= p.n_tiles && g * mt <= num_sms; ++g) {
-        if (p.n_tiles % g) continue;
-        const double eff = (double)M / ((double)mt * bn) * (double)(g * mt) / num_sms;
+        const int most = (p.n_tiles + g - 1) / g;
+        const double eff = (double)M / ((double)mt * bn) * (double)(g * mt) / num_sms *
+                           ((double)p.n_tiles / g / most);
         if (eff > best + 1e-9) {
           best = eff;
           bbn = bn;
@@ -1162,7 +1173,6 @@ const char *configure(int M, int N, int K, int num_sms, bool defer, TcParams &p,
       p.total = (long long)p.n_tiles * p.m_tiles * p.KB;
       p.grid = bg * bmt;
       p.dp_groups = bg;
-      p.dp_tpc = p.n_tiles / bg;
       p.stages = st > 8 ? 8 : st;
       uint32_t c2 = 32;
       while (c2 < (uint32_t)p.BN) c2 <<= 1;

@@ -159,14 +159,17 @@ __global__ void __launch_bounds__(TPB, TPB == NORM_THREADS_WIDE && NV <= 4 ? 4 :
   }
 }
 
-// grid (M, ceil((H + 2G) / ROPE_HEADS)), block ROPE_HEADS * dh/2: rotate q and
-// k heads at the row's position;
-// q -> q_out fp32 (if given) and qb_out, k and v -> cache (if write_kv).  With a
-// split view the projection is completed from the GEMM's split-tile partials.  Positions,
-// the RoPE table, the page table and the bias are written before the pass,
-// so they are read before the wait on the projection.
+// grid (ceil(M / rpb), ceil((H + 2G) / ROPE_HEADS)), block ROPE_HEADS * dh/2:
+// rotate q and k heads at the row's position; q -> q_out fp32 (if given) and
+// qb_out, k and v -> cache (if write_kv) and rows_out (if given).  With a
+// split view the projection is completed from the GEMM's split-tile
+// partials.  Positions, the RoPE table, the page table and the bias are
+// written before the pass, so they are read before the wait on the
+// projection.  RPB > 1 (a prefill chunk, no split view): the CTA's RPB rows
+// are loaded together, one round trip for all of them.
 constexpr int ROPE_HEADS = 8;  // heads per CTA
-template <typename T>
+constexpr int ROPE_RPB = 8;    // rows per CTA of a many-row pass
+template <typename T, int RPB>
 __global__ void k_rope_scatter(const float *qkv, const float2 *rope, const int32_t *pos, int M,
                                int rpb, int H, int G, int dh, int layer, const KVView *views,
                                const int32_t *rowdoc, KVView single, float *q_out,
@@ -179,24 +182,83 @@ __global__ void k_rope_scatter(const float *qkv, const float2 *rope, const int32
   if (hh >= H + 2 * G) return;
   const int Nqkv = (H + 2 * G) * dh;
   const int n1 = hh * dh + t, n2 = n1 + half;
-  // rows r0 .. r1-1 (one for a pass of a few rows; several for a prefill
-  // chunk, where one row per CTA spent its time starting CTAs); the first
-  // row's position, table entries and split tile are read before the wait
+  const int kv = hh < H + G ? 0 : 1, gk = hh - H - kv * G;
+  // the row's cache entry (o) and rows_out entry (ro), for k and v heads
+  auto kv_dst = [&](int i, int p, T *&c, size_t &o, size_t &ro) {
+    c = nullptr;
+    if (hh >= H && write_kv) {
+      const KVView v = views ? views[rowdoc[i]] : single;
+      c = (T *)v.pages;
+      o = v.offset(layer, kv, gk, p);
+      // rows_out: K then V, each [M][L][G][dh]
+      ro = ((((size_t)kv * M + i) * L + layer) * G + gk) * dh;
+    }
+  };
+  auto out = [&](int i, float x1, float x2, float2 cs, T *c, size_t o, size_t ro) {
+    if (hh < H + G) {
+      const float r1r = x1 * cs.x - x2 * cs.y;
+      const float r2r = x2 * cs.x + x1 * cs.y;
+      x1 = r1r;
+      x2 = r2r;
+    }
+    if (hh < H) {
+      if (q_out) {
+        float *qo = q_out + (size_t)i * H * dh + (size_t)hh * dh;
+        qo[t] = x1;
+        qo[t + half] = x2;
+      }
+      if (qb_out) {
+        __nv_bfloat16 *qb = qb_out + (size_t)i * H * dh + (size_t)hh * dh;
+        qb[t] = __float2bfloat16_rn(x1 * qscale);
+        qb[t + half] = __float2bfloat16_rn(x2 * qscale);
+      }
+      return;
+    }
+    if (!c) return;
+    st(c, o + t, x1);
+    st(c, o + t + half, x2);
+    if (rows_out) {
+      st(rows_out, ro + t, x1);
+      st(rows_out, ro + t + half, x2);
+    }
+  };
+  if constexpr (RPB > 1) {
+    const int r0 = blockIdx.x * RPB, nr = min(RPB, M - r0);
+    int p[RPB];
+    float2 cs[RPB];
+    T *c[RPB];
+    size_t o[RPB], ro[RPB];
+#pragma unroll
+    for (int k = 0; k < RPB; ++k) {
+      p[k] = k < nr ? pos[r0 + k] : 0;
+      cs[k] = hh < H + G && k < nr ? rope[(size_t)p[k] * half + t] : make_float2(1.f, 0.f);
+      c[k] = nullptr;
+      if (k < nr) kv_dst(r0 + k, p[k], c[k], o[k], ro[k]);
+    }
+    pdl_wait();
+    ts.waited();
+    float x1[RPB], x2[RPB];
+#pragma unroll
+    for (int k = 0; k < RPB; ++k) {
+      const float *x = qkv + (size_t)(r0 + k) * Nqkv;
+      x1[k] = k < nr ? x[n1] : 0.f;
+      x2[k] = k < nr ? x[n2] : 0.f;
+    }
+#pragma unroll
+    for (int k = 0; k < RPB; ++k)
+      if (k < nr) out(r0 + k, x1[k], x2[k], cs[k], c[k], o[k], ro[k]);
+    return;
+  }
+  // rows r0 .. r1-1 one after another; the first row's position, table
+  // entries and split tile are read before the wait
   const int r0 = blockIdx.x * rpb, r1 = min(M, r0 + rpb);
   for (int i = r0; i < r1; ++i) {
     const int p = pos[i];
     float2 cs = make_float2(1.f, 0.f);
     if (hh < H + G) cs = rope[(size_t)p * half + t];
-    T *c = nullptr;
+    T *c;
     size_t o = 0, ro = 0;
-    if (hh >= H && write_kv) {
-      const KVView v = views ? views[rowdoc[i]] : single;
-      const int kv = hh < H + G ? 0 : 1;
-      c = (T *)v.pages;
-      o = v.offset(layer, kv, hh - H - kv * G, p);
-      // rows_out: K then V, each [M][L][G][dh]
-      ro = ((((size_t)kv * M + i) * L + layer) * G + (hh - H - kv * G)) * dh;
-    }
+    kv_dst(i, p, c, o, ro);
     // dh divides 128: both halves of the head lie in one feature tile
     SplitTile stl{0, 0, 0};
     float b1 = 0.f, b2 = 0.f;
@@ -222,32 +284,7 @@ __global__ void k_rope_scatter(const float *qkv, const float2 *rope, const int32
       x1 = x[n1];
       x2 = x[n2];
     }
-    if (hh < H + G) {
-      const float r1r = x1 * cs.x - x2 * cs.y;
-      const float r2r = x2 * cs.x + x1 * cs.y;
-      x1 = r1r;
-      x2 = r2r;
-    }
-    if (hh < H) {
-      if (q_out) {
-        float *qo = q_out + (size_t)i * H * dh + (size_t)hh * dh;
-        qo[t] = x1;
-        qo[t + half] = x2;
-      }
-      if (qb_out) {
-        __nv_bfloat16 *qb = qb_out + (size_t)i * H * dh + (size_t)hh * dh;
-        qb[t] = __float2bfloat16_rn(x1 * qscale);
-        qb[t + half] = __float2bfloat16_rn(x2 * qscale);
-      }
-      continue;
-    }
-    if (!c) continue;
-    st(c, o + t, x1);
-    st(c, o + t + half, x2);
-    if (rows_out) {
-      st(rows_out, ro + t, x1);
-      st(rows_out, ro + t + half, x2);
-    }
+    out(i, x1, x2, cs, c, o, ro);
   }
 }
 
@@ -465,19 +502,24 @@ void launch_rope_scatter(const float *qkv, const float2 *rope, const int32_t *po
                          KVView single, float *q_out, void *qb_out, float qscale, bool write_kv,
                          cudaStream_t s, const SplitView *sv, void *rows_out) {
   if (M <= 0) return;
-  const int rpb = M >= 1024 ? 8 : 1;  // rows per CTA
+  const SplitView v = sv ? *sv : SplitView{};
+  // a prefill chunk: several rows per CTA (one row per CTA spent its time
+  // starting CTAs), loaded together when the projection is complete
+  const int rpb = M >= 1024 ? ROPE_RPB : 1;
+  const bool batched = rpb > 1 && !v.ws;
   dim3 grid((M + rpb - 1) / rpb, (dm.H + 2 * dm.G + ROPE_HEADS - 1) / ROPE_HEADS);
   const int threads = ROPE_HEADS * dm.dh / 2;
   int wk = write_kv ? 1 : 0;
-  const SplitView v = sv ? *sv : SplitView{};
+  auto go = [&](auto *tag) {
+    using T = std::remove_pointer_t<decltype(tag)>;
+    launch_pdl(batched ? k_rope_scatter<T, ROPE_RPB> : k_rope_scatter<T, 1>, grid, threads, 0, s,
+               qkv, rope, pos, M, rpb, dm.H, dm.G, dm.dh, layer, views, rowdoc, single, q_out,
+               (__nv_bfloat16 *)qb_out, qscale, wk, v, (T *)rows_out, dm.L);
+  };
   if (dm.dtype == KVR_DTYPE_BF16)
-    launch_pdl(k_rope_scatter<__nv_bfloat16>, grid, threads, 0, s, qkv, rope, pos, M, rpb, dm.H,
-               dm.G, dm.dh, layer, views, rowdoc, single, q_out, (__nv_bfloat16 *)qb_out, qscale,
-               wk, v, (__nv_bfloat16 *)rows_out, dm.L);
+    go((__nv_bfloat16 *)nullptr);
   else
-    launch_pdl(k_rope_scatter<float>, grid, threads, 0, s, qkv, rope, pos, M, rpb, dm.H, dm.G,
-               dm.dh, layer, views, rowdoc, single, q_out, (__nv_bfloat16 *)qb_out, qscale, wk,
-               v, (float *)rows_out, dm.L);
+    go((float *)nullptr);
 }
 
 void launch_swiglu(const float *gu, int M, int F, void *act, int dtype, cudaStream_t s) {

@@ -63,11 +63,12 @@ def test_lm_head_matches_fp64_matmul(model):
     assert rel(got, f64(x) @ f64(lm).T) <= 1e-3
 
 
-@pytest.mark.parametrize("M", [512, 4096])
+@pytest.mark.parametrize("M", [512, 904, 4096])
 def test_many_row_projections_match_fp64_matmul(M):
     # a prefill chunk's row counts: the grouped data-parallel tiling (whole
-    # tiles per CTA, token tiles of up to 256 rows with a ragged last one);
-    # the fp64 reference on a sample of rows from every token tile
+    # tiles per CTA, token tiles of up to 256 rows with a ragged last one;
+    # at 904 rows gate/up's 224 feature tiles in 38 groups of 5 or 6); the
+    # fp64 reference on a sample of rows from every token tile
     cfg = synth.preset("llama8b", n_layers=1)
     m = kv.Model(cfg, None, seed=0, max_context=512, max_rows=4096)
     d, F = cfg["d_model"], cfg["ffn"]
