@@ -224,8 +224,8 @@ def run_reference(args, cfg, rank):
 # DRAM bytes (read + write) of one gate/up GEMM launch at this workload's shape
 # (40 x 28672 x 4096), from one ncu capture of that launch; reported only while the
 # GEMM kernel's source is the one the capture was taken on.
-GU_TRAFFIC_BYTES = 235280384 + 2372864
-GU_TRAFFIC_SOURCE_SHA256 = "8c50084a4dde7e11d5b7e916f8acb26422331cd7d45204691d56920573cc9aa6"
+GU_TRAFFIC_BYTES = 235281920 + 2391808
+GU_TRAFFIC_SOURCE_SHA256 = "c781d22d35957a5c5c4aba8ccf399d42580e2d37d3d470495c2b3b372a9e1547"
 
 
 def workload_config(cfg: dict, world: int) -> dict:
