@@ -31,13 +31,15 @@ Pin status (what each function is checked against, in tests/test_oracle_*.py):
   logits_all / answer_logprob -- the textbook decoder run over C' + query.
   transplant           -- identity (all positions) and no-op (none) cases.
   random               -- published SplitMix64 test vectors, uniformity.
-  attention score      -- special cases: zero W_q gives uniform scores (ties ->
+  attention score      -- the reading computed from two textbook forwards (the
+                          fresh span queries of C', the stale pool keys of C,
+                          softmax over the pool, summed over layers, heads and
+                          span rows); zero W_q gives uniform scores (ties ->
                           EditLocal set); the scores sum to layers*heads*|S|.
-                          Otherwise parity unpinned.
-  cacheblend score     -- special cases: an edit that changes no token gives
-                          all-zero deviation; zero attention/MLP output
-                          projections give zero deviation.  Otherwise parity
-                          unpinned.
+  cacheblend score     -- the layer-1 K/V deviation between two textbook
+                          forwards (C' and C) over the pool; equal to the
+                          deviation a full-suffix repair leaves; an edit that
+                          changes no token gives all-zero deviation.
   topk                 -- hand-written golden cases with ties and NaN.
 """
 from __future__ import annotations
