@@ -502,8 +502,11 @@ def main():
         cache.repair_read(new, EDIT_START, A, k_out=k_rows, v_out=v_rows)
     barrier()
     e2e_s = max_over_ranks((time.perf_counter() - t0) / args.steps, "cuda")
-    h2d = int(new.nbytes + 4 * K_BUDGET + 4 * M)
-    d2h = int(k_rows.nbytes + v_rows.nbytes + 4 * K_BUDGET)
+    # what the two calls copy: kvr_select the new tokens in, the count, the
+    # device flag and the K positions out; kvr_repair_read the new tokens and
+    # the M positions of P in, the rows' K and V and the device flag out
+    h2d = int(2 * new.nbytes + 4 * M)
+    d2h = int(4 * (K_BUDGET + 2) + k_rows.nbytes + v_rows.nbytes + 4)
 
     # selector time, reported apart from the repair (the paper's protocol): each
     # policy on this cache, median of 3 after one warm-up; and the repair alone
